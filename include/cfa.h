@@ -1,0 +1,320 @@
+/*
+ * cfa.h -- C ABI of the chunked tensor-materialization loader.
+ *
+ * The loader brings a model checkpoint ("the blob": one contiguous byte stream holding every
+ * tensor of the model) from host memory into a serving engine's final per-parameter layout on
+ * one GPU.  It follows the refined tensor-materialization automaton of InstantInfer
+ * (arXiv 2607.18957, section 4.2 "Tensor Materialization", refined CFA model):
+ *
+ *   - the blob is cut into equal-length chunks, the last one possibly partial;
+ *   - the tensor <-> chunk association (tensor.chunks / chunk.tensors) is precomputed once,
+ *     here by cfa_plan_create;
+ *   - each chunk moves InDisk -> InMem -> InGPU -> Destroyed through a two-stage pipeline
+ *     (section 4.2, dependency (i)): host staging into a pinned slot, then a host->device copy
+ *     into a device staging slot;
+ *   - once a chunk is InGPU, one batched GPU kernel copies and assembles every tensor piece
+ *     that lies in it into its destination (dependency (ii)), which moves those tensors from
+ *     Alloc to Loaded;
+ *   - the chunk's staging slot is released once all its pieces are written (dependency (iii)).
+ *
+ * Beyond what the paper states, the kernel also fuses the serving engine's layout transforms
+ * (several checkpoint tensors written at row offsets of one fused destination, e.g. q/k/v into
+ * one qkv weight), an optional fp32 -> bf16 round-to-nearest-even cast, and an optional
+ * per-tensor 64-bit additive checksum of the destination element bits.
+ *
+ * Conventions for every function below:
+ *   - The return value is a cfa_status: CFA_OK (0) on success, a negative CFA_ERR_* code
+ *     otherwise.  No function aborts, throws, traps the GPU or spins without a bound.
+ *   - cfa_last_error(plan) gives a human-readable detail of the last failure on that plan;
+ *     cfa_last_error(NULL) gives the detail of the last failure of cfa_plan_create on the
+ *     calling thread.
+ *   - "device pointer" means an address in the global memory of the plan's CUDA device;
+ *     "host pointer" means ordinary process memory.
+ *   - Streams are CUDA runtime streams (cudaStream_t); NULL is the legacy default stream.
+ *   - All integers are little-endian, as on both the host and the GPU.
+ */
+#ifndef CFA_H
+#define CFA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t, declared here so that this header needs no CUDA header. */
+typedef struct CUstream_st *cfa_stream;
+
+typedef int cfa_status;
+
+#define CFA_OK            0
+#define CFA_ERR_INVAL    (-1)  /* bad argument, bad option, or malformed manifest entry */
+#define CFA_ERR_OVERLAP  (-2)  /* two pieces (or two destinations) write the same bytes */
+#define CFA_ERR_OOB      (-3)  /* an entry reads past the blob or writes past its destination */
+#define CFA_ERR_COVERAGE (-4)  /* strict mode: some destination byte is written by no entry */
+#define CFA_ERR_CUDA     (-5)  /* a CUDA runtime call failed; detail in cfa_last_error */
+#define CFA_ERR_SOURCE   (-6)  /* the source callback reported an error */
+#define CFA_ERR_TIMEOUT  (-7)  /* a host wait reached its deadline; nothing was cancelled */
+#define CFA_ERR_BUSY     (-8)  /* the plan is in use by another thread */
+#define CFA_ERR_NOMEM    (-9)  /* a host or device allocation failed */
+#define CFA_ERR_DTYPE    (-10) /* source and destination dtypes do not match the entry's cast */
+#define CFA_ERR_ALIGN    (-11) /* an offset, pointer or size breaks an alignment rule */
+#define CFA_ERR_DEVICE   (-12) /* the unpack kernel's own descriptor check failed (debug mode) */
+
+/* Element types.  Only the element size matters for plain copies; 1-byte types cover int8,
+ * uint8 and the fp8 formats. */
+#define CFA_DTYPE_U8    1
+#define CFA_DTYPE_BF16  2
+#define CFA_DTYPE_F16   3
+#define CFA_DTYPE_F32   4
+#define CFA_DTYPE_I32   5
+#define CFA_DTYPE_I64   6
+#define CFA_DTYPE_F64   7
+
+#define CFA_MAX_DIMS    8
+#define CFA_MAX_LAYERS  65536
+
+/* cfa_tensor_entry.flags */
+#define CFA_ENTRY_CAST_BF16 0x1u /* source fp32, destination bf16, round to nearest even */
+#define CFA_ENTRY_CKSUM     0x2u /* accumulate this entry's checksum (see cfa_get_checksums) */
+
+/* Passed as `layer` to cfa_wait_layer / cfa_get_layer_times: the whole load. */
+#define CFA_ALL (-1)
+
+/*
+ * One checkpoint tensor (one tensor component of section 4.2).
+ *
+ *   name            optional, copied by cfa_plan_create; used only in error messages.
+ *   src_dtype       CFA_DTYPE_* of the elements in the blob.
+ *   ndim, shape     logical shape, row-major and contiguous in the blob; ndim 0 is a scalar.
+ *                   Zero-element tensors are valid and load nothing.
+ *   blob_offset     byte offset of element 0 in the blob; a multiple of the source element size.
+ *   dst_index       index into the cfa_dst array.
+ *   layer           readiness group, 0 <= layer < CFA_MAX_LAYERS (cfa_wait_layer).
+ *   dst_row_offset  where the tensor starts inside its destination, in destination rows.
+ *                   For a destination of ndim >= 2, a row is its last dimension R = shape[-1]:
+ *                   the entry's last dimension must equal R and the entry fills
+ *                   numel / R consecutive rows starting at dst_row_offset.  For a destination
+ *                   of ndim <= 1 a row is one element.  This is how fused layouts are written:
+ *                   q, k, v at rows 0, Hq, Hq + Hkv of qkv; gate, up at rows 0, I of gate_up;
+ *                   expert e's w1, w3 at rows 2Ie, 2Ie + I of the [E*2I, H] view of w13.
+ *   flags           CFA_ENTRY_*.  Without CFA_ENTRY_CAST_BF16 the destination dtype must
+ *                   equal src_dtype; with it, src_dtype must be F32 and the destination BF16.
+ */
+typedef struct cfa_tensor_entry {
+    const char *name;
+    int32_t src_dtype;
+    int32_t ndim;
+    int64_t shape[CFA_MAX_DIMS];
+    uint64_t blob_offset;
+    int32_t dst_index;
+    int32_t layer;
+    int64_t dst_row_offset;
+    uint32_t flags;
+    uint32_t reserved; /* must be 0 */
+} cfa_tensor_entry;
+
+/*
+ * One destination parameter of the serving engine (a Loaded tensor of section 4.2).
+ * dev_ptr is a device pointer owned by the caller, aligned to its element size (16-byte
+ * alignment is what makes the vector path apply), and it must stay valid for every load that
+ * uses the plan.  Destinations must not overlap one another in memory.
+ */
+typedef struct cfa_dst {
+    void *dev_ptr;
+    int32_t dtype;
+    int32_t ndim;
+    int64_t shape[CFA_MAX_DIMS];
+} cfa_dst;
+
+/* cfa_plan_opts.flags */
+#define CFA_OPT_STRICT_COVERAGE 0x1u  /* every destination byte must be written exactly once */
+#define CFA_OPT_HOST_ONLY       0x2u  /* build and validate on the host only: no CUDA call is made,
+                                         cfa_plan_get_pieces works, loads return CFA_ERR_INVAL */
+#define CFA_OPT_TIMING          0x4u  /* record per-chunk timing events (cfa_get_stats, timeline) */
+#define CFA_OPT_NO_BULK         0x8u  /* never use the TMA bulk-copy kernel */
+#define CFA_OPT_DEBUG_CHECKS    0x10u /* the kernel re-checks every descriptor against the chunk
+                                         and reports CFA_ERR_DEVICE instead of touching memory */
+#define CFA_OPT_NO_MERGE        0x20u /* DEVICE sources: one launch per chunk instead of one
+                                         launch per contiguous run of chunks */
+
+typedef struct cfa_plan_opts {
+    uint64_t chunk_bytes;     /* chunk length S, a multiple of 256; default 512 MiB */
+    int32_t host_slots;       /* pinned host staging slots of S bytes (0 = none, else >= 2); default 2 */
+    int32_t dev_slots;        /* device staging slots of S bytes (0 = none, else >= 2); default 2 */
+    int32_t fill_threads;     /* host threads copying pageable sources into pinned slots; default 8 */
+    int32_t device;           /* CUDA device ordinal; -1 = the current device */
+    uint32_t slab_bytes;      /* destination bytes per block-level work item, a multiple of 4096;
+                                 default 65536 */
+    uint32_t tiny_bytes;      /* pieces with fewer destination bytes go warp-per-descriptor;
+                                 default 8192 */
+    uint32_t flags;           /* CFA_OPT_*; default CFA_OPT_STRICT_COVERAGE */
+    uint32_t reserved;        /* must be 0 */
+    void *workspace;          /* optional device memory for the staging slots (NULL = plan allocates) */
+    uint64_t workspace_bytes; /* must be >= dev_slots * chunk_bytes when workspace is given */
+} cfa_plan_opts;
+
+/* Fills *opts with the defaults listed above. */
+void cfa_plan_opts_default(cfa_plan_opts *opts);
+
+/* Source kinds (cfa_source.kind). */
+#define CFA_SRC_HOST     1 /* pageable host memory; copied into pinned slots by host threads */
+#define CFA_SRC_PINNED   2 /* page-locked host memory; copied straight to the device slots */
+#define CFA_SRC_CALLBACK 3 /* fill(user, blob_offset, dst, len) writes the bytes into a pinned slot */
+#define CFA_SRC_DEVICE   4 /* device memory already holding the blob; no staging, no copies */
+
+/* Writes blob bytes [blob_offset, blob_offset + len) to host memory dst and returns 0, or
+ * returns non-zero on failure.  It runs on a CUDA host-function thread and must not call CUDA. */
+typedef int (*cfa_fill_fn)(void *user, uint64_t blob_offset, void *dst, uint64_t len);
+
+/*
+ * Where the blob's bytes come from.  With period_bytes == 0, blob byte o is base[o].  With
+ * period_bytes > 0 (a multiple of chunk_bytes), the blob is periodic and byte o is
+ * base[o % period_bytes]; this streams a blob larger than memory from a smaller pool.  base must
+ * be 256-byte aligned for PINNED and DEVICE sources.  The source must stay valid until the load
+ * has completed (cfa_wait_layer(CFA_ALL) returned CFA_OK).
+ */
+typedef struct cfa_source {
+    int32_t kind;
+    int32_t reserved;
+    const void *base;
+    uint64_t period_bytes;
+    cfa_fill_fn fill;
+    void *user;
+} cfa_source;
+
+typedef struct cfa_plan cfa_plan;
+
+typedef struct cfa_stats {
+    uint64_t blob_bytes;
+    uint64_t n_entries, n_dsts, n_chunks, n_layers;
+    uint64_t n_pieces;        /* tensor x chunk intersections */
+    uint64_t n_slabs;         /* block-level work items (vector path) */
+    uint64_t n_bulk;          /* block-level work items (TMA bulk path) */
+    uint64_t n_tiny;          /* warp-level work items */
+    uint64_t bytes_read;      /* algorithmic bytes one load reads from staging */
+    uint64_t bytes_written;   /* algorithmic bytes one load writes into destinations */
+    uint64_t descriptor_bytes;
+    uint64_t loads;           /* loads enqueued on this plan */
+    uint64_t kernel_launches; /* unpack kernel launches enqueued by the last load */
+    double plan_ms;           /* host time spent in cfa_plan_create */
+    /* CFA_OPT_TIMING only, valid once the last load has completed: */
+    double load_ms;           /* first enqueued operation to last unpack, device clock */
+    double h2d_ms;            /* sum over chunks of the host->device copy time */
+    double unpack_ms;         /* sum over launches of the unpack kernel time */
+} cfa_stats;
+
+/* A piece (tensor x chunk) as the plan builder cut it; for inspection and tests. */
+typedef struct cfa_piece {
+    uint32_t chunk;
+    uint32_t entry;
+    uint64_t src_offset;      /* byte offset in the blob */
+    uint32_t dst_index;
+    uint32_t cast;
+    uint64_t dst_offset;      /* byte offset inside the destination */
+    uint64_t n_elems;
+} cfa_piece;
+
+/*
+ * Validates the manifest, precomputes the chunk <-> tensor mapping (section 4.2) and cuts
+ * every tensor into pieces, then, unless CFA_OPT_HOST_ONLY is set, uploads the descriptor table
+ * to the device and allocates the staging slots, the streams and the events.
+ *
+ *   entries, n_entries  the checkpoint's tensors (host memory; copied, may be freed on return).
+ *   dsts, n_dsts        the destinations (host array; copied; dev_ptr stays caller-owned).
+ *   blob_bytes          length of the blob; every entry must lie inside it.
+ *   opts                NULL for the defaults.
+ *   out                 receives the plan; set to NULL on failure.
+ *
+ * Errors: CFA_ERR_INVAL, CFA_ERR_DTYPE, CFA_ERR_ALIGN, CFA_ERR_OOB, CFA_ERR_OVERLAP,
+ * CFA_ERR_COVERAGE (strict mode), CFA_ERR_NOMEM, CFA_ERR_CUDA.  Nothing is left allocated.
+ */
+cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
+                           const cfa_dst *dsts, size_t n_dsts, uint64_t blob_bytes,
+                           const cfa_plan_opts *opts, cfa_plan **out);
+
+/*
+ * Enqueues one complete load of the blob into the destinations and returns without waiting.
+ * Every chunk goes through: host staging (HOST: copied by the plan's fill threads; CALLBACK:
+ * written by src->fill; PINNED and DEVICE: none), a host->device copy on the plan's copy
+ * stream (none for DEVICE), and one unpack kernel on `stream` that writes all pieces of the
+ * chunk (DEVICE sources merge contiguous chunks into one launch).  The load is ordered after
+ * all work enqueued on `stream` before this call, and work enqueued on `stream` after this
+ * call sees every destination written.  Per-layer readiness is published through
+ * cfa_wait_layer.  Loads on one plan run in the order they were enqueued; the checksums and
+ * layer events always refer to the most recently enqueued load.
+ *
+ * Errors: CFA_ERR_INVAL (bad source, host-only plan, or a staging kind the plan has no slots
+ * for), CFA_ERR_ALIGN, CFA_ERR_CUDA.  Failures that happen later (the callback, a CUDA error)
+ * are latched and returned by cfa_wait_layer / cfa_get_checksums for that load.
+ */
+cfa_status cfa_load_async(cfa_plan *plan, const cfa_source *src, cfa_stream stream);
+
+/*
+ * Waits until readiness group `layer` of the last load is Loaded (all its tensors written), or
+ * the whole load with layer == CFA_ALL.
+ *   consumer != NULL: makes that stream wait on the GPU (no host blocking) and returns.
+ *   consumer == NULL: blocks the host, polling without spinning on the GPU, until the group is
+ *                     ready or timeout_ns (< 0: no limit) has passed; then CFA_ERR_TIMEOUT.
+ * Errors: CFA_ERR_INVAL (unknown layer, no load yet), CFA_ERR_TIMEOUT, CFA_ERR_SOURCE,
+ * CFA_ERR_CUDA, CFA_ERR_DEVICE.
+ */
+cfa_status cfa_wait_layer(cfa_plan *plan, int32_t layer, cfa_stream consumer, int64_t timeout_ns);
+
+/*
+ * Copies the per-entry checksums of the last load to host_out[0 .. n) (n <= n_entries), in entry
+ * order.  An entry's checksum is the sum, modulo 2^64, of its destination elements' bit patterns
+ * read as unsigned integers of the destination element size (after the cast).  Entries without
+ * CFA_ENTRY_CKSUM read 0.  Blocks until the load has completed.
+ */
+cfa_status cfa_get_checksums(cfa_plan *plan, uint64_t *host_out, size_t n);
+
+/* Fills *out.  Blocks until the last load has completed if CFA_OPT_TIMING is set. */
+cfa_status cfa_get_stats(cfa_plan *plan, cfa_stats *out);
+
+/*
+ * Milliseconds from the first operation of the last load to the moment each readiness group was
+ * Loaded, for groups 0 .. n-1 (CFA_OPT_TIMING plans; blocks until the load completes).
+ */
+cfa_status cfa_get_layer_times(cfa_plan *plan, float *ms_out, size_t n);
+
+/*
+ * Number of readiness groups and pieces of the plan; then the pieces themselves, in chunk order
+ * (at most cap of them into out).  Host-only; works on CFA_OPT_HOST_ONLY plans.
+ */
+cfa_status cfa_plan_info(const cfa_plan *plan, uint64_t *n_layers, uint64_t *n_pieces,
+                         uint64_t *n_chunks);
+cfa_status cfa_plan_get_pieces(const cfa_plan *plan, cfa_piece *out, size_t cap, size_t *n_out);
+
+/*
+ * Unpacks chunks [chunk_begin, chunk_end) that the caller has already placed in device memory:
+ * blob byte o of those chunks is at chunk_src + (o - chunk_begin * chunk_bytes).  chunk_src is a
+ * device pointer, 256-byte aligned.  One kernel launch on `stream`; checksums accumulate into
+ * the plan's checksum buffer (cleared by cfa_load_async, or by cfa_reset_checksums).  This is the
+ * bare "InGPU -> Loaded" transition of section 4.2 for callers that manage their own staging.
+ */
+cfa_status cfa_unpack_chunks_async(cfa_plan *plan, uint32_t chunk_begin, uint32_t chunk_end,
+                                   const void *chunk_src, cfa_stream stream);
+
+/* Zeroes the plan's checksum buffer on `stream`. */
+cfa_status cfa_reset_checksums(cfa_plan *plan, cfa_stream stream);
+
+/*
+ * Waits for all work of the plan to finish, then frees everything the plan owns (descriptor
+ * table, staging slots, pinned slots, streams, events, checksum buffer, threads).  The
+ * destinations stay allocated.  Accepts NULL.
+ */
+cfa_status cfa_plan_destroy(cfa_plan *plan);
+
+/* Detail of the last failure (see the conventions above).  Never NULL. */
+const char *cfa_last_error(const cfa_plan *plan);
+
+/* Name of a status code, e.g. "CFA_ERR_OVERLAP". */
+const char *cfa_status_name(cfa_status st);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CFA_H */

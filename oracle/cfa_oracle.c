@@ -1,0 +1,207 @@
+/*
+ * ORACLE -- plain, slow CPU restatement of what tensor materialization computes.
+ *
+ * Test infrastructure only: the test suite, the smoke check and the benchmark's CPU-baseline
+ * leg use it; the loader library never does, and this file shares no code, header or table with
+ * it.
+ *
+ * What it computes (InstantInfer, section 4.2, refined CFA model, and Theorem 2): the chunked,
+ * pipelined loader must leave every tensor in exactly the state the naive loader leaves it in:
+ * the naive loader takes the tensors one by one and writes each tensor's elements into its
+ * destination.  This file is that naive loader, element by element, in the order the definition
+ * states:
+ *
+ *   for each entry t:
+ *     D      = destination t.dst
+ *     es_s   = element size of t's source dtype
+ *     es_d   = 2 if t casts fp32 -> bf16, else es_s (and D's dtype must equal the source dtype)
+ *     n      = product of t.shape
+ *     row    = D's last dimension R when D has >= 2 dimensions (t.shape[-1] must equal R),
+ *              one element when D has <= 1 dimension
+ *     base   = t.row_offset * (elements per row) * es_d     (bytes into D)
+ *     for i in 0 .. n-1:
+ *         x = little-endian es_s-byte integer at blob[t.blob_offset + i * es_s]
+ *         y = cast ? rne_bf16(x) : x
+ *         write y as es_d little-endian bytes at D[base + i * es_d]
+ *         cover[D][each written byte] += 1
+ *         if t checksums: ck[t] = (ck[t] + y) mod 2^64
+ *
+ * and, in strict mode, every byte of every destination must end with cover == 1.
+ *
+ * rne_bf16 (round to nearest, ties to even, on the bit pattern; IEEE 754-2008 roundTiesToEven
+ * applied to dropping the low 16 bits of a binary32): NaN -> 0x7FC0; otherwise add 0x7FFF plus
+ * the lowest kept bit, then drop the low 16 bits.  Inf stays Inf, values past the largest finite
+ * bf16 round to Inf, subnormals round like any other value, signed zeros keep their sign.
+ */
+#include <stdint.h>
+#include <stddef.h>
+
+/* The oracle's own dtype codes (its Python wrapper maps dtype names onto these). */
+enum { ORC_U8 = 1, ORC_BF16 = 2, ORC_F16 = 3, ORC_F32 = 4, ORC_I32 = 5, ORC_I64 = 6, ORC_F64 = 7 };
+
+/* Entry flags as the wrapper passes them. */
+enum { ORC_CAST = 1, ORC_CKSUM = 2 };
+
+/* Result codes. */
+enum {
+    ORC_OK = 0,
+    ORC_E_INVAL = 1,    /* unknown dtype, bad dimension count, negative size or offset */
+    ORC_E_DTYPE = 2,    /* source / destination dtypes do not fit the entry's cast flag */
+    ORC_E_ALIGN = 3,    /* blob offset not a multiple of the source element size */
+    ORC_E_OOB = 4,      /* reads outside the blob or writes outside the destination */
+    ORC_E_SHAPE = 5,    /* last dimension differs from the destination row */
+    ORC_E_OVERLAP = 6,  /* some destination byte written more than once */
+    ORC_E_COVERAGE = 7, /* some destination byte never written */
+};
+
+static int orc_elem_size(int32_t dt)
+{
+    switch (dt) {
+    case ORC_U8: return 1;
+    case ORC_BF16: return 2;
+    case ORC_F16: return 2;
+    case ORC_F32: return 4;
+    case ORC_I32: return 4;
+    case ORC_I64: return 8;
+    case ORC_F64: return 8;
+    default: return 0;
+    }
+}
+
+uint16_t oracle_rne_bf16(uint32_t u)
+{
+    const uint32_t exponent = u & 0x7F800000u;
+    const uint32_t mantissa = u & 0x007FFFFFu;
+    if (exponent == 0x7F800000u && mantissa != 0u) return 0x7FC0u; /* any NaN */
+    const uint32_t lowest_kept_bit = (u >> 16) & 1u;
+    return (uint16_t)((u + 0x7FFFu + lowest_kept_bit) >> 16);
+}
+
+void oracle_rne_bf16_array(const uint32_t *in, uint16_t *out, uint64_t n)
+{
+    for (uint64_t i = 0; i < n; ++i) out[i] = oracle_rne_bf16(in[i]);
+}
+
+static uint64_t read_le(const uint8_t *p, int nbytes)
+{
+    uint64_t x = 0;
+    for (int k = 0; k < nbytes; ++k) x |= (uint64_t)p[k] << (8 * k);
+    return x;
+}
+
+static void write_le(uint8_t *p, uint64_t y, int nbytes)
+{
+    for (int k = 0; k < nbytes; ++k) p[k] = (uint8_t)(y >> (8 * k));
+}
+
+/*
+ * Unpacks every entry whose destination buffer is given.
+ *
+ *   e_*            entry columns (n_entries); e_shape is n_entries x 8, row-major.
+ *   d_*            destination columns (n_dsts); d_shape is n_dsts x 8.
+ *   d_buf[j]       host buffer of destination j (its full byte size), or NULL: entries into a
+ *                  NULL destination are still validated but not executed.
+ *   d_cover[j]     optional per-byte write counters of destination j (NULL to skip).
+ *   blob           holds blob bytes [blob_begin, blob_end).
+ *   blob_bytes     length of the whole blob (for the bounds rule).
+ *   cksum          n_entries accumulators, added to (the caller zeroes them).
+ *   bad_entry      receives the first failing entry, or -1.
+ * Returns ORC_OK or the first failure's code.  An entry whose bytes lie outside
+ * [blob_begin, blob_end) but inside the blob is skipped like a NULL destination.
+ */
+int oracle_unpack(uint64_t n_entries, const int32_t *e_dtype, const int32_t *e_ndim,
+                  const int64_t *e_shape, const uint64_t *e_offset, const int32_t *e_dst,
+                  const int64_t *e_row, const uint32_t *e_flags,
+                  uint64_t n_dsts, const int32_t *d_dtype, const int32_t *d_ndim,
+                  const int64_t *d_shape, uint8_t *const *d_buf, uint32_t *const *d_cover,
+                  const uint8_t *blob, uint64_t blob_begin, uint64_t blob_end,
+                  uint64_t blob_bytes, uint64_t *cksum, int64_t *bad_entry)
+{
+    *bad_entry = -1;
+    for (uint64_t t = 0; t < n_entries; ++t) {
+        const int es_s = orc_elem_size(e_dtype[t]);
+        if (es_s == 0 || e_ndim[t] < 0 || e_ndim[t] > 8) { *bad_entry = (int64_t)t; return ORC_E_INVAL; }
+        if (e_dst[t] < 0 || (uint64_t)e_dst[t] >= n_dsts) { *bad_entry = (int64_t)t; return ORC_E_INVAL; }
+        const uint64_t j = (uint64_t)e_dst[t];
+        const int es_dt = orc_elem_size(d_dtype[j]);
+        if (es_dt == 0 || d_ndim[j] < 0 || d_ndim[j] > 8) { *bad_entry = (int64_t)t; return ORC_E_INVAL; }
+        const int cast = (e_flags[t] & ORC_CAST) != 0;
+
+        /* dtypes */
+        if (cast) {
+            if (e_dtype[t] != ORC_F32 || d_dtype[j] != ORC_BF16) { *bad_entry = (int64_t)t; return ORC_E_DTYPE; }
+        } else if (e_dtype[t] != d_dtype[j]) {
+            *bad_entry = (int64_t)t;
+            return ORC_E_DTYPE;
+        }
+        const int es_d = cast ? 2 : es_s;
+
+        /* element counts */
+        uint64_t n = 1;
+        for (int k = 0; k < e_ndim[t]; ++k) {
+            if (e_shape[8 * t + k] < 0) { *bad_entry = (int64_t)t; return ORC_E_INVAL; }
+            n *= (uint64_t)e_shape[8 * t + k];
+        }
+        uint64_t d_numel = 1;
+        for (int k = 0; k < d_ndim[j]; ++k) {
+            if (d_shape[8 * j + k] < 0) { *bad_entry = (int64_t)t; return ORC_E_INVAL; }
+            d_numel *= (uint64_t)d_shape[8 * j + k];
+        }
+
+        /* placement inside the destination */
+        if (e_row[t] < 0) { *bad_entry = (int64_t)t; return ORC_E_OOB; }
+        uint64_t row_elems;
+        if (d_ndim[j] >= 2) {
+            row_elems = (uint64_t)d_shape[8 * j + d_ndim[j] - 1];
+            if (n > 0) {
+                if (e_ndim[t] < 1 || (uint64_t)e_shape[8 * t + e_ndim[t] - 1] != row_elems) {
+                    *bad_entry = (int64_t)t;
+                    return ORC_E_SHAPE;
+                }
+            }
+        } else {
+            row_elems = 1;
+        }
+        const uint64_t base_elem = (uint64_t)e_row[t] * row_elems;
+        if (base_elem + n > d_numel) { *bad_entry = (int64_t)t; return ORC_E_OOB; }
+        const uint64_t base = base_elem * (uint64_t)es_d;
+
+        /* source range */
+        if (e_offset[t] % (uint64_t)es_s != 0) { *bad_entry = (int64_t)t; return ORC_E_ALIGN; }
+        if (e_offset[t] + n * (uint64_t)es_s > blob_bytes) { *bad_entry = (int64_t)t; return ORC_E_OOB; }
+
+        if (d_buf[j] == NULL || n == 0) continue;
+        if (e_offset[t] < blob_begin || e_offset[t] + n * (uint64_t)es_s > blob_end) continue;
+
+        const uint8_t *src = blob + (e_offset[t] - blob_begin);
+        uint8_t *dst = d_buf[j] + base;
+        uint32_t *cover = d_cover ? d_cover[j] : NULL;
+        uint64_t ck = 0;
+        for (uint64_t i = 0; i < n; ++i) {
+            const uint64_t x = read_le(src + i * (uint64_t)es_s, es_s);
+            const uint64_t y = cast ? (uint64_t)oracle_rne_bf16((uint32_t)x) : x;
+            write_le(dst + i * (uint64_t)es_d, y, es_d);
+            if (cover)
+                for (int k = 0; k < es_d; ++k) cover[base + i * (uint64_t)es_d + (uint64_t)k] += 1u;
+            ck += y;
+        }
+        if (e_flags[t] & ORC_CKSUM) cksum[t] += ck;
+    }
+    return ORC_OK;
+}
+
+/* Strict-mode rule: every byte of every checked destination covered exactly once.  Returns
+ * ORC_OK, ORC_E_OVERLAP or ORC_E_COVERAGE and the failing destination in *bad_dst. */
+int oracle_check_cover(uint64_t n_dsts, const uint64_t *d_nbytes, uint32_t *const *d_cover,
+                       int64_t *bad_dst)
+{
+    *bad_dst = -1;
+    for (uint64_t j = 0; j < n_dsts; ++j) {
+        if (d_cover[j] == NULL) continue;
+        for (uint64_t b = 0; b < d_nbytes[j]; ++b) {
+            if (d_cover[j][b] > 1u) { *bad_dst = (int64_t)j; return ORC_E_OVERLAP; }
+            if (d_cover[j][b] == 0u) { *bad_dst = (int64_t)j; return ORC_E_COVERAGE; }
+        }
+    }
+    return ORC_OK;
+}

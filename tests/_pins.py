@@ -1,0 +1,323 @@
+"""Pins of the oracle: checks against what the paper and the mathematics fix, not against the
+oracle's own formulas.  Each function raises AssertionError on a mismatch.  They take `lib` so
+that test_oracle_mutants.py can run them against deliberately broken builds of the oracle.
+
+What pins what:
+  rne_golden          hand-derived IEEE roundTiesToEven cases (tests/golden/rne_cases.txt)
+  rne_vs_torch        a library routine: torch's CPU float32 -> bfloat16 conversion
+  rne_vs_nearest      the definition of round-to-nearest-even, evaluated in fp64
+  golden_manifests    hand-written manifests with their loaded bytes typed out by hand
+  one_to_one          closed form: a 1:1 cast-free load copies blob slices (numpy sum checksums)
+  concat_reference    fused layouts equal numpy/torch concatenation and stacking of the parts
+  cast_reference      cast entries equal torch's conversion of the source values
+  invariants          exact-once coverage, byte conservation, repack(unpack(blob)) == blob,
+                      entry-order invariance (Theorem 2), padding independence
+  validation          malformed manifests are rejected with the right class of error
+"""
+import numpy as np
+import torch
+
+import oracle
+from workloads import DTYPE_SIZE, Manifest, dense_config, moe_config, tiny_config
+
+from _golden import manifest_case, rne_cases
+
+
+# ---------------------------------------------------------------------------------------------
+# the cast
+# ---------------------------------------------------------------------------------------------
+def _torch_bf16_bits(u32):
+    f = torch.from_numpy(np.ascontiguousarray(u32, dtype=np.uint32).view(np.float32))
+    return f.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+def _is_nan32(u32):
+    u32 = np.asarray(u32, dtype=np.uint32)
+    return ((u32 & 0x7F800000) == 0x7F800000) & ((u32 & 0x007FFFFF) != 0)
+
+
+def check_rne_block(u32, lib=None):
+    """Oracle cast of u32 vs torch: equal on non-NaN inputs; NaN -> 0x7FC0 (torch: any NaN)."""
+    got = oracle.rne_bf16(u32, lib=lib)
+    ref = _torch_bf16_bits(u32)
+    nan = _is_nan32(u32)
+    bad = (~nan) & (got != ref)
+    assert not bad.any(), f"rne differs from torch at {hex(int(u32[bad][0]))}: " \
+                          f"{hex(int(got[bad][0]))} vs {hex(int(ref[bad][0]))}"
+    if nan.any():
+        assert (got[nan] == 0x7FC0).all(), "NaN must map to 0x7FC0"
+        r = ref[nan]
+        assert (((r & 0x7F80) == 0x7F80) & ((r & 0x007F) != 0)).all()
+
+
+def rne_golden(lib=None):
+    for u, want in rne_cases():
+        got = oracle.rne_bf16_scalar(u, lib=lib)
+        assert got == want, f"rne({u:#010x}) = {got:#06x}, want {want:#06x}"
+
+
+def rne_vs_torch(lib=None):
+    """Every upper half x the lower halves that decide rounding (0, 1, 0x7FFF, 0x8000, 0x8001,
+    0xFFFF) plus random patterns."""
+    hi = np.arange(1 << 16, dtype=np.uint32) << 16
+    lows = np.array([0, 1, 0x7FFF, 0x8000, 0x8001, 0xFFFF], dtype=np.uint32)
+    u = (hi[:, None] | lows[None, :]).ravel()
+    check_rne_block(u, lib)
+    rng = np.random.default_rng(11)
+    check_rne_block(rng.integers(0, 1 << 32, size=1 << 20, dtype=np.uint64).astype(np.uint32),
+                    lib)
+
+
+def _bf16_value(b16):
+    return np.asarray(b16, dtype=np.uint32).__lshift__(16).view(np.float32).astype(np.float64)
+
+
+def rne_vs_nearest(lib=None):
+    """For finite x the result must be the nearer of the two bf16 neighbours that bracket x
+    (truncation toward zero and one unit further out, the latter possibly infinity as the
+    overflow threshold), the even one on a tie."""
+    rng = np.random.default_rng(12)
+    u = rng.integers(0, 1 << 32, size=1 << 20, dtype=np.uint64).astype(np.uint32)
+    u = np.concatenate([u, (u & 0xFFFF0000) | 0x8000, np.arange(1 << 16, dtype=np.uint32)])
+    u = u[~_is_nan32(u) & ((u & 0x7F800000) != 0x7F800000)]  # finite only
+    x = u.view(np.float32).astype(np.float64)
+    lo = (u >> 16).astype(np.uint32)                       # toward zero
+    hi = lo + 1                                            # one bf16 unit further from zero
+    vlo = _bf16_value(lo)
+    # value of `hi` as if the exponent were unbounded (2^128 for the step past the max)
+    ulp = np.abs(_bf16_value(lo | 1) - _bf16_value(lo & ~np.uint32(1)))
+    ulp = np.where(ulp == 0, np.ldexp(1.0, -133), ulp)     # subnormal/zero spacing is 2^-133
+    vhi = vlo + np.sign(x + (x == 0)) * ulp
+    dlo, dhi = np.abs(x - vlo), np.abs(vhi - x)
+    want = np.where(dlo < dhi, lo, np.where(dhi < dlo, hi, np.where(lo & 1, hi, lo)))
+    got = oracle.rne_bf16(u, lib=lib).astype(np.uint32)
+    bad = got != want.astype(np.uint32)
+    assert not bad.any(), f"rne({int(u[bad][0]):#010x}) = {int(got[bad][0]):#06x}, " \
+                          f"nearest-even gives {int(want[bad][0]):#06x}"
+
+
+# ---------------------------------------------------------------------------------------------
+# unpacking
+# ---------------------------------------------------------------------------------------------
+def golden_manifests(lib=None):
+    for name in ("fused_tiny.txt", "moe_tiny.txt"):
+        m, blob, exp_dst, exp_ck = manifest_case(name)
+        r = oracle.unpack(m, blob, lib=lib, fill=0xEE)
+        assert r.status == 0, (name, r.status_name, r.bad_entry)
+        for j, want in exp_dst.items():
+            assert np.array_equal(r.dst[j], want), (name, j, r.dst[j], want)
+        assert np.array_equal(r.cksum, exp_ck), (name, r.cksum, exp_ck)
+
+
+def _blob(m):
+    return m.blob_range(0, m.blob_bytes)
+
+
+def _elem_view(buf, dtype):
+    es = DTYPE_SIZE[dtype]
+    return buf.view({1: np.uint8, 2: np.uint16, 4: np.uint32, 8: np.uint64}[es])
+
+
+def one_to_one(lib=None):
+    m = tiny_config(seed=21, n=60, lo=2, hi=6000, align=2, jitter=5)
+    blob = _blob(m)
+    r = oracle.unpack(m, blob, lib=lib)
+    assert r.status == 0
+    for i in range(m.n_entries):
+        off, nb = int(m.e_offset[i]), m.e_nbytes(i)
+        sl = blob[off:off + nb]
+        assert np.array_equal(r.dst[int(m.e_dst[i])], sl), i
+        assert int(r.cksum[i]) == int(sl.view(np.uint16).astype(np.uint64).sum()), i
+
+
+def _expected_by_concat(m, blob):
+    """Destination bytes built by concatenating each destination's parts in row order, with
+    torch doing the casts: no offsets are computed."""
+    out = {}
+    for j in range(m.n_dsts):
+        parts = []
+        for i in sorted(m.entries_of_dst(j), key=lambda i: int(m.e_row[i])):
+            off, nb = int(m.e_offset[i]), m.e_nbytes(i)
+            sl = blob[off:off + nb]
+            if m.e_cast[i]:
+                sl = _torch_bf16_bits(sl.view(np.uint32)).view(np.uint8)
+            parts.append(sl)
+        out[j] = np.concatenate(parts) if parts else np.zeros(0, np.uint8)
+        assert out[j].size == m.d_nbytes(j)
+    return out
+
+
+def _mini_dense(src="bf16", seed=31, **kw):
+    kw.setdefault("align", 2 if src == "bf16" else 4)
+    kw.setdefault("jitter", 3)
+    return dense_config("mini_dense", seed, layers=2, hidden=64, n_q=4, n_kv=2, head_dim=16,
+                        inter=96, vocab=100, src_dtype=src, **kw)
+
+
+def _mini_moe(seed=41, **kw):
+    kw.setdefault("align", 2)
+    kw.setdefault("jitter", 3)
+    return moe_config("mini_moe", seed, layers=2, hidden=32, n_q=4, n_kv=2, head_dim=8,
+                      inter=48, n_experts=3, vocab=50, n_extra=25, **kw)
+
+
+def _check_against_concat(m, lib):
+    blob = _blob(m)
+    r = oracle.unpack(m, blob, lib=lib, fill=0x5A)
+    assert r.status == 0, (r.status_name, r.bad_entry)
+    exp = _expected_by_concat(m, blob)
+    for j in range(m.n_dsts):
+        assert np.array_equal(r.dst[j], exp[j]), (m.name, m.d_name[j])
+    # checksums: sum of each entry's destination elements, cut out of the expected bytes in the
+    # same row order
+    for j in range(m.n_dsts):
+        pos = 0
+        for i in sorted(m.entries_of_dst(j), key=lambda i: int(m.e_row[i])):
+            nb = m.e_numel(i) * DTYPE_SIZE[str(m.d_dtype[j])]
+            want = int(_elem_view(exp[j][pos:pos + nb], str(m.d_dtype[j])).astype(np.uint64)
+                       .sum(dtype=np.uint64))
+            assert int(r.cksum[i]) == want, (m.name, m.e_name[i])
+            pos += nb
+
+
+def concat_reference(lib=None):
+    m = _mini_dense()
+    # the fused layout itself: q, k, v rows and gate, up rows in that order
+    for j in range(m.n_dsts):
+        names = [m.e_name[i].rsplit(".", 2)[-2]
+                 for i in sorted(m.entries_of_dst(j), key=lambda i: int(m.e_row[i]))]
+        if m.d_name[j].endswith("qkv_proj.weight"):
+            assert names == ["q_proj", "k_proj", "v_proj"]
+        if m.d_name[j].endswith("gate_up_proj.weight"):
+            assert names == ["gate_proj", "up_proj"]
+    _check_against_concat(m, lib)
+    mm = _mini_moe()
+    _check_against_concat(mm, lib)
+    # stacking: w13[e] == cat(w1_e, w3_e), w2[e] == w2_e, through numpy reshapes
+    blob = _blob(mm)
+    r = oracle.unpack(mm, blob, lib=lib)
+    for j in range(mm.n_dsts):
+        if not mm.d_name[j].endswith("w13_weight"):
+            continue
+        E, I2, H = mm.d_shape_tuple(j)
+        w13 = r.dst[j].view(np.uint16).reshape(E, I2, H)
+        pre = mm.d_name[j].rsplit("experts.", 1)[0] + "experts."
+        idx = {mm.e_name[i]: i for i in mm.entries_of_dst(j)}
+        for e in range(E):
+            parts = []
+            for w in ("w1", "w3"):
+                i = idx[f"{pre}{e}.{w}.weight"]
+                off = int(mm.e_offset[i])
+                parts.append(blob[off:off + mm.e_nbytes(i)].view(np.uint16).reshape(I2 // 2, H))
+            assert np.array_equal(w13[e], np.concatenate(parts, axis=0)), (j, e)
+
+
+def cast_reference(lib=None):
+    m = _mini_dense("f32", seed=32)
+    assert m.e_cast.all()
+    _check_against_concat(m, lib)
+
+
+def invariants(lib=None):
+    m = _mini_moe(seed=43)
+    blob = _blob(m)
+    r = oracle.unpack(m, blob, lib=lib, cover=True)
+    assert r.status == 0
+    # exactly-once coverage
+    st, bad = oracle.check_cover(r, lib=lib)
+    assert st == 0, (oracle.STATUS_NAME[st], bad)
+    assert all((c == 1).all() for c in r.cover.values())
+    # bytes conserved (cast-free: source bytes == destination bytes)
+    assert m.total_src_bytes() == sum(v.size for v in r.dst.values())
+    # repack(unpack(blob)) == blob on the bytes entries cover; positions come from summing
+    # part sizes in row order, not from the row-offset formula
+    back = np.zeros_like(blob)
+    covered = np.zeros(blob.size, dtype=bool)
+    for j in range(m.n_dsts):
+        pos = 0
+        for i in sorted(m.entries_of_dst(j), key=lambda i: int(m.e_row[i])):
+            off, nb = int(m.e_offset[i]), m.e_nbytes(i)
+            back[off:off + nb] = r.dst[j][pos:pos + nb]
+            covered[off:off + nb] = True
+            pos += nb
+    assert np.array_equal(back[covered], blob[covered])
+    # entry-order invariance (Theorem 2: any order reaching the same per-tensor states)
+    perm = np.random.default_rng(5).permutation(m.n_entries)
+    mp = _permuted(m, perm)
+    rp = oracle.unpack(mp, blob, lib=lib)
+    assert rp.status == 0
+    for j in range(m.n_dsts):
+        assert np.array_equal(rp.dst[j], r.dst[j])
+    assert np.array_equal(rp.cksum, r.cksum[perm])
+    # padding independence: bytes no entry covers do not matter
+    noisy = blob.copy()
+    noisy[~covered] ^= 0xA5
+    rn = oracle.unpack(m, noisy, lib=lib)
+    for j in range(m.n_dsts):
+        assert np.array_equal(rn.dst[j], r.dst[j])
+    # a window of the blob that holds every byte of the selected destinations is enough
+    j = max(range(m.n_dsts), key=m.d_nbytes)
+    es = m.entries_of_dst(j)
+    lo = min(int(m.e_offset[i]) for i in es)
+    hi = max(int(m.e_offset[i]) + m.e_nbytes(i) for i in es)
+    rw = oracle.unpack(m, blob[lo:hi], blob_begin=lo, dsts=[j], lib=lib)
+    assert rw.status == 0 and np.array_equal(rw.dst[j], r.dst[j])
+    assert all(int(rw.cksum[i]) == int(r.cksum[i]) for i in es)
+
+
+def _permuted(m, perm):
+    ents = []
+    for i in perm:
+        i = int(i)
+        ents.append({"name": m.e_name[i], "dtype": str(m.e_dtype[i]),
+                     "shape": m.e_shape_tuple(i), "offset": int(m.e_offset[i]),
+                     "dst": int(m.e_dst[i]), "row": int(m.e_row[i]),
+                     "cast": bool(m.e_cast[i]), "cksum": bool(m.e_cksum[i]),
+                     "layer": int(m.e_layer[i])})
+    dsts = [{"name": m.d_name[j], "dtype": str(m.d_dtype[j]), "shape": m.d_shape_tuple(j)}
+            for j in range(m.n_dsts)]
+    return Manifest(m.name, ents, dsts, m.blob_bytes, m.blob_kind, m.seed, m.period,
+                    m.chunk_bytes)
+
+
+def _variant(m, i, **change):
+    ents = []
+    for k in range(m.n_entries):
+        e = {"name": m.e_name[k], "dtype": str(m.e_dtype[k]), "shape": m.e_shape_tuple(k),
+             "offset": int(m.e_offset[k]), "dst": int(m.e_dst[k]), "row": int(m.e_row[k]),
+             "cast": bool(m.e_cast[k]), "cksum": bool(m.e_cksum[k]),
+             "layer": int(m.e_layer[k])}
+        if k == i:
+            e.update(change)
+        ents.append(e)
+    dsts = [{"name": m.d_name[j], "dtype": str(m.d_dtype[j]), "shape": m.d_shape_tuple(j)}
+            for j in range(m.n_dsts)]
+    return Manifest(m.name, ents, dsts, m.blob_bytes, m.blob_kind, m.seed)
+
+
+def validation(lib=None):
+    m, blob, _, _ = manifest_case("fused_tiny.txt")
+    # q is entry 0 (bf16 [2, 2] at offset 4 into qkv rows 0..1); norm is entry 3 (cast)
+    cases = [
+        (_variant(m, 0, offset=32), oracle.ORC_E_OOB),         # reads past the 34-byte blob
+        (_variant(m, 0, offset=5), oracle.ORC_E_ALIGN),        # not a multiple of 2
+        (_variant(m, 0, row=3), oracle.ORC_E_OOB),             # rows 3..4 of a 4-row dst
+        (_variant(m, 0, dtype="f16"), oracle.ORC_E_DTYPE),     # bf16 destination
+        (_variant(m, 3, cast=False), oracle.ORC_E_DTYPE),      # f32 into bf16 without cast
+        (_variant(m, 0, shape=(1, 4)), oracle.ORC_E_SHAPE),    # last dim 4 != row length 2
+        (_variant(m, 5, row=2), oracle.ORC_E_OOB),             # bias[2:4] of a 3-element dst
+    ]
+    for mv, code in cases:
+        r = oracle.unpack(mv, blob, lib=lib)
+        assert r.status == code, (oracle.STATUS_NAME[r.status], oracle.STATUS_NAME[code])
+    # overlap and gap are decided by coverage
+    r = oracle.unpack(_variant(m, 1, row=1), blob, cover=True, lib=lib)   # k onto q's row 1
+    assert r.status == 0
+    assert oracle.check_cover(r, lib=lib)[0] == oracle.ORC_E_OVERLAP
+    r = oracle.unpack(_variant(m, 4, shape=(0,)), blob, cover=True, lib=lib)  # bias[0] unset
+    assert r.status == 0
+    assert oracle.check_cover(r, lib=lib)[0] == oracle.ORC_E_COVERAGE
+
+
+ALL_PINS = [rne_golden, rne_vs_torch, rne_vs_nearest, golden_manifests, one_to_one,
+            concat_reference, cast_reference, invariants, validation]

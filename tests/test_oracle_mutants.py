@@ -1,0 +1,74 @@
+"""The pins are strong enough: each plausible mistake planted in a copy of the oracle (a dropped
+term, a wrong index, a swapped operand) makes at least one pin fail.  The mistakes are planted
+in temporary copies compiled on the CPU; the oracle itself is untouched."""
+import os
+import subprocess
+import sys
+
+import pytest
+
+import oracle
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+# Runs every pin against one compiled mutant in a child process (a mutant that writes out of
+# bounds may crash, which also counts as caught) and prints the pins that failed.
+_RUNNER = r"""
+import sys
+sys.path[:0] = [sys.argv[1], sys.argv[2]]
+import _pins, oracle
+lib = oracle.load_variant(sys.argv[3])
+failed = []
+for pin in _pins.ALL_PINS:
+    try:
+        pin(lib=lib)
+    except AssertionError:
+        failed.append(pin.__name__)
+print("FAILED:" + ",".join(failed))
+"""
+
+# (name, text in cfa_oracle.c, replacement)
+MUTANTS = [
+    ("rne_drops_lsb", "u + 0x7FFFu + lowest_kept_bit", "u + 0x7FFFu"),
+    ("rne_truncates", "(u + 0x7FFFu + lowest_kept_bit) >> 16", "u >> 16"),
+    ("rne_rounds_half_up", "u + 0x7FFFu + lowest_kept_bit", "u + 0x8000u"),
+    ("rne_nan_passthrough", "return 0x7FC0u; /* any NaN */", "return (uint16_t)(u >> 16);"),
+    ("rne_nan_test_wrong", "mantissa != 0u) return", "mantissa == 0u) return"),
+    ("row_offset_dropped", "(uint64_t)e_row[t] * row_elems", "(uint64_t)e_row[t]"),
+    ("row_is_first_dim", "d_shape[8 * j + d_ndim[j] - 1]", "d_shape[8 * j]"),
+    ("base_uses_src_size", "base_elem * (uint64_t)es_d", "base_elem * (uint64_t)es_s"),
+    ("big_endian_read", "x |= (uint64_t)p[k] << (8 * k)",
+     "x |= (uint64_t)p[k] << (8 * (nbytes - 1 - k))"),
+    ("src_stride_wrong", "src + i * (uint64_t)es_s", "src + i * (uint64_t)es_d"),
+    ("dst_stride_wrong", "dst + i * (uint64_t)es_d", "dst + i * (uint64_t)es_s"),
+    ("checksum_of_source", "ck += y;", "ck += x;"),
+    ("checksum_misses_last", "ck += y;", "if (i + 1 < n) ck += y;"),
+    ("cast_ignored", "const uint64_t y = cast ? (uint64_t)oracle_rne_bf16((uint32_t)x) : x;",
+     "const uint64_t y = x;"),
+    ("oob_check_off_by_elem", "if (base_elem + n > d_numel)", "if (base_elem + n > d_numel + 1)"),
+    ("cover_not_counted", "+= 1u;", "+= 0u;"),
+]
+
+
+@pytest.fixture(scope="module")
+def mutant_dir(tmp_path_factory):
+    return tmp_path_factory.mktemp("oracle_mutants")
+
+
+@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
+def test_pins_catch_mutant(name, old, new, mutant_dir):
+    src = open(oracle.SOURCE_PATH).read()
+    assert src.count(old) == 1, f"mutation site for {name} not unique"
+    c = os.path.join(mutant_dir, f"{name}.c")
+    so = os.path.join(mutant_dir, f"{name}.so")
+    with open(c, "w") as f:
+        f.write(src.replace(old, new))
+    subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", c, "-o", so], check=True)
+    root = os.path.dirname(HERE)
+    r = subprocess.run([sys.executable, "-c", _RUNNER, HERE, root, so],
+                       capture_output=True, text=True, timeout=600)
+    if r.returncode != 0:
+        return  # the mutant crashed the pins' process: caught
+    line = [ln for ln in r.stdout.splitlines() if ln.startswith("FAILED:")][-1]
+    failed = [x for x in line[len("FAILED:"):].split(",") if x]
+    assert failed, f"no pin caught mutant {name}"
