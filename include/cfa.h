@@ -60,7 +60,8 @@ typedef int cfa_status;
 #define CFA_ERR_NOMEM    (-9)  /* a host or device allocation failed */
 #define CFA_ERR_DTYPE    (-10) /* source and destination dtypes do not match the entry's cast */
 #define CFA_ERR_ALIGN    (-11) /* an offset, pointer or size breaks an alignment rule */
-#define CFA_ERR_DEVICE   (-12) /* the unpack kernel's own descriptor check failed (debug mode) */
+#define CFA_ERR_DEVICE   (-12) /* the unpack kernel's own descriptor check failed */
+#define CFA_ERR_SHAPE    (-13) /* an entry's last dimension differs from its destination's row */
 
 /* Element types.  Only the element size matters for plain copies; 1-byte types cover int8,
  * uint8 and the fp8 formats. */
@@ -134,15 +135,15 @@ typedef struct cfa_dst {
                                          cfa_plan_get_pieces works, loads return CFA_ERR_INVAL */
 #define CFA_OPT_TIMING          0x4u  /* record per-chunk timing events (cfa_get_stats, timeline) */
 #define CFA_OPT_NO_BULK         0x8u  /* never use the TMA bulk-copy kernel */
-#define CFA_OPT_DEBUG_CHECKS    0x10u /* the kernel re-checks every descriptor against the chunk
-                                         and reports CFA_ERR_DEVICE instead of touching memory */
-#define CFA_OPT_NO_MERGE        0x20u /* DEVICE sources: one launch per chunk instead of one
+#define CFA_OPT_NO_MERGE        0x10u /* DEVICE sources: one launch per chunk instead of one
                                          launch per contiguous run of chunks */
 
 typedef struct cfa_plan_opts {
     uint64_t chunk_bytes;     /* chunk length S, a multiple of 256; default 512 MiB */
-    int32_t host_slots;       /* pinned host staging slots of S bytes (0 = none, else >= 2); default 2 */
-    int32_t dev_slots;        /* device staging slots of S bytes (0 = none, else >= 2); default 2 */
+    int32_t host_slots;       /* pinned host staging slots of S bytes, allocated by the first HOST
+                                 or CALLBACK load (0 = none); default 2 */
+    int32_t dev_slots;        /* device staging slots of S bytes, allocated by cfa_plan_create
+                                 (0 = none: DEVICE sources only); default 2 */
     int32_t fill_threads;     /* host threads copying pageable sources into pinned slots; default 8 */
     int32_t device;           /* CUDA device ordinal; -1 = the current device */
     uint32_t slab_bytes;      /* destination bytes per block-level work item, a multiple of 4096;
@@ -312,6 +313,11 @@ const char *cfa_last_error(const cfa_plan *plan);
 
 /* Name of a status code, e.g. "CFA_ERR_OVERLAP". */
 const char *cfa_status_name(cfa_status st);
+
+/* sizeof of the ABI struct with this name ("cfa_tensor_entry", "cfa_dst", "cfa_plan_opts",
+ * "cfa_source", "cfa_stats", "cfa_piece"), or 0 for an unknown name; lets a binding check its
+ * own copies of the layouts.  Host-only. */
+size_t cfa_abi_sizeof(const char *type_name);
 
 #ifdef __cplusplus
 }

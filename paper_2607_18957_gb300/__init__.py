@@ -1,0 +1,289 @@
+"""GB300 loader of model checkpoints into a serving engine's final parameter layout.
+
+Python face of the C ABI in include/cfa.h (libcfa.so, built in-tree by `build.py`).  Every
+step of a load runs in the library (host plan builder in C, staging pipeline on CUDA streams,
+unpack kernels for sm_103a); this module only marshals arguments.  PyTorch is used for device
+memory and streams only, and is imported lazily.
+
+    entries = make_entries(dtype=[...], shape=[...], offset=[...], dst=[...], row=[...])
+    plan = Plan(entries, dsts=[(tensor.data_ptr(), "bf16", tensor.shape), ...],
+                blob_bytes=n)
+    plan.load_async(Source.pinned(ptr))      # enqueue; returns at once
+    plan.wait_layer(3)                       # readiness group 3 Loaded
+    plan.wait_layer()                        # whole load
+    ck = plan.checksums()
+"""
+import ctypes
+
+import numpy as np
+
+from . import _lib
+from ._lib import ALL, DTYPE, ENTRY_DTYPE, DST_DTYPE, PIECE_DTYPE  # noqa: F401
+
+__all__ = ["Plan", "Source", "CfaError", "make_entries", "make_dsts", "ALL", "library_path"]
+
+
+class CfaError(RuntimeError):
+    def __init__(self, status, detail):
+        self.status = status
+        self.name = _lib.STATUS.get(status, str(status))
+        super().__init__(f"{self.name}: {detail}")
+
+
+def library_path():
+    return _lib.LIB_PATH
+
+
+def _check(st, plan_handle=None):
+    if st != _lib.CFA_OK:
+        lib = _lib.load()
+        detail = lib.cfa_last_error(plan_handle)
+        raise CfaError(st, detail.decode(errors="replace") if detail else "")
+
+
+def _stream_handle(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def make_entries(dtype, shape, offset, dst, row=None, cast=None, cksum=None, layer=None,
+                 names=None):
+    """Builds the cfa_tensor_entry array from columns.
+
+    dtype   sequence of dtype names ("bf16", "f32", ...), or of CFA_DTYPE_* codes
+    shape   sequence of shapes (tuples), or an [N, 8] int array plus `ndim` via a tuple
+            (shape_array, ndim_array)
+    offset  blob byte offsets;  dst  destination indices;  row  destination row offsets
+    cast, cksum  booleans (default: no cast, checksum on);  layer  readiness groups (default 0)
+    names   optional list of str (kept alive by the returned object)
+    """
+    n = len(dst)
+    e = np.zeros(n, dtype=ENTRY_DTYPE)
+    codes = [DTYPE[str(x)] if not isinstance(x, (int, np.integer)) else int(x) for x in dtype]
+    e["src_dtype"] = np.asarray(codes, dtype=np.int32) if n else 0
+    if isinstance(shape, tuple) and len(shape) == 2 and isinstance(shape[0], np.ndarray):
+        e["shape"] = shape[0]
+        e["ndim"] = shape[1]
+    else:
+        for i, s in enumerate(shape):
+            s = tuple(int(x) for x in s)
+            e["ndim"][i] = len(s)
+            e["shape"][i, :len(s)] = s
+    e["blob_offset"] = np.asarray(offset, dtype=np.uint64) if n else 0
+    e["dst_index"] = np.asarray(dst, dtype=np.int32) if n else 0
+    if row is not None:
+        e["dst_row_offset"] = np.asarray(row, dtype=np.int64)
+    fl = np.zeros(n, dtype=np.uint32)
+    if cast is not None:
+        fl |= np.asarray(cast, dtype=bool).astype(np.uint32) * _lib.ENTRY_CAST_BF16
+    if cksum is None:
+        fl |= _lib.ENTRY_CKSUM
+    else:
+        fl |= np.asarray(cksum, dtype=bool).astype(np.uint32) * _lib.ENTRY_CKSUM
+    e["flags"] = fl
+    if layer is not None:
+        e["layer"] = np.asarray(layer, dtype=np.int32)
+    keep = None
+    if names is not None:
+        blob = b"".join(s.encode() + b"\0" for s in names)
+        keep = ctypes.create_string_buffer(blob, len(blob))
+        base = ctypes.addressof(keep)
+        offs = np.zeros(n, dtype=np.uint64)
+        pos = 0
+        for i, s in enumerate(names):
+            offs[i] = base + pos
+            pos += len(s.encode()) + 1
+        e["name"] = offs
+    return _Entries(e, keep)
+
+
+class _Entries:
+    def __init__(self, arr, keep):
+        self.arr = arr
+        self.keep = keep
+
+    def __len__(self):
+        return len(self.arr)
+
+
+def make_dsts(dsts):
+    """[(device pointer, dtype name or code, shape), ...] -> cfa_dst array."""
+    d = np.zeros(len(dsts), dtype=DST_DTYPE)
+    for j, (ptr, dt, shape) in enumerate(dsts):
+        s = tuple(int(x) for x in shape)
+        d["dev_ptr"][j] = int(ptr)
+        d["dtype"][j] = DTYPE[str(dt)] if not isinstance(dt, (int, np.integer)) else int(dt)
+        d["ndim"][j] = len(s)
+        d["shape"][j, :len(s)] = s
+    return d
+
+
+class Source:
+    """Where the blob comes from (cfa_source)."""
+
+    def __init__(self, kind, base=0, period=0, fill=None, user=None):
+        self.kind, self.base, self.period, self.fill, self.user = kind, base, period, fill, user
+
+    @classmethod
+    def host(cls, ptr, period=0):
+        """Pageable host memory, copied into pinned slots by the plan's threads."""
+        return cls(_lib.SRC_HOST, ptr, period)
+
+    @classmethod
+    def pinned(cls, ptr, period=0):
+        """Page-locked host memory, copied straight to the device."""
+        return cls(_lib.SRC_PINNED, ptr, period)
+
+    @classmethod
+    def device(cls, ptr, period=0):
+        """Device memory that already holds the blob (no staging, no copies)."""
+        return cls(_lib.SRC_DEVICE, ptr, period)
+
+    @classmethod
+    def callback(cls, fill_fn_ptr, user_ptr=0):
+        """A C function int fill(void *user, uint64 off, void *dst, uint64 len), as an address
+        (for example from ctypes.cast(ctypes_function, c_void_p).value)."""
+        return cls(_lib.SRC_CALLBACK, 0, 0, fill_fn_ptr, user_ptr)
+
+    def to_c(self):
+        s = _lib.Source()
+        s.kind = self.kind
+        s.base = self.base or None
+        s.period_bytes = self.period
+        s.fill = self.fill or None
+        s.user = self.user or None
+        return s
+
+
+class Plan:
+    """A loading plan (cfa_plan): validated manifest, chunk <-> tensor mapping, descriptor table,
+    staging slots, streams and events."""
+
+    def __init__(self, entries, dsts, blob_bytes, chunk_bytes=512 << 20, host_slots=2,
+                 dev_slots=2, fill_threads=8, slab_bytes=65536, tiny_bytes=8192, strict=True,
+                 host_only=False, timing=False, no_bulk=False, no_merge=False, device=-1,
+                 workspace=0, workspace_bytes=0):
+        lib = _lib.load()
+        self._lib = lib
+        self._handle = None
+        if not isinstance(entries, _Entries):
+            entries = _Entries(np.ascontiguousarray(entries, dtype=ENTRY_DTYPE), None)
+        self._entries = entries
+        if not isinstance(dsts, np.ndarray):
+            dsts = make_dsts(dsts)
+        self._dsts = np.ascontiguousarray(dsts, dtype=DST_DTYPE)
+        o = _lib.PlanOpts()
+        lib.cfa_plan_opts_default(ctypes.byref(o))
+        o.chunk_bytes = chunk_bytes
+        o.host_slots = host_slots
+        o.dev_slots = dev_slots
+        o.fill_threads = fill_threads
+        o.device = device
+        o.slab_bytes = slab_bytes
+        o.tiny_bytes = tiny_bytes
+        o.flags = ((_lib.OPT_STRICT_COVERAGE if strict else 0) |
+                   (_lib.OPT_HOST_ONLY if host_only else 0) |
+                   (_lib.OPT_TIMING if timing else 0) |
+                   (_lib.OPT_NO_BULK if no_bulk else 0) |
+                   (_lib.OPT_NO_MERGE if no_merge else 0))
+        o.workspace = workspace or None
+        o.workspace_bytes = workspace_bytes
+        h = ctypes.c_void_p()
+        ea = entries.arr
+        st = lib.cfa_plan_create(ea.ctypes.data if len(ea) else None, len(ea),
+                                 self._dsts.ctypes.data if len(self._dsts) else None,
+                                 len(self._dsts), int(blob_bytes), ctypes.byref(o),
+                                 ctypes.byref(h))
+        _check(st, None)
+        self._handle = h
+        self.n_entries = len(ea)
+        self.chunk_bytes = chunk_bytes
+        self._sources = []
+
+    # -- loading -------------------------------------------------------------------------------
+    def load_async(self, source, stream=None):
+        """Enqueues one full load; returns at once.  Keeps `source` alive until the next load."""
+        s = source.to_c()
+        self._sources = [source, s]
+        st = self._lib.cfa_load_async(self._handle, ctypes.byref(s),
+                                      ctypes.c_void_p(_stream_handle(stream)))
+        _check(st, self._handle)
+
+    def wait_layer(self, layer=ALL, stream=None, timeout_ns=-1, host=None):
+        """Waits for readiness group `layer` (ALL = the whole load).  With a stream (or host=False
+        and the current stream) the stream waits on the GPU; otherwise the host blocks."""
+        if stream is None and host is False:
+            stream = _stream_handle(None)
+        h = None if stream is None else ctypes.c_void_p(_stream_handle(stream))
+        st = self._lib.cfa_wait_layer(self._handle, layer, h, timeout_ns)
+        _check(st, self._handle)
+
+    def try_wait_layer(self, layer=ALL, timeout_ns=0):
+        """Host wait that returns the status code instead of raising."""
+        return self._lib.cfa_wait_layer(self._handle, layer, None, timeout_ns)
+
+    def checksums(self, n=None):
+        n = self.n_entries if n is None else n
+        out = np.zeros(n, dtype=np.uint64)
+        st = self._lib.cfa_get_checksums(self._handle, out.ctypes.data if n else None, n)
+        _check(st, self._handle)
+        return out
+
+    def stats(self):
+        s = _lib.Stats()
+        _check(self._lib.cfa_get_stats(self._handle, ctypes.byref(s)), self._handle)
+        return {name: getattr(s, name) for name, _ in _lib.Stats._fields_}
+
+    def layer_times(self, n=None):
+        if n is None:
+            n = self.info()["n_layers"]
+        out = np.zeros(n, dtype=np.float32)
+        _check(self._lib.cfa_get_layer_times(self._handle, out.ctypes.data if n else None, n),
+               self._handle)
+        return out
+
+    def info(self):
+        a, b, c = ctypes.c_uint64(), ctypes.c_uint64(), ctypes.c_uint64()
+        _check(self._lib.cfa_plan_info(self._handle, ctypes.byref(a), ctypes.byref(b),
+                                       ctypes.byref(c)), self._handle)
+        return {"n_layers": a.value, "n_pieces": b.value, "n_chunks": c.value}
+
+    def pieces(self):
+        n = self.info()["n_pieces"]
+        out = np.zeros(n, dtype=PIECE_DTYPE)
+        got = ctypes.c_size_t()
+        _check(self._lib.cfa_plan_get_pieces(self._handle, out.ctypes.data if n else None, n,
+                                             ctypes.byref(got)), self._handle)
+        return out[:got.value]
+
+    def unpack_chunks_async(self, chunk_begin, chunk_end, src_ptr, stream=None):
+        st = self._lib.cfa_unpack_chunks_async(self._handle, chunk_begin, chunk_end,
+                                               ctypes.c_void_p(src_ptr),
+                                               ctypes.c_void_p(_stream_handle(stream)))
+        _check(st, self._handle)
+
+    def reset_checksums(self, stream=None):
+        _check(self._lib.cfa_reset_checksums(self._handle,
+                                             ctypes.c_void_p(_stream_handle(stream))),
+               self._handle)
+
+    def close(self):
+        if self._handle is not None:
+            self._lib.cfa_plan_destroy(self._handle)
+            self._handle = None
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

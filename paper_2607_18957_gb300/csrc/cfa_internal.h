@@ -1,0 +1,87 @@
+/*
+ * Internal structures shared by the host plan builder (cfa_plan.c), the kernels
+ * (cfa_unpack.cu) and the runtime (cfa_runtime.cu).  Not part of the C ABI.
+ */
+#ifndef CFA_INTERNAL_H
+#define CFA_INTERNAL_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#include "cfa.h"
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/*
+ * One unit of GPU work: a contiguous run of elements of one piece (tensor x chunk).
+ * 32 bytes, read once per work item.
+ *   src   blob byte offset of the first source element (the launch adds its source base)
+ *   dst   device address of the first destination element
+ *   n     element count
+ *   ck    checksum slot (the entry index), or CFA_NO_CK
+ *   mode  bits 0-1: log2 of the source element size; bits 2-3: log2 of the destination element
+ *         size; bit 4: fp32 -> bf16 round-to-nearest-even cast
+ */
+typedef struct cfa_work {
+    uint64_t src;
+    uint64_t dst;
+    uint32_t n;
+    uint32_t ck;
+    uint32_t mode;
+    uint32_t pad;
+} cfa_work;
+
+#define CFA_NO_CK 0xFFFFFFFFu
+
+/* Work classes: one specialised kernel each.  0..3 = plain copy of 1, 2, 4, 8-byte elements;
+ * 4 = fp32 -> bf16 cast. */
+#define CFA_N_CLASSES 5
+#define CFA_CLASS_CAST 4
+#define CFA_MODE_CAST 0x10u
+#define CFA_MODE(src_log2, dst_log2, cast) \
+    ((uint32_t)(src_log2) | ((uint32_t)(dst_log2) << 2) | ((cast) ? CFA_MODE_CAST : 0u))
+
+/* Host side of a plan: everything cfa_plan_create computes before touching the GPU. */
+typedef struct cfa_host_plan {
+    cfa_plan_opts opts;
+    uint64_t blob_bytes;
+    uint64_t chunk_bytes;
+    uint32_t n_chunks;
+    uint32_t n_layers;
+    size_t n_entries, n_dsts;
+    cfa_tensor_entry *entries; /* copies; names point into `names` */
+    char **names;
+    cfa_dst *dsts;
+    cfa_piece *pieces; /* sorted by (chunk, src offset) */
+    size_t n_pieces;
+    /* work items ordered by (class, chunk): class k of chunk c owns
+     * [first[k * (n_chunks + 1) + c], first[k * (n_chunks + 1) + c + 1]) of each array, so the
+     * items of one class over a run of chunks are contiguous */
+    cfa_work *slabs; /* block-level, LSU vector path */
+    size_t n_slabs;
+    uint32_t *slab_first;
+    cfa_work *bulk;  /* block-level, TMA bulk path (cast-free, 16-byte aligned) */
+    size_t n_bulk;
+    uint32_t *bulk_first;
+    cfa_work *tiny;  /* warp-level */
+    size_t n_tiny;
+    uint32_t *tiny_first;
+    int64_t *layer_last_chunk; /* n_layers; -1 = the group has no bytes */
+    uint64_t bytes_read, bytes_written;
+    int any_cksum;
+} cfa_host_plan;
+
+cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries,
+                               const cfa_dst *dsts, size_t n_dsts, uint64_t blob_bytes,
+                               const cfa_plan_opts *opts, cfa_host_plan *out, char *err,
+                               size_t errlen);
+void cfa_host_plan_free(cfa_host_plan *hp);
+int cfa_dtype_size(int32_t dtype);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CFA_INTERNAL_H */

@@ -1,0 +1,825 @@
+/*
+ * Runtime of the loader: the C ABI of cfa.h on top of the host plan (cfa_plan.c) and the unpack
+ * kernels (cfa_unpack.cu).
+ *
+ * InstantInfer section 4.2 runs each chunk through InDisk -> InMem -> InGPU -> Destroyed with
+ *   (i)   (C_i, InMem) -> (C_{i+1}, InDisk) and (C_i, InGPU) -> (C_{i+1}, InMem): one chunk at a
+ *         time per data path, the paths overlapping (a two-stage pipeline);
+ *   (ii)  (C_i, InGPU) -> (T_j, Alloc): a chunk on the GPU lets its tensors be assembled;
+ *   (iii) (T_j, Loaded) -> (C_i, InGPU): a chunk is destroyed once all its tensors are loaded.
+ * Here every state transition is a CUDA stream operation and every dependency a CUDA event, all
+ * enqueued at once by cfa_load_async, so the host never blocks inside a load:
+ *
+ *   fill stream   wait(host slot free) -> host function: copy chunk c into pinned slot c mod H
+ *                 (pageable or callback sources only) -> record(filled)
+ *   copy stream   wait(filled) -> wait(device slot free) -> cudaMemcpyAsync H2D into device slot
+ *                 c mod D -> record(host slot free) -> record(h2d done)
+ *   caller stream wait(h2d done) -> unpack kernel for chunk c -> record(device slot free)
+ *                 -> record(layer l ready) for each readiness group whose last chunk is c
+ *
+ * Each stream runs one chunk at a time (dependency (i)); the three streams overlap; the slot
+ * events carry dependencies (ii) and (iii).  A device source skips staging: its chunks already
+ * sit in device memory, and contiguous chunks are unpacked by one launch.
+ */
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <atomic>
+#include <chrono>
+#include <condition_variable>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <functional>
+#include <memory>
+#include <mutex>
+#include <new>
+#include <thread>
+#include <vector>
+
+#include "cfa_internal.h"
+
+extern "C" int cfa_unpack_blocks_per_sm(int cls);
+extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_t n_slabs,
+                                         const cfa_work *tiny, uint32_t n_tiny,
+                                         uint64_t src_base, uint64_t src_lo, uint64_t src_hi,
+                                         unsigned long long *ck, int *status, int grid_cap,
+                                         cudaStream_t stream);
+
+namespace {
+
+thread_local char g_create_err[512];
+
+/* ---- a small thread pool for host staging copies ---------------------------------------- */
+class Pool {
+  public:
+    explicit Pool(int n)
+    {
+        for (int i = 0; i < n; ++i) threads_.emplace_back([this] { loop(); });
+    }
+    ~Pool()
+    {
+        {
+            std::lock_guard<std::mutex> g(mu_);
+            stop_ = true;
+        }
+        cv_.notify_all();
+        for (auto &t : threads_) t.join();
+    }
+    /* Runs f(0 .. nparts-1) on the pool and the calling thread; returns when all are done. */
+    void run(int nparts, const std::function<void(int)> &f)
+    {
+        if (threads_.empty() || nparts <= 1) {
+            for (int k = 0; k < nparts; ++k) f(k);
+            return;
+        }
+        {
+            std::lock_guard<std::mutex> g(mu_);
+            fn_.store(&f);
+            total_.store(nparts);
+            pending_.store(nparts);
+            next_.store(0);
+            ++gen_;
+        }
+        cv_.notify_all();
+        work();
+        std::unique_lock<std::mutex> lk(mu_);
+        done_.wait(lk, [this] { return pending_.load() == 0; });
+    }
+
+  private:
+    void work()
+    {
+        for (;;) {
+            const int k = next_.fetch_add(1);
+            if (k >= total_.load()) return;
+            (*fn_.load())(k);
+            if (pending_.fetch_sub(1) == 1) {
+                std::lock_guard<std::mutex> g(mu_);
+                done_.notify_all();
+            }
+        }
+    }
+    void loop()
+    {
+        uint64_t seen = 0;
+        for (;;) {
+            {
+                std::unique_lock<std::mutex> lk(mu_);
+                cv_.wait(lk, [&] { return stop_ || gen_ != seen; });
+                if (stop_) return;
+                seen = gen_;
+            }
+            work();
+        }
+    }
+    std::vector<std::thread> threads_;
+    std::mutex mu_;
+    std::condition_variable cv_, done_;
+    std::atomic<const std::function<void(int)> *> fn_{nullptr};
+    std::atomic<int> total_{0}, pending_{0}, next_{0};
+    uint64_t gen_ = 0;
+    bool stop_ = false;
+};
+
+struct LoadCtx;
+
+struct FillJob {
+    LoadCtx *ctx;
+    uint32_t chunk;
+    int host_slot;
+};
+
+struct LoadCtx {
+    cfa_plan *plan;
+    cfa_source src;
+    std::atomic<int> error{0};
+    std::vector<FillJob> jobs;
+};
+
+struct DeviceGuard {
+    int prev = -1;
+    bool ok = false;
+    explicit DeviceGuard(int dev)
+    {
+        if (cudaGetDevice(&prev) != cudaSuccess) prev = -1;
+        ok = cudaSetDevice(dev) == cudaSuccess;
+    }
+    ~DeviceGuard()
+    {
+        if (prev >= 0) cudaSetDevice(prev);
+    }
+};
+
+} // namespace
+
+struct cfa_plan {
+    cfa_host_plan hp{};
+    bool host_only = false;
+    int device = 0;
+    int grid_cap[CFA_N_CLASSES] = {0};
+    cfa_work *d_slabs = nullptr, *d_tiny = nullptr;
+    unsigned long long *d_ck = nullptr;
+    int *d_status = nullptr;
+    uint8_t *d_slots = nullptr;
+    bool own_slots = false;
+    uint64_t slot_bytes = 0;
+    int n_dev_slots = 0;
+    uint8_t *h_slots = nullptr;
+    int n_host_slots = 0;
+    cudaStream_t fill_stream = nullptr, copy_stream = nullptr, aux_stream = nullptr;
+    std::vector<cudaEvent_t> ev_dev_free, ev_h2d, ev_host_free, ev_filled, ev_layer;
+    cudaEvent_t ev_begin = nullptr, ev_all = nullptr;
+    std::vector<cudaEvent_t> t_h2d0, t_h2d1, t_k0, t_k1;
+    std::vector<std::vector<uint32_t>> layers_ending; /* per chunk */
+    std::vector<uint32_t> layers_empty;
+    std::unique_ptr<Pool> pool;
+    std::vector<std::unique_ptr<LoadCtx>> loads;
+    LoadCtx *last = nullptr;
+    std::mutex mu;
+    char err[512] = {0};
+    uint64_t n_loads = 0;
+    uint64_t last_launches = 0;
+    uint32_t last_h2d = 0;
+    double plan_ms = 0;
+};
+
+namespace {
+
+void set_err(cfa_plan *p, const char *fmt, ...)
+{
+    char *buf = p ? p->err : g_create_err;
+    size_t n = p ? sizeof(p->err) : sizeof(g_create_err);
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, n, fmt, ap);
+    va_end(ap);
+}
+
+#define CK(p, call)                                                                        \
+    do {                                                                                   \
+        cudaError_t e_ = (call);                                                           \
+        if (e_ != cudaSuccess) {                                                           \
+            set_err((p), "%s failed: %s", #call, cudaGetErrorString(e_));                  \
+            return CFA_ERR_CUDA;                                                           \
+        }                                                                                  \
+    } while (0)
+
+void CUDART_CB fill_host_fn(void *arg)
+{
+    FillJob *j = static_cast<FillJob *>(arg);
+    LoadCtx *ctx = j->ctx;
+    cfa_plan *p = ctx->plan;
+    if (ctx->error.load()) return;
+    const uint64_t S = p->hp.chunk_bytes;
+    const uint64_t off = (uint64_t)j->chunk * S;
+    const uint64_t len = std::min<uint64_t>(S, p->hp.blob_bytes - off);
+    uint8_t *dst = p->h_slots + (uint64_t)j->host_slot * S;
+    const uint64_t part = 16ull << 20;
+    const int nparts = (int)((len + part - 1) / part);
+    const cfa_source &src = ctx->src;
+    p->pool->run(nparts, [&](int k) {
+        const uint64_t a = (uint64_t)k * part;
+        const uint64_t b = std::min<uint64_t>(len, a + part);
+        if (src.kind == CFA_SRC_HOST) {
+            const uint64_t so = src.period_bytes ? (off % src.period_bytes) : off;
+            std::memcpy(dst + a, static_cast<const uint8_t *>(src.base) + so + a, b - a);
+        } else if (src.fill(src.user, off + a, dst + a, b - a) != 0) {
+            int zero = 0;
+            ctx->error.compare_exchange_strong(zero, CFA_ERR_SOURCE);
+        }
+    });
+}
+
+/* Unpacks chunks [c0, c1), whose blob byte o sits at device address src_base + o: one launch
+ * per work class present in those chunks (normally one). */
+cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, cudaStream_t s)
+{
+    const cfa_host_plan &hp = p->hp;
+    const uint64_t lo = (uint64_t)c0 * hp.chunk_bytes;
+    const uint64_t hi = std::min<uint64_t>(hp.blob_bytes, (uint64_t)c1 * hp.chunk_bytes);
+    const size_t row = (size_t)hp.n_chunks + 1;
+    for (int k = 0; k < CFA_N_CLASSES; ++k) {
+        const uint32_t s0 = hp.slab_first[k * row + c0], s1 = hp.slab_first[k * row + c1];
+        const uint32_t t0 = hp.tiny_first[k * row + c0], t1 = hp.tiny_first[k * row + c1];
+        if (s1 == s0 && t1 == t0) continue;
+        const bool timing =
+            (hp.opts.flags & CFA_OPT_TIMING) && p->last_launches < p->t_k0.size();
+        if (timing) CK(p, cudaEventRecord(p->t_k0[p->last_launches], s));
+        CK(p, cfa_launch_unpack(k, p->d_slabs + s0, s1 - s0, p->d_tiny + t0, t1 - t0, src_base,
+                                lo, hi, p->d_ck, p->d_status, p->grid_cap[k], s));
+        if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], s));
+        p->last_launches++;
+    }
+    return CFA_OK;
+}
+
+cfa_status record_layers(cfa_plan *p, uint32_t c0, uint32_t c1, cudaStream_t s)
+{
+    for (uint32_t c = c0; c < c1; ++c)
+        for (uint32_t l : p->layers_ending[c]) CK(p, cudaEventRecord(p->ev_layer[l], s));
+    return CFA_OK;
+}
+
+cfa_status make_event(cfa_plan *p, cudaEvent_t *ev, bool timing)
+{
+    CK(p, cudaEventCreateWithFlags(ev, timing ? cudaEventDefault : cudaEventDisableTiming));
+    return CFA_OK;
+}
+
+void release(cfa_plan *p)
+{
+    if (!p) return;
+    if (!p->host_only) {
+        DeviceGuard g(p->device);
+        if (p->fill_stream) cudaStreamSynchronize(p->fill_stream);
+        if (p->copy_stream) cudaStreamSynchronize(p->copy_stream);
+        if (p->ev_all) cudaEventSynchronize(p->ev_all);
+        if (p->aux_stream) cudaStreamSynchronize(p->aux_stream);
+        auto kill = [](std::vector<cudaEvent_t> &v) {
+            for (cudaEvent_t e : v)
+                if (e) cudaEventDestroy(e);
+            v.clear();
+        };
+        kill(p->ev_dev_free);
+        kill(p->ev_h2d);
+        kill(p->ev_host_free);
+        kill(p->ev_filled);
+        kill(p->ev_layer);
+        kill(p->t_h2d0);
+        kill(p->t_h2d1);
+        kill(p->t_k0);
+        kill(p->t_k1);
+        if (p->ev_begin) cudaEventDestroy(p->ev_begin);
+        if (p->ev_all) cudaEventDestroy(p->ev_all);
+        if (p->fill_stream) cudaStreamDestroy(p->fill_stream);
+        if (p->copy_stream) cudaStreamDestroy(p->copy_stream);
+        if (p->aux_stream) cudaStreamDestroy(p->aux_stream);
+        if (p->d_slabs) cudaFree(p->d_slabs);
+        if (p->d_tiny) cudaFree(p->d_tiny);
+        if (p->d_ck) cudaFree(p->d_ck);
+        if (p->d_status) cudaFree(p->d_status);
+        if (p->own_slots && p->d_slots) cudaFree(p->d_slots);
+        if (p->h_slots) cudaFreeHost(p->h_slots);
+    }
+    p->pool.reset();
+    cfa_host_plan_free(&p->hp);
+    delete p;
+}
+
+cfa_status setup_device(cfa_plan *p)
+{
+    cfa_host_plan &hp = p->hp;
+    const cfa_plan_opts &o = hp.opts;
+    if (o.device >= 0) p->device = o.device;
+    else CK(nullptr, cudaGetDevice(&p->device));
+    DeviceGuard g(p->device);
+    if (!g.ok) {
+        set_err(nullptr, "cannot select CUDA device %d", p->device);
+        return CFA_ERR_CUDA;
+    }
+    int sms = 0;
+    CK(nullptr, cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device));
+    for (int k = 0; k < CFA_N_CLASSES; ++k) {
+        const int per_sm = cfa_unpack_blocks_per_sm(k);
+        if (sms <= 0 || per_sm <= 0) {
+            set_err(nullptr, "unpack kernel %d cannot run on device %d (sm=%d, blocks/sm=%d)", k,
+                    p->device, sms, per_sm);
+            return CFA_ERR_CUDA;
+        }
+        p->grid_cap[k] = sms * per_sm;
+    }
+
+    auto upload = [&](cfa_work **d, const cfa_work *h, size_t n) -> cfa_status {
+        const size_t bytes = (n ? n : 1) * sizeof(cfa_work);
+        if (cudaMalloc(d, bytes) != cudaSuccess) {
+            set_err(nullptr, "cudaMalloc of %zu descriptor bytes failed", bytes);
+            return CFA_ERR_NOMEM;
+        }
+        if (n) CK(nullptr, cudaMemcpy(*d, h, n * sizeof(cfa_work), cudaMemcpyHostToDevice));
+        return CFA_OK;
+    };
+    cfa_status st = upload(&p->d_slabs, hp.slabs, hp.n_slabs);
+    if (st) return st;
+    st = upload(&p->d_tiny, hp.tiny, hp.n_tiny);
+    if (st) return st;
+    const size_t ck_bytes = (hp.n_entries ? hp.n_entries : 1) * sizeof(unsigned long long);
+    if (cudaMalloc(&p->d_ck, ck_bytes) != cudaSuccess ||
+        cudaMalloc(&p->d_status, sizeof(int)) != cudaSuccess) {
+        set_err(nullptr, "cudaMalloc of the checksum buffer failed");
+        return CFA_ERR_NOMEM;
+    }
+    CK(nullptr, cudaMemset(p->d_ck, 0, ck_bytes));
+    CK(nullptr, cudaMemset(p->d_status, 0, sizeof(int)));
+
+    p->n_dev_slots = o.dev_slots;
+    p->n_host_slots = o.host_slots;
+    p->slot_bytes = std::min<uint64_t>(hp.chunk_bytes, (hp.blob_bytes + 255) / 256 * 256);
+    if (p->n_dev_slots > 0 && p->slot_bytes > 0) {
+        if (o.workspace) {
+            p->d_slots = static_cast<uint8_t *>(o.workspace);
+        } else {
+            if (cudaMalloc(&p->d_slots, (uint64_t)p->n_dev_slots * p->slot_bytes) !=
+                cudaSuccess) {
+                cudaGetLastError();
+                set_err(nullptr, "cudaMalloc of %d staging slots of %llu bytes failed",
+                        p->n_dev_slots, (unsigned long long)p->slot_bytes);
+                return CFA_ERR_NOMEM;
+            }
+            p->own_slots = true;
+        }
+    }
+    CK(nullptr, cudaStreamCreateWithFlags(&p->fill_stream, cudaStreamNonBlocking));
+    CK(nullptr, cudaStreamCreateWithFlags(&p->copy_stream, cudaStreamNonBlocking));
+    CK(nullptr, cudaStreamCreateWithFlags(&p->aux_stream, cudaStreamNonBlocking));
+    const bool timing = (o.flags & CFA_OPT_TIMING) != 0;
+    auto events = [&](std::vector<cudaEvent_t> &v, size_t n, bool t) -> cfa_status {
+        v.assign(n, nullptr);
+        for (auto &e : v) {
+            cfa_status s = make_event(nullptr, &e, t);
+            if (s) return s;
+        }
+        return CFA_OK;
+    };
+    if ((st = events(p->ev_dev_free, p->n_dev_slots, false))) return st;
+    if ((st = events(p->ev_h2d, p->n_dev_slots, false))) return st;
+    if ((st = events(p->ev_host_free, p->n_host_slots, false))) return st;
+    if ((st = events(p->ev_filled, p->n_host_slots, false))) return st;
+    if ((st = events(p->ev_layer, hp.n_layers, timing))) return st;
+    if ((st = make_event(nullptr, &p->ev_begin, timing))) return st;
+    if ((st = make_event(nullptr, &p->ev_all, timing))) return st;
+    if (timing) {
+        if ((st = events(p->t_h2d0, hp.n_chunks, true))) return st;
+        if ((st = events(p->t_h2d1, hp.n_chunks, true))) return st;
+        if ((st = events(p->t_k0, 2 * ((size_t)hp.n_chunks + 1), true))) return st;
+        if ((st = events(p->t_k1, 2 * ((size_t)hp.n_chunks + 1), true))) return st;
+    }
+    if (o.fill_threads > 1) p->pool.reset(new Pool(o.fill_threads - 1));
+    else p->pool.reset(new Pool(0));
+    return CFA_OK;
+}
+
+cfa_status check_status_word(cfa_plan *p)
+{
+    int h = 0;
+    CK(p, cudaStreamWaitEvent(p->aux_stream, p->ev_all, 0));
+    CK(p, cudaMemcpyAsync(&h, p->d_status, sizeof(int), cudaMemcpyDeviceToHost, p->aux_stream));
+    CK(p, cudaStreamSynchronize(p->aux_stream));
+    if (h) {
+        set_err(p, "the unpack kernel rejected a work item outside its chunk");
+        return CFA_ERR_DEVICE;
+    }
+    return CFA_OK;
+}
+
+cfa_status wait_event_host(cfa_plan *p, cudaEvent_t ev, int64_t timeout_ns)
+{
+    const auto t0 = std::chrono::steady_clock::now();
+    int64_t sleep_us = 10;
+    for (;;) {
+        const cudaError_t q = cudaEventQuery(ev);
+        if (q == cudaSuccess) return CFA_OK;
+        if (q != cudaErrorNotReady) {
+            set_err(p, "cudaEventQuery failed: %s", cudaGetErrorString(q));
+            return CFA_ERR_CUDA;
+        }
+        if (timeout_ns >= 0) {
+            const int64_t el = std::chrono::duration_cast<std::chrono::nanoseconds>(
+                                   std::chrono::steady_clock::now() - t0)
+                                   .count();
+            if (el >= timeout_ns) {
+                set_err(p, "wait timed out after %lld ns", (long long)timeout_ns);
+                return CFA_ERR_TIMEOUT;
+            }
+        }
+        std::this_thread::sleep_for(std::chrono::microseconds(sleep_us));
+        sleep_us = std::min<int64_t>(sleep_us * 2, 1000);
+    }
+}
+
+} // namespace
+
+extern "C" {
+
+cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
+                           const cfa_dst *dsts, size_t n_dsts, uint64_t blob_bytes,
+                           const cfa_plan_opts *opts, cfa_plan **out)
+{
+    if (!out) {
+        set_err(nullptr, "out is NULL");
+        return CFA_ERR_INVAL;
+    }
+    *out = nullptr;
+    const auto t0 = std::chrono::steady_clock::now();
+    cfa_plan *p = new (std::nothrow) cfa_plan();
+    if (!p) {
+        set_err(nullptr, "out of host memory");
+        return CFA_ERR_NOMEM;
+    }
+    cfa_status st = cfa_host_plan_build(entries, n_entries, dsts, n_dsts, blob_bytes, opts,
+                                        &p->hp, g_create_err, sizeof(g_create_err));
+    if (st) {
+        delete p;
+        return st;
+    }
+    const cfa_host_plan &hp = p->hp;
+    p->host_only = (hp.opts.flags & CFA_OPT_HOST_ONLY) != 0;
+    p->layers_ending.assign(hp.n_chunks, {});
+    for (uint32_t l = 0; l < hp.n_layers; ++l) {
+        if (hp.layer_last_chunk[l] < 0) p->layers_empty.push_back(l);
+        else p->layers_ending[(size_t)hp.layer_last_chunk[l]].push_back(l);
+    }
+    if (!p->host_only) {
+        st = setup_device(p);
+        if (st) {
+            char keep[sizeof(g_create_err)];
+            std::memcpy(keep, g_create_err, sizeof keep);
+            release(p);
+            std::memcpy(g_create_err, keep, sizeof keep);
+            return st;
+        }
+    }
+    p->plan_ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0)
+                     .count();
+    *out = p;
+    return CFA_OK;
+}
+
+cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_)
+{
+    if (!p || !src) return CFA_ERR_INVAL;
+    if (p->host_only) {
+        set_err(p, "host-only plan cannot load");
+        return CFA_ERR_INVAL;
+    }
+    std::unique_lock<std::mutex> lk(p->mu, std::try_to_lock);
+    if (!lk.owns_lock()) {
+        set_err(p, "plan in use by another thread");
+        return CFA_ERR_BUSY;
+    }
+    const cfa_host_plan &hp = p->hp;
+    const uint64_t S = hp.chunk_bytes;
+    const int kind = src->kind;
+    if (kind < CFA_SRC_HOST || kind > CFA_SRC_DEVICE || src->reserved) {
+        set_err(p, "unknown source kind %d", kind);
+        return CFA_ERR_INVAL;
+    }
+    if (src->period_bytes && (src->period_bytes % S != 0 || kind == CFA_SRC_CALLBACK)) {
+        set_err(p, "period_bytes must be a multiple of chunk_bytes (not for callbacks)");
+        return CFA_ERR_INVAL;
+    }
+    if (kind == CFA_SRC_CALLBACK ? !src->fill : (!src->base && hp.blob_bytes)) {
+        set_err(p, "source has no base pointer or fill function");
+        return CFA_ERR_INVAL;
+    }
+    if ((kind == CFA_SRC_PINNED || kind == CFA_SRC_DEVICE) && ((uintptr_t)src->base & 255u)) {
+        set_err(p, "pinned and device sources must be 256-byte aligned");
+        return CFA_ERR_ALIGN;
+    }
+    const bool staged = kind == CFA_SRC_HOST || kind == CFA_SRC_CALLBACK;
+    if (kind != CFA_SRC_DEVICE && hp.n_chunks && (p->n_dev_slots == 0 || !p->d_slots)) {
+        set_err(p, "plan has no device staging slots (dev_slots = 0)");
+        return CFA_ERR_INVAL;
+    }
+    if (staged && hp.n_chunks && p->n_host_slots == 0) {
+        set_err(p, "plan has no pinned host slots (host_slots = 0)");
+        return CFA_ERR_INVAL;
+    }
+    DeviceGuard g(p->device);
+    cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream_);
+
+    /* contexts of loads that have fully completed are no longer referenced by host functions */
+    if (!p->loads.empty() && cudaEventQuery(p->ev_all) == cudaSuccess &&
+        cudaStreamQuery(p->fill_stream) == cudaSuccess)
+        p->loads.clear();
+    if (staged && hp.n_chunks && !p->h_slots) {
+        if (cudaHostAlloc(&p->h_slots, (uint64_t)p->n_host_slots * S, cudaHostAllocDefault) !=
+            cudaSuccess) {
+            cudaGetLastError();
+            p->h_slots = nullptr;
+            set_err(p, "cudaHostAlloc of %d pinned slots of %llu bytes failed", p->n_host_slots,
+                    (unsigned long long)S);
+            return CFA_ERR_NOMEM;
+        }
+    }
+    std::unique_ptr<LoadCtx> ctx(new (std::nothrow) LoadCtx());
+    if (!ctx) return CFA_ERR_NOMEM;
+    ctx->plan = p;
+    ctx->src = *src;
+    if (staged) {
+        ctx->jobs.resize(hp.n_chunks);
+        for (uint32_t c = 0; c < hp.n_chunks; ++c)
+            ctx->jobs[c] = FillJob{ctx.get(), c, (int)(c % (uint32_t)p->n_host_slots)};
+    }
+    LoadCtx *cx = ctx.get();
+    p->loads.push_back(std::move(ctx));
+    p->last = cx;
+    p->n_loads++;
+    p->last_launches = 0;
+    p->last_h2d = 0;
+    const bool timing = (hp.opts.flags & CFA_OPT_TIMING) != 0;
+
+    /* the load starts after the previous load of this plan and after prior work on cs */
+    CK(p, cudaStreamWaitEvent(cs, p->ev_all, 0));
+    CK(p, cudaEventRecord(p->ev_begin, cs));
+    CK(p, cudaStreamWaitEvent(p->fill_stream, p->ev_begin, 0));
+    CK(p, cudaStreamWaitEvent(p->copy_stream, p->ev_begin, 0));
+    if (hp.any_cksum)
+        CK(p, cudaMemsetAsync(p->d_ck, 0, hp.n_entries * sizeof(unsigned long long), cs));
+    CK(p, cudaMemsetAsync(p->d_status, 0, sizeof(int), cs));
+    for (uint32_t l : p->layers_empty) CK(p, cudaEventRecord(p->ev_layer[l], cs));
+
+    if (kind == CFA_SRC_DEVICE) {
+        const uint64_t base = (uint64_t)(uintptr_t)src->base;
+        const bool merge = !(hp.opts.flags & CFA_OPT_NO_MERGE);
+        const uint32_t per_run =
+            merge ? (src->period_bytes ? (uint32_t)(src->period_bytes / S) : hp.n_chunks) : 1u;
+        for (uint32_t c0 = 0; c0 < hp.n_chunks;) {
+            const uint32_t c1 = std::min<uint32_t>(hp.n_chunks, c0 + std::max(per_run, 1u));
+            /* blob byte o of this run sits at base + (o mod period), i.e. base - c0*S + o when
+             * the run starts on a period boundary */
+            uint64_t run_base;
+            if (src->period_bytes) {
+                const uint64_t o0 = (uint64_t)c0 * S;
+                run_base = base + o0 % src->period_bytes - o0;
+            } else {
+                run_base = base;
+            }
+            cfa_status st = launch(p, c0, c1, run_base, cs);
+            if (st) return st;
+            if ((st = record_layers(p, c0, c1, cs))) return st;
+            c0 = c1;
+        }
+    } else {
+        for (uint32_t c = 0; c < hp.n_chunks; ++c) {
+            const int ds = (int)(c % (uint32_t)p->n_dev_slots);
+            const uint64_t off = (uint64_t)c * S;
+            const uint64_t len = std::min<uint64_t>(S, hp.blob_bytes - off);
+            const void *hsrc;
+            int hs = -1;
+            if (staged) {
+                hs = (int)(c % (uint32_t)p->n_host_slots);
+                CK(p, cudaStreamWaitEvent(p->fill_stream, p->ev_host_free[hs], 0));
+                CK(p, cudaLaunchHostFunc(p->fill_stream, fill_host_fn, &cx->jobs[c]));
+                CK(p, cudaEventRecord(p->ev_filled[hs], p->fill_stream));
+                CK(p, cudaStreamWaitEvent(p->copy_stream, p->ev_filled[hs], 0));
+                hsrc = p->h_slots + (uint64_t)hs * S;
+            } else {
+                const uint64_t so = src->period_bytes ? off % src->period_bytes : off;
+                hsrc = static_cast<const uint8_t *>(src->base) + so;
+            }
+            uint8_t *dslot = p->d_slots + (uint64_t)ds * p->slot_bytes;
+            CK(p, cudaStreamWaitEvent(p->copy_stream, p->ev_dev_free[ds], 0));
+            if (timing) CK(p, cudaEventRecord(p->t_h2d0[c], p->copy_stream));
+            CK(p, cudaMemcpyAsync(dslot, hsrc, len, cudaMemcpyHostToDevice, p->copy_stream));
+            if (timing) CK(p, cudaEventRecord(p->t_h2d1[c], p->copy_stream));
+            p->last_h2d++;
+            if (staged) CK(p, cudaEventRecord(p->ev_host_free[hs], p->copy_stream));
+            CK(p, cudaEventRecord(p->ev_h2d[ds], p->copy_stream));
+            CK(p, cudaStreamWaitEvent(cs, p->ev_h2d[ds], 0));
+            cfa_status st = launch(p, c, c + 1, (uint64_t)(uintptr_t)dslot - off, cs);
+            if (st) return st;
+            CK(p, cudaEventRecord(p->ev_dev_free[ds], cs));
+            if ((st = record_layers(p, c, c + 1, cs))) return st;
+        }
+    }
+    CK(p, cudaEventRecord(p->ev_all, cs));
+    return CFA_OK;
+}
+
+cfa_status cfa_wait_layer(cfa_plan *p, int32_t layer, cfa_stream consumer, int64_t timeout_ns)
+{
+    if (!p || p->host_only) return CFA_ERR_INVAL;
+    if (!p->last) {
+        set_err(p, "no load has been enqueued");
+        return CFA_ERR_INVAL;
+    }
+    cudaEvent_t ev;
+    if (layer == CFA_ALL) ev = p->ev_all;
+    else if (layer >= 0 && (uint32_t)layer < p->hp.n_layers) ev = p->ev_layer[layer];
+    else {
+        set_err(p, "unknown readiness group %d", layer);
+        return CFA_ERR_INVAL;
+    }
+    DeviceGuard g(p->device);
+    if (consumer) {
+        CK(p, cudaStreamWaitEvent(reinterpret_cast<cudaStream_t>(consumer), ev, 0));
+        const int e = p->last->error.load();
+        return e ? e : CFA_OK;
+    }
+    cfa_status st = wait_event_host(p, ev, timeout_ns);
+    if (st) return st;
+    const int e = p->last->error.load();
+    if (e) {
+        set_err(p, "the source callback failed");
+        return e;
+    }
+    if (layer == CFA_ALL) return check_status_word(p);
+    return CFA_OK;
+}
+
+cfa_status cfa_get_checksums(cfa_plan *p, uint64_t *host_out, size_t n)
+{
+    if (!p || p->host_only || (n && !host_out) || n > p->hp.n_entries) return CFA_ERR_INVAL;
+    if (!p->last) {
+        set_err(p, "no load has been enqueued");
+        return CFA_ERR_INVAL;
+    }
+    cfa_status st = cfa_wait_layer(p, CFA_ALL, nullptr, -1);
+    if (st) return st;
+    if (!n) return CFA_OK;
+    DeviceGuard g(p->device);
+    CK(p, cudaStreamWaitEvent(p->aux_stream, p->ev_all, 0));
+    CK(p, cudaMemcpyAsync(host_out, p->d_ck, n * sizeof(uint64_t), cudaMemcpyDeviceToHost,
+                          p->aux_stream));
+    CK(p, cudaStreamSynchronize(p->aux_stream));
+    return CFA_OK;
+}
+
+cfa_status cfa_get_stats(cfa_plan *p, cfa_stats *s)
+{
+    if (!p || !s) return CFA_ERR_INVAL;
+    const cfa_host_plan &hp = p->hp;
+    std::memset(s, 0, sizeof *s);
+    s->blob_bytes = hp.blob_bytes;
+    s->n_entries = hp.n_entries;
+    s->n_dsts = hp.n_dsts;
+    s->n_chunks = hp.n_chunks;
+    s->n_layers = hp.n_layers;
+    s->n_pieces = hp.n_pieces;
+    s->n_slabs = hp.n_slabs;
+    s->n_bulk = hp.n_bulk;
+    s->n_tiny = hp.n_tiny;
+    s->bytes_read = hp.bytes_read;
+    s->bytes_written = hp.bytes_written;
+    s->descriptor_bytes = (hp.n_slabs + hp.n_bulk + hp.n_tiny) * sizeof(cfa_work);
+    s->loads = p->n_loads;
+    s->kernel_launches = p->last_launches;
+    s->plan_ms = p->plan_ms;
+    if ((hp.opts.flags & CFA_OPT_TIMING) && p->last && !p->host_only) {
+        DeviceGuard g(p->device);
+        CK(p, cudaEventSynchronize(p->ev_all));
+        float ms = 0;
+        CK(p, cudaEventElapsedTime(&ms, p->ev_begin, p->ev_all));
+        s->load_ms = ms;
+        for (uint32_t c = 0; c < p->last_h2d && c < p->t_h2d0.size(); ++c) {
+            CK(p, cudaEventElapsedTime(&ms, p->t_h2d0[c], p->t_h2d1[c]));
+            s->h2d_ms += ms;
+        }
+        for (uint64_t k = 0; k < p->last_launches && k < p->t_k0.size(); ++k) {
+            CK(p, cudaEventElapsedTime(&ms, p->t_k0[k], p->t_k1[k]));
+            s->unpack_ms += ms;
+        }
+    }
+    return CFA_OK;
+}
+
+cfa_status cfa_get_layer_times(cfa_plan *p, float *ms_out, size_t n)
+{
+    if (!p || p->host_only || (n && !ms_out) || n > p->hp.n_layers) return CFA_ERR_INVAL;
+    if (!(p->hp.opts.flags & CFA_OPT_TIMING) || !p->last) {
+        set_err(p, "layer times need a CFA_OPT_TIMING plan and a load");
+        return CFA_ERR_INVAL;
+    }
+    DeviceGuard g(p->device);
+    CK(p, cudaEventSynchronize(p->ev_all));
+    for (size_t l = 0; l < n; ++l)
+        CK(p, cudaEventElapsedTime(&ms_out[l], p->ev_begin, p->ev_layer[l]));
+    return CFA_OK;
+}
+
+cfa_status cfa_plan_info(const cfa_plan *p, uint64_t *n_layers, uint64_t *n_pieces,
+                         uint64_t *n_chunks)
+{
+    if (!p) return CFA_ERR_INVAL;
+    if (n_layers) *n_layers = p->hp.n_layers;
+    if (n_pieces) *n_pieces = p->hp.n_pieces;
+    if (n_chunks) *n_chunks = p->hp.n_chunks;
+    return CFA_OK;
+}
+
+cfa_status cfa_plan_get_pieces(const cfa_plan *p, cfa_piece *out, size_t cap, size_t *n_out)
+{
+    if (!p || (cap && !out)) return CFA_ERR_INVAL;
+    const size_t n = std::min(cap, p->hp.n_pieces);
+    if (n) std::memcpy(out, p->hp.pieces, n * sizeof(cfa_piece));
+    if (n_out) *n_out = n;
+    return CFA_OK;
+}
+
+cfa_status cfa_unpack_chunks_async(cfa_plan *p, uint32_t chunk_begin, uint32_t chunk_end,
+                                   const void *chunk_src, cfa_stream stream)
+{
+    if (!p || p->host_only || chunk_begin > chunk_end || chunk_end > p->hp.n_chunks ||
+        (!chunk_src && chunk_end > chunk_begin)) {
+        if (p) set_err(p, "bad chunk range or source");
+        return CFA_ERR_INVAL;
+    }
+    if ((uintptr_t)chunk_src & 255u) {
+        set_err(p, "chunk_src must be 256-byte aligned");
+        return CFA_ERR_ALIGN;
+    }
+    std::unique_lock<std::mutex> lk(p->mu, std::try_to_lock);
+    if (!lk.owns_lock()) return CFA_ERR_BUSY;
+    DeviceGuard g(p->device);
+    const uint64_t base =
+        (uint64_t)(uintptr_t)chunk_src - (uint64_t)chunk_begin * p->hp.chunk_bytes;
+    const uint64_t saved = p->last_launches;
+    p->last_launches = p->t_k0.size(); /* no timing events for direct launches */
+    cfa_status st = launch(p, chunk_begin, chunk_end, base, reinterpret_cast<cudaStream_t>(stream));
+    p->last_launches = saved;
+    return st;
+}
+
+cfa_status cfa_reset_checksums(cfa_plan *p, cfa_stream stream)
+{
+    if (!p || p->host_only) return CFA_ERR_INVAL;
+    DeviceGuard g(p->device);
+    CK(p, cudaMemsetAsync(p->d_ck, 0, (p->hp.n_entries ? p->hp.n_entries : 1) * 8,
+                          reinterpret_cast<cudaStream_t>(stream)));
+    CK(p, cudaMemsetAsync(p->d_status, 0, sizeof(int), reinterpret_cast<cudaStream_t>(stream)));
+    return CFA_OK;
+}
+
+cfa_status cfa_plan_destroy(cfa_plan *p)
+{
+    release(p);
+    return CFA_OK;
+}
+
+const char *cfa_last_error(const cfa_plan *p) { return p ? p->err : g_create_err; }
+
+const char *cfa_status_name(cfa_status st)
+{
+    switch (st) {
+    case CFA_OK: return "CFA_OK";
+    case CFA_ERR_INVAL: return "CFA_ERR_INVAL";
+    case CFA_ERR_OVERLAP: return "CFA_ERR_OVERLAP";
+    case CFA_ERR_OOB: return "CFA_ERR_OOB";
+    case CFA_ERR_COVERAGE: return "CFA_ERR_COVERAGE";
+    case CFA_ERR_CUDA: return "CFA_ERR_CUDA";
+    case CFA_ERR_SOURCE: return "CFA_ERR_SOURCE";
+    case CFA_ERR_TIMEOUT: return "CFA_ERR_TIMEOUT";
+    case CFA_ERR_BUSY: return "CFA_ERR_BUSY";
+    case CFA_ERR_NOMEM: return "CFA_ERR_NOMEM";
+    case CFA_ERR_DTYPE: return "CFA_ERR_DTYPE";
+    case CFA_ERR_ALIGN: return "CFA_ERR_ALIGN";
+    case CFA_ERR_DEVICE: return "CFA_ERR_DEVICE";
+    case CFA_ERR_SHAPE: return "CFA_ERR_SHAPE";
+    default: return "CFA_ERR_UNKNOWN";
+    }
+}
+
+size_t cfa_abi_sizeof(const char *type_name)
+{
+    if (!type_name) return 0;
+    if (!std::strcmp(type_name, "cfa_tensor_entry")) return sizeof(cfa_tensor_entry);
+    if (!std::strcmp(type_name, "cfa_dst")) return sizeof(cfa_dst);
+    if (!std::strcmp(type_name, "cfa_plan_opts")) return sizeof(cfa_plan_opts);
+    if (!std::strcmp(type_name, "cfa_source")) return sizeof(cfa_source);
+    if (!std::strcmp(type_name, "cfa_stats")) return sizeof(cfa_stats);
+    if (!std::strcmp(type_name, "cfa_piece")) return sizeof(cfa_piece);
+    return 0;
+}
+
+} /* extern "C" */

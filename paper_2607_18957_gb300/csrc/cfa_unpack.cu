@@ -1,0 +1,410 @@
+/*
+ * Unpack kernels: the "InGPU -> Loaded" transition of InstantInfer section 4.2 (dependency (ii):
+ * once a chunk is in GPU memory, its bytes are copied and assembled into every tensor it
+ * carries).  One launch handles every work item of one chunk, or of a run of chunks that sit
+ * contiguously in device memory.
+ *
+ * The work is pure data movement plus integer arithmetic, so it is bound by HBM bandwidth:
+ * every source byte is read once from the staging buffer and every destination byte written
+ * once.  Design points:
+ *   - block-per-slab: a slab (tens of KiB of one piece) is copied by a whole CTA with 16-byte
+ *     vector loads and stores, several in flight per thread;
+ *   - warp-per-descriptor: pieces below the tiny threshold are handled by one warp each, eight
+ *     per CTA, so the ~200k small tensors of an MoE checkpoint do not each pay for a CTA;
+ *   - a persistent grid (a few CTAs per SM) walks the work list, so the launch cost does not
+ *     grow with the number of work items;
+ *   - source and destination offsets that differ modulo 16 are realigned in registers (two
+ *     aligned loads and a funnel shift per 16-byte store), so stores stay 16 bytes wide;
+ *   - the fp32 -> bf16 cast rounds to nearest even on the bit pattern with integer operations;
+ *   - checksums are sums modulo 2^64 of the destination element bit patterns, reduced inside the
+ *     CTA or warp and added with one 64-bit atomic per (CTA, run of same-tensor slabs) or per
+ *     tiny piece; integer addition is associative, so the result does not depend on the order.
+ */
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "cfa_internal.h"
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kUnroll = 4;
+constexpr int kMinBlocks = 4; /* 64 registers per thread at most */
+
+struct UnpackArgs {
+    const cfa_work *slabs;
+    const cfa_work *tiny;
+    uint32_t n_slabs;
+    uint32_t n_tiny;
+    uint64_t src_base; /* device address of blob byte 0 for this launch */
+    uint64_t src_lo;   /* blob bytes [src_lo, src_hi) are readable in this launch */
+    uint64_t src_hi;
+    unsigned long long *ck;
+    int *status;
+};
+
+/* ---- memory operations ------------------------------------------------------------------ */
+
+/* Streaming 16-byte load of staging data: read once, never by L1. */
+__device__ __forceinline__ uint4 ld_stream(const void *p)
+{
+    uint4 v;
+    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+        : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+        : "l"(p));
+    return v;
+}
+
+/* 16-byte load that may be shared with the neighbouring thread (realignment path). */
+__device__ __forceinline__ uint4 ld_shared_line(const void *p)
+{
+    uint4 v;
+    asm("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+        : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+        : "l"(p));
+    return v;
+}
+
+/* Streaming 16-byte store: written once, not read again by this kernel. */
+__device__ __forceinline__ void st_stream(void *p, uint4 v)
+{
+    asm volatile("st.global.cs.v4.u32 [%0], {%1, %2, %3, %4};" ::"l"(p), "r"(v.x), "r"(v.y),
+                 "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+template <int ES> struct Elem;
+template <> struct Elem<1> { typedef uint8_t T; };
+template <> struct Elem<2> { typedef uint16_t T; };
+template <> struct Elem<4> { typedef uint32_t T; };
+template <> struct Elem<8> { typedef unsigned long long T; };
+
+/* Sum of the ES-byte little-endian integers in a 16-byte vector. */
+template <int ES> __device__ __forceinline__ uint64_t vsum(uint4 v);
+template <> __device__ __forceinline__ uint64_t vsum<1>(uint4 v)
+{
+    return (uint64_t)(__vsadu4(v.x, 0u) + __vsadu4(v.y, 0u) + __vsadu4(v.z, 0u) +
+                      __vsadu4(v.w, 0u));
+}
+template <> __device__ __forceinline__ uint64_t vsum<2>(uint4 v)
+{
+    const uint32_t lo = (v.x & 0xFFFFu) + (v.y & 0xFFFFu) + (v.z & 0xFFFFu) + (v.w & 0xFFFFu);
+    const uint32_t hi = (v.x >> 16) + (v.y >> 16) + (v.z >> 16) + (v.w >> 16);
+    return (uint64_t)lo + hi;
+}
+template <> __device__ __forceinline__ uint64_t vsum<4>(uint4 v)
+{
+    return (uint64_t)v.x + v.y + v.z + v.w;
+}
+template <> __device__ __forceinline__ uint64_t vsum<8>(uint4 v)
+{
+    return (((uint64_t)v.y << 32) | v.x) + (((uint64_t)v.w << 32) | v.z);
+}
+
+/* Bytes k .. k+15 of the 32-byte concatenation a:b (little-endian), 0 < k < 16. */
+__device__ __forceinline__ uint4 funnel16(uint4 a, uint4 b, uint32_t k)
+{
+    const uint32_t s = (k & 3u) * 8u;
+    uint32_t w0, w1, w2, w3, w4;
+    switch (k >> 2) {
+    case 0: w0 = a.x; w1 = a.y; w2 = a.z; w3 = a.w; w4 = b.x; break;
+    case 1: w0 = a.y; w1 = a.z; w2 = a.w; w3 = b.x; w4 = b.y; break;
+    case 2: w0 = a.z; w1 = a.w; w2 = b.x; w3 = b.y; w4 = b.z; break;
+    default: w0 = a.w; w1 = b.x; w2 = b.y; w3 = b.z; w4 = b.w; break;
+    }
+    uint4 o;
+    o.x = __funnelshift_r(w0, w1, s);
+    o.y = __funnelshift_r(w1, w2, s);
+    o.z = __funnelshift_r(w2, w3, s);
+    o.w = __funnelshift_r(w3, w4, s);
+    return o;
+}
+
+/* fp32 bit pattern -> bf16 bit pattern, round to nearest, ties to even.  Adding 0x7FFF plus the
+ * lowest kept bit carries into bit 16 exactly when the dropped half is above one half ulp, or
+ * equal to it with an odd kept part.  NaNs become the quiet NaN 0x7FC0. */
+__device__ __forceinline__ uint32_t bf16_rne(uint32_t u)
+{
+    const uint32_t rounded = (u + 0x7FFFu + ((u >> 16) & 1u)) >> 16;
+    return ((u & 0x7FFFFFFFu) > 0x7F800000u) ? 0x7FC0u : rounded;
+}
+
+/* ---- copy of one contiguous run --------------------------------------------------------- */
+
+template <int ES>
+__device__ __forceinline__ uint64_t copy_elems(const uint8_t *src, uint8_t *dst, uint32_t n,
+                                               uint32_t tid, uint32_t nthr)
+{
+    typedef typename Elem<ES>::T T;
+    uint64_t acc = 0;
+    for (uint32_t e = tid; e < n; e += nthr) {
+        const T v = reinterpret_cast<const T *>(src)[e];
+        reinterpret_cast<T *>(dst)[e] = v;
+        acc += (uint64_t)v;
+    }
+    return acc;
+}
+
+/* Copies nbytes (a multiple of ES) from src to dst; thread tid of nthr.  Returns this thread's
+ * share of the checksum. */
+template <int ES, int U>
+__device__ uint64_t copy_run(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst,
+                             uint64_t nbytes, uint32_t tid, uint32_t nthr)
+{
+    uint64_t acc = 0;
+    /* head: elements until the destination is 16-byte aligned */
+    uint32_t head = (uint32_t)((16u - ((uintptr_t)dst & 15u)) & 15u);
+    if (head > nbytes) head = (uint32_t)nbytes;
+    acc += copy_elems<ES>(src, dst, head / ES, tid, nthr);
+    src += head;
+    dst += head;
+    nbytes -= head;
+
+    /* runs hold at most 2^32 elements of at most 8 bytes, so vector indices fit 32 bits */
+    const uint32_t nvec = (uint32_t)(nbytes >> 4);
+    const uint32_t k = (uint32_t)((uintptr_t)src & 15u);
+    uint4 *d = reinterpret_cast<uint4 *>(dst);
+    if (k == 0) {
+        const uint4 *s = reinterpret_cast<const uint4 *>(src);
+        const uint32_t step = nthr * U;
+        for (uint32_t base = 0; base < nvec; base += step) {
+            uint4 v[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const uint32_t i = base + u * nthr + tid;
+                if (i < nvec) v[u] = ld_stream(s + i);
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const uint32_t i = base + u * nthr + tid;
+                if (i < nvec) {
+                    st_stream(d + i, v[u]);
+                    acc += vsum<ES>(v[u]);
+                }
+            }
+        }
+    } else {
+        /* source off by k bytes: every 16-byte store takes bytes k..k+15 of two aligned
+         * vectors, both of which hold needed bytes, so nothing outside the run is read */
+        const uint4 *s = reinterpret_cast<const uint4 *>(src - k);
+        for (uint32_t i = tid; i < nvec; i += nthr) {
+            const uint4 o = funnel16(ld_shared_line(s + i), ld_shared_line(s + i + 1), k);
+            st_stream(d + i, o);
+            acc += vsum<ES>(o);
+        }
+    }
+    /* tail */
+    const uint64_t body = (uint64_t)nvec << 4;
+    acc += copy_elems<ES>(src + body, dst + body, (uint32_t)((nbytes - body) / ES), tid, nthr);
+    return acc;
+}
+
+/* n fp32 elements at src -> n bf16 elements at dst. */
+template <int U>
+__device__ uint64_t cast_run(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst,
+                             uint64_t n, uint32_t tid, uint32_t nthr)
+{
+    uint64_t acc = 0;
+    uint32_t h = (uint32_t)(((16u - ((uintptr_t)dst & 15u)) & 15u) >> 1);
+    if (h > n) h = (uint32_t)n;
+    for (uint32_t e = tid; e < h; e += nthr) {
+        const uint32_t y = bf16_rne(reinterpret_cast<const uint32_t *>(src)[e]);
+        reinterpret_cast<uint16_t *>(dst)[e] = (uint16_t)y;
+        acc += y;
+    }
+    src += 4u * h;
+    dst += 2u * h;
+    n -= h;
+
+    const uint32_t ng = (uint32_t)(n >> 3); /* groups of 8: 32 source bytes, one 16-byte store */
+    uint4 *d = reinterpret_cast<uint4 *>(dst);
+    if (((uintptr_t)src & 15u) == 0) {
+        const uint4 *s = reinterpret_cast<const uint4 *>(src);
+        const uint32_t step = nthr * U;
+        for (uint32_t base = 0; base < ng; base += step) {
+            uint4 a[U], b[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const uint32_t g = base + u * nthr + tid;
+                if (g < ng) {
+                    a[u] = ld_stream(s + 2 * g);
+                    b[u] = ld_stream(s + 2 * g + 1);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const uint32_t g = base + u * nthr + tid;
+                if (g < ng) {
+                    const uint32_t r0 = bf16_rne(a[u].x), r1 = bf16_rne(a[u].y);
+                    const uint32_t r2 = bf16_rne(a[u].z), r3 = bf16_rne(a[u].w);
+                    const uint32_t r4 = bf16_rne(b[u].x), r5 = bf16_rne(b[u].y);
+                    const uint32_t r6 = bf16_rne(b[u].z), r7 = bf16_rne(b[u].w);
+                    uint4 o;
+                    o.x = r0 | (r1 << 16);
+                    o.y = r2 | (r3 << 16);
+                    o.z = r4 | (r5 << 16);
+                    o.w = r6 | (r7 << 16);
+                    st_stream(d + g, o);
+                    acc += (uint64_t)(r0 + r1 + r2 + r3) + (r4 + r5 + r6 + r7);
+                }
+            }
+        }
+    } else {
+        const uint32_t *s = reinterpret_cast<const uint32_t *>(src);
+        for (uint32_t g = tid; g < ng; g += nthr) {
+            uint32_t r[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q) r[q] = bf16_rne(s[8 * g + q]);
+            uint4 o;
+            o.x = r[0] | (r[1] << 16);
+            o.y = r[2] | (r[3] << 16);
+            o.z = r[4] | (r[5] << 16);
+            o.w = r[6] | (r[7] << 16);
+            st_stream(d + g, o);
+            acc += (uint64_t)(r[0] + r[1] + r[2] + r[3]) + (r[4] + r[5] + r[6] + r[7]);
+        }
+    }
+    const uint64_t body = (uint64_t)ng << 3;
+    for (uint64_t e = body + tid; e < n; e += nthr) {
+        const uint32_t y = bf16_rne(reinterpret_cast<const uint32_t *>(src)[e]);
+        reinterpret_cast<uint16_t *>(dst)[e] = (uint16_t)y;
+        acc += y;
+    }
+    return acc;
+}
+
+/* Checks a work item against the launch's readable source range and its kernel's class. */
+template <int CLS>
+__device__ __forceinline__ bool item_ok(const cfa_work &w, const UnpackArgs &a)
+{
+    const uint32_t sl = w.mode & 3u;
+    const uint64_t src_bytes = (uint64_t)w.n << sl;
+    const uint32_t want_mode = CLS == CFA_CLASS_CAST ? CFA_MODE(2, 1, 1) : CFA_MODE(CLS, CLS, 0);
+    const uint32_t dl = (w.mode >> 2) & 3u;
+    return w.mode == want_mode && w.n != 0 && w.src >= a.src_lo && w.src <= a.src_hi &&
+           src_bytes <= a.src_hi - w.src && (w.src & ((1ull << sl) - 1)) == 0 &&
+           (w.dst & ((1ull << dl) - 1)) == 0;
+}
+
+template <int CLS, int U>
+__device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs &a, uint32_t tid,
+                                             uint32_t nthr)
+{
+    const uint8_t *src = reinterpret_cast<const uint8_t *>(a.src_base + w.src);
+    uint8_t *dst = reinterpret_cast<uint8_t *>(w.dst);
+    if constexpr (CLS == CFA_CLASS_CAST)
+        return cast_run<(U > 2 ? 2 : U)>(src, dst, w.n, tid, nthr);
+    else
+        return copy_run<(1 << CLS), U>(src, dst, (uint64_t)w.n << CLS, tid, nthr);
+}
+
+__device__ __forceinline__ uint64_t warp_sum(uint64_t v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, o);
+    return v;
+}
+
+/* Adds the CTA's accumulated checksum to slot ck; every thread of the CTA must call it. */
+__device__ __forceinline__ void block_flush(uint64_t &acc, uint32_t ck, unsigned long long *out,
+                                            unsigned long long *red)
+{
+    const uint64_t v = warp_sum(acc);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        unsigned long long t = 0;
+#pragma unroll
+        for (int q = 0; q < kWarps; ++q) t += red[q];
+        atomicAdd(out + ck, t);
+    }
+    __syncthreads();
+    acc = 0;
+}
+
+/* One launch: the block-level items of one class (first), then its warp-level items. */
+template <int CLS>
+__global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_unpack_kernel(const UnpackArgs a)
+{
+    __shared__ unsigned long long red[kWarps];
+    const uint32_t n_groups = (a.n_tiny + kWarps - 1) / kWarps;
+    const uint32_t n_items = a.n_slabs + n_groups;
+    const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
+    uint64_t acc = 0;
+    uint32_t acc_ck = CFA_NO_CK;
+
+    for (uint32_t item = blockIdx.x; item < n_items; item += gridDim.x) {
+        if (item < a.n_slabs) {
+            const cfa_work w = a.slabs[item]; /* the same 32 bytes for every thread */
+            if (!item_ok<CLS>(w, a)) {
+                if (threadIdx.x == 0) atomicCAS(a.status, 0, 1);
+                continue;
+            }
+            if (w.ck != acc_ck) {
+                if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
+                acc = 0;
+                acc_ck = w.ck;
+            }
+            acc += run_item<CLS, kUnroll>(w, a, threadIdx.x, kThreads);
+        } else {
+            if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
+            acc_ck = CFA_NO_CK;
+            const uint32_t t = (item - a.n_slabs) * kWarps + warp;
+            if (t < a.n_tiny) {
+                const cfa_work w = a.tiny[t];
+                if (!item_ok<CLS>(w, a)) {
+                    if (lane == 0) atomicCAS(a.status, 0, 1);
+                } else {
+                    const uint64_t v = warp_sum(run_item<CLS, 1>(w, a, lane, 32u));
+                    if (lane == 0 && w.ck != CFA_NO_CK) atomicAdd(a.ck + w.ck, v);
+                }
+            }
+        }
+    }
+    if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
+}
+
+typedef void (*kernel_fn)(const UnpackArgs);
+const kernel_fn kKernels[CFA_N_CLASSES] = {cfa_unpack_kernel<0>, cfa_unpack_kernel<1>,
+                                           cfa_unpack_kernel<2>, cfa_unpack_kernel<3>,
+                                           cfa_unpack_kernel<CFA_CLASS_CAST>};
+
+} // namespace
+
+/* Resident CTAs per SM of the class-cls kernel (0 if it cannot run). */
+extern "C" int cfa_unpack_blocks_per_sm(int cls)
+{
+    if (cls < 0 || cls >= CFA_N_CLASSES) return 0;
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kKernels[cls], kThreads, 0) !=
+        cudaSuccess)
+        return 0;
+    return n;
+}
+
+/* Launches the class-cls unpack over the given work items; grid_cap bounds the persistent grid. */
+extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_t n_slabs,
+                                         const cfa_work *tiny, uint32_t n_tiny,
+                                         uint64_t src_base, uint64_t src_lo, uint64_t src_hi,
+                                         unsigned long long *ck, int *status, int grid_cap,
+                                         cudaStream_t stream)
+{
+    if (cls < 0 || cls >= CFA_N_CLASSES || grid_cap <= 0) return cudaErrorInvalidValue;
+    const uint64_t items = (uint64_t)n_slabs + (n_tiny + kWarps - 1) / kWarps;
+    if (items == 0) return cudaSuccess;
+    UnpackArgs a;
+    a.slabs = slabs;
+    a.tiny = tiny;
+    a.n_slabs = n_slabs;
+    a.n_tiny = n_tiny;
+    a.src_base = src_base;
+    a.src_lo = src_lo;
+    a.src_hi = src_hi;
+    a.ck = ck;
+    a.status = status;
+    const uint64_t grid = items < (uint64_t)grid_cap ? items : (uint64_t)grid_cap;
+    kKernels[cls]<<<(unsigned)grid, kThreads, 0, stream>>>(a);
+    return cudaGetLastError();
+}

@@ -1,0 +1,219 @@
+"""The loader library on the host (no GPU): it loads, exports every function cfa.h declares,
+agrees with the binding's struct layouts, and its plan builder (validation, tensor x chunk
+pieces, fused placement) agrees with the oracle.  Plans here are CFA_OPT_HOST_ONLY: no CUDA
+call is made."""
+import os
+import re
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2607_18957_gb300 as cfa
+from paper_2607_18957_gb300 import _lib
+from paper_2607_18957_gb300 import build as cfa_build
+from workloads import DTYPE_SIZE, dense_config, moe_config, tiny_config
+from workloads.harness import entries_for
+
+import _pins
+from _golden import manifest_case
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built_library():
+    cfa_build.build()
+    return _lib.load()
+
+
+def header_functions():
+    text = open(os.path.join(ROOT, "include", "cfa.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(cfa_\w+)\s*\(", text)))
+
+
+def test_exports_every_declared_function(built_library):
+    names = header_functions()
+    assert len(names) >= 15
+    for n in names:
+        assert hasattr(built_library, n), n
+    assert set(names) == set(_lib.SIGNATURES), "binding and header disagree"
+
+
+def test_struct_layouts_match():
+    lib = _lib.load()  # raises on a mismatch
+    assert lib.cfa_abi_sizeof(b"cfa_tensor_entry") == 112
+    assert lib.cfa_abi_sizeof(b"nonsense") == 0
+    assert lib.cfa_status_name(-2) == b"CFA_ERR_OVERLAP"
+
+
+FAKE_BASE = 0x7F00_0000_0000
+
+
+def fake_dsts(m, misalign=0, guard=256):
+    out, pos = [], guard
+    for j in range(m.n_dsts):
+        es = DTYPE_SIZE[str(m.d_dtype[j])]
+        pos = (pos + 255) // 256 * 256 + (misalign // es) * es
+        out.append((FAKE_BASE + pos, str(m.d_dtype[j]), m.d_shape_tuple(j)))
+        pos += m.d_nbytes(j) + guard
+    return out
+
+
+def host_plan(m, chunk_bytes=512 << 20, misalign=0, **kw):
+    return cfa.Plan(entries_for(m, with_names=True), fake_dsts(m, misalign), m.blob_bytes,
+                    chunk_bytes=chunk_bytes, host_only=True, **kw)
+
+
+def execute_pieces_on_cpu(m, pieces, blob):
+    """Applies the plan's pieces with numpy/torch: no offsets are recomputed here."""
+    out = {j: np.zeros(m.d_nbytes(j), np.uint8) for j in range(m.n_dsts)}
+    for pc in pieces:
+        i = int(pc["entry"])
+        es_s = DTYPE_SIZE[str(m.e_dtype[i])]
+        n = int(pc["n_elems"])
+        src = blob[int(pc["src_offset"]):int(pc["src_offset"]) + n * es_s]
+        if pc["cast"]:
+            f = torch.from_numpy(src.view(np.float32).copy())
+            src = f.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint8)
+        o = int(pc["dst_offset"])
+        out[int(pc["dst_index"])][o:o + src.size] = src
+    return out
+
+
+def mini_configs():
+    return [
+        tiny_config(seed=51, n=40, lo=2, hi=20000, align=2, jitter=7),
+        dense_config("d", 52, 2, 64, 4, 2, 16, 96, 100, align=2, jitter=3),
+        dense_config("d32", 53, 2, 64, 4, 2, 16, 96, 100, src_dtype="f32", align=4, jitter=2),
+        moe_config("m", 54, 2, 32, 4, 2, 8, 48, 3, 50, n_extra=30, align=2, jitter=3),
+    ]
+
+
+@pytest.mark.parametrize("chunk", [256, 4096 + 256, 1 << 20, 512 << 20])
+def test_plan_pieces_reproduce_the_oracle(chunk):
+    for m in mini_configs():
+        blob = m.blob_range(0, m.blob_bytes)
+        with host_plan(m, chunk_bytes=chunk) as p:
+            pcs = p.pieces()
+            info = p.info()
+        assert info["n_chunks"] == -(-m.blob_bytes // chunk)
+        # every piece lies inside one chunk
+        es = np.array([DTYPE_SIZE[str(m.e_dtype[int(i)])] for i in pcs["entry"]])
+        start = pcs["src_offset"].astype(np.int64)
+        end = start + pcs["n_elems"].astype(np.int64) * es
+        assert (start // chunk == pcs["chunk"]).all()
+        assert ((end - 1) // chunk == pcs["chunk"]).all()
+        # chunk-major order
+        assert (np.diff(pcs["chunk"].astype(np.int64)) >= 0).all()
+        got = execute_pieces_on_cpu(m, pcs, blob)
+        ref = oracle.unpack(m, blob)
+        assert ref.status == 0
+        for j in range(m.n_dsts):
+            assert np.array_equal(got[j], ref.dst[j]), (m.name, chunk, m.d_name[j])
+
+
+def test_golden_manifests_through_the_plan():
+    for name in ("fused_tiny.txt", "moe_tiny.txt"):
+        m, blob, exp_dst, _ = manifest_case(name)
+        with host_plan(m, chunk_bytes=256) as p:
+            got = execute_pieces_on_cpu(m, p.pieces(), blob)
+        for j, want in exp_dst.items():
+            assert np.array_equal(got[j], want), (name, j)
+
+
+_ORACLE_TO_CFA = {oracle.ORC_E_INVAL: "CFA_ERR_INVAL", oracle.ORC_E_DTYPE: "CFA_ERR_DTYPE",
+                  oracle.ORC_E_ALIGN: "CFA_ERR_ALIGN", oracle.ORC_E_OOB: "CFA_ERR_OOB",
+                  oracle.ORC_E_SHAPE: "CFA_ERR_SHAPE", oracle.ORC_E_OVERLAP: "CFA_ERR_OVERLAP",
+                  oracle.ORC_E_COVERAGE: "CFA_ERR_COVERAGE"}
+
+
+def _plan_status(m, **kw):
+    try:
+        host_plan(m, chunk_bytes=256, **kw).close()
+        return "CFA_OK"
+    except cfa.CfaError as e:
+        return e.name
+
+
+def test_validation_agrees_with_the_oracle():
+    m, blob, _, _ = manifest_case("fused_tiny.txt")
+    cases = [
+        (dict(i=0, offset=32), None), (dict(i=0, offset=5), None), (dict(i=0, row=3), None),
+        (dict(i=0, dtype="f16"), None), (dict(i=3, cast=False), None),
+        (dict(i=0, shape=(1, 4)), None), (dict(i=5, row=2), None),
+        (dict(i=1, row=1), "cover"), (dict(i=4, shape=(0,)), "cover"),
+    ]
+    for change, how in cases:
+        i = change.pop("i")
+        mv = _pins._variant(m, i, **change)
+        r = oracle.unpack(mv, blob, cover=(how == "cover"))
+        code = oracle.check_cover(r)[0] if how == "cover" else r.status
+        assert code != 0
+        assert _plan_status(mv) == _ORACLE_TO_CFA[code], (change, oracle.STATUS_NAME[code])
+    # the valid manifest passes both
+    assert oracle.unpack(m, blob).status == 0 and _plan_status(m) == "CFA_OK"
+    # non-strict mode accepts the gap
+    gap = _pins._variant(m, 4, shape=(0,))
+    assert _plan_status(gap, strict=False) == "CFA_OK"
+
+
+def test_destinations_overlapping_in_memory_are_rejected():
+    m, _, _, _ = manifest_case("fused_tiny.txt")
+    d = fake_dsts(m)
+    d[1] = (d[0][0] + 8, d[1][1], d[1][2])  # norm starts inside qkv
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Plan(entries_for(m), d, m.blob_bytes, host_only=True)
+    assert e.value.name == "CFA_ERR_OVERLAP"
+
+
+def test_bad_options_and_misaligned_destination():
+    m, _, _, _ = manifest_case("fused_tiny.txt")
+    with pytest.raises(cfa.CfaError) as e:
+        host_plan(m, chunk_bytes=100)
+    assert e.value.name == "CFA_ERR_INVAL"
+    with pytest.raises(cfa.CfaError) as e:
+        host_plan(m, slab_bytes=1000)
+    assert e.value.name == "CFA_ERR_INVAL"
+    d = fake_dsts(m)
+    d[0] = (d[0][0] + 1, d[0][1], d[0][2])
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Plan(entries_for(m), d, m.blob_bytes, host_only=True)
+    assert e.value.name == "CFA_ERR_ALIGN"
+
+
+def test_empty_manifest_and_zero_sized_entries():
+    from workloads import Manifest
+    with cfa.Plan(cfa.make_entries([], [], [], []), [], 0, host_only=True) as p:
+        assert p.info() == {"n_layers": 0, "n_pieces": 0, "n_chunks": 0}
+    ents = [{"name": "a", "dtype": "bf16", "shape": (0, 4), "offset": 0, "dst": 0, "row": 0},
+            {"name": "b", "dtype": "bf16", "shape": (2,), "offset": 0, "dst": 1, "row": 0,
+             "layer": 2}]
+    dsts = [{"name": "A", "dtype": "bf16", "shape": (0, 4)},
+            {"name": "B", "dtype": "bf16", "shape": (2,)}]
+    m = Manifest("zero", ents, dsts, 4, "bits", 0)
+    with host_plan(m) as p:
+        assert p.info()["n_pieces"] == 1 and p.info()["n_layers"] == 3
+
+
+def test_host_only_plan_refuses_to_load():
+    m, _, _, _ = manifest_case("fused_tiny.txt")
+    with host_plan(m) as p:
+        with pytest.raises(cfa.CfaError) as e:
+            p.load_async(cfa.Source.host(1), stream=0)
+        assert e.value.name == "CFA_ERR_INVAL"
+
+
+def test_full_size_manifests_plan_on_the_host():
+    import workloads
+    for name in ("llama3_8b_bf16", "llama3_70b_bf16"):
+        m = workloads.named_config(name)
+        with host_plan(m, chunk_bytes=m.chunk_bytes) as p:
+            st = p.stats()
+            assert st["bytes_written"] == m.total_dst_bytes()
+            assert st["n_chunks"] == -(-m.blob_bytes // m.chunk_bytes)
+            assert st["n_layers"] == m.n_groups()
+            pcs = p.pieces()
+            assert int(pcs["n_elems"].sum()) == sum(m.e_numel(i) for i in range(m.n_entries))

@@ -26,9 +26,11 @@
  *            656 <= c < 660 -> a signed zero.  That is about 0.5 % ties, 0.5 % subnormals and
  *            a few zeros, and never NaN or Inf.
  */
+#define _POSIX_C_SOURCE 200809L
 #include <math.h>
 #include <stdint.h>
 #include <string.h>
+#include <time.h>
 
 static inline uint64_t wl_word(uint64_t seed, uint64_t w)
 {
@@ -115,6 +117,45 @@ int wl_fill_f32mix(uint64_t seed, uint64_t off, uint64_t len, uint8_t *out)
         out[4 * i + 1] = (uint8_t)(v >> 8);
         out[4 * i + 2] = (uint8_t)(v >> 16);
         out[4 * i + 3] = (uint8_t)(v >> 24);
+    }
+    return 0;
+}
+
+/*
+ * A fill callback with the loader's source signature, so that tests and the benchmark can
+ * stream a blob that exists only as its generator definition.  `user` points to a
+ * wl_cb_source.  Optional fault injection on the host: fail_from (return an error for ranges
+ * reaching that blob offset) and delay_us (sleep before every call).
+ */
+typedef struct wl_cb_source {
+    int32_t kind; /* 0 = bits, 1 = f32mix */
+    int32_t reserved;
+    uint64_t seed;
+    uint64_t period;    /* 0 = none */
+    uint64_t fail_from; /* UINT64_MAX = never */
+    uint64_t delay_us;
+} wl_cb_source;
+
+int wl_fill_cb(void *user, uint64_t off, void *dst, uint64_t len)
+{
+    const wl_cb_source *s = (const wl_cb_source *)user;
+    if (s->delay_us) {
+        struct timespec ts;
+        ts.tv_sec = (time_t)(s->delay_us / 1000000u);
+        ts.tv_nsec = (long)(s->delay_us % 1000000u) * 1000L;
+        nanosleep(&ts, NULL);
+    }
+    if (off + len > s->fail_from) return 1;
+    uint8_t *out = (uint8_t *)dst;
+    while (len) {
+        uint64_t o = s->period ? off % s->period : off;
+        uint64_t take = s->period ? s->period - o : len;
+        if (take > len) take = len;
+        if (s->kind == 0) wl_fill_bits(s->seed, o, take, out);
+        else if (wl_fill_f32mix(s->seed, o, take, out) != 0) return 2;
+        out += take;
+        off += take;
+        len -= take;
     }
     return 0;
 }
