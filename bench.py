@@ -1,0 +1,410 @@
+#!/usr/bin/env python3
+"""Benchmark of the GB300 checkpoint loader.
+
+One step = one complete load of a synthetic Llama-3-8B-shaped bf16 checkpoint (32 layers, q/k/v
+and gate/up fused; 16.06 GB) into its final per-parameter layout, i.e. every stage of the path:
+chunked staging, host->device transfer (e2e only), the unpack kernel with fused layouts and
+per-tensor checksums, readiness events, and the checksum read-back (e2e only).
+
+Printed on one JSON line (rank 0):
+  value      unpacked GB/s into the final layout, kernel only: the blob already sits in HBM
+             (device source); algorithmic bytes = every source byte read once + every
+             destination byte written once, over the device time of K steps
+  e2e        the same metric end to end through the C ABI with a pinned HOST blob: every step
+             copies the whole checkpoint host->device (cudaMemcpyAsync on the loader's copy
+             stream) and reads the checksums back; also seconds per model and the fraction of
+             the measured host->device bandwidth
+  roofline   the unpack kernel against the measured HBM copy bandwidth
+  cpu_baseline  the oracle (plain CPU loader) on a bounded sample, on this host's cores
+
+--impl reference times the oracle as the reference arm.  --gpus N runs N independent replicas
+(one process per GPU under torchrun); nothing in the path is sharded or exchanged.
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "unpacked GB/s into final layout (% of HBM peak); end-to-end H2D load s per model"
+UNIT = "GB/s"
+HBM_FALLBACK_GBS = 6800.0
+L2_BYTES = 129e6
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama3_8b_bf16")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--e2e-steps", type=int, default=None,
+                    help="steps of the end-to-end measurement (default: min(steps, 20))")
+    return ap.parse_args()
+
+
+# ------------------------------------------------------------------------------------------
+def make_workload(name):
+    import workloads
+    if name in workloads.NAMED_CONFIGS:
+        return workloads.named_config(name)
+    if name == "llama3_8b_bf16_2layer_v32k":  # small case for ncu captures (~1.4 GB blob)
+        return workloads.dense_config(name, 2, layers=2, hidden=4096, n_q=32, n_kv=8,
+                                      head_dim=128, inter=14336, vocab=32000)
+    raise SystemExit(f"unknown workload {name}")
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": HBM_FALLBACK_GBS}, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    for f in ("cfa_unpack.cu",):
+        with open(os.path.join(ROOT, "paper_2607_18957_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def recorded_traffic(workload):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+    except OSError:
+        return None
+    r = rec.get(workload)
+    if not r or r.get("kernel_sha256") != kernel_source_hash():
+        return None
+    return r.get("dram_bytes_per_launch")
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled while the timed region runs."""
+
+    FIELDS = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid):
+        self.uuid = uuid
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 10:
+                    continue
+                if self.uuid and parts[1] != self.uuid and not self.uuid.endswith(parts[1]) \
+                        and not parts[1].endswith(self.uuid):
+                    continue
+                rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        mhz = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        maxs = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            for k, nm in enumerate(names):
+                if r[6 + k].lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(mhz) if mhz else None,
+                "sm_max_mhz": max(maxs) if maxs else None,
+                "samples": len(rows), "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------------------------------------
+def cpu_baseline(m, seconds, steps=None):
+    """The oracle, as it stands, on destinations in blob order until `seconds` of CPU time (or
+    one destination per step for the reference arm).  Generation of the sample's blob bytes is
+    outside the timed region.  Returns (GB/s, bytes, secs, description, per-step times)."""
+    import numpy as np
+
+    import oracle
+    from workloads import DTYPE_SIZE
+    order = sorted(range(m.n_dsts),
+                   key=lambda j: min(int(m.e_offset[i]) for i in m.entries_of_dst(j)))
+    done_bytes, busy, used, step_times = 0, 0.0, [], []
+    k = 0
+    while True:
+        j = order[k % len(order)]
+        k += 1
+        es = m.entries_of_dst(j)
+        lo = min(int(m.e_offset[i]) for i in es)
+        hi = max(int(m.e_offset[i]) + m.e_nbytes(i) for i in es)
+        window = m.blob_range(lo, hi - lo)
+        t0 = time.perf_counter()
+        r = oracle.unpack(m, window, blob_begin=lo, dsts=[j])
+        dt = time.perf_counter() - t0
+        assert r.status == 0
+        nb = sum(m.e_nbytes(i) for i in es) + m.d_nbytes(j)
+        done_bytes += nb
+        busy += dt
+        used.append(m.d_name[j])
+        step_times.append((dt, nb))
+        del window, r
+        if steps is not None:
+            if len(step_times) >= steps:
+                break
+        elif busy >= seconds or k >= len(order):
+            break
+    desc = (f"{len(used)} destination tensor(s) of {m.name} in blob order ({used[0]} ...), "
+            f"{done_bytes / 1e9:.2f} GB of algorithmic bytes, single thread")
+    return done_bytes / busy / 1e9, done_bytes, busy, desc, step_times
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    m = make_workload(args.workload)
+    cores = 1
+    # warm-up steps, then K timed steps, each one destination tensor through the oracle
+    cpu_baseline(m, 0, steps=max(args.warmup, 1))
+    gbs, nbytes, busy, desc, times = cpu_baseline(m, 0, steps=args.steps)
+    ms = 1e3 * sum(t for t, _ in times) / len(times)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(gbs, 4), "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "u16", "data": "synthetic (seeded generator)",
+        "config": {"workload": m.name, "step": "one destination tensor per step, in blob order",
+                   "parallelism": "replicas"},
+        "cpu_baseline": {"value": round(gbs, 4), "unit": UNIT, "cores": cores, "kind": "oracle",
+                         "sample": desc},
+        "e2e": {"value": round(gbs, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------------------------------
+def run_ours(args):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    import paper_2607_18957_gb300 as cfa
+    from workloads.harness import DeviceDsts, entries_for, pinned_blob
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl")
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    def sum_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.SUM)
+        return float(t.item())
+
+    m = make_workload(args.workload)
+    t_setup = time.time()
+    host = pinned_blob(m)                      # the checkpoint in page-locked host memory
+    dev_blob = torch.empty(m.source_bytes(), dtype=torch.uint8, device="cuda")
+    dev_blob.copy_(host)
+    dsts = DeviceDsts(m)
+    entries = entries_for(m)
+    stream = torch.cuda.current_stream()
+    setup_s = time.time() - t_setup
+
+    # ---------------- kernel only: the blob already resident in HBM -------------------------
+    plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                    dev_slots=0, host_slots=0)
+    st = plan.stats()
+    algo_bytes = st["bytes_read"] + st["bytes_written"]
+    src = cfa.Source.device(dev_blob.data_ptr(), period=m.period or 0)
+    for _ in range(args.warmup):
+        plan.load_async(src, stream)
+    torch.cuda.synchronize()
+    launches_per_load = plan.stats()["kernel_launches"]
+
+    props = torch.cuda.get_device_properties(local)
+    uuid = str(getattr(props, "uuid", "") or "")
+    if uuid and not uuid.startswith("GPU-"):
+        uuid = "GPU-" + uuid
+    sampler = ClockSampler(uuid)
+    sampler.start()
+    time.sleep(0.3)
+    barrier()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for k in range(args.steps):
+        ev[k][0].record(stream)
+        plan.load_async(src, stream)
+        ev[k][1].record(stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    kernel_ms = t0.elapsed_time(t1)
+    per_load = [a.elapsed_time(b) for a, b in ev]
+    ck_dev = plan.checksums()
+    plan.close()
+    total_ms = max_over_ranks(kernel_ms)
+    value = sum_over_ranks(algo_bytes * args.steps) / (total_ms / 1e3) / 1e9
+
+    # ---------------- end to end: pinned host blob -> final layout through the C ABI ---------
+    e2e = None
+    h2d_gbs = None
+    if not args.no_e2e:
+        # host->device copy bandwidth of this machine, 1 GiB pinned, best of 10
+        gib = 1 << 30
+        hsrc = host[:gib] if host.numel() >= gib else torch.empty(gib, dtype=torch.uint8,
+                                                                 pin_memory=True)
+        dtmp = torch.empty(gib, dtype=torch.uint8, device="cuda")
+        best = None
+        for _ in range(12):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            dtmp.copy_(hsrc, non_blocking=True)
+            b.record(stream)
+            b.synchronize()
+            t = a.elapsed_time(b)
+            best = t if best is None else min(best, t)
+        h2d_gbs = gib / (best / 1e3) / 1e9
+        del dtmp
+        e2e_steps = args.e2e_steps or min(args.steps, 20)
+        plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                        dev_slots=2, host_slots=0)
+        hsrc_all = cfa.Source.pinned(host.data_ptr(), period=m.period or 0)
+        for _ in range(min(args.warmup, 3)):
+            plan.load_async(hsrc_all, stream)
+            plan.checksums()
+        barrier()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        marks = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
+        a.record(stream)
+        for k in range(e2e_steps):
+            plan.load_async(hsrc_all, stream)   # H2D of the whole checkpoint + unpack
+            ck = plan.checksums()                # D2H of the step's result
+            marks[k].record(stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e2e_ms = max_over_ranks(a.elapsed_time(b)) / e2e_steps
+        step_ms = [a.elapsed_time(marks[0])] + [marks[k - 1].elapsed_time(marks[k])
+                                                for k in range(1, e2e_steps)]
+        assert np.array_equal(ck, ck_dev), "end-to-end checksums differ from the kernel-only run"
+        plan.close()
+        e2e_gbs = sum_over_ranks(algo_bytes) / (e2e_ms / 1e3) / 1e9
+        e2e = {"value": round(e2e_gbs, 3), "unit": UNIT,
+               "h2d_bytes_per_step": m.blob_bytes, "d2h_bytes_per_step": 8 * m.n_entries,
+               "seconds_per_model": round(e2e_ms / 1e3, 5),
+               "h2d_gbs_measured": round(h2d_gbs, 2),
+               "frac_of_h2d": round((m.blob_bytes / (e2e_ms / 1e3) / 1e9) / h2d_gbs, 4),
+               "steps": e2e_steps, "step_ms_median": round(statistics.median(step_ms), 2),
+               "step_ms_max": round(max(step_ms), 2),
+               "source": f"pinned host blob, 2 device staging slots of {m.chunk_bytes >> 20} MiB"}
+    clocks = sampler.stop()
+
+    # ---------------- the oracle on this host -------------------------------------------------
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        gbs, nb, busy, desc, _ = cpu_baseline(m, args.cpu_seconds)
+        cpu = {"value": round(gbs, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": desc}
+
+    if rank != 0:
+        if world > 1:
+            dist.destroy_process_group()
+        return
+    peaks, peak_kind = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", HBM_FALLBACK_GBS))
+    avg_launch_ms = statistics.mean(per_load)
+    achieved = algo_bytes / (avg_launch_ms / 1e3) / 1e9
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "u16",
+        "data": "synthetic (seeded counter-based generator; random bf16 bit patterns)",
+        "config": {"workload": m.name, "blob_bytes": m.blob_bytes, "tensors": m.n_entries,
+                   "destinations": m.n_dsts, "algorithmic_bytes_per_step": algo_bytes,
+                   "chunk_bytes": m.chunk_bytes, "kernel_source": "device-resident blob",
+                   "l2": f"no flush: inputs {m.blob_bytes / 1e9:.2f} GB > L2 "
+                         f"{L2_BYTES / 1e6:.0f} MB",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
+                     "unit": "GB/s", "frac": round(achieved / peak, 4),
+                     "traffic": recorded_traffic(m.name), "peak_source": peak_kind,
+                     "kernel": "cfa_unpack_kernel<1> (bf16 copy class)",
+                     "launch_ms": round(avg_launch_ms, 4)},
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+        "gpu_launches": int(launches_per_load * args.steps),
+        "clocks": clocks,
+        "setup_s": round(setup_s, 2),
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -106,6 +106,27 @@ def _ptr_array(arrs):
     return out
 
 
+def _columns(m):
+    """The manifest's columns in the oracle's own codes (marshalling only; cached on m)."""
+    c = getattr(m, "_oracle_columns", None)
+    if c is None:
+        c = (np.array([_DTYPE_CODE[str(x)] for x in m.e_dtype], dtype=np.int32),
+             np.array([_DTYPE_CODE[str(x)] for x in m.d_dtype], dtype=np.int32),
+             (m.e_cast.astype(np.uint32) * _CAST) | (m.e_cksum.astype(np.uint32) * _CKSUM),
+             np.ascontiguousarray(m.e_ndim, dtype=np.int32),
+             np.ascontiguousarray(m.e_shape, dtype=np.int64),
+             np.ascontiguousarray(m.e_offset, dtype=np.uint64),
+             np.ascontiguousarray(m.e_dst, dtype=np.int32),
+             np.ascontiguousarray(m.e_row, dtype=np.int64),
+             np.ascontiguousarray(m.d_ndim, dtype=np.int32),
+             np.ascontiguousarray(m.d_shape, dtype=np.int64))
+        try:
+            m._oracle_columns = c
+        except AttributeError:
+            pass
+    return c
+
+
 def unpack(m, blob, blob_begin=0, dsts=None, cover=False, fill=0, lib=None):
     """Runs the naive loader over manifest `m`.
 
@@ -120,16 +141,8 @@ def unpack(m, blob, blob_begin=0, dsts=None, cover=False, fill=0, lib=None):
     lib = lib or _load()
     n, nd = m.n_entries, m.n_dsts
     sel = range(nd) if dsts is None else sorted(set(int(j) for j in dsts))
-    e_dtype = np.array([_DTYPE_CODE[str(x)] for x in m.e_dtype], dtype=np.int32)
-    d_dtype = np.array([_DTYPE_CODE[str(x)] for x in m.d_dtype], dtype=np.int32)
-    e_flags = (m.e_cast.astype(np.uint32) * _CAST) | (m.e_cksum.astype(np.uint32) * _CKSUM)
-    e_ndim = np.ascontiguousarray(m.e_ndim, dtype=np.int32)
-    e_shape = np.ascontiguousarray(m.e_shape, dtype=np.int64)
-    e_off = np.ascontiguousarray(m.e_offset, dtype=np.uint64)
-    e_dst = np.ascontiguousarray(m.e_dst, dtype=np.int32)
-    e_row = np.ascontiguousarray(m.e_row, dtype=np.int64)
-    d_ndim = np.ascontiguousarray(m.d_ndim, dtype=np.int32)
-    d_shape = np.ascontiguousarray(m.d_shape, dtype=np.int64)
+    (e_dtype, d_dtype, e_flags, e_ndim, e_shape, e_off, e_dst, e_row, d_ndim,
+     d_shape) = _columns(m)
     bufs = [None] * nd
     covs = [None] * nd
     for j in sel:

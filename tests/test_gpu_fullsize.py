@@ -1,0 +1,167 @@
+"""GPU parity at the full sizes of the five workloads, in the launch configurations the
+benchmark times: every destination byte and every checksum against the oracle (run per batch of
+destinations on regenerated blob windows, on all host cores).  Also the per-layer readiness
+times of the 70B-shaped streaming load."""
+import os
+from concurrent.futures import ThreadPoolExecutor
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2607_18957_gb300 as cfa
+import workloads
+from workloads.harness import CallbackSource, DeviceDsts, entries_for
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def cuda_device():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.set_device(0)
+    yield
+    torch.cuda.empty_cache()
+
+
+def _threads():
+    return max(1, min(16, len(os.sched_getaffinity(0))))
+
+
+def verify_all(m, d, ck, max_batch=1 << 29, max_count=50_000):
+    """Every destination byte and every checksum of `m` against the oracle."""
+    nbytes = m.e_nbytes_array()
+    offs = m.e_offset.astype(np.int64)
+    de = m.dst_entries()
+    batches, j0, acc = [], 0, 0
+    for j in range(m.n_dsts):
+        acc += m.d_nbytes(j)
+        if acc >= max_batch or j + 1 - j0 >= max_count or j == m.n_dsts - 1:
+            batches.append((j0, j + 1))
+            j0, acc = j + 1, 0
+
+    def work(b):
+        a, z = b
+        ents = np.concatenate([de[j] for j in range(a, z)])
+        if ents.size == 0:
+            return ents, np.zeros(0, np.uint64), []
+        lo = int(offs[ents].min())
+        hi = int((offs[ents] + nbytes[ents]).max())
+        window = m.blob_range(lo, hi - lo, threads=2)
+        r = oracle.unpack(m, window, blob_begin=lo, dsts=range(a, z))
+        assert r.status == 0, r.status_name
+        got = d.host_region(a, z)
+        bad = [m.d_name[j] for j in range(a, z) if not np.array_equal(got[j], r.dst[j])]
+        return ents, r.cksum[ents], bad
+
+    bad_all, n_ck = [], 0
+    with ThreadPoolExecutor(_threads()) as ex:
+        for ents, want, bad in ex.map(work, batches):
+            bad_all += bad
+            assert np.array_equal(ck[ents], want), f"{m.name}: checksums differ"
+            n_ck += ents.size
+    assert not bad_all, f"{m.name}: destinations differ from the oracle: {bad_all[:5]}"
+    assert n_ck == m.n_entries
+
+
+def device_source_blob(m):
+    """The blob (or one period of it) in device memory, generated on the host piecewise."""
+    n = m.source_bytes()
+    dev = torch.empty(n, dtype=torch.uint8, device="cuda")
+    piece = 2 << 30
+    stage = torch.empty(min(piece, n), dtype=torch.uint8, pin_memory=True)
+    for o in range(0, n, piece):
+        k = min(piece, n - o)
+        workloads.gen.fill_ptr(m.blob_kind, m.seed, o, k, stage.data_ptr())
+        dev[o:o + k].copy_(stage[:k])
+    return dev
+
+
+def _load(m, d, src, **kw):
+    with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                  **kw) as plan:
+        plan.load_async(src)
+        plan.wait_layer()
+        ck = plan.checksums()
+        st = plan.stats()
+        times = plan.layer_times() if kw.get("timing") else None
+    return ck, st, times
+
+
+def test_full_tiny_1000():
+    m = workloads.named_config("tiny_1000")
+    d = DeviceDsts(m)
+    blob = device_source_blob(m)
+    ck, _, _ = _load(m, d, cfa.Source.device(blob.data_ptr()), dev_slots=0, host_slots=0)
+    verify_all(m, d, ck)
+    assert d.guards_intact()
+
+
+def test_full_llama3_8b_bf16():
+    m = workloads.named_config("llama3_8b_bf16")
+    d = DeviceDsts(m)
+    blob = device_source_blob(m)
+    # the benchmark's kernel-only configuration: blob resident in HBM, one merged launch
+    ck, st, _ = _load(m, d, cfa.Source.device(blob.data_ptr()), dev_slots=0, host_slots=0)
+    assert st["kernel_launches"] == 1
+    verify_all(m, d, ck)
+    assert d.guards_intact()
+    del blob
+    # the benchmark's end-to-end configuration: pinned host blob through the staging slots
+    host = torch.empty(m.blob_bytes, dtype=torch.uint8, pin_memory=True)
+    m.fill_source_ptr(host.data_ptr())
+    d.buf.fill_(0xA5)
+    ck2, st2, _ = _load(m, d, cfa.Source.pinned(host.data_ptr()), host_slots=0)
+    assert st2["kernel_launches"] == st2["n_chunks"]
+    assert np.array_equal(ck, ck2)
+    verify_all(m, d, ck2)
+
+
+def test_full_llama3_8b_f32_rne():
+    m = workloads.named_config("llama3_8b_f32_rne")
+    d = DeviceDsts(m)
+    blob = device_source_blob(m)
+    ck, _, _ = _load(m, d, cfa.Source.device(blob.data_ptr()), dev_slots=0, host_slots=0)
+    verify_all(m, d, ck)
+    assert d.guards_intact()
+
+
+def test_full_mixtral_8x7b_bf16():
+    m = workloads.named_config("mixtral_8x7b_bf16")
+    d = DeviceDsts(m)
+    blob = device_source_blob(m)
+    ck, st, _ = _load(m, d, cfa.Source.device(blob.data_ptr()), dev_slots=0, host_slots=0)
+    assert st["n_tiny"] >= 200_000
+    verify_all(m, d, ck)
+    del blob
+    torch.cuda.empty_cache()
+    # the same checkpoint streamed through the callback source and the staging ring
+    d.buf.fill_(0xA5)
+    cb = CallbackSource(m)
+    ck2, _, _ = _load(m, d, cb.source(), fill_threads=16)
+    assert np.array_equal(ck, ck2)
+    verify_all(m, d, ck2)
+
+
+def test_full_llama3_70b_bf16_streamed():
+    m = workloads.named_config("llama3_70b_bf16")
+    d = DeviceDsts(m)
+    pool = torch.empty(m.period, dtype=torch.uint8, pin_memory=True)
+    m.fill_source_ptr(pool.data_ptr())
+    ck, st, times = _load(m, d, cfa.Source.pinned(pool.data_ptr(), period=m.period),
+                          timing=True)
+    assert st["n_chunks"] == 132
+    # readiness groups follow blob order: embedding, layers 0..79, head
+    assert np.all(np.diff(times) >= -1e-3), times
+    assert times[-1] <= st["load_ms"] + 1e-3
+    verify_all(m, d, ck)
+    # and from a device-resident pool, one launch per period
+    dpool = pool.to("cuda")
+    d.buf.fill_(0xA5)
+    ck2, st2, _ = _load(m, d, cfa.Source.device(dpool.data_ptr(), period=m.period),
+                        dev_slots=0, host_slots=0)
+    assert st2["kernel_launches"] == -(-st2["n_chunks"] // (m.period // m.chunk_bytes))
+    assert np.array_equal(ck, ck2)
+    assert d.guards_intact()

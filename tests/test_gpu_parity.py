@@ -146,7 +146,7 @@ def test_element_sizes_1_4_8():
     ents, dsts, off = [], [], 0
     for k, (dt, es) in enumerate([("u8", 1), ("i32", 4), ("i64", 8), ("f64", 8), ("u8", 1)]):
         n = int(rng.integers(1, 70000))
-        off += int(rng.integers(0, 5)) * es
+        off = (off + es - 1) // es * es + int(rng.integers(0, 5)) * es
         dsts.append({"name": f"d{k}", "dtype": dt, "shape": (n,)})
         ents.append({"name": f"e{k}", "dtype": dt, "shape": (n,), "offset": off, "dst": k,
                      "row": 0, "layer": k})

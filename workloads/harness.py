@@ -52,6 +52,14 @@ class DeviceDsts:
     def host_bytes(self, j):
         return self.view(j).cpu().numpy()
 
+    def host_region(self, j0, j1):
+        """Destinations j0 .. j1-1 with one device->host copy: {j: uint8 array}."""
+        lo = self.offsets[j0]
+        hi = self.offsets[j1 - 1] + self.m.d_nbytes(j1 - 1)
+        h = self.buf[lo:hi].cpu().numpy()
+        return {j: h[self.offsets[j] - lo:self.offsets[j] - lo + self.m.d_nbytes(j)]
+                for j in range(j0, j1)}
+
     def guards_intact(self):
         """True if every byte outside the destinations still holds GUARD_BYTE."""
         import torch
