@@ -114,7 +114,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                 "-lms", "100"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
         except OSError:
             self.proc = None
 
@@ -342,6 +342,7 @@ def run_ours(args):
         e2e_ms = max_over_ranks(a.elapsed_time(b)) / e2e_steps
         step_ms = [a.elapsed_time(marks[0])] + [marks[k - 1].elapsed_time(marks[k])
                                                 for k in range(1, e2e_steps)]
+        print("e2e step ms:", [round(x, 1) for x in step_ms], file=sys.stderr)
         assert np.array_equal(ck, ck_dev), "end-to-end checksums differ from the kernel-only run"
         plan.close()
         e2e_gbs = sum_over_ranks(algo_bytes) / (e2e_ms / 1e3) / 1e9
