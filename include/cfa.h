@@ -298,6 +298,44 @@ cfa_status cfa_plan_get_pieces(const cfa_plan *plan, cfa_piece *out, size_t cap,
 cfa_status cfa_unpack_chunks_async(cfa_plan *plan, uint32_t chunk_begin, uint32_t chunk_end,
                                    const void *chunk_src, cfa_stream stream);
 
+/*
+ * Unpacks a blob that already sits in device memory into its destinations WITHOUT ALLOCATING
+ * ANYTHING -- no cudaMalloc, no cudaFree, no host heap.  The paper has no counterpart: it is for
+ * callers that cannot allocate, such as a serving engine whose memory pool already owns the
+ * device, code running under CUDA stream capture (where cudaMalloc and cudaFree are not
+ * allowed), or a restricted runtime with no allocator.  It is cfa_plan_create +
+ * cfa_load_async(DEVICE source) + cfa_get_checksums' buffer in one call, with these
+ * differences:
+ *   - no plan: every entry is validated on its own (dtype, shape, bounds, alignment), but the
+ *     coverage and overlap checks of cfa_plan_create are not made; destinations must not
+ *     overlap one another and entries must not write the same bytes;
+ *   - the work descriptors live in a fixed device array inside this library of
+ *     CFA_NOALLOC_MAX_ITEMS entries (16384 x 32 bytes = 512 KiB, plus a status word), held by
+ *     every GPU that loads the library until the process exits.  A tensor needs one work item
+ *     per 2 MiB of destination bytes, one in all below 8 KiB; a manifest that needs more is
+ *     rejected with CFA_ERR_INVAL before any GPU work, and `err` says so;
+ *   - all calls on a device share that array: calls serialise on the host, but calls whose GPU
+ *     work may overlap (different streams, no ordering between them) race on it;
+ *   - the first call on a device does a one-time set-up (it looks up the array's device address
+ *     and the kernels' occupancy); make it before any stream capture.
+ *
+ *   entries, n_entries, dsts, n_dsts   as for cfa_plan_create (host arrays, read during the call)
+ *   blob_dev, blob_bytes   the blob in device memory (256-byte aligned); must stay valid and
+ *                          unchanged until the unpack has run on `stream`
+ *   cksum_dev              device array of n_entries uint64 receiving the checksums
+ *                          (cleared by the call), or NULL for none
+ *   stream                 all GPU work is enqueued here; the call returns without waiting, after
+ *                          the descriptors have been handed to the driver
+ *   err, err_len           optional buffer for a message on failure (NULL for none)
+ * Errors: CFA_ERR_INVAL (NULL argument, bad entry, too many work items), CFA_ERR_DTYPE,
+ * CFA_ERR_SHAPE, CFA_ERR_OOB, CFA_ERR_ALIGN, CFA_ERR_CUDA.
+ */
+#define CFA_NOALLOC_MAX_ITEMS 16384
+cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t n_entries,
+                              const cfa_dst *dsts, size_t n_dsts, const void *blob_dev,
+                              uint64_t blob_bytes, uint64_t *cksum_dev, cfa_stream stream,
+                              char *err, size_t err_len);
+
 /* Zeroes the plan's checksum buffer on `stream`. */
 cfa_status cfa_reset_checksums(cfa_plan *plan, cfa_stream stream);
 

@@ -83,6 +83,8 @@ SIGNATURES = {
     "cfa_last_error": (ctypes.c_char_p, [_P]),
     "cfa_status_name": (ctypes.c_char_p, [ctypes.c_int]),
     "cfa_abi_sizeof": (_SZ, [ctypes.c_char_p]),
+    "cfa_unpack_noalloc": (ctypes.c_int, [_P, _SZ, _P, _SZ, _P, _U64, _P, _P, ctypes.c_char_p,
+                                          _SZ]),
 }
 
 _lib = None
