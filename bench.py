@@ -49,6 +49,10 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--no-attribution", action="store_true",
+                    help="skip the end-to-end attribution measurements")
+    ap.add_argument("--bulk", action="store_true",
+                    help="copy aligned slabs with the TMA bulk kernel (for comparison)")
     ap.add_argument("--e2e-steps", type=int, default=None,
                     help="steps of the end-to-end measurement (default: min(steps, 20))")
     return ap.parse_args()
@@ -76,7 +80,7 @@ def measured_peaks():
 
 def kernel_source_hash():
     h = hashlib.sha256()
-    for f in ("cfa_unpack.cu",):
+    for f in ("cfa_unpack.cu", "cfa_bulk.cu"):
         with open(os.path.join(ROOT, "paper_2607_18957_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()
@@ -153,6 +157,75 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------------------------
+def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
+    """Where end-to-end time goes: the host link for pinned and pageable memory, host memcpy
+    with the loader's fill threads, a load from a pageable copy of the checkpoint through the
+    pinned staging ring, and (CFA_OPT_TIMING) per-layer readiness of one pinned load."""
+    from concurrent.futures import ThreadPoolExecutor
+
+    import numpy as np
+    import torch
+
+    import paper_2607_18957_gb300 as cfa
+    out = {"h2d_pinned_gbs": round(h2d_gbs, 2)}
+    gib = 1 << 30
+    threads = max(1, len(os.sched_getaffinity(0)))
+    pageable = np.empty(m.source_bytes(), dtype=np.uint8)
+    pageable[:] = host.numpy()                                   # the same bytes, pageable
+    dtmp = torch.empty(gib, dtype=torch.uint8, device="cuda")
+    src_t = torch.from_numpy(pageable[:gib])
+    best = min(_timed(lambda: dtmp.copy_(src_t), stream) for _ in range(5))
+    out["h2d_pageable_gbs"] = round(gib / best / 1e6, 2)
+    del dtmp
+    dst = np.empty(4 * gib, dtype=np.uint8)
+    part = (4 * gib) // threads
+
+    def cp(k):
+        np.copyto(dst[k * part:(k + 1) * part], pageable[k * part:(k + 1) * part])
+    with ThreadPoolExecutor(threads) as ex:
+        list(ex.map(cp, range(threads)))                         # warm
+        t0 = time.perf_counter()
+        list(ex.map(cp, range(threads)))
+        out["host_memcpy_gbs"] = round(4 * gib / (time.perf_counter() - t0) / 1e9, 2)
+    out["host_threads"] = threads
+    del dst
+    plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                    dev_slots=2, host_slots=2, fill_threads=threads, bulk=args.bulk)
+    src = cfa.Source.host(pageable.ctypes.data, period=m.period or 0)
+    plan.load_async(src, stream)
+    plan.checksums()
+    ms = min(_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
+             for _ in range(2))
+    plan.close()
+    out["e2e_pageable_s_per_model"] = round(ms / 1e3, 4)
+    out["e2e_pageable_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
+    del pageable
+    plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                    dev_slots=2, host_slots=0, timing=True, bulk=args.bulk)
+    plan.load_async(cfa.Source.pinned(host.data_ptr(), period=m.period or 0), stream)
+    plan.wait_layer()
+    t = plan.layer_times()
+    st = plan.stats()
+    plan.close()
+    out["layer_ready_ms"] = {"first_group": round(float(t[0]), 2),
+                             "median_group": round(float(np.median(t)), 2),
+                             "last_group": round(float(t[-1]), 2),
+                             "groups": int(t.size), "load_ms": round(st["load_ms"], 2),
+                             "h2d_ms": round(st["h2d_ms"], 2),
+                             "unpack_ms": round(st["unpack_ms"], 2)}
+    return out
+
+
+def _timed(fn, stream):
+    import torch
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    fn()
+    b.record(stream)
+    b.synchronize()
+    return a.elapsed_time(b)
+
+
 def cpu_baseline(m, seconds, steps=None):
     """The oracle, as it stands, on destinations in blob order until `seconds` of CPU time (or
     one destination per step for the reference arm).  Generation of the sample's blob bytes is
@@ -263,7 +336,7 @@ def run_ours(args):
 
     # ---------------- kernel only: the blob already resident in HBM -------------------------
     plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                    dev_slots=0, host_slots=0)
+                    dev_slots=0, host_slots=0, bulk=args.bulk)
     st = plan.stats()
     algo_bytes = st["bytes_read"] + st["bytes_written"]
     src = cfa.Source.device(dev_blob.data_ptr(), period=m.period or 0)
@@ -322,7 +395,7 @@ def run_ours(args):
         del dtmp
         e2e_steps = args.e2e_steps or min(args.steps, 20)
         plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                        dev_slots=2, host_slots=0)
+                        dev_slots=2, host_slots=0, bulk=args.bulk)
         hsrc_all = cfa.Source.pinned(host.data_ptr(), period=m.period or 0)
         for _ in range(min(args.warmup, 3)):
             plan.load_async(hsrc_all, stream)
@@ -354,6 +427,8 @@ def run_ours(args):
                "steps": e2e_steps, "step_ms_median": round(statistics.median(step_ms), 2),
                "step_ms_max": round(max(step_ms), 2),
                "source": f"pinned host blob, 2 device staging slots of {m.chunk_bytes >> 20} MiB"}
+        if not args.no_attribution:
+            e2e["attribution"] = attribution(m, host, dsts, entries, stream, args, h2d_gbs)
     clocks = sampler.stop()
 
     # ---------------- the oracle on this host -------------------------------------------------
@@ -367,6 +442,12 @@ def run_ours(args):
         if world > 1:
             dist.destroy_process_group()
         return
+    if st["n_bulk"]:
+        kernel_name = "cfa_bulk_kernel (TMA bulk copies) + cfa_unpack_kernel (heads, tails, tiny)"
+    elif bool(m.e_cast.any()):
+        kernel_name = "cfa_unpack_kernel<4> (fp32 -> bf16 cast class)"
+    else:
+        kernel_name = "cfa_unpack_kernel (16-byte vector copy)"
     peaks, peak_kind = measured_peaks()
     peak = float(peaks.get("hbm_gbs", HBM_FALLBACK_GBS))
     avg_launch_ms = statistics.mean(per_load)
@@ -386,7 +467,7 @@ def run_ours(args):
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
                      "unit": "GB/s", "frac": round(achieved / peak, 4),
                      "traffic": recorded_traffic(m.name), "peak_source": peak_kind,
-                     "kernel": "cfa_unpack_kernel<1> (bf16 copy class)",
+                     "kernel": kernel_name,
                      "launch_ms": round(avg_launch_ms, 4)},
         "e2e": e2e,
         "cpu_baseline": cpu,

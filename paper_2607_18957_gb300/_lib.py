@@ -15,7 +15,7 @@ STATUS = {0: "CFA_OK", -1: "CFA_ERR_INVAL", -2: "CFA_ERR_OVERLAP", -3: "CFA_ERR_
           -12: "CFA_ERR_DEVICE", -13: "CFA_ERR_SHAPE"}
 DTYPE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7}
 ENTRY_CAST_BF16, ENTRY_CKSUM = 0x1, 0x2
-OPT_STRICT_COVERAGE, OPT_HOST_ONLY, OPT_TIMING, OPT_NO_BULK, OPT_NO_MERGE = 0x1, 0x2, 0x4, 0x8, 0x10
+OPT_STRICT_COVERAGE, OPT_HOST_ONLY, OPT_TIMING, OPT_BULK, OPT_NO_MERGE = 0x1, 0x2, 0x4, 0x8, 0x10
 SRC_HOST, SRC_PINNED, SRC_CALLBACK, SRC_DEVICE = 1, 2, 3, 4
 ALL = -1
 

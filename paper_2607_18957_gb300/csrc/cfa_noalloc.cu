@@ -31,7 +31,8 @@
 extern "C" int cfa_unpack_blocks_per_sm(int cls);
 extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_t n_slabs,
                                          const cfa_work *tiny, uint32_t n_tiny,
-                                         uint64_t src_base, uint64_t src_lo, uint64_t src_hi,
+                                         uint64_t src_base, uint64_t src_period,
+                                         uint64_t src_lo, uint64_t src_hi,
                                          unsigned long long *ck, int *status, int grid_cap,
                                          cudaStream_t stream);
 
@@ -281,7 +282,7 @@ extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t
         if (!count[k][0] && !count[k][1]) continue;
         e = cfa_launch_unpack(k, scratch->items + base[k][0], count[k][0],
                               scratch->items + base[k][1], count[k][1],
-                              (uint64_t)(uintptr_t)blob_dev, 0, blob_bytes,
+                              (uint64_t)(uintptr_t)blob_dev, 0, 0, blob_bytes,
                               reinterpret_cast<unsigned long long *>(cksum_dev), &scratch->status,
                               g_grid_cap[dev][k], stream);
     }

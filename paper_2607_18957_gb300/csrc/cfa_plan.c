@@ -25,7 +25,7 @@
 /* The TMA bulk kernel takes cast-free slabs whose source, destination and length are all
  * multiples of 16 bytes. */
 #ifndef CFA_BULK_READY
-#define CFA_BULK_READY 0
+#define CFA_BULK_READY 1
 #endif
 
 int cfa_dtype_size(int32_t dt)
@@ -441,7 +441,7 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
     out->tiny_first = (uint32_t *)calloc(nf, sizeof(uint32_t));
     if (!out->slab_first || !out->bulk_first || !out->tiny_first) { st = CFA_ERR_NOMEM; goto done; }
     {
-        const int use_bulk = CFA_BULK_READY && !(o.flags & CFA_OPT_NO_BULK);
+        const int use_bulk = CFA_BULK_READY && (o.flags & CFA_OPT_BULK);
         const uint64_t slab = o.slab_bytes;
         /* pass 1: items in chunk order, tagged with their class in `pad` */
         for (size_t p = 0; p < n_pieces; ++p) {

@@ -40,9 +40,16 @@
 #include "cfa_internal.h"
 
 extern "C" int cfa_unpack_blocks_per_sm(int cls);
+extern "C" int cfa_bulk_blocks_per_sm(int log2es);
+extern "C" cudaError_t cfa_launch_bulk(int log2es, const cfa_work *items, uint32_t n_items,
+                                       uint64_t src_base, uint64_t src_period,
+                                       uint64_t src_lo, uint64_t src_hi,
+                                       unsigned long long *ck, int *status, int grid_cap,
+                                       cudaStream_t stream);
 extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_t n_slabs,
                                          const cfa_work *tiny, uint32_t n_tiny,
-                                         uint64_t src_base, uint64_t src_lo, uint64_t src_hi,
+                                         uint64_t src_base, uint64_t src_period,
+                                         uint64_t src_lo, uint64_t src_hi,
                                          unsigned long long *ck, int *status, int grid_cap,
                                          cudaStream_t stream);
 
@@ -158,7 +165,8 @@ struct cfa_plan {
     bool host_only = false;
     int device = 0;
     int grid_cap[CFA_N_CLASSES] = {0};
-    cfa_work *d_slabs = nullptr, *d_tiny = nullptr;
+    int bulk_grid_cap[4] = {0};
+    cfa_work *d_slabs = nullptr, *d_tiny = nullptr, *d_bulk = nullptr;
     unsigned long long *d_ck = nullptr;
     int *d_status = nullptr;
     uint8_t *d_slots = nullptr;
@@ -231,23 +239,36 @@ void CUDART_CB fill_host_fn(void *arg)
     });
 }
 
-/* Unpacks chunks [c0, c1), whose blob byte o sits at device address src_base + o: one launch
- * per work class present in those chunks (normally one). */
-cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, cudaStream_t s)
+/* Unpacks chunks [c0, c1), whose blob byte o sits at device address src_base + o (or
+ * src_base + (o mod period) for a periodic source): per work class present in those chunks
+ * (normally one), a TMA bulk launch for its aligned cast-free slabs and a vector launch for
+ * everything else. */
+cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint64_t period,
+                  cudaStream_t s)
 {
     const cfa_host_plan &hp = p->hp;
     const uint64_t lo = (uint64_t)c0 * hp.chunk_bytes;
     const uint64_t hi = std::min<uint64_t>(hp.blob_bytes, (uint64_t)c1 * hp.chunk_bytes);
     const size_t row = (size_t)hp.n_chunks + 1;
+    const bool timing_on = (hp.opts.flags & CFA_OPT_TIMING) != 0;
+    for (int k = 0; k < CFA_N_CLASSES && hp.n_bulk; ++k) {
+        const uint32_t b0 = hp.bulk_first[k * row + c0], b1 = hp.bulk_first[k * row + c1];
+        if (b1 == b0) continue;
+        const bool timing = timing_on && p->last_launches < p->t_k0.size();
+        if (timing) CK(p, cudaEventRecord(p->t_k0[p->last_launches], s));
+        CK(p, cfa_launch_bulk(k, p->d_bulk + b0, b1 - b0, src_base, period, lo, hi, p->d_ck,
+                              p->d_status, p->bulk_grid_cap[k], s));
+        if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], s));
+        p->last_launches++;
+    }
     for (int k = 0; k < CFA_N_CLASSES; ++k) {
         const uint32_t s0 = hp.slab_first[k * row + c0], s1 = hp.slab_first[k * row + c1];
         const uint32_t t0 = hp.tiny_first[k * row + c0], t1 = hp.tiny_first[k * row + c1];
         if (s1 == s0 && t1 == t0) continue;
-        const bool timing =
-            (hp.opts.flags & CFA_OPT_TIMING) && p->last_launches < p->t_k0.size();
+        const bool timing = timing_on && p->last_launches < p->t_k0.size();
         if (timing) CK(p, cudaEventRecord(p->t_k0[p->last_launches], s));
         CK(p, cfa_launch_unpack(k, p->d_slabs + s0, s1 - s0, p->d_tiny + t0, t1 - t0, src_base,
-                                lo, hi, p->d_ck, p->d_status, p->grid_cap[k], s));
+                                period, lo, hi, p->d_ck, p->d_status, p->grid_cap[k], s));
         if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], s));
         p->last_launches++;
     }
@@ -297,6 +318,7 @@ void release(cfa_plan *p)
         if (p->aux_stream) cudaStreamDestroy(p->aux_stream);
         if (p->d_slabs) cudaFree(p->d_slabs);
         if (p->d_tiny) cudaFree(p->d_tiny);
+        if (p->d_bulk) cudaFree(p->d_bulk);
         if (p->d_ck) cudaFree(p->d_ck);
         if (p->d_status) cudaFree(p->d_status);
         if (p->own_slots && p->d_slots) cudaFree(p->d_slots);
@@ -329,6 +351,16 @@ cfa_status setup_device(cfa_plan *p)
         }
         p->grid_cap[k] = sms * per_sm;
     }
+    if (hp.n_bulk) {
+        for (int k = 0; k < 4; ++k) {
+            const int per_sm = cfa_bulk_blocks_per_sm(k);
+            if (per_sm <= 0) {
+                set_err(nullptr, "bulk kernel %d cannot run on device %d", k, p->device);
+                return CFA_ERR_CUDA;
+            }
+            p->bulk_grid_cap[k] = sms * per_sm;
+        }
+    }
 
     auto upload = [&](cfa_work **d, const cfa_work *h, size_t n) -> cfa_status {
         const size_t bytes = (n ? n : 1) * sizeof(cfa_work);
@@ -342,6 +374,8 @@ cfa_status setup_device(cfa_plan *p)
     cfa_status st = upload(&p->d_slabs, hp.slabs, hp.n_slabs);
     if (st) return st;
     st = upload(&p->d_tiny, hp.tiny, hp.n_tiny);
+    if (st) return st;
+    st = upload(&p->d_bulk, hp.bulk, hp.n_bulk);
     if (st) return st;
     const size_t ck_bytes = (hp.n_entries ? hp.n_entries : 1) * sizeof(unsigned long long);
     if (cudaMalloc(&p->d_ck, ck_bytes) != cudaSuccess ||
@@ -391,8 +425,9 @@ cfa_status setup_device(cfa_plan *p)
     if (timing) {
         if ((st = events(p->t_h2d0, hp.n_chunks, true))) return st;
         if ((st = events(p->t_h2d1, hp.n_chunks, true))) return st;
-        if ((st = events(p->t_k0, 2 * ((size_t)hp.n_chunks + 1), true))) return st;
-        if ((st = events(p->t_k1, 2 * ((size_t)hp.n_chunks + 1), true))) return st;
+        const size_t nk = 2 * CFA_N_CLASSES * ((size_t)hp.n_chunks + 1);
+        if ((st = events(p->t_k0, nk, true))) return st;
+        if ((st = events(p->t_k1, nk, true))) return st;
     }
     if (o.fill_threads > 1) p->pool.reset(new Pool(o.fill_threads - 1));
     else p->pool.reset(new Pool(0));
@@ -570,22 +605,13 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
     for (uint32_t l : p->layers_empty) CK(p, cudaEventRecord(p->ev_layer[l], cs));
 
     if (kind == CFA_SRC_DEVICE) {
+        /* the blob already sits in device memory: no staging; one launch over all chunks (per
+         * work class), or one per chunk with CFA_OPT_NO_MERGE for finer readiness events */
         const uint64_t base = (uint64_t)(uintptr_t)src->base;
-        const bool merge = !(hp.opts.flags & CFA_OPT_NO_MERGE);
-        const uint32_t per_run =
-            merge ? (src->period_bytes ? (uint32_t)(src->period_bytes / S) : hp.n_chunks) : 1u;
+        const uint32_t per_run = (hp.opts.flags & CFA_OPT_NO_MERGE) ? 1u : hp.n_chunks;
         for (uint32_t c0 = 0; c0 < hp.n_chunks;) {
-            const uint32_t c1 = std::min<uint32_t>(hp.n_chunks, c0 + std::max(per_run, 1u));
-            /* blob byte o of this run sits at base + (o mod period), i.e. base - c0*S + o when
-             * the run starts on a period boundary */
-            uint64_t run_base;
-            if (src->period_bytes) {
-                const uint64_t o0 = (uint64_t)c0 * S;
-                run_base = base + o0 % src->period_bytes - o0;
-            } else {
-                run_base = base;
-            }
-            cfa_status st = launch(p, c0, c1, run_base, cs);
+            const uint32_t c1 = std::min<uint32_t>(hp.n_chunks, c0 + per_run);
+            cfa_status st = launch(p, c0, c1, base, src->period_bytes, cs);
             if (st) return st;
             if ((st = record_layers(p, c0, c1, cs))) return st;
             c0 = c1;
@@ -617,7 +643,7 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             if (staged) CK(p, cudaEventRecord(p->ev_host_free[hs], p->copy_stream));
             CK(p, cudaEventRecord(p->ev_h2d[ds], p->copy_stream));
             CK(p, cudaStreamWaitEvent(cs, p->ev_h2d[ds], 0));
-            cfa_status st = launch(p, c, c + 1, (uint64_t)(uintptr_t)dslot - off, cs);
+            cfa_status st = launch(p, c, c + 1, (uint64_t)(uintptr_t)dslot - off, 0, cs);
             if (st) return st;
             CK(p, cudaEventRecord(p->ev_dev_free[ds], cs));
             if ((st = record_layers(p, c, c + 1, cs))) return st;
@@ -766,7 +792,8 @@ cfa_status cfa_unpack_chunks_async(cfa_plan *p, uint32_t chunk_begin, uint32_t c
         (uint64_t)(uintptr_t)chunk_src - (uint64_t)chunk_begin * p->hp.chunk_bytes;
     const uint64_t saved = p->last_launches;
     p->last_launches = p->t_k0.size(); /* no timing events for direct launches */
-    cfa_status st = launch(p, chunk_begin, chunk_end, base, reinterpret_cast<cudaStream_t>(stream));
+    cfa_status st =
+        launch(p, chunk_begin, chunk_end, base, 0, reinterpret_cast<cudaStream_t>(stream));
     p->last_launches = saved;
     return st;
 }

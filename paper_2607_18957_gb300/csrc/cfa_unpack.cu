@@ -37,8 +37,9 @@ struct UnpackArgs {
     const cfa_work *tiny;
     uint32_t n_slabs;
     uint32_t n_tiny;
-    uint64_t src_base; /* device address of blob byte 0 for this launch */
-    uint64_t src_lo;   /* blob bytes [src_lo, src_hi) are readable in this launch */
+    uint64_t src_base;   /* device address of blob byte 0 for this launch */
+    uint64_t src_period; /* 0, or P: blob byte o sits at src_base + (o mod P) */
+    uint64_t src_lo;     /* blob bytes [src_lo, src_hi) are readable in this launch */
     uint64_t src_hi;
     unsigned long long *ck;
     int *status;
@@ -291,7 +292,8 @@ template <int CLS, int U>
 __device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs &a, uint32_t tid,
                                              uint32_t nthr)
 {
-    const uint8_t *src = reinterpret_cast<const uint8_t *>(a.src_base + w.src);
+    const uint64_t off = a.src_period ? w.src % a.src_period : w.src;
+    const uint8_t *src = reinterpret_cast<const uint8_t *>(a.src_base + off);
     uint8_t *dst = reinterpret_cast<uint8_t *>(w.dst);
     if constexpr (CLS == CFA_CLASS_CAST)
         return cast_run<(U > 2 ? 2 : U)>(src, dst, w.n, tid, nthr);
@@ -384,10 +386,13 @@ extern "C" int cfa_unpack_blocks_per_sm(int cls)
     return n;
 }
 
-/* Launches the class-cls unpack over the given work items; grid_cap bounds the persistent grid. */
+/* Launches the class-cls unpack over the given work items; grid_cap bounds the persistent grid.
+ * Blob byte o is read at src_base + o, or at src_base + (o mod src_period) for a periodic
+ * source (a work item never straddles a period: periods are whole chunks). */
 extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_t n_slabs,
                                          const cfa_work *tiny, uint32_t n_tiny,
-                                         uint64_t src_base, uint64_t src_lo, uint64_t src_hi,
+                                         uint64_t src_base, uint64_t src_period,
+                                         uint64_t src_lo, uint64_t src_hi,
                                          unsigned long long *ck, int *status, int grid_cap,
                                          cudaStream_t stream)
 {
@@ -400,6 +405,7 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
     a.n_slabs = n_slabs;
     a.n_tiny = n_tiny;
     a.src_base = src_base;
+    a.src_period = src_period;
     a.src_lo = src_lo;
     a.src_hi = src_hi;
     a.ck = ck;

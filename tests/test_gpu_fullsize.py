@@ -167,11 +167,11 @@ def test_full_llama3_70b_bf16_streamed():
     assert np.all(np.diff(times) >= -1e-3), times
     assert times[-1] <= st["load_ms"] + 1e-3
     verify_all(m, d, ck)
-    # and from a device-resident pool, one launch per period
+    # and from a device-resident pool: one merged launch per kernel over all 132 chunks
     dpool = pool.to("cuda")
     d.buf.fill_(0xA5)
     ck2, st2, _ = _load(m, d, cfa.Source.device(dpool.data_ptr(), period=m.period),
                         dev_slots=0, host_slots=0)
-    assert st2["kernel_launches"] == -(-st2["n_chunks"] // (m.period // m.chunk_bytes))
+    assert st2["kernel_launches"] <= 2
     assert np.array_equal(ck, ck2)
     assert d.guards_intact()

@@ -133,6 +133,26 @@ def test_parity_work_splits(slab, tiny):
         load_and_compare(m, "device", chunk=1 << 20, slab_bytes=slab, tiny_bytes=tiny)
 
 
+@pytest.mark.parametrize("cfg", list(CONFIGS))
+@pytest.mark.parametrize("kind", ["device", "pinned", "callback"])
+@pytest.mark.parametrize("chunk", [4096 + 256, 1 << 20])
+def test_parity_bulk_path(cfg, kind, chunk):
+    """With CFA_OPT_BULK the aligned cast-free slabs go through the TMA bulk kernel."""
+    m = CONFIGS[cfg]()
+    st = load_and_compare(m, kind, chunk=chunk, bulk=True)
+    if cfg == "dense_f32":
+        assert st["n_bulk"] == 0  # casts never take the bulk path
+
+
+def test_bulk_path_takes_every_aligned_slab():
+    m = dense_config("dense_aligned", 67, layers=2, hidden=512, n_q=8, n_kv=2, head_dim=64,
+                     inter=1536, vocab=1000, align=256)
+    st = load_and_compare(m, "device", chunk=1 << 20, bulk=True)
+    assert st["n_bulk"] > 0 and st["n_slabs"] == 0
+    st = load_and_compare(m, "device", chunk=1 << 20)
+    assert st["n_bulk"] == 0 and st["n_slabs"] > 0
+
+
 def test_parity_aligned_full_tiny_workload():
     """The 1,000-tensor 256-byte-aligned workload at full size (about 125 MiB)."""
     m = tiny_config(seed=1)
