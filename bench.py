@@ -170,7 +170,8 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
     out = {"h2d_pinned_gbs": round(h2d_gbs, 2)}
     gib = 1 << 30
     threads = max(1, len(os.sched_getaffinity(0)))
-    pageable = np.empty(m.source_bytes(), dtype=np.uint8)
+    raw = np.empty(m.source_bytes() + 256, dtype=np.uint8)
+    pageable = raw[(-raw.ctypes.data) % 256:][:m.source_bytes()]  # 256-byte aligned view
     pageable[:] = host.numpy()                                   # the same bytes, pageable
     dtmp = torch.empty(gib, dtype=torch.uint8, device="cuda")
     src_t = torch.from_numpy(pageable[:gib])
@@ -199,7 +200,21 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
     plan.close()
     out["e2e_pageable_s_per_model"] = round(ms / 1e3, 4)
     out["e2e_pageable_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
-    del pageable
+    # the same pageable bytes read in place by the unpack kernel over NVLink-C2C (no staging)
+    plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                    dev_slots=0, host_slots=0, bulk=args.bulk)
+    src = cfa.Source.host_direct(pageable.ctypes.data, period=m.period or 0)
+    try:
+        plan.load_async(src, stream)
+        plan.checksums()
+        ms = min(_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
+                 for _ in range(2))
+        out["e2e_direct_pageable_s_per_model"] = round(ms / 1e3, 4)
+        out["e2e_direct_pageable_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
+    except cfa.CfaError as e:
+        out["e2e_direct_pageable"] = f"unavailable: {e}"
+    plan.close()
+    del pageable, raw
     plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
                     dev_slots=2, host_slots=0, timing=True, bulk=args.bulk)
     plan.load_async(cfa.Source.pinned(host.data_ptr(), period=m.period or 0), stream)

@@ -167,6 +167,12 @@ void cfa_plan_opts_default(cfa_plan_opts *opts);
 #define CFA_SRC_PINNED   2 /* page-locked host memory; copied straight to the device slots */
 #define CFA_SRC_CALLBACK 3 /* fill(user, blob_offset, dst, len) writes the bytes into a pinned slot */
 #define CFA_SRC_DEVICE   4 /* device memory already holding the blob; no staging, no copies */
+#define CFA_SRC_HOST_DIRECT 5 /* host memory that the unpack kernel reads in place over the host
+                                 link, one launch per chunk: no staging slots, no copy engine.
+                                 Page-locked memory always qualifies; pageable memory needs a
+                                 device that can access it (cudaDevAttrPageableMemoryAccess:
+                                 Grace-Blackwell and Grace-Hopper over NVLink-C2C), otherwise
+                                 the load is refused with CFA_ERR_INVAL before any GPU work */
 
 /* Writes blob bytes [blob_offset, blob_offset + len) to host memory dst and returns 0, or
  * returns non-zero on failure.  It runs on a CUDA host-function thread and must not call CUDA. */
@@ -176,7 +182,7 @@ typedef int (*cfa_fill_fn)(void *user, uint64_t blob_offset, void *dst, uint64_t
  * Where the blob's bytes come from.  With period_bytes == 0, blob byte o is base[o].  With
  * period_bytes > 0 (a multiple of chunk_bytes), the blob is periodic and byte o is
  * base[o % period_bytes]; this streams a blob larger than memory from a smaller pool.  base must
- * be 256-byte aligned for PINNED and DEVICE sources.  The source must stay valid until the load
+ * be 256-byte aligned for PINNED, DEVICE and HOST_DIRECT sources.  The source must stay valid until the load
  * has completed (cfa_wait_layer(CFA_ALL) returned CFA_OK).
  */
 typedef struct cfa_source {

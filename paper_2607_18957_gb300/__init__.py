@@ -144,6 +144,12 @@ class Source:
         return cls(_lib.SRC_DEVICE, ptr, period)
 
     @classmethod
+    def host_direct(cls, ptr, period=0):
+        """Host memory (pageable or page-locked) that the unpack kernel reads in place over the
+        host link; pageable memory needs a device with pageable memory access."""
+        return cls(_lib.SRC_HOST_DIRECT, ptr, period)
+
+    @classmethod
     def callback(cls, fill_fn_ptr, user_ptr=0):
         """A C function int fill(void *user, uint64 off, void *dst, uint64 len), as an address
         (for example from ctypes.cast(ctypes_function, c_void_p).value)."""

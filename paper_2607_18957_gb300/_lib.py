@@ -16,7 +16,7 @@ STATUS = {0: "CFA_OK", -1: "CFA_ERR_INVAL", -2: "CFA_ERR_OVERLAP", -3: "CFA_ERR_
 DTYPE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7}
 ENTRY_CAST_BF16, ENTRY_CKSUM = 0x1, 0x2
 OPT_STRICT_COVERAGE, OPT_HOST_ONLY, OPT_TIMING, OPT_BULK, OPT_NO_MERGE = 0x1, 0x2, 0x4, 0x8, 0x10
-SRC_HOST, SRC_PINNED, SRC_CALLBACK, SRC_DEVICE = 1, 2, 3, 4
+SRC_HOST, SRC_PINNED, SRC_CALLBACK, SRC_DEVICE, SRC_HOST_DIRECT = 1, 2, 3, 4, 5
 ALL = -1
 
 # cfa_tensor_entry and cfa_dst as numpy records (fast for 10^5 entries)

@@ -164,6 +164,7 @@ struct cfa_plan {
     cfa_host_plan hp{};
     bool host_only = false;
     int device = 0;
+    int pageable_access = 0; /* the device can read pageable host memory in place */
     int grid_cap[CFA_N_CLASSES] = {0};
     int bulk_grid_cap[4] = {0};
     cfa_work *d_slabs = nullptr, *d_tiny = nullptr, *d_bulk = nullptr;
@@ -342,6 +343,8 @@ cfa_status setup_device(cfa_plan *p)
     }
     int sms = 0;
     CK(nullptr, cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device));
+    CK(nullptr, cudaDeviceGetAttribute(&p->pageable_access, cudaDevAttrPageableMemoryAccess,
+                                       p->device));
     for (int k = 0; k < CFA_N_CLASSES; ++k) {
         const int per_sm = cfa_unpack_blocks_per_sm(k);
         if (sms <= 0 || per_sm <= 0) {
@@ -535,7 +538,7 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
     const cfa_host_plan &hp = p->hp;
     const uint64_t S = hp.chunk_bytes;
     const int kind = src->kind;
-    if (kind < CFA_SRC_HOST || kind > CFA_SRC_DEVICE || src->reserved) {
+    if (kind < CFA_SRC_HOST || kind > CFA_SRC_HOST_DIRECT || src->reserved) {
         set_err(p, "unknown source kind %d", kind);
         return CFA_ERR_INVAL;
     }
@@ -547,12 +550,30 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
         set_err(p, "source has no base pointer or fill function");
         return CFA_ERR_INVAL;
     }
-    if ((kind == CFA_SRC_PINNED || kind == CFA_SRC_DEVICE) && ((uintptr_t)src->base & 255u)) {
-        set_err(p, "pinned and device sources must be 256-byte aligned");
+    if ((kind == CFA_SRC_PINNED || kind == CFA_SRC_DEVICE || kind == CFA_SRC_HOST_DIRECT) &&
+        ((uintptr_t)src->base & 255u)) {
+        set_err(p, "pinned, device and direct host sources must be 256-byte aligned");
         return CFA_ERR_ALIGN;
     }
     const bool staged = kind == CFA_SRC_HOST || kind == CFA_SRC_CALLBACK;
-    if (kind != CFA_SRC_DEVICE && hp.n_chunks && (p->n_dev_slots == 0 || !p->d_slots)) {
+    const bool in_place = kind == CFA_SRC_DEVICE || kind == CFA_SRC_HOST_DIRECT;
+    if (kind == CFA_SRC_HOST_DIRECT && hp.blob_bytes) {
+        /* page-locked memory is mapped for the device; pageable memory is readable in place
+         * only where the device shares the host's page tables */
+        cudaPointerAttributes at;
+        std::memset(&at, 0, sizeof at);
+        if (cudaPointerGetAttributes(&at, src->base) != cudaSuccess) {
+            cudaGetLastError();
+            at.type = cudaMemoryTypeUnregistered;
+        }
+        const bool mapped = at.type == cudaMemoryTypeHost || at.type == cudaMemoryTypeManaged;
+        if (!mapped && !p->pageable_access) {
+            set_err(p, "this device cannot read pageable host memory in place; use a HOST "
+                       "source or page-locked memory");
+            return CFA_ERR_INVAL;
+        }
+    }
+    if (!in_place && hp.n_chunks && (p->n_dev_slots == 0 || !p->d_slots)) {
         set_err(p, "plan has no device staging slots (dev_slots = 0)");
         return CFA_ERR_INVAL;
     }
@@ -604,11 +625,14 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
     CK(p, cudaMemsetAsync(p->d_status, 0, sizeof(int), cs));
     for (uint32_t l : p->layers_empty) CK(p, cudaEventRecord(p->ev_layer[l], cs));
 
-    if (kind == CFA_SRC_DEVICE) {
-        /* the blob already sits in device memory: no staging; one launch over all chunks (per
-         * work class), or one per chunk with CFA_OPT_NO_MERGE for finer readiness events */
+    if (in_place) {
+        /* the kernel reads the blob where it is: device memory (one launch over all chunks per
+         * work class, or one per chunk with CFA_OPT_NO_MERGE) or host memory over the host link
+         * (one launch per chunk, so readiness events follow the stream of chunks) */
         const uint64_t base = (uint64_t)(uintptr_t)src->base;
-        const uint32_t per_run = (hp.opts.flags & CFA_OPT_NO_MERGE) ? 1u : hp.n_chunks;
+        const uint32_t per_run =
+            (kind == CFA_SRC_HOST_DIRECT || (hp.opts.flags & CFA_OPT_NO_MERGE)) ? 1u
+                                                                                 : hp.n_chunks;
         for (uint32_t c0 = 0; c0 < hp.n_chunks;) {
             const uint32_t c1 = std::min<uint32_t>(hp.n_chunks, c0 + per_run);
             cfa_status st = launch(p, c0, c1, base, src->period_bytes, cs);

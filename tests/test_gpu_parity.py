@@ -54,7 +54,24 @@ def make_source(kind, m, blob, keep):
         cb = CallbackSource(m)
         keep.append(cb)
         return cb.source()
+    if kind == "direct_pageable":
+        h = aligned_host_copy(blob)
+        keep.append(h)
+        return cfa.Source.host_direct(h.ctypes.data)
+    if kind == "direct_pinned":
+        h = torch.from_numpy(blob).pin_memory()
+        keep.append(h)
+        return cfa.Source.host_direct(h.data_ptr())
     raise ValueError(kind)
+
+
+def aligned_host_copy(blob, align=256):
+    """A pageable copy of `blob` starting on an `align`-byte boundary."""
+    buf = np.empty(blob.size + align, dtype=np.uint8)
+    off = (-buf.ctypes.data) % align
+    h = buf[off:off + blob.size]
+    h[:] = blob
+    return h
 
 
 def load_and_compare(m, kind, chunk, misalign=0, **kw):
@@ -102,7 +119,8 @@ CONFIGS = {"tiny": cfg_tiny, "dense": cfg_dense, "dense_f32": cfg_dense_f32, "mo
 
 
 @pytest.mark.parametrize("cfg", list(CONFIGS))
-@pytest.mark.parametrize("kind", ["device", "pinned", "host", "callback"])
+@pytest.mark.parametrize("kind", ["device", "pinned", "host", "callback", "direct_pageable",
+                                  "direct_pinned"])
 def test_parity_sources(cfg, kind):
     m = CONFIGS[cfg]()
     load_and_compare(m, kind, chunk=1 << 20)
@@ -293,8 +311,11 @@ def test_periodic_source():
     blob, ref = reference(m)
     pool_h = torch.from_numpy(m.blob_range(0, m.period)).pin_memory()
     pool_d = pool_h.to("cuda")
+    pool_pg = aligned_host_copy(m.blob_range(0, m.period))
     for src in (cfa.Source.pinned(pool_h.data_ptr(), period=m.period),
-                cfa.Source.device(pool_d.data_ptr(), period=m.period)):
+                cfa.Source.device(pool_d.data_ptr(), period=m.period),
+                cfa.Source.host_direct(pool_pg.ctypes.data, period=m.period),
+                cfa.Source.host(pool_pg.ctypes.data, period=m.period)):
         d = DeviceDsts(m)
         with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=1 << 20) as plan:
             plan.load_async(src)
