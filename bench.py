@@ -61,12 +61,13 @@ def parse_args():
 # ------------------------------------------------------------------------------------------
 def make_workload(name):
     import workloads
-    if name in workloads.NAMED_CONFIGS:
-        return workloads.named_config(name)
     if name == "llama3_8b_bf16_2layer_v32k":  # small case for ncu captures (~1.4 GB blob)
         return workloads.dense_config(name, 2, layers=2, hidden=4096, n_q=32, n_kv=8,
                                       head_dim=128, inter=14336, vocab=32000)
-    raise SystemExit(f"unknown workload {name}")
+    try:
+        return workloads.named_config(name)
+    except KeyError:
+        raise SystemExit(f"unknown workload {name}")
 
 
 def measured_peaks():
@@ -258,7 +259,7 @@ def cpu_baseline(m, seconds, steps=None):
         k += 1
         es = m.entries_of_dst(j)
         lo = min(int(m.e_offset[i]) for i in es)
-        hi = max(int(m.e_offset[i]) + m.e_nbytes(i) for i in es)
+        hi = max(int(m.e_offset[i]) + m.e_extent(i) for i in es)
         window = m.blob_range(lo, hi - lo)
         t0 = time.perf_counter()
         r = oracle.unpack(m, window, blob_begin=lo, dsts=[j])

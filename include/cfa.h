@@ -88,8 +88,8 @@ typedef int cfa_status;
  *
  *   name            optional, copied by cfa_plan_create; used only in error messages.
  *   src_dtype       CFA_DTYPE_* of the elements in the blob.
- *   ndim, shape     logical shape, row-major and contiguous in the blob; ndim 0 is a scalar.
- *                   Zero-element tensors are valid and load nothing.
+ *   ndim, shape     logical shape, row-major; ndim 0 is a scalar.  Zero-element tensors are
+ *                   valid and load nothing.
  *   blob_offset     byte offset of element 0 in the blob; a multiple of the source element size.
  *   dst_index       index into the cfa_dst array.
  *   layer           readiness group, 0 <= layer < CFA_MAX_LAYERS (cfa_wait_layer).
@@ -102,6 +102,13 @@ typedef int cfa_status;
  *                   expert e's w1, w3 at rows 2Ie, 2Ie + I of the [E*2I, H] view of w13.
  *   flags           CFA_ENTRY_*.  Without CFA_ENTRY_CAST_BF16 the destination dtype must
  *                   equal src_dtype; with it, src_dtype must be F32 and the destination BF16.
+ *   src_row_stride  0 when the tensor's elements are contiguous in the blob.  Otherwise the
+ *                   tensor is read as numel / shape[-1] rows of shape[-1] elements whose first
+ *                   elements lie src_row_stride source elements apart (>= shape[-1]): a column
+ *                   slice of a larger row-major checkpoint tensor.  This is how a
+ *                   tensor-parallel rank reads its shard of a row-parallel weight (columns
+ *                   [r K / R, (r + 1) K / R) of o_proj, down_proj, w2); column-parallel shards
+ *                   (row ranges) are contiguous and need no stride.
  */
 typedef struct cfa_tensor_entry {
     const char *name;
@@ -113,7 +120,7 @@ typedef struct cfa_tensor_entry {
     int32_t layer;
     int64_t dst_row_offset;
     uint32_t flags;
-    uint32_t reserved; /* must be 0 */
+    uint32_t src_row_stride;
 } cfa_tensor_entry;
 
 /*
@@ -203,6 +210,7 @@ typedef struct cfa_stats {
     uint64_t n_slabs;         /* block-level work items (vector path) */
     uint64_t n_bulk;          /* block-level work items (TMA bulk path) */
     uint64_t n_tiny;          /* warp-level work items */
+    uint64_t n_strided;       /* block-level work items over rows of column slices */
     uint64_t bytes_read;      /* algorithmic bytes one load reads from staging */
     uint64_t bytes_written;   /* algorithmic bytes one load writes into destinations */
     uint64_t descriptor_bytes;
@@ -215,7 +223,10 @@ typedef struct cfa_stats {
     double unpack_ms;         /* sum over launches of the unpack kernel time */
 } cfa_stats;
 
-/* A piece (tensor x chunk) as the plan builder cut it; for inspection and tests. */
+/* A piece (tensor x chunk) as the plan builder cut it; for inspection and tests.  A piece is
+ * `rows` runs of n_elems / rows elements each; run k starts at source byte
+ * src_offset + k * src_row_stride * (source element size) and fills the destination
+ * contiguously from dst_offset on.  Contiguous pieces have rows = 1. */
 typedef struct cfa_piece {
     uint32_t chunk;
     uint32_t entry;
@@ -224,6 +235,8 @@ typedef struct cfa_piece {
     uint32_t cast;
     uint64_t dst_offset;      /* byte offset inside the destination */
     uint64_t n_elems;
+    uint32_t rows;
+    uint32_t src_row_stride;  /* source elements between run starts (rows > 1) */
 } cfa_piece;
 
 /*

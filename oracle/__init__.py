@@ -57,7 +57,7 @@ def _bind(path):
     lib.oracle_rne_bf16.restype = ctypes.c_uint16
     lib.oracle_rne_bf16_array.argtypes = [P, P, U64]
     lib.oracle_rne_bf16_array.restype = None
-    lib.oracle_unpack.argtypes = [U64, P, P, P, P, P, P, P, U64, P, P, P, P, P, P, U64,
+    lib.oracle_unpack.argtypes = [U64, P, P, P, P, P, P, P, P, U64, P, P, P, P, P, P, U64,
                                   U64, U64, P, P]
     lib.oracle_unpack.restype = ctypes.c_int
     lib.oracle_check_cover.argtypes = [U64, P, P, P]
@@ -119,7 +119,9 @@ def _columns(m):
              np.ascontiguousarray(m.e_dst, dtype=np.int32),
              np.ascontiguousarray(m.e_row, dtype=np.int64),
              np.ascontiguousarray(m.d_ndim, dtype=np.int32),
-             np.ascontiguousarray(m.d_shape, dtype=np.int64))
+             np.ascontiguousarray(m.d_shape, dtype=np.int64),
+             np.ascontiguousarray(getattr(m, "e_stride", np.zeros(m.n_entries)),
+                                  dtype=np.uint32))
         try:
             m._oracle_columns = c
         except AttributeError:
@@ -142,7 +144,7 @@ def unpack(m, blob, blob_begin=0, dsts=None, cover=False, fill=0, lib=None):
     n, nd = m.n_entries, m.n_dsts
     sel = range(nd) if dsts is None else sorted(set(int(j) for j in dsts))
     (e_dtype, d_dtype, e_flags, e_ndim, e_shape, e_off, e_dst, e_row, d_ndim,
-     d_shape) = _columns(m)
+     d_shape, e_stride) = _columns(m)
     bufs = [None] * nd
     covs = [None] * nd
     for j in sel:
@@ -156,7 +158,7 @@ def unpack(m, blob, blob_begin=0, dsts=None, cover=False, fill=0, lib=None):
     bad = ctypes.c_int64(-1)
     st = lib.oracle_unpack(
         n, e_dtype.ctypes.data, e_ndim.ctypes.data, e_shape.ctypes.data, e_off.ctypes.data,
-        e_dst.ctypes.data, e_row.ctypes.data, e_flags.ctypes.data,
+        e_dst.ctypes.data, e_row.ctypes.data, e_flags.ctypes.data, e_stride.ctypes.data,
         nd, d_dtype.ctypes.data, d_ndim.ctypes.data, d_shape.ctypes.data,
         _ptr_array(bufs), _ptr_array(covs) if cover else None,
         blob.ctypes.data if blob.size else None, blob_begin, blob_begin + blob.size,

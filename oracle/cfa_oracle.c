@@ -19,8 +19,10 @@
  *     row    = D's last dimension R when D has >= 2 dimensions (t.shape[-1] must equal R),
  *              one element when D has <= 1 dimension
  *     base   = t.row_offset * (elements per row) * es_d     (bytes into D)
+ *     C      = t.shape[-1];  stride = t.src_row_stride, or C when it is 0 (contiguous)
  *     for i in 0 .. n-1:
- *         x = little-endian es_s-byte integer at blob[t.blob_offset + i * es_s]
+ *         src_i = (i / C) * stride + (i mod C)     (element i of row i / C of a column slice)
+ *         x = little-endian es_s-byte integer at blob[t.blob_offset + src_i * es_s]
  *         y = cast ? rne_bf16(x) : x
  *         write y as es_d little-endian bytes at D[base + i * es_d]
  *         cover[D][each written byte] += 1
@@ -97,7 +99,8 @@ static void write_le(uint8_t *p, uint64_t y, int nbytes)
 /*
  * Unpacks every entry whose destination buffer is given.
  *
- *   e_*            entry columns (n_entries); e_shape is n_entries x 8, row-major.
+ *   e_*            entry columns (n_entries); e_shape is n_entries x 8, row-major;
+ *                  e_stride may be NULL (every entry contiguous).
  *   d_*            destination columns (n_dsts); d_shape is n_dsts x 8.
  *   d_buf[j]       host buffer of destination j (its full byte size), or NULL: entries into a
  *                  NULL destination are still validated but not executed.
@@ -111,7 +114,7 @@ static void write_le(uint8_t *p, uint64_t y, int nbytes)
  */
 int oracle_unpack(uint64_t n_entries, const int32_t *e_dtype, const int32_t *e_ndim,
                   const int64_t *e_shape, const uint64_t *e_offset, const int32_t *e_dst,
-                  const int64_t *e_row, const uint32_t *e_flags,
+                  const int64_t *e_row, const uint32_t *e_flags, const uint32_t *e_stride,
                   uint64_t n_dsts, const int32_t *d_dtype, const int32_t *d_ndim,
                   const int64_t *d_shape, uint8_t *const *d_buf, uint32_t *const *d_cover,
                   const uint8_t *blob, uint64_t blob_begin, uint64_t blob_end,
@@ -166,19 +169,28 @@ int oracle_unpack(uint64_t n_entries, const int32_t *e_dtype, const int32_t *e_n
         if (base_elem + n > d_numel) { *bad_entry = (int64_t)t; return ORC_E_OOB; }
         const uint64_t base = base_elem * (uint64_t)es_d;
 
+        /* source layout: rows of C elements, `stride` elements apart */
+        const uint64_t C = e_ndim[t] >= 1 ? (uint64_t)e_shape[8 * t + e_ndim[t] - 1] : 1;
+        const uint64_t given = e_stride ? (uint64_t)e_stride[t] : 0;
+        if (given != 0 && (e_ndim[t] < 1 || given < C)) { *bad_entry = (int64_t)t; return ORC_E_INVAL; }
+        const uint64_t stride = given ? given : C;
+        /* elements the entry spans in the blob, from its first to its last element */
+        const uint64_t extent = n == 0 ? 0 : (n / C - 1) * stride + C;
+
         /* source range */
         if (e_offset[t] % (uint64_t)es_s != 0) { *bad_entry = (int64_t)t; return ORC_E_ALIGN; }
-        if (e_offset[t] + n * (uint64_t)es_s > blob_bytes) { *bad_entry = (int64_t)t; return ORC_E_OOB; }
+        if (e_offset[t] + extent * (uint64_t)es_s > blob_bytes) { *bad_entry = (int64_t)t; return ORC_E_OOB; }
 
         if (d_buf[j] == NULL || n == 0) continue;
-        if (e_offset[t] < blob_begin || e_offset[t] + n * (uint64_t)es_s > blob_end) continue;
+        if (e_offset[t] < blob_begin || e_offset[t] + extent * (uint64_t)es_s > blob_end) continue;
 
         const uint8_t *src = blob + (e_offset[t] - blob_begin);
         uint8_t *dst = d_buf[j] + base;
         uint32_t *cover = d_cover ? d_cover[j] : NULL;
         uint64_t ck = 0;
         for (uint64_t i = 0; i < n; ++i) {
-            const uint64_t x = read_le(src + i * (uint64_t)es_s, es_s);
+            const uint64_t src_i = (i / C) * stride + (i % C);
+            const uint64_t x = read_le(src + src_i * (uint64_t)es_s, es_s);
             const uint64_t y = cast ? (uint64_t)oracle_rne_bf16((uint32_t)x) : x;
             write_le(dst + i * (uint64_t)es_d, y, es_d);
             if (cover)

@@ -51,7 +51,7 @@ def _stream_handle(stream):
 
 
 def make_entries(dtype, shape, offset, dst, row=None, cast=None, cksum=None, layer=None,
-                 names=None):
+                 names=None, src_row_stride=None):
     """Builds the cfa_tensor_entry array from columns.
 
     dtype   sequence of dtype names ("bf16", "f32", ...), or of CFA_DTYPE_* codes
@@ -60,6 +60,8 @@ def make_entries(dtype, shape, offset, dst, row=None, cast=None, cksum=None, lay
     offset  blob byte offsets;  dst  destination indices;  row  destination row offsets
     cast, cksum  booleans (default: no cast, checksum on);  layer  readiness groups (default 0)
     names   optional list of str (kept alive by the returned object)
+    src_row_stride  source elements between row starts for strided (column-slice) entries;
+            0 = contiguous (default)
     """
     n = len(dst)
     e = np.zeros(n, dtype=ENTRY_DTYPE)
@@ -87,6 +89,8 @@ def make_entries(dtype, shape, offset, dst, row=None, cast=None, cksum=None, lay
     e["flags"] = fl
     if layer is not None:
         e["layer"] = np.asarray(layer, dtype=np.int32)
+    if src_row_stride is not None:
+        e["src_row_stride"] = np.asarray(src_row_stride, dtype=np.uint32)
     keep = None
     if names is not None:
         blob = b"".join(s.encode() + b"\0" for s in names)

@@ -23,7 +23,7 @@ ALL = -1
 ENTRY_DTYPE = np.dtype([("name", "<u8"), ("src_dtype", "<i4"), ("ndim", "<i4"),
                         ("shape", "<i8", (8,)), ("blob_offset", "<u8"), ("dst_index", "<i4"),
                         ("layer", "<i4"), ("dst_row_offset", "<i8"), ("flags", "<u4"),
-                        ("reserved", "<u4")])
+                        ("src_row_stride", "<u4")])
 DST_DTYPE = np.dtype([("dev_ptr", "<u8"), ("dtype", "<i4"), ("ndim", "<i4"),
                       ("shape", "<i8", (8,))])
 
@@ -49,7 +49,7 @@ class Source(ctypes.Structure):
 class Stats(ctypes.Structure):
     _fields_ = [(n, ctypes.c_uint64) for n in (
         "blob_bytes", "n_entries", "n_dsts", "n_chunks", "n_layers", "n_pieces", "n_slabs",
-        "n_bulk", "n_tiny", "bytes_read", "bytes_written", "descriptor_bytes", "loads",
+        "n_bulk", "n_tiny", "n_strided", "bytes_read", "bytes_written", "descriptor_bytes", "loads",
         "kernel_launches")] + [(n, ctypes.c_double) for n in (
             "plan_ms", "load_ms", "h2d_ms", "unpack_ms")]
 
@@ -58,12 +58,13 @@ class Piece(ctypes.Structure):
     _fields_ = [("chunk", ctypes.c_uint32), ("entry", ctypes.c_uint32),
                 ("src_offset", ctypes.c_uint64), ("dst_index", ctypes.c_uint32),
                 ("cast", ctypes.c_uint32), ("dst_offset", ctypes.c_uint64),
-                ("n_elems", ctypes.c_uint64)]
+                ("n_elems", ctypes.c_uint64), ("rows", ctypes.c_uint32),
+                ("src_row_stride", ctypes.c_uint32)]
 
 
 PIECE_DTYPE = np.dtype([("chunk", "<u4"), ("entry", "<u4"), ("src_offset", "<u8"),
                         ("dst_index", "<u4"), ("cast", "<u4"), ("dst_offset", "<u8"),
-                        ("n_elems", "<u8")])
+                        ("n_elems", "<u8"), ("rows", "<u4"), ("src_row_stride", "<u4")])
 
 # Every function cfa.h declares, with its ctypes signature.
 _P, _U64, _I32, _SZ = ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int32, ctypes.c_size_t

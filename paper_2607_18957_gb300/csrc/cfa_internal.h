@@ -33,6 +33,22 @@ typedef struct cfa_work {
     uint32_t pad;
 } cfa_work;
 
+/*
+ * A block of rows of a strided piece (a column slice of a larger checkpoint tensor): row k
+ * starts at source blob offset src + k * stride * (source element size) and lands at
+ * dst + k * cols * (destination element size).  40 bytes.
+ */
+typedef struct cfa_swork {
+    uint64_t src;
+    uint64_t dst;
+    uint32_t rows;
+    uint32_t cols;   /* elements per row */
+    uint32_t stride; /* source elements between row starts */
+    uint32_t ck;
+    uint32_t mode;
+    uint32_t cls;    /* work class, used while the plan is built */
+} cfa_swork;
+
 #define CFA_NO_CK 0xFFFFFFFFu
 
 /* Work classes: one specialised kernel each.  0..3 = plain copy of 1, 2, 4, 8-byte elements;
@@ -68,6 +84,9 @@ typedef struct cfa_host_plan {
     cfa_work *tiny;  /* warp-level */
     size_t n_tiny;
     uint32_t *tiny_first;
+    cfa_swork *strided; /* block-level, rows of column slices */
+    size_t n_strided;
+    uint32_t *strided_first;
     int64_t *layer_last_chunk; /* n_layers; -1 = the group has no bytes */
     uint64_t bytes_read, bytes_written;
     int any_cksum;

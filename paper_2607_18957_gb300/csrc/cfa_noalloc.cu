@@ -98,9 +98,11 @@ cfa_status place(const cfa_tensor_entry &e, const cfa_dst *dsts, size_t n_dsts,
 {
     *es_s = dtype_size(e.src_dtype);
     if (!*es_s || e.ndim < 0 || e.ndim > CFA_MAX_DIMS || e.dst_index < 0 ||
-        (size_t)e.dst_index >= n_dsts || e.reserved ||
+        (size_t)e.dst_index >= n_dsts || e.src_row_stride ||
         (e.flags & ~(CFA_ENTRY_CAST_BF16 | CFA_ENTRY_CKSUM)))
-        return fail(CFA_ERR_INVAL, "bad dtype, ndim, flags or destination index", i);
+        return fail(CFA_ERR_INVAL,
+                    "bad dtype, ndim, flags or destination index, or a strided entry (strided "
+                    "entries need cfa_plan_create)", i);
     const cfa_dst &d = dsts[e.dst_index];
     const int es_dst = dtype_size(d.dtype);
     if (!es_dst || d.ndim < 0 || d.ndim > CFA_MAX_DIMS)

@@ -105,6 +105,9 @@ typedef struct {
     uint64_t n;       /* elements */
     int es_s, es_d;   /* element sizes */
     uint64_t dst_off; /* byte offset inside the destination */
+    uint64_t cols;    /* elements per row (the last dimension) */
+    uint64_t stride;  /* source elements between row starts; == cols when contiguous */
+    uint64_t extent;  /* source bytes from the first to the last element */
 } ent_info;
 
 typedef struct {
@@ -148,6 +151,66 @@ static int mul_overflows(uint64_t a, uint64_t b, uint64_t *out)
     return 0;
 }
 
+/* Class and source blob offset of an item of either descriptor kind. */
+static void item_key(const vec *v, size_t q, uint32_t *cls, uint64_t *src)
+{
+    if (v->elem == sizeof(cfa_swork)) {
+        const cfa_swork *w = (const cfa_swork *)v->p + q;
+        *cls = w->cls;
+        *src = w->src;
+    } else {
+        const cfa_work *w = (const cfa_work *)v->p + q;
+        *cls = w->pad;
+        *src = w->src;
+    }
+}
+
+/* Reorders the items of v (in chunk order) by (class, chunk), stably, and fills
+ * first[class * (n_chunks + 1) + chunk] with each group's start. */
+static cfa_status partition_by_class(vec *v, uint32_t *first, uint32_t n_chunks, uint64_t S,
+                                     char *err, size_t errlen)
+{
+    if (v->n >= UINT32_MAX) {
+        fail(err, errlen, "too many work items; raise slab_bytes");
+        return CFA_ERR_INVAL;
+    }
+    const size_t row = (size_t)n_chunks + 1, nf = (size_t)CFA_N_CLASSES * row;
+    for (size_t q = 0; q < v->n; ++q) {
+        uint32_t k;
+        uint64_t src;
+        item_key(v, q, &k, &src);
+        first[(size_t)k * row + (size_t)(src / S) + 1]++;
+    }
+    uint32_t run = 0;
+    for (size_t idx = 0; idx < nf; ++idx) {
+        if (idx % row == 0) {
+            first[idx] = run;
+        } else {
+            run += first[idx];
+            first[idx] = run;
+        }
+    }
+    char *sorted = (char *)malloc((v->n ? v->n : 1) * v->elem);
+    uint32_t *cursor = (uint32_t *)malloc(nf * sizeof(uint32_t));
+    if (!sorted || !cursor) {
+        free(sorted);
+        free(cursor);
+        return CFA_ERR_NOMEM;
+    }
+    memcpy(cursor, first, nf * sizeof(uint32_t));
+    for (size_t q = 0; q < v->n; ++q) {
+        uint32_t k;
+        uint64_t src;
+        item_key(v, q, &k, &src);
+        const uint32_t to = cursor[(size_t)k * row + (size_t)(src / S)]++;
+        memcpy(sorted + (size_t)to * v->elem, (const char *)v->p + q * v->elem, v->elem);
+    }
+    free(cursor);
+    free(v->p);
+    v->p = sorted;
+    return CFA_OK;
+}
+
 void cfa_host_plan_free(cfa_host_plan *hp)
 {
     if (!hp) return;
@@ -164,6 +227,8 @@ void cfa_host_plan_free(cfa_host_plan *hp)
     free(hp->bulk_first);
     free(hp->tiny);
     free(hp->tiny_first);
+    free(hp->strided);
+    free(hp->strided_first);
     free(hp->layer_last_chunk);
     memset(hp, 0, sizeof *hp);
 }
@@ -178,10 +243,11 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
     span *spans = NULL;
     dspan *ds = NULL;
     uint64_t *dst_bytes = NULL;
-    vec slabs = {0}, bulk = {0}, tiny = {0};
+    vec slabs = {0}, bulk = {0}, tiny = {0}, strided = {0};
     if (!out) return CFA_ERR_INVAL;
     memset(out, 0, sizeof *out);
     slabs.elem = bulk.elem = tiny.elem = sizeof(cfa_work);
+    strided.elem = sizeof(cfa_swork);
 
     /* 1. options */
     cfa_plan_opts o;
@@ -286,7 +352,7 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
     for (size_t i = 0; i < n_entries; ++i) {
         const cfa_tensor_entry *e = &entries[i];
         const int es_s = cfa_dtype_size(e->src_dtype);
-        if (!es_s || e->ndim < 0 || e->ndim > CFA_MAX_DIMS || e->reserved ||
+        if (!es_s || e->ndim < 0 || e->ndim > CFA_MAX_DIMS ||
             (e->flags & ~(CFA_ENTRY_CAST_BF16 | CFA_ENTRY_CKSUM))) {
             fail(err, errlen, "entry %zu (%s): bad dtype, ndim or flags", i, ename(e));
             st = CFA_ERR_INVAL;
@@ -346,18 +412,32 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
             st = CFA_ERR_ALIGN;
             goto done;
         }
-        src_len = n * (uint64_t)es_s; /* cannot overflow: n <= d_numel and es_s <= 8 ... */
-        dst_len = n * (uint64_t)es_d;
-        if (src_len / (uint64_t)es_s != n || e->blob_offset > blob_bytes ||
+        /* source layout: rows of `cols` elements, `stride` elements apart */
+        const uint64_t cols = e->ndim >= 1 ? (uint64_t)e->shape[e->ndim - 1] : 1;
+        if (e->src_row_stride && (e->ndim < 1 || e->src_row_stride < cols)) {
+            fail(err, errlen, "entry %zu (%s): source row stride below the row length", i,
+                 ename(e));
+            st = CFA_ERR_INVAL;
+            goto done;
+        }
+        const uint64_t stride = e->src_row_stride ? e->src_row_stride : cols;
+        uint64_t extent_elems = 0;
+        if (n && mul_overflows(n / cols - 1, stride, &extent_elems)) extent_elems = UINT64_MAX;
+        if (n) extent_elems = extent_elems > UINT64_MAX - cols ? UINT64_MAX : extent_elems + cols;
+        if (mul_overflows(extent_elems, (uint64_t)es_s, &src_len) || e->blob_offset > blob_bytes ||
             src_len > blob_bytes - e->blob_offset) {
             fail(err, errlen, "entry %zu (%s): reads past the end of the blob", i, ename(e));
             st = CFA_ERR_OOB;
             goto done;
         }
+        dst_len = n * (uint64_t)es_d;
         info[i].n = n;
         info[i].es_s = es_s;
         info[i].es_d = es_d;
         info[i].dst_off = first * (uint64_t)es_d;
+        info[i].cols = cols;
+        info[i].stride = stride;
+        info[i].extent = src_len;
         (void)dst_len;
     }
 
@@ -399,39 +479,76 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         }
     }
 
-    /* 3. pieces = tensor x chunk */
-    size_t n_pieces = 0;
-    for (size_t i = 0; i < n_entries; ++i) {
-        if (!info[i].n) continue;
-        const uint64_t a = entries[i].blob_offset;
-        const uint64_t b = a + info[i].n * (uint64_t)info[i].es_s;
-        n_pieces += (size_t)((b - 1) / S - a / S + 1);
-    }
-    out->pieces = (cfa_piece *)malloc((n_pieces ? n_pieces : 1) * sizeof(cfa_piece));
-    if (!out->pieces) { st = CFA_ERR_NOMEM; goto done; }
+    /* 3. pieces = tensor x chunk.  A contiguous tensor gives one piece per chunk it touches.
+     * A column slice gives one strided piece per run of whole rows inside a chunk, and its rows
+     * that cross a chunk boundary are cut into contiguous pieces at the boundary. */
     {
-        size_t p = 0;
+        vec pv = {0};
+        pv.elem = sizeof(cfa_piece);
         for (size_t i = 0; i < n_entries; ++i) {
-            if (!info[i].n) continue;
-            const uint64_t a = entries[i].blob_offset;
-            const uint64_t b = a + info[i].n * (uint64_t)info[i].es_s;
-            for (uint64_t c = a / S; c * S < b; ++c) {
-                const uint64_t lo = a > c * S ? a : c * S;
-                const uint64_t hi = b < (c + 1) * S ? b : (c + 1) * S;
-                cfa_piece *pc = &out->pieces[p++];
-                pc->chunk = (uint32_t)c;
-                pc->entry = (uint32_t)i;
-                pc->src_offset = lo;
-                pc->dst_index = (uint32_t)entries[i].dst_index;
-                pc->cast = (entries[i].flags & CFA_ENTRY_CAST_BF16) ? 1u : 0u;
-                pc->dst_offset = info[i].dst_off +
-                                 (lo - a) / (uint64_t)info[i].es_s * (uint64_t)info[i].es_d;
-                pc->n_elems = (hi - lo) / (uint64_t)info[i].es_s;
+            const ent_info *in = &info[i];
+            if (!in->n) continue;
+            cfa_piece pc;
+            memset(&pc, 0, sizeof pc);
+            pc.entry = (uint32_t)i;
+            pc.dst_index = (uint32_t)entries[i].dst_index;
+            pc.cast = (entries[i].flags & CFA_ENTRY_CAST_BF16) ? 1u : 0u;
+            pc.rows = 1;
+            const uint64_t es_s = (uint64_t)in->es_s, es_d = (uint64_t)in->es_d;
+            const uint64_t a0 = entries[i].blob_offset;
+            /* contiguous runs [lo, hi) of source bytes whose first element is element e0 */
+#define CFA_EMIT_RUN(LO, HI, E0)                                                             \
+    do {                                                                                     \
+        for (uint64_t c_ = (LO) / S; c_ * S < (HI); ++c_) {                                  \
+            const uint64_t lo_ = (LO) > c_ * S ? (LO) : c_ * S;                               \
+            const uint64_t hi_ = (HI) < (c_ + 1) * S ? (HI) : (c_ + 1) * S;                   \
+            pc.chunk = (uint32_t)c_;                                                         \
+            pc.rows = 1;                                                                     \
+            pc.src_row_stride = 0;                                                           \
+            pc.src_offset = lo_;                                                             \
+            pc.n_elems = (hi_ - lo_) / es_s;                                                 \
+            pc.dst_offset = in->dst_off + ((E0) + (lo_ - (LO)) / es_s) * es_d;              \
+            if (vec_push(&pv, &pc)) { free(pv.p); st = CFA_ERR_NOMEM; goto done; }           \
+        }                                                                                    \
+    } while (0)
+            if (in->stride == in->cols) {
+                CFA_EMIT_RUN(a0, a0 + in->n * es_s, 0);
+                continue;
             }
+            const uint64_t rows = in->n / in->cols;
+            const uint64_t row_bytes = in->cols * es_s, step = in->stride * es_s;
+            for (uint64_t r = 0; r < rows;) {
+                const uint64_t a = a0 + r * step;
+                const uint64_t c = a / S;
+                if (a + row_bytes <= (c + 1) * S) {
+                    /* rows r .. r+k-1 lie entirely inside chunk c */
+                    uint64_t k = 1 + ((c + 1) * S - (a + row_bytes)) / step;
+                    if (k > rows - r) k = rows - r;
+                    if (k > UINT32_MAX) k = UINT32_MAX;
+                    pc.chunk = (uint32_t)c;
+                    pc.src_offset = a;
+                    pc.rows = (uint32_t)k;
+                    pc.src_row_stride = k > 1 ? (uint32_t)in->stride : 0;
+                    pc.n_elems = k * in->cols;
+                    pc.dst_offset = in->dst_off + r * in->cols * es_d;
+                    if (vec_push(&pv, &pc)) { free(pv.p); st = CFA_ERR_NOMEM; goto done; }
+                    r += k;
+                } else {
+                    CFA_EMIT_RUN(a, a + row_bytes, r * in->cols);
+                    r += 1;
+                }
+            }
+#undef CFA_EMIT_RUN
+        }
+        out->pieces = (cfa_piece *)pv.p;
+        out->n_pieces = pv.n;
+        if (!out->pieces) {
+            out->pieces = (cfa_piece *)malloc(sizeof(cfa_piece));
+            if (!out->pieces) { st = CFA_ERR_NOMEM; goto done; }
         }
     }
+    const size_t n_pieces = out->n_pieces;
     qsort(out->pieces, n_pieces, sizeof(cfa_piece), cmp_piece);
-    out->n_pieces = n_pieces;
 
     /* 4. work items, ordered by (class, chunk) */
     const uint32_t n_chunks = (uint32_t)n_chunks64;
@@ -439,21 +556,49 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
     out->slab_first = (uint32_t *)calloc(nf, sizeof(uint32_t));
     out->bulk_first = (uint32_t *)calloc(nf, sizeof(uint32_t));
     out->tiny_first = (uint32_t *)calloc(nf, sizeof(uint32_t));
-    if (!out->slab_first || !out->bulk_first || !out->tiny_first) { st = CFA_ERR_NOMEM; goto done; }
+    out->strided_first = (uint32_t *)calloc(nf, sizeof(uint32_t));
+    if (!out->slab_first || !out->bulk_first || !out->tiny_first || !out->strided_first) {
+        st = CFA_ERR_NOMEM;
+        goto done;
+    }
     {
         const int use_bulk = CFA_BULK_READY && (o.flags & CFA_OPT_BULK);
         const uint64_t slab = o.slab_bytes;
-        /* pass 1: items in chunk order, tagged with their class in `pad` */
+        /* pass 1: items in chunk order, tagged with their class */
         for (size_t p = 0; p < n_pieces; ++p) {
             const cfa_piece *pc = &out->pieces[p];
             const ent_info *in = &info[pc->entry];
             const cfa_tensor_entry *e = &entries[pc->entry];
+            const uint32_t ck = (e->flags & CFA_ENTRY_CKSUM) ? pc->entry : CFA_NO_CK;
+            const uint32_t mode = CFA_MODE(log2_small(in->es_s), log2_small(in->es_d), pc->cast);
+            const uint32_t cls = pc->cast ? CFA_CLASS_CAST : (uint32_t)log2_small(in->es_s);
+            const uint64_t a0 = (uint64_t)(uintptr_t)dsts[pc->dst_index].dev_ptr + pc->dst_offset;
+            if (pc->rows > 1) {
+                /* blocks of whole rows, about slab_bytes of destination each */
+                const uint64_t row_d = in->cols * (uint64_t)in->es_d;
+                uint64_t per = row_d ? slab / row_d : 1;
+                if (per == 0) per = 1;
+                for (uint64_t r = 0; r < pc->rows; r += per) {
+                    const uint64_t k = pc->rows - r < per ? pc->rows - r : per;
+                    cfa_swork sw;
+                    memset(&sw, 0, sizeof sw);
+                    sw.src = pc->src_offset + r * in->stride * (uint64_t)in->es_s;
+                    sw.dst = a0 + r * row_d;
+                    sw.rows = (uint32_t)k;
+                    sw.cols = (uint32_t)in->cols;
+                    sw.stride = (uint32_t)in->stride;
+                    sw.ck = ck;
+                    sw.mode = mode;
+                    sw.cls = cls;
+                    if (vec_push(&strided, &sw)) { st = CFA_ERR_NOMEM; goto done; }
+                }
+                continue;
+            }
             cfa_work w;
             memset(&w, 0, sizeof w);
-            w.ck = (e->flags & CFA_ENTRY_CKSUM) ? pc->entry : CFA_NO_CK;
-            w.mode = CFA_MODE(log2_small(in->es_s), log2_small(in->es_d), pc->cast);
-            w.pad = pc->cast ? CFA_CLASS_CAST : (uint32_t)log2_small(in->es_s);
-            const uint64_t a0 = (uint64_t)(uintptr_t)dsts[pc->dst_index].dev_ptr + pc->dst_offset;
+            w.ck = ck;
+            w.mode = mode;
+            w.pad = cls;
             const uint64_t nb = pc->n_elems * (uint64_t)in->es_d;
             if (nb < o.tiny_bytes) {
                 w.src = pc->src_offset;
@@ -481,52 +626,11 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
             }
         }
         /* pass 2: stable partition by class (items are in chunk order already) */
-        vec *lists[3] = {&slabs, &bulk, &tiny};
-        uint32_t *firsts[3] = {out->slab_first, out->bulk_first, out->tiny_first};
-        for (int li = 0; li < 3; ++li) {
-            vec *v = lists[li];
-            if (v->n >= UINT32_MAX) {
-                fail(err, errlen, "too many work items; raise slab_bytes");
-                st = CFA_ERR_INVAL;
-                goto done;
-            }
-            cfa_work *src_items = (cfa_work *)v->p;
-            cfa_work *sorted = (cfa_work *)malloc((v->n ? v->n : 1) * sizeof(cfa_work));
-            if (!sorted) { st = CFA_ERR_NOMEM; goto done; }
-            /* count per (class, chunk) */
-            uint32_t *first = firsts[li];
-            for (size_t q = 0; q < v->n; ++q) {
-                const uint32_t k = src_items[q].pad;
-                const uint64_t blob_off = src_items[q].src;
-                const uint32_t c = (uint32_t)(blob_off / S);
-                first[(size_t)k * (n_chunks + 1) + c + 1]++;
-            }
-            /* exclusive prefix over the (class, chunk) grid */
-            uint32_t run = 0;
-            for (size_t k = 0; k < CFA_N_CLASSES; ++k) {
-                for (uint32_t c = 0; c <= n_chunks; ++c) {
-                    const size_t idx = k * ((size_t)n_chunks + 1) + c;
-                    if (c == 0) {
-                        first[idx] = run;
-                    } else {
-                        run += first[idx];
-                        first[idx] = run;
-                    }
-                }
-            }
-            /* scatter, keeping chunk order inside each class */
-            uint32_t *cursor = (uint32_t *)malloc(nf * sizeof(uint32_t));
-            if (!cursor) { free(sorted); st = CFA_ERR_NOMEM; goto done; }
-            memcpy(cursor, first, nf * sizeof(uint32_t));
-            for (size_t q = 0; q < v->n; ++q) {
-                const uint32_t k = src_items[q].pad;
-                const uint32_t c = (uint32_t)(src_items[q].src / S);
-                sorted[cursor[(size_t)k * (n_chunks + 1) + c]++] = src_items[q];
-            }
-            free(cursor);
-            free(v->p);
-            v->p = sorted;
-        }
+        if ((st = partition_by_class(&slabs, out->slab_first, n_chunks, S, err, errlen))) goto done;
+        if ((st = partition_by_class(&bulk, out->bulk_first, n_chunks, S, err, errlen))) goto done;
+        if ((st = partition_by_class(&tiny, out->tiny_first, n_chunks, S, err, errlen))) goto done;
+        if ((st = partition_by_class(&strided, out->strided_first, n_chunks, S, err, errlen)))
+            goto done;
     }
 
     /* 5. readiness groups: last chunk carrying one of their bytes */
@@ -535,8 +639,7 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
     for (uint32_t l = 0; l < n_layers; ++l) out->layer_last_chunk[l] = -1;
     for (size_t i = 0; i < n_entries; ++i) {
         if (!info[i].n) continue;
-        const uint64_t last =
-            (entries[i].blob_offset + info[i].n * (uint64_t)info[i].es_s - 1) / S;
+        const uint64_t last = (entries[i].blob_offset + info[i].extent - 1) / S;
         int64_t *slot = &out->layer_last_chunk[entries[i].layer];
         if ((int64_t)last > *slot) *slot = (int64_t)last;
         out->bytes_read += info[i].n * (uint64_t)info[i].es_s;
@@ -572,7 +675,9 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
     out->n_bulk = bulk.n;
     out->tiny = (cfa_work *)tiny.p;
     out->n_tiny = tiny.n;
-    slabs.p = bulk.p = tiny.p = NULL;
+    out->strided = (cfa_swork *)strided.p;
+    out->n_strided = strided.n;
+    slabs.p = bulk.p = tiny.p = strided.p = NULL;
 
 done:
     free(info);
@@ -582,6 +687,7 @@ done:
     free(slabs.p);
     free(bulk.p);
     free(tiny.p);
+    free(strided.p);
     if (st != CFA_OK) cfa_host_plan_free(out);
     return st;
 }

@@ -41,6 +41,12 @@
 
 extern "C" int cfa_unpack_blocks_per_sm(int cls);
 extern "C" int cfa_bulk_blocks_per_sm(int log2es);
+extern "C" int cfa_strided_blocks_per_sm(int cls);
+extern "C" cudaError_t cfa_launch_strided(int cls, const cfa_swork *items, uint32_t n_items,
+                                          uint64_t src_base, uint64_t src_period,
+                                          uint64_t src_lo, uint64_t src_hi,
+                                          unsigned long long *ck, int *status, int grid_cap,
+                                          cudaStream_t stream);
 extern "C" cudaError_t cfa_launch_bulk(int log2es, const cfa_work *items, uint32_t n_items,
                                        uint64_t src_base, uint64_t src_period,
                                        uint64_t src_lo, uint64_t src_hi,
@@ -167,7 +173,9 @@ struct cfa_plan {
     int pageable_access = 0; /* the device can read pageable host memory in place */
     int grid_cap[CFA_N_CLASSES] = {0};
     int bulk_grid_cap[4] = {0};
+    int strided_grid_cap[CFA_N_CLASSES] = {0};
     cfa_work *d_slabs = nullptr, *d_tiny = nullptr, *d_bulk = nullptr;
+    cfa_swork *d_strided = nullptr;
     unsigned long long *d_ck = nullptr;
     int *d_status = nullptr;
     uint8_t *d_slots = nullptr;
@@ -262,6 +270,16 @@ cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint
         if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], s));
         p->last_launches++;
     }
+    for (int k = 0; k < CFA_N_CLASSES && hp.n_strided; ++k) {
+        const uint32_t r0 = hp.strided_first[k * row + c0], r1 = hp.strided_first[k * row + c1];
+        if (r1 == r0) continue;
+        const bool timing = timing_on && p->last_launches < p->t_k0.size();
+        if (timing) CK(p, cudaEventRecord(p->t_k0[p->last_launches], s));
+        CK(p, cfa_launch_strided(k, p->d_strided + r0, r1 - r0, src_base, period, lo, hi,
+                                 p->d_ck, p->d_status, p->strided_grid_cap[k], s));
+        if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], s));
+        p->last_launches++;
+    }
     for (int k = 0; k < CFA_N_CLASSES; ++k) {
         const uint32_t s0 = hp.slab_first[k * row + c0], s1 = hp.slab_first[k * row + c1];
         const uint32_t t0 = hp.tiny_first[k * row + c0], t1 = hp.tiny_first[k * row + c1];
@@ -320,6 +338,7 @@ void release(cfa_plan *p)
         if (p->d_slabs) cudaFree(p->d_slabs);
         if (p->d_tiny) cudaFree(p->d_tiny);
         if (p->d_bulk) cudaFree(p->d_bulk);
+        if (p->d_strided) cudaFree(p->d_strided);
         if (p->d_ck) cudaFree(p->d_ck);
         if (p->d_status) cudaFree(p->d_status);
         if (p->own_slots && p->d_slots) cudaFree(p->d_slots);
@@ -354,6 +373,14 @@ cfa_status setup_device(cfa_plan *p)
         }
         p->grid_cap[k] = sms * per_sm;
     }
+    for (int k = 0; k < CFA_N_CLASSES && hp.n_strided; ++k) {
+        const int per_sm = cfa_strided_blocks_per_sm(k);
+        if (per_sm <= 0) {
+            set_err(nullptr, "strided kernel %d cannot run on device %d", k, p->device);
+            return CFA_ERR_CUDA;
+        }
+        p->strided_grid_cap[k] = sms * per_sm;
+    }
     if (hp.n_bulk) {
         for (int k = 0; k < 4; ++k) {
             const int per_sm = cfa_bulk_blocks_per_sm(k);
@@ -380,6 +407,16 @@ cfa_status setup_device(cfa_plan *p)
     if (st) return st;
     st = upload(&p->d_bulk, hp.bulk, hp.n_bulk);
     if (st) return st;
+    {
+        const size_t bytes = (hp.n_strided ? hp.n_strided : 1) * sizeof(cfa_swork);
+        if (cudaMalloc(&p->d_strided, bytes) != cudaSuccess) {
+            set_err(nullptr, "cudaMalloc of %zu descriptor bytes failed", bytes);
+            return CFA_ERR_NOMEM;
+        }
+        if (hp.n_strided)
+            CK(nullptr, cudaMemcpy(p->d_strided, hp.strided, hp.n_strided * sizeof(cfa_swork),
+                                   cudaMemcpyHostToDevice));
+    }
     const size_t ck_bytes = (hp.n_entries ? hp.n_entries : 1) * sizeof(unsigned long long);
     if (cudaMalloc(&p->d_ck, ck_bytes) != cudaSuccess ||
         cudaMalloc(&p->d_status, sizeof(int)) != cudaSuccess) {
@@ -428,7 +465,7 @@ cfa_status setup_device(cfa_plan *p)
     if (timing) {
         if ((st = events(p->t_h2d0, hp.n_chunks, true))) return st;
         if ((st = events(p->t_h2d1, hp.n_chunks, true))) return st;
-        const size_t nk = 2 * CFA_N_CLASSES * ((size_t)hp.n_chunks + 1);
+        const size_t nk = 3 * CFA_N_CLASSES * ((size_t)hp.n_chunks + 1);
         if ((st = events(p->t_k0, nk, true))) return st;
         if ((st = events(p->t_k1, nk, true))) return st;
     }
@@ -740,9 +777,11 @@ cfa_status cfa_get_stats(cfa_plan *p, cfa_stats *s)
     s->n_slabs = hp.n_slabs;
     s->n_bulk = hp.n_bulk;
     s->n_tiny = hp.n_tiny;
+    s->n_strided = hp.n_strided;
     s->bytes_read = hp.bytes_read;
     s->bytes_written = hp.bytes_written;
-    s->descriptor_bytes = (hp.n_slabs + hp.n_bulk + hp.n_tiny) * sizeof(cfa_work);
+    s->descriptor_bytes = (hp.n_slabs + hp.n_bulk + hp.n_tiny) * sizeof(cfa_work) +
+                          hp.n_strided * sizeof(cfa_swork);
     s->loads = p->n_loads;
     s->kernel_launches = p->last_launches;
     s->plan_ms = p->plan_ms;

@@ -368,6 +368,73 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_unpack_kernel(const 
     if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
 }
 
+/* ---- column slices: blocks of strided rows -------------------------------------------- */
+
+struct StridedArgs {
+    const cfa_swork *items;
+    uint32_t n_items;
+    uint32_t pad;
+    uint64_t src_base;
+    uint64_t src_period;
+    uint64_t src_lo, src_hi;
+    unsigned long long *ck;
+    int *status;
+};
+
+template <int CLS>
+__device__ __forceinline__ bool sitem_ok(const cfa_swork &w, const StridedArgs &a)
+{
+    const uint32_t want_mode = CLS == CFA_CLASS_CAST ? CFA_MODE(2, 1, 1) : CFA_MODE(CLS, CLS, 0);
+    if (w.mode != want_mode || w.rows == 0 || w.cols == 0 || w.stride < w.cols) return false;
+    const uint32_t sl = w.mode & 3u, dl = (w.mode >> 2) & 3u;
+    const uint64_t extent = ((uint64_t)(w.rows - 1) * w.stride + w.cols) << sl;
+    return w.src >= a.src_lo && w.src <= a.src_hi && extent <= a.src_hi - w.src &&
+           (w.src & ((1ull << sl) - 1)) == 0 && (w.dst & ((1ull << dl) - 1)) == 0;
+}
+
+/* Each CTA takes blocks of rows; its warps take the rows of a block in turn and copy each row
+ * like a contiguous run (16-byte vectors, realigned when source and destination disagree mod
+ * 16, four vectors in flight per lane). */
+template <int CLS>
+__global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_strided_kernel(const StridedArgs a)
+{
+    constexpr int SES = CLS == CFA_CLASS_CAST ? 4 : (1 << CLS);
+    constexpr int DES = CLS == CFA_CLASS_CAST ? 2 : (1 << CLS);
+    __shared__ unsigned long long red[kWarps];
+    const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
+    uint64_t acc = 0;
+    uint32_t acc_ck = CFA_NO_CK;
+    for (uint32_t item = blockIdx.x; item < a.n_items; item += gridDim.x) {
+        const cfa_swork w = a.items[item];
+        if (!sitem_ok<CLS>(w, a)) {
+            if (threadIdx.x == 0) atomicCAS(a.status, 0, 1);
+            continue;
+        }
+        if (w.ck != acc_ck) {
+            if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
+            acc = 0;
+            acc_ck = w.ck;
+        }
+        const uint64_t off = a.src_period ? w.src % a.src_period : w.src;
+        const uint8_t *src = reinterpret_cast<const uint8_t *>(a.src_base + off);
+        uint8_t *dst = reinterpret_cast<uint8_t *>(w.dst);
+        for (uint32_t r = warp; r < w.rows; r += kWarps) {
+            const uint8_t *s = src + (uint64_t)r * w.stride * SES;
+            uint8_t *d = dst + (uint64_t)r * w.cols * DES;
+            if constexpr (CLS == CFA_CLASS_CAST)
+                acc += cast_run<2>(s, d, w.cols, lane, 32u);
+            else
+                acc += copy_run<DES, kUnroll>(s, d, (uint64_t)w.cols * DES, lane, 32u);
+        }
+    }
+    if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
+}
+
+typedef void (*strided_fn)(const StridedArgs);
+const strided_fn kStrided[CFA_N_CLASSES] = {cfa_strided_kernel<0>, cfa_strided_kernel<1>,
+                                            cfa_strided_kernel<2>, cfa_strided_kernel<3>,
+                                            cfa_strided_kernel<CFA_CLASS_CAST>};
+
 typedef void (*kernel_fn)(const UnpackArgs);
 const kernel_fn kKernels[CFA_N_CLASSES] = {cfa_unpack_kernel<0>, cfa_unpack_kernel<1>,
                                            cfa_unpack_kernel<2>, cfa_unpack_kernel<3>,
@@ -412,5 +479,40 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
     a.status = status;
     const uint64_t grid = items < (uint64_t)grid_cap ? items : (uint64_t)grid_cap;
     kKernels[cls]<<<(unsigned)grid, kThreads, 0, stream>>>(a);
+    return cudaGetLastError();
+}
+
+/* Resident CTAs per SM of the class-cls strided kernel (0 if it cannot run). */
+extern "C" int cfa_strided_blocks_per_sm(int cls)
+{
+    if (cls < 0 || cls >= CFA_N_CLASSES) return 0;
+    int n = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kStrided[cls], kThreads, 0) !=
+        cudaSuccess)
+        return 0;
+    return n;
+}
+
+/* Launches the class-cls unpack of strided row blocks (column slices of checkpoint tensors). */
+extern "C" cudaError_t cfa_launch_strided(int cls, const cfa_swork *items, uint32_t n_items,
+                                          uint64_t src_base, uint64_t src_period,
+                                          uint64_t src_lo, uint64_t src_hi,
+                                          unsigned long long *ck, int *status, int grid_cap,
+                                          cudaStream_t stream)
+{
+    if (cls < 0 || cls >= CFA_N_CLASSES || grid_cap <= 0) return cudaErrorInvalidValue;
+    if (n_items == 0) return cudaSuccess;
+    StridedArgs a;
+    a.items = items;
+    a.n_items = n_items;
+    a.pad = 0;
+    a.src_base = src_base;
+    a.src_period = src_period;
+    a.src_lo = src_lo;
+    a.src_hi = src_hi;
+    a.ck = ck;
+    a.status = status;
+    const uint32_t grid = n_items < (uint32_t)grid_cap ? n_items : (uint32_t)grid_cap;
+    kStrided[cls]<<<grid, kThreads, 0, stream>>>(a);
     return cudaGetLastError();
 }

@@ -37,7 +37,8 @@ def manifest_case(name):
             entries.append({"name": t[1], "dtype": t[2],
                             "shape": tuple(int(x) for x in t[3].split(",")),
                             "offset": int(t[4]), "dst": int(t[5]), "row": int(t[6]),
-                            "cast": bool(int(t[7])), "cksum": True, "layer": 0})
+                            "cast": bool(int(t[7])), "cksum": True, "layer": 0,
+                            "stride": int(t[8]) if len(t) > 8 else 0})
         elif key == "expect_dst":
             exp_dst[int(t[1])] = np.array([int(x, 16) for x in t[2:]], dtype=np.uint8)
         elif key == "expect_cksum":

@@ -13,6 +13,9 @@ What pins what:
   invariants          exact-once coverage, byte conservation, repack(unpack(blob)) == blob,
                       entry-order invariance (Theorem 2), padding independence
   validation          malformed manifests are rejected with the right class of error
+  tp_shards           tensor-parallel shards: each equals numpy slicing of the full tensor, and
+                      the shards of all ranks reassemble (numpy concatenate) into the unsharded
+                      load
 """
 import numpy as np
 import torch
@@ -100,7 +103,7 @@ def rne_vs_nearest(lib=None):
 # unpacking
 # ---------------------------------------------------------------------------------------------
 def golden_manifests(lib=None):
-    for name in ("fused_tiny.txt", "moe_tiny.txt"):
+    for name in ("fused_tiny.txt", "moe_tiny.txt", "tp_shard_tiny.txt"):
         m, blob, exp_dst, exp_ck = manifest_case(name)
         r = oracle.unpack(m, blob, lib=lib, fill=0xEE)
         assert r.status == 0, (name, r.status_name, r.bad_entry)
@@ -130,6 +133,22 @@ def one_to_one(lib=None):
         assert int(r.cksum[i]) == int(sl.view(np.uint16).astype(np.uint64).sum()), i
 
 
+def _source_elements(m, blob, i):
+    """Entry i's source bytes in element order: the blob slice, or for a column slice the
+    leading columns of a (rows, stride) numpy view of the bytes it spans."""
+    off, nb = int(m.e_offset[i]), m.e_nbytes(i)
+    stride = int(m.e_stride[i])
+    if stride == 0:
+        return blob[off:off + nb]
+    es = DTYPE_SIZE[str(m.e_dtype[i])]
+    cols = int(m.e_shape[i, m.e_ndim[i] - 1])
+    rows = nb // es // cols
+    span = np.zeros(rows * stride * es, dtype=np.uint8)
+    ext = m.e_extent(i)
+    span[:ext] = blob[off:off + ext]
+    return np.ascontiguousarray(span.reshape(rows, stride * es)[:, :cols * es]).ravel()
+
+
 def _expected_by_concat(m, blob):
     """Destination bytes built by concatenating each destination's parts in row order, with
     torch doing the casts: no offsets are computed."""
@@ -137,8 +156,7 @@ def _expected_by_concat(m, blob):
     for j in range(m.n_dsts):
         parts = []
         for i in sorted(m.entries_of_dst(j), key=lambda i: int(m.e_row[i])):
-            off, nb = int(m.e_offset[i]), m.e_nbytes(i)
-            sl = blob[off:off + nb]
+            sl = _source_elements(m, blob, i)
             if m.e_cast[i]:
                 sl = _torch_bf16_bits(sl.view(np.uint32)).view(np.uint8)
             parts.append(sl)
@@ -158,7 +176,7 @@ def _mini_moe(seed=41, **kw):
     kw.setdefault("align", 2)
     kw.setdefault("jitter", 3)
     return moe_config("mini_moe", seed, layers=2, hidden=32, n_q=4, n_kv=2, head_dim=8,
-                      inter=48, n_experts=3, vocab=50, n_extra=25, **kw)
+                      inter=48, n_experts=3, vocab=52, n_extra=25, **kw)
 
 
 def _check_against_concat(m, lib):
@@ -273,7 +291,7 @@ def _permuted(m, perm):
                      "shape": m.e_shape_tuple(i), "offset": int(m.e_offset[i]),
                      "dst": int(m.e_dst[i]), "row": int(m.e_row[i]),
                      "cast": bool(m.e_cast[i]), "cksum": bool(m.e_cksum[i]),
-                     "layer": int(m.e_layer[i])})
+                     "layer": int(m.e_layer[i]), "stride": int(m.e_stride[i])})
     dsts = [{"name": m.d_name[j], "dtype": str(m.d_dtype[j]), "shape": m.d_shape_tuple(j)}
             for j in range(m.n_dsts)]
     return Manifest(m.name, ents, dsts, m.blob_bytes, m.blob_kind, m.seed, m.period,
@@ -286,7 +304,7 @@ def _variant(m, i, **change):
         e = {"name": m.e_name[k], "dtype": str(m.e_dtype[k]), "shape": m.e_shape_tuple(k),
              "offset": int(m.e_offset[k]), "dst": int(m.e_dst[k]), "row": int(m.e_row[k]),
              "cast": bool(m.e_cast[k]), "cksum": bool(m.e_cksum[k]),
-             "layer": int(m.e_layer[k])}
+             "layer": int(m.e_layer[k]), "stride": int(m.e_stride[k])}
         if k == i:
             e.update(change)
         ents.append(e)
@@ -319,5 +337,90 @@ def validation(lib=None):
     assert oracle.check_cover(r, lib=lib)[0] == oracle.ORC_E_COVERAGE
 
 
+def tp_shards(lib=None):
+    """Rank shards against numpy slicing, and the ranks together against the unsharded load."""
+    for build, src in ((_mini_dense, "bf16"), (_mini_dense, "f32"), (_mini_moe, None)):
+        for tp in (2, 4):
+            kw = {} if src is None else {"src": src}
+            full = build(seed=35, **kw)
+            blob = _blob(full)
+            rf = oracle.unpack(full, blob, lib=lib)
+            assert rf.status == 0
+            ranks = []
+            for rank in range(tp):
+                m = build(seed=35, tp=tp, rank=rank, **kw)
+                assert m.blob_bytes == full.blob_bytes
+                r = oracle.unpack(m, blob, lib=lib)
+                assert r.status == 0, (m.name, tp, rank, r.status_name)
+                exp = _expected_by_concat(m, blob)
+                for j in range(m.n_dsts):
+                    assert np.array_equal(r.dst[j], exp[j]), (tp, rank, m.d_name[j])
+                ranks.append((m, r))
+            _check_reassembly(full, rf, ranks, tp)
+
+
+def _check_reassembly(full, rf, ranks, tp):
+    """Shards of all ranks, concatenated the way the split cut them, give the unsharded
+    destinations: row-parallel weights along columns, vocabulary and column-parallel weights
+    (each fused part separately) along rows."""
+    def dst(m, r, name):
+        j = m.d_name.index(name)
+        return r.dst[j].view(np.uint16).reshape(m.d_shape_tuple(j))
+
+    names = full.d_name
+    for name in names:
+        jf = names.index(name)
+        want = rf.dst[jf].view(np.uint16).reshape(full.d_shape_tuple(jf))
+        parts = [dst(m, r, name) for m, r in ranks]
+        if name.endswith("gate_up_proj.weight"):
+            halves = [np.split(p, 2, axis=0) for p in parts]
+            got = np.concatenate([h[0] for h in halves] + [h[1] for h in halves], axis=0)
+        elif name.endswith(("o_proj.weight", "down_proj.weight", "w2_weight")):
+            got = np.concatenate(parts, axis=-1)
+        elif name.endswith(("embed_tokens.weight", "lm_head.weight", "q_proj.weight",
+                            "gate_proj.weight", "up_proj.weight")):
+            got = np.concatenate(parts, axis=0)
+        elif name.endswith("w13_weight"):
+            halves = [np.split(p, 2, axis=1) for p in parts]
+            got = np.concatenate([h[0] for h in halves] + [h[1] for h in halves], axis=1)
+        elif name.endswith("qkv_proj.weight"):
+            continue  # checked below, per part
+        else:
+            got = parts[0]  # replicated: norms, router, extras
+            for p in parts[1:]:
+                assert np.array_equal(p, got), name
+        assert np.array_equal(got, want), name
+    # fused qkv: q rows split over ranks; k and v split, or replicated per kv head
+    m0 = ranks[0][0]
+    qkv = [n for n in names if n.endswith("qkv_proj.weight")]
+    for name in qkv:
+        jf = names.index(name)
+        want = rf.dst[jf].view(np.uint16).reshape(full.d_shape_tuple(jf))
+        parts = [dst(m, r, name) for m, r in ranks]
+        rows_r = parts[0].shape[0]
+        q_rows_r = (want.shape[0] - 2 * _kv_rows(full, name)) // tp
+        kv_r = (rows_r - q_rows_r) // 2
+        q = np.concatenate([p[:q_rows_r] for p in parts], axis=0)
+        assert np.array_equal(q, want[:q_rows_r * tp]), name
+        kv_full = _kv_rows(full, name)
+        for which, base in (("k", q_rows_r * tp), ("v", q_rows_r * tp + kv_full)):
+            off = q_rows_r if which == "k" else q_rows_r + kv_r
+            shards = [p[off:off + kv_r] for p in parts]
+            if kv_r * tp == kv_full:
+                got = np.concatenate(shards, axis=0)
+                assert np.array_equal(got, want[base:base + kv_full]), (name, which)
+            else:  # replicated heads: every shard is one of the full kv heads
+                for s in shards:
+                    heads = want[base:base + kv_full].reshape(-1, kv_r, want.shape[1])
+                    assert any(np.array_equal(s, h) for h in heads), (name, which)
+    del m0
+
+
+def _kv_rows(full, qkv_name):
+    prefix = qkv_name.rsplit("qkv_proj", 1)[0]
+    i = full.e_name.index(prefix + "k_proj.weight")
+    return int(full.e_shape[i, 0])
+
+
 ALL_PINS = [rne_golden, rne_vs_torch, rne_vs_nearest, golden_manifests, one_to_one,
-            concat_reference, cast_reference, invariants, validation]
+            concat_reference, cast_reference, invariants, validation, tp_shards]

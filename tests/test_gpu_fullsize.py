@@ -42,7 +42,7 @@ def release_device_memory():
 
 def verify_all(m, d, ck, max_batch=1 << 29, max_count=50_000):
     """Every destination byte and every checksum of `m` against the oracle."""
-    nbytes = m.e_nbytes_array()
+    nbytes = m.e_extent_array()
     offs = m.e_offset.astype(np.int64)
     de = m.dst_entries()
     batches, j0, acc = [], 0, 0
@@ -151,6 +151,27 @@ def test_full_mixtral_8x7b_bf16():
     d.buf.fill_(0xA5)
     cb = CallbackSource(m)
     ck2, _, _ = _load(m, d, cb.source(), fill_threads=16)
+    assert np.array_equal(ck, ck2)
+    verify_all(m, d, ck2)
+
+
+def test_full_llama3_70b_bf16_tensor_parallel_rank():
+    """Rank 3 of 8 of the 70B checkpoint: row ranges of q/k/v, gate/up, embed, lm_head and
+    column slices of o and down, read from the whole (periodic) checkpoint."""
+    m = workloads.named_config("llama3_70b_bf16_tp8r3")
+    d = DeviceDsts(m)
+    pool = torch.empty(m.period, dtype=torch.uint8, pin_memory=True)
+    m.fill_source_ptr(pool.data_ptr())
+    dpool = pool.to("cuda")
+    ck, st, _ = _load(m, d, cfa.Source.device(dpool.data_ptr(), period=m.period),
+                      dev_slots=0, host_slots=0)
+    assert st["n_strided"] > 0
+    verify_all(m, d, ck)
+    assert d.guards_intact()
+    # the same shard read in place from the pinned pool over the host link
+    d.buf.fill_(0xA5)
+    ck2, _, _ = _load(m, d, cfa.Source.host_direct(pool.data_ptr(), period=m.period),
+                      dev_slots=0, host_slots=0)
     assert np.array_equal(ck, ck2)
     verify_all(m, d, ck2)
 

@@ -115,7 +115,25 @@ def cfg_moe():
                       inter=512, n_experts=4, vocab=500, n_extra=3000, align=2, jitter=3)
 
 
-CONFIGS = {"tiny": cfg_tiny, "dense": cfg_dense, "dense_f32": cfg_dense_f32, "moe": cfg_moe}
+def cfg_dense_tp():
+    return dense_config("dense_tp2r1", 68, layers=2, hidden=512, n_q=8, n_kv=2, head_dim=64,
+                        inter=1536, vocab=1000, align=2, jitter=5, tp=2, rank=1)
+
+
+def cfg_f32_tp():
+    return dense_config("dense_f32_tp4r3", 69, layers=2, hidden=512, n_q=8, n_kv=2,
+                        head_dim=64, inter=1536, vocab=1000, src_dtype="f32", align=4,
+                        jitter=3, tp=4, rank=3)
+
+
+def cfg_moe_tp():
+    return moe_config("moe_tp2r0", 70, layers=2, hidden=256, n_q=4, n_kv=2, head_dim=64,
+                      inter=512, n_experts=4, vocab=500, n_extra=300, align=2, jitter=3,
+                      tp=2, rank=0)
+
+
+CONFIGS = {"tiny": cfg_tiny, "dense": cfg_dense, "dense_f32": cfg_dense_f32, "moe": cfg_moe,
+           "dense_tp": cfg_dense_tp, "f32_tp": cfg_f32_tp, "moe_tp": cfg_moe_tp}
 
 
 @pytest.mark.parametrize("cfg", list(CONFIGS))

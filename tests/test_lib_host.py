@@ -73,13 +73,18 @@ def execute_pieces_on_cpu(m, pieces, blob):
     for pc in pieces:
         i = int(pc["entry"])
         es_s = DTYPE_SIZE[str(m.e_dtype[i])]
-        n = int(pc["n_elems"])
-        src = blob[int(pc["src_offset"]):int(pc["src_offset"]) + n * es_s]
-        if pc["cast"]:
-            f = torch.from_numpy(src.view(np.float32).copy())
-            src = f.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint8)
+        rows = int(pc["rows"])
+        cols = int(pc["n_elems"]) // rows
+        step = int(pc["src_row_stride"]) * es_s if rows > 1 else cols * es_s
         o = int(pc["dst_offset"])
-        out[int(pc["dst_index"])][o:o + src.size] = src
+        for k in range(rows):
+            a = int(pc["src_offset"]) + k * step
+            src = blob[a:a + cols * es_s]
+            if pc["cast"]:
+                f = torch.from_numpy(src.view(np.float32).copy())
+                src = f.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint8)
+            out[int(pc["dst_index"])][o:o + src.size] = src
+            o += src.size
     return out
 
 
@@ -89,6 +94,12 @@ def mini_configs():
         dense_config("d", 52, 2, 64, 4, 2, 16, 96, 100, align=2, jitter=3),
         dense_config("d32", 53, 2, 64, 4, 2, 16, 96, 100, src_dtype="f32", align=4, jitter=2),
         moe_config("m", 54, 2, 32, 4, 2, 8, 48, 3, 50, n_extra=30, align=2, jitter=3),
+        # tensor-parallel ranks: column slices read with a source row stride
+        dense_config("d_tp2r1", 55, 2, 64, 4, 2, 16, 96, 100, align=2, jitter=3, tp=2, rank=1),
+        dense_config("d32_tp4r2", 56, 2, 64, 4, 2, 16, 96, 100, src_dtype="f32", align=4,
+                     jitter=2, tp=4, rank=2),
+        moe_config("m_tp2r0", 57, 2, 32, 4, 2, 8, 48, 3, 52, n_extra=30, align=2, jitter=3,
+                   tp=2, rank=0),
     ]
 
 
@@ -103,7 +114,10 @@ def test_plan_pieces_reproduce_the_oracle(chunk):
         # every piece lies inside one chunk
         es = np.array([DTYPE_SIZE[str(m.e_dtype[int(i)])] for i in pcs["entry"]])
         start = pcs["src_offset"].astype(np.int64)
-        end = start + pcs["n_elems"].astype(np.int64) * es
+        rows = pcs["rows"].astype(np.int64)
+        cols = pcs["n_elems"].astype(np.int64) // rows
+        step = np.where(rows > 1, pcs["src_row_stride"].astype(np.int64), cols)
+        end = start + ((rows - 1) * step + cols) * es
         assert (start // chunk == pcs["chunk"]).all()
         assert ((end - 1) // chunk == pcs["chunk"]).all()
         # chunk-major order
@@ -182,6 +196,16 @@ def test_bad_options_and_misaligned_destination():
     with pytest.raises(cfa.CfaError) as e:
         cfa.Plan(entries_for(m), d, m.blob_bytes, host_only=True)
     assert e.value.name == "CFA_ERR_ALIGN"
+
+
+def test_strided_entries_are_validated_like_the_oracle():
+    m, blob, _, _ = manifest_case("tp_shard_tiny.txt")
+    assert _plan_status(m) == "CFA_OK" and oracle.unpack(m, blob).status == 0
+    # a stride shorter than the row, and a column slice reading past the blob
+    for change, name in ((dict(stride=1), "CFA_ERR_INVAL"), (dict(offset=40), "CFA_ERR_OOB")):
+        mv = _pins._variant(m, 2, **change)
+        assert _plan_status(mv) == name
+        assert _ORACLE_TO_CFA[oracle.unpack(mv, blob).status] == name
 
 
 def test_empty_manifest_and_zero_sized_entries():

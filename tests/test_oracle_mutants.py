@@ -39,7 +39,8 @@ MUTANTS = [
     ("base_uses_src_size", "base_elem * (uint64_t)es_d", "base_elem * (uint64_t)es_s"),
     ("big_endian_read", "x |= (uint64_t)p[k] << (8 * k)",
      "x |= (uint64_t)p[k] << (8 * (nbytes - 1 - k))"),
-    ("src_stride_wrong", "src + i * (uint64_t)es_s", "src + i * (uint64_t)es_d"),
+    ("src_stride_wrong", "read_le(src + src_i * (uint64_t)es_s, es_s)",
+     "read_le(src + src_i * (uint64_t)es_d, es_s)"),
     ("dst_stride_wrong", "dst + i * (uint64_t)es_d", "dst + i * (uint64_t)es_s"),
     ("checksum_of_source", "ck += y;", "ck += x;"),
     ("checksum_misses_last", "ck += y;", "if (i + 1 < n) ck += y;"),
@@ -47,6 +48,10 @@ MUTANTS = [
      "const uint64_t y = x;"),
     ("oob_check_off_by_elem", "if (base_elem + n > d_numel)", "if (base_elem + n > d_numel + 1)"),
     ("cover_not_counted", "+= 1u;", "+= 0u;"),
+    ("stride_ignored", "const uint64_t src_i = (i / C) * stride + (i % C);",
+     "const uint64_t src_i = i;"),
+    ("stride_uses_row_length", "const uint64_t stride = given ? given : C;",
+     "const uint64_t stride = C;"),
 ]
 
 

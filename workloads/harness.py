@@ -16,7 +16,8 @@ def entries_for(m, with_names=False):
     return cfa.make_entries(dtype=list(m.e_dtype), shape=(m.e_shape, m.e_ndim),
                             offset=m.e_offset, dst=m.e_dst, row=m.e_row, cast=m.e_cast,
                             cksum=m.e_cksum, layer=m.e_layer,
-                            names=m.e_name if with_names else None)
+                            names=m.e_name if with_names else None,
+                            src_row_stride=m.e_stride)
 
 
 class DeviceDsts:
@@ -115,8 +116,8 @@ def device_blob(m, host=None):
 
 
 def entry_host_bytes(m, i):
-    """Source bytes of entry i, regenerated from the blob definition."""
-    return m.blob_range(int(m.e_offset[i]), m.e_nbytes(i))
+    """Blob bytes entry i spans (its source bytes, plus the gaps of a column slice)."""
+    return m.blob_range(int(m.e_offset[i]), m.e_extent(i))
 
 
 __all__ = ["entries_for", "DeviceDsts", "CallbackSource", "pinned_blob", "device_blob",
