@@ -211,7 +211,8 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
         ms = min(_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
                  for _ in range(2))
         out["e2e_direct_pageable_s_per_model"] = round(ms / 1e3, 4)
-        out["e2e_direct_pageable_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
+        # the kernel reads only the bytes the entries cover (a tensor-parallel rank: its shard)
+        out["e2e_direct_pageable_link_gbs"] = round(plan.stats()["bytes_read"] / ms / 1e6, 2)
     except cfa.CfaError as e:
         out["e2e_direct_pageable"] = f"unavailable: {e}"
     plan.close()

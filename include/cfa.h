@@ -79,6 +79,11 @@ typedef int cfa_status;
 /* cfa_tensor_entry.flags */
 #define CFA_ENTRY_CAST_BF16 0x1u /* source fp32, destination bf16, round to nearest even */
 #define CFA_ENTRY_CKSUM     0x2u /* accumulate this entry's checksum (see cfa_get_checksums) */
+#define CFA_ENTRY_CONVERT   0x4u /* convert to the destination dtype; supported pairs:
+                                    f32 -> bf16, f32 -> f16, f16 -> bf16 (round to nearest,
+                                    ties to even; NaN -> 0x7FC0 for bf16, sign | 0x7E00 for
+                                    f16; overflow -> infinity), bf16 -> f32 and f16 -> f32
+                                    (exact, NaN payloads kept) */
 
 /* Passed as `layer` to cfa_wait_layer / cfa_get_layer_times: the whole load. */
 #define CFA_ALL (-1)
@@ -100,8 +105,10 @@ typedef int cfa_status;
  *                   of ndim <= 1 a row is one element.  This is how fused layouts are written:
  *                   q, k, v at rows 0, Hq, Hq + Hkv of qkv; gate, up at rows 0, I of gate_up;
  *                   expert e's w1, w3 at rows 2Ie, 2Ie + I of the [E*2I, H] view of w13.
- *   flags           CFA_ENTRY_*.  Without CFA_ENTRY_CAST_BF16 the destination dtype must
- *                   equal src_dtype; with it, src_dtype must be F32 and the destination BF16.
+ *   flags           CFA_ENTRY_*.  Without CFA_ENTRY_CAST_BF16 or CFA_ENTRY_CONVERT the
+ *                   destination dtype must equal src_dtype; with CFA_ENTRY_CAST_BF16, src_dtype
+ *                   must be F32 and the destination BF16; with CFA_ENTRY_CONVERT the pair must
+ *                   be one CFA_ENTRY_CONVERT lists.
  *   src_row_stride  0 when the tensor's elements are contiguous in the blob.  Otherwise the
  *                   tensor is read as numel / shape[-1] rows of shape[-1] elements whose first
  *                   elements lie src_row_stride source elements apart (>= shape[-1]): a column
@@ -232,7 +239,8 @@ typedef struct cfa_piece {
     uint32_t entry;
     uint64_t src_offset;      /* byte offset in the blob */
     uint32_t dst_index;
-    uint32_t cast;
+    uint32_t conv;            /* 0 = copy; 1 f32->bf16, 2 f32->f16, 3 f16->bf16, 4 bf16->f32,
+                                 5 f16->f32 */
     uint64_t dst_offset;      /* byte offset inside the destination */
     uint64_t n_elems;
     uint32_t rows;

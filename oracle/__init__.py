@@ -29,7 +29,10 @@ _lib = None
 # The oracle's own dtype codes (cfa_oracle.c); dtype names are the manifest's.
 _DTYPE_CODE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7}
 _ELEM = {"u8": 1, "bf16": 2, "f16": 2, "f32": 4, "i32": 4, "i64": 8, "f64": 8}
-_CAST, _CKSUM = 1, 2
+_CONVERT, _CKSUM = 1, 2
+# conversion ids of oracle_convert_array
+CONV = {("f32", "bf16"): 1, ("f32", "f16"): 2, ("f16", "bf16"): 3, ("bf16", "f32"): 4,
+        ("f16", "f32"): 5}
 
 ORC_OK, ORC_E_INVAL, ORC_E_DTYPE, ORC_E_ALIGN, ORC_E_OOB, ORC_E_SHAPE, ORC_E_OVERLAP, \
     ORC_E_COVERAGE = range(8)
@@ -44,7 +47,8 @@ def build(force=False):
         return _LIB_PATH
     fd, tmp = tempfile.mkstemp(suffix=".so", dir=_HERE)
     os.close(fd)
-    subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", _SRC, "-o", tmp], check=True)
+    subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", _SRC, "-o", tmp, "-lm"],
+                   check=True)
     os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
 
@@ -62,6 +66,10 @@ def _bind(path):
     lib.oracle_unpack.restype = ctypes.c_int
     lib.oracle_check_cover.argtypes = [U64, P, P, P]
     lib.oracle_check_cover.restype = ctypes.c_int
+    lib.oracle_convert_array.argtypes = [ctypes.c_int, P, P, U64]
+    lib.oracle_convert_array.restype = None
+    lib.oracle_f32_to_f16.argtypes = [ctypes.c_uint32]
+    lib.oracle_f32_to_f16.restype = ctypes.c_uint16
     return lib
 
 
@@ -84,6 +92,20 @@ def rne_bf16(u32, lib=None):
     out = np.empty(a.shape, dtype=np.uint16)
     (lib or _load()).oracle_rne_bf16_array(a.ctypes.data, out.ctypes.data, a.size)
     return out
+
+
+def convert(src_dtype, dst_dtype, bits, lib=None):
+    """Converts an array of source bit patterns (uint16 or uint32) to destination bit patterns
+    with the oracle's conversion for that dtype pair."""
+    conv = CONV[(src_dtype, dst_dtype)]
+    a = np.ascontiguousarray(bits, dtype=np.uint16 if src_dtype in ("f16", "bf16") else np.uint32)
+    out = np.empty(a.shape, dtype=np.uint16 if dst_dtype in ("f16", "bf16") else np.uint32)
+    (lib or _load()).oracle_convert_array(conv, a.ctypes.data, out.ctypes.data, a.size)
+    return out
+
+
+def f32_to_f16_scalar(u, lib=None):
+    return int((lib or _load()).oracle_f32_to_f16(int(u) & 0xFFFFFFFF))
 
 
 class OracleResult:
@@ -112,7 +134,7 @@ def _columns(m):
     if c is None:
         c = (np.array([_DTYPE_CODE[str(x)] for x in m.e_dtype], dtype=np.int32),
              np.array([_DTYPE_CODE[str(x)] for x in m.d_dtype], dtype=np.int32),
-             (m.e_cast.astype(np.uint32) * _CAST) | (m.e_cksum.astype(np.uint32) * _CKSUM),
+             (m.e_cast.astype(np.uint32) * _CONVERT) | (m.e_cksum.astype(np.uint32) * _CKSUM),
              np.ascontiguousarray(m.e_ndim, dtype=np.int32),
              np.ascontiguousarray(m.e_shape, dtype=np.int64),
              np.ascontiguousarray(m.e_offset, dtype=np.uint64),

@@ -13,8 +13,9 @@
  *
  *   for each entry t:
  *     D      = destination t.dst
- *     es_s   = element size of t's source dtype
- *     es_d   = 2 if t casts fp32 -> bf16, else es_s (and D's dtype must equal the source dtype)
+ *     es_s   = element size of t's source dtype;  es_d = element size of D's dtype
+ *              (equal to the source dtype unless t converts: f32 -> bf16, f32 -> f16,
+ *              f16 -> bf16, bf16 -> f32, f16 -> f32)
  *     n      = product of t.shape
  *     row    = D's last dimension R when D has >= 2 dimensions (t.shape[-1] must equal R),
  *              one element when D has <= 1 dimension
@@ -23,7 +24,7 @@
  *     for i in 0 .. n-1:
  *         src_i = (i / C) * stride + (i mod C)     (element i of row i / C of a column slice)
  *         x = little-endian es_s-byte integer at blob[t.blob_offset + src_i * es_s]
- *         y = cast ? rne_bf16(x) : x
+ *         y = converts ? convert(x) : x
  *         write y as es_d little-endian bytes at D[base + i * es_d]
  *         cover[D][each written byte] += 1
  *         if t checksums: ck[t] = (ck[t] + y) mod 2^64
@@ -34,15 +35,37 @@
  * applied to dropping the low 16 bits of a binary32): NaN -> 0x7FC0; otherwise add 0x7FFF plus
  * the lowest kept bit, then drop the low 16 bits.  Inf stays Inf, values past the largest finite
  * bf16 round to Inf, subnormals round like any other value, signed zeros keep their sign.
+ *
+ * The other conversions follow the IEEE 754 binary16 definition (1 sign, 5 exponent bits with
+ * bias 15, 10 fraction bits; subnormals m * 2^-24): f16 -> f32 is exact (the value as a double,
+ * then as a float, which holds every binary16 value; NaN keeps its payload in the top fraction
+ * bits); f32 -> f16 takes the exact value and rounds it to the nearest binary16 with ties to
+ * even (nearbyint in the default rounding mode), overflowing to infinity from 65520 up, NaN ->
+ * sign | 0x7E00; f16 -> bf16 is f16 -> f32 then rne_bf16; bf16 -> f32 appends 16 zero bits.
  */
+#include <math.h>
 #include <stdint.h>
 #include <stddef.h>
+#include <string.h>
 
 /* The oracle's own dtype codes (its Python wrapper maps dtype names onto these). */
 enum { ORC_U8 = 1, ORC_BF16 = 2, ORC_F16 = 3, ORC_F32 = 4, ORC_I32 = 5, ORC_I64 = 6, ORC_F64 = 7 };
 
 /* Entry flags as the wrapper passes them. */
-enum { ORC_CAST = 1, ORC_CKSUM = 2 };
+enum { ORC_CONVERT = 1, ORC_CKSUM = 2 };
+
+/* Conversions, by (source, destination) dtype. */
+enum { ORC_NONE = 0, ORC_F32_BF16, ORC_F32_F16, ORC_F16_BF16, ORC_BF16_F32, ORC_F16_F32 };
+
+static int orc_conversion(int32_t s, int32_t d)
+{
+    if (s == ORC_F32 && d == ORC_BF16) return ORC_F32_BF16;
+    if (s == ORC_F32 && d == ORC_F16) return ORC_F32_F16;
+    if (s == ORC_F16 && d == ORC_BF16) return ORC_F16_BF16;
+    if (s == ORC_BF16 && d == ORC_F32) return ORC_BF16_F32;
+    if (s == ORC_F16 && d == ORC_F32) return ORC_F16_F32;
+    return ORC_NONE;
+}
 
 /* Result codes. */
 enum {
@@ -82,6 +105,70 @@ uint16_t oracle_rne_bf16(uint32_t u)
 void oracle_rne_bf16_array(const uint32_t *in, uint16_t *out, uint64_t n)
 {
     for (uint64_t i = 0; i < n; ++i) out[i] = oracle_rne_bf16(in[i]);
+}
+
+uint32_t oracle_f16_to_f32(uint16_t h)
+{
+    const uint32_t s = h >> 15, e = (h >> 10) & 31u, m = h & 1023u;
+    if (e == 31u) return (s << 31) | 0x7F800000u | (m << 13); /* infinity or NaN */
+    const double v = e == 0 ? ldexp((double)m, -24) : ldexp(1024.0 + (double)m, (int)e - 25);
+    const float f = (float)(s ? -v : v);
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    return u;
+}
+
+uint16_t oracle_f32_to_f16(uint32_t u)
+{
+    const uint16_t sign = (uint16_t)((u >> 16) & 0x8000u);
+    if ((u & 0x7F800000u) == 0x7F800000u && (u & 0x007FFFFFu)) return sign | 0x7E00u;
+    float f;
+    memcpy(&f, &u, 4);
+    const double v = fabs((double)f);
+    if (isinf(v) || v >= 65520.0) return sign | 0x7C00u; /* 65504 + half an ulp (16) */
+    if (v < ldexp(1.0, -14)) {                           /* subnormal: m * 2^-24 */
+        const double m = nearbyint(ldexp(v, 24));         /* may round up to 1024 = 2^-14 */
+        return sign | (uint16_t)m;
+    }
+    int e2;
+    frexp(v, &e2);          /* v = fr * 2^e2, 0.5 <= fr < 1 */
+    int E = e2 - 1;         /* 2^E <= v < 2^(E+1) */
+    double m = nearbyint(ldexp(v, 10 - E)); /* 1024 <= m <= 2048 */
+    if (m == 2048.0) {
+        m = 1024.0;
+        E += 1;
+    }
+    if (E > 15) return sign | 0x7C00u;
+    return sign | (uint16_t)((E + 15) << 10) | (uint16_t)(m - 1024.0);
+}
+
+uint32_t oracle_bf16_to_f32(uint16_t b) { return (uint32_t)b << 16; }
+
+uint16_t oracle_f16_to_bf16(uint16_t h) { return oracle_rne_bf16(oracle_f16_to_f32(h)); }
+
+static uint64_t orc_convert(int conv, uint64_t x)
+{
+    switch (conv) {
+    case ORC_F32_BF16: return oracle_rne_bf16((uint32_t)x);
+    case ORC_F32_F16: return oracle_f32_to_f16((uint32_t)x);
+    case ORC_F16_BF16: return oracle_f16_to_bf16((uint16_t)x);
+    case ORC_BF16_F32: return oracle_bf16_to_f32((uint16_t)x);
+    case ORC_F16_F32: return oracle_f16_to_f32((uint16_t)x);
+    default: return x;
+    }
+}
+
+/* Array forms for the pins (one conversion over n elements). */
+void oracle_convert_array(int conv, const void *in, void *out, uint64_t n)
+{
+    const int in16 = conv == ORC_F16_BF16 || conv == ORC_BF16_F32 || conv == ORC_F16_F32;
+    const int out16 = conv == ORC_F32_BF16 || conv == ORC_F32_F16 || conv == ORC_F16_BF16;
+    for (uint64_t i = 0; i < n; ++i) {
+        const uint64_t x = in16 ? ((const uint16_t *)in)[i] : ((const uint32_t *)in)[i];
+        const uint64_t y = orc_convert(conv, x);
+        if (out16) ((uint16_t *)out)[i] = (uint16_t)y;
+        else ((uint32_t *)out)[i] = (uint32_t)y;
+    }
 }
 
 static uint64_t read_le(const uint8_t *p, int nbytes)
@@ -128,16 +215,15 @@ int oracle_unpack(uint64_t n_entries, const int32_t *e_dtype, const int32_t *e_n
         const uint64_t j = (uint64_t)e_dst[t];
         const int es_dt = orc_elem_size(d_dtype[j]);
         if (es_dt == 0 || d_ndim[j] < 0 || d_ndim[j] > 8) { *bad_entry = (int64_t)t; return ORC_E_INVAL; }
-        const int cast = (e_flags[t] & ORC_CAST) != 0;
+        const int converts = (e_flags[t] & ORC_CONVERT) != 0;
 
         /* dtypes */
-        if (cast) {
-            if (e_dtype[t] != ORC_F32 || d_dtype[j] != ORC_BF16) { *bad_entry = (int64_t)t; return ORC_E_DTYPE; }
-        } else if (e_dtype[t] != d_dtype[j]) {
+        const int conv = converts ? orc_conversion(e_dtype[t], d_dtype[j]) : ORC_NONE;
+        if (converts ? conv == ORC_NONE : e_dtype[t] != d_dtype[j]) {
             *bad_entry = (int64_t)t;
             return ORC_E_DTYPE;
         }
-        const int es_d = cast ? 2 : es_s;
+        const int es_d = es_dt;
 
         /* element counts */
         uint64_t n = 1;
@@ -191,7 +277,7 @@ int oracle_unpack(uint64_t n_entries, const int32_t *e_dtype, const int32_t *e_n
         for (uint64_t i = 0; i < n; ++i) {
             const uint64_t src_i = (i / C) * stride + (i % C);
             const uint64_t x = read_le(src + src_i * (uint64_t)es_s, es_s);
-            const uint64_t y = cast ? (uint64_t)oracle_rne_bf16((uint32_t)x) : x;
+            const uint64_t y = converts ? orc_convert(conv, x) : x;
             write_le(dst + i * (uint64_t)es_d, y, es_d);
             if (cover)
                 for (int k = 0; k < es_d; ++k) cover[base + i * (uint64_t)es_d + (uint64_t)k] += 1u;

@@ -58,7 +58,8 @@ def make_entries(dtype, shape, offset, dst, row=None, cast=None, cksum=None, lay
     shape   sequence of shapes (tuples), or an [N, 8] int array plus `ndim` via a tuple
             (shape_array, ndim_array)
     offset  blob byte offsets;  dst  destination indices;  row  destination row offsets
-    cast, cksum  booleans (default: no cast, checksum on);  layer  readiness groups (default 0)
+    cast, cksum  booleans (default: no conversion, checksum on); cast converts the source
+            elements to the destination's dtype (CFA_ENTRY_CONVERT);  layer  readiness groups
     names   optional list of str (kept alive by the returned object)
     src_row_stride  source elements between row starts for strided (column-slice) entries;
             0 = contiguous (default)
@@ -81,7 +82,7 @@ def make_entries(dtype, shape, offset, dst, row=None, cast=None, cksum=None, lay
         e["dst_row_offset"] = np.asarray(row, dtype=np.int64)
     fl = np.zeros(n, dtype=np.uint32)
     if cast is not None:
-        fl |= np.asarray(cast, dtype=bool).astype(np.uint32) * _lib.ENTRY_CAST_BF16
+        fl |= np.asarray(cast, dtype=bool).astype(np.uint32) * _lib.ENTRY_CONVERT
     if cksum is None:
         fl |= _lib.ENTRY_CKSUM
     else:

@@ -14,7 +14,7 @@ STATUS = {0: "CFA_OK", -1: "CFA_ERR_INVAL", -2: "CFA_ERR_OVERLAP", -3: "CFA_ERR_
           -8: "CFA_ERR_BUSY", -9: "CFA_ERR_NOMEM", -10: "CFA_ERR_DTYPE", -11: "CFA_ERR_ALIGN",
           -12: "CFA_ERR_DEVICE", -13: "CFA_ERR_SHAPE"}
 DTYPE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7}
-ENTRY_CAST_BF16, ENTRY_CKSUM = 0x1, 0x2
+ENTRY_CAST_BF16, ENTRY_CKSUM, ENTRY_CONVERT = 0x1, 0x2, 0x4
 OPT_STRICT_COVERAGE, OPT_HOST_ONLY, OPT_TIMING, OPT_BULK, OPT_NO_MERGE = 0x1, 0x2, 0x4, 0x8, 0x10
 SRC_HOST, SRC_PINNED, SRC_CALLBACK, SRC_DEVICE, SRC_HOST_DIRECT = 1, 2, 3, 4, 5
 ALL = -1
@@ -57,13 +57,13 @@ class Stats(ctypes.Structure):
 class Piece(ctypes.Structure):
     _fields_ = [("chunk", ctypes.c_uint32), ("entry", ctypes.c_uint32),
                 ("src_offset", ctypes.c_uint64), ("dst_index", ctypes.c_uint32),
-                ("cast", ctypes.c_uint32), ("dst_offset", ctypes.c_uint64),
+                ("conv", ctypes.c_uint32), ("dst_offset", ctypes.c_uint64),
                 ("n_elems", ctypes.c_uint64), ("rows", ctypes.c_uint32),
                 ("src_row_stride", ctypes.c_uint32)]
 
 
 PIECE_DTYPE = np.dtype([("chunk", "<u4"), ("entry", "<u4"), ("src_offset", "<u8"),
-                        ("dst_index", "<u4"), ("cast", "<u4"), ("dst_offset", "<u8"),
+                        ("dst_index", "<u4"), ("conv", "<u4"), ("dst_offset", "<u8"),
                         ("n_elems", "<u8"), ("rows", "<u4"), ("src_row_stride", "<u4")])
 
 # Every function cfa.h declares, with its ctypes signature.

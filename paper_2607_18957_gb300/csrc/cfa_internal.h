@@ -51,13 +51,33 @@ typedef struct cfa_swork {
 
 #define CFA_NO_CK 0xFFFFFFFFu
 
+/* Element conversions (cfa_work.mode bits 4-7, cfa_piece.conv). */
+#define CFA_CONV_NONE 0
+#define CFA_CONV_F32_BF16 1
+#define CFA_CONV_F32_F16 2
+#define CFA_CONV_F16_BF16 3
+#define CFA_CONV_BF16_F32 4
+#define CFA_CONV_F16_F32 5
+#define CFA_N_CONV 6
+
 /* Work classes: one specialised kernel each.  0..3 = plain copy of 1, 2, 4, 8-byte elements;
- * 4 = fp32 -> bf16 cast. */
-#define CFA_N_CLASSES 5
-#define CFA_CLASS_CAST 4
-#define CFA_MODE_CAST 0x10u
-#define CFA_MODE(src_log2, dst_log2, cast) \
-    ((uint32_t)(src_log2) | ((uint32_t)(dst_log2) << 2) | ((cast) ? CFA_MODE_CAST : 0u))
+ * 3 + conv = conversion `conv`. */
+#define CFA_N_CLASSES 9
+#define CFA_CLASS_OF_CONV(conv) (3 + (conv))
+#define CFA_MODE(src_log2, dst_log2, conv) \
+    ((uint32_t)(src_log2) | ((uint32_t)(dst_log2) << 2) | ((uint32_t)(conv) << 4))
+#define CFA_MODE_CONV(mode) (((mode) >> 4) & 15u)
+
+/* Conversion for a (source, destination) dtype pair, 0 if the pair has none. */
+static inline int cfa_conversion(int32_t src, int32_t dst)
+{
+    if (src == CFA_DTYPE_F32 && dst == CFA_DTYPE_BF16) return CFA_CONV_F32_BF16;
+    if (src == CFA_DTYPE_F32 && dst == CFA_DTYPE_F16) return CFA_CONV_F32_F16;
+    if (src == CFA_DTYPE_F16 && dst == CFA_DTYPE_BF16) return CFA_CONV_F16_BF16;
+    if (src == CFA_DTYPE_BF16 && dst == CFA_DTYPE_F32) return CFA_CONV_BF16_F32;
+    if (src == CFA_DTYPE_F16 && dst == CFA_DTYPE_F32) return CFA_CONV_F16_F32;
+    return CFA_CONV_NONE;
+}
 
 /* Host side of a plan: everything cfa_plan_create computes before touching the GPU. */
 typedef struct cfa_host_plan {

@@ -94,12 +94,12 @@ cfa_status fail(cfa_status st, const char *msg, size_t i)
 /* Placement of one entry: element count, element sizes and destination byte offset. */
 cfa_status place(const cfa_tensor_entry &e, const cfa_dst *dsts, size_t n_dsts,
                  uint64_t blob_bytes, size_t i, uint64_t *n_out, int *es_s, int *es_d,
-                 uint64_t *dst_off)
+                 uint64_t *dst_off, int *conv)
 {
     *es_s = dtype_size(e.src_dtype);
     if (!*es_s || e.ndim < 0 || e.ndim > CFA_MAX_DIMS || e.dst_index < 0 ||
         (size_t)e.dst_index >= n_dsts || e.src_row_stride ||
-        (e.flags & ~(CFA_ENTRY_CAST_BF16 | CFA_ENTRY_CKSUM)))
+        (e.flags & ~(CFA_ENTRY_CAST_BF16 | CFA_ENTRY_CKSUM | CFA_ENTRY_CONVERT)))
         return fail(CFA_ERR_INVAL,
                     "bad dtype, ndim, flags or destination index, or a strided entry (strided "
                     "entries need cfa_plan_create)", i);
@@ -107,11 +107,13 @@ cfa_status place(const cfa_tensor_entry &e, const cfa_dst *dsts, size_t n_dsts,
     const int es_dst = dtype_size(d.dtype);
     if (!es_dst || d.ndim < 0 || d.ndim > CFA_MAX_DIMS)
         return fail(CFA_ERR_INVAL, "bad destination dtype or ndim", i);
-    const bool cast = (e.flags & CFA_ENTRY_CAST_BF16) != 0;
-    if (cast ? (e.src_dtype != CFA_DTYPE_F32 || d.dtype != CFA_DTYPE_BF16)
-             : (e.src_dtype != d.dtype))
+    const bool converts = (e.flags & (CFA_ENTRY_CAST_BF16 | CFA_ENTRY_CONVERT)) != 0;
+    *conv = converts ? cfa_conversion(e.src_dtype, d.dtype) : CFA_CONV_NONE;
+    if (converts ? (*conv == CFA_CONV_NONE ||
+                    ((e.flags & CFA_ENTRY_CAST_BF16) && *conv != CFA_CONV_F32_BF16))
+                 : (e.src_dtype != d.dtype))
         return fail(CFA_ERR_DTYPE, "dtype does not match the destination", i);
-    *es_d = cast ? 2 : *es_s;
+    *es_d = es_dst;
     uint64_t n = 1, d_numel = 1;
     for (int k = 0; k < e.ndim; ++k) {
         if (e.shape[k] < 0) return fail(CFA_ERR_INVAL, "negative dimension", i);
@@ -206,11 +208,12 @@ extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t
     uint32_t count[CFA_N_CLASSES][2] = {};
     for (size_t i = 0; i < n_entries; ++i) {
         uint64_t n, off;
-        int es_s, es_d;
-        cfa_status st = place(entries[i], dsts, n_dsts, blob_bytes, i, &n, &es_s, &es_d, &off);
+        int es_s, es_d, conv;
+        cfa_status st =
+            place(entries[i], dsts, n_dsts, blob_bytes, i, &n, &es_s, &es_d, &off, &conv);
         if (st) return st;
         if (!n) continue;
-        const int cls = (entries[i].flags & CFA_ENTRY_CAST_BF16) ? CFA_CLASS_CAST : log2_es(es_s);
+        const int cls = conv ? CFA_CLASS_OF_CONV(conv) : log2_es(es_s);
         const uint64_t nb = n * (uint64_t)es_d;
         const uint64_t items = nb < kTinyBytes ? 1 : (nb + kSlabBytes - 1) / kSlabBytes;
         uint64_t total = items;
@@ -234,14 +237,13 @@ extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t
         }
     for (size_t i = 0; i < n_entries; ++i) {
         uint64_t n, off;
-        int es_s, es_d;
-        place(entries[i], dsts, n_dsts, blob_bytes, i, &n, &es_s, &es_d, &off);
+        int es_s, es_d, conv;
+        place(entries[i], dsts, n_dsts, blob_bytes, i, &n, &es_s, &es_d, &off, &conv);
         if (!n) continue;
-        const bool cast = (entries[i].flags & CFA_ENTRY_CAST_BF16) != 0;
-        const int cls = cast ? CFA_CLASS_CAST : log2_es(es_s);
+        const int cls = conv ? CFA_CLASS_OF_CONV(conv) : log2_es(es_s);
         cfa_work w;
         w.ck = (cksum_dev && (entries[i].flags & CFA_ENTRY_CKSUM)) ? (uint32_t)i : CFA_NO_CK;
-        w.mode = CFA_MODE(log2_es(es_s), log2_es(es_d), cast);
+        w.mode = CFA_MODE(log2_es(es_s), log2_es(es_d), conv);
         w.pad = (uint32_t)cls;
         const uint64_t dst0 = (uint64_t)(uintptr_t)dsts[entries[i].dst_index].dev_ptr + off;
         const uint64_t nb = n * (uint64_t)es_d;

@@ -104,6 +104,7 @@ static int vec_push(vec *v, const void *x)
 typedef struct {
     uint64_t n;       /* elements */
     int es_s, es_d;   /* element sizes */
+    int conv;         /* CFA_CONV_* */
     uint64_t dst_off; /* byte offset inside the destination */
     uint64_t cols;    /* elements per row (the last dimension) */
     uint64_t stride;  /* source elements between row starts; == cols when contiguous */
@@ -353,7 +354,7 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         const cfa_tensor_entry *e = &entries[i];
         const int es_s = cfa_dtype_size(e->src_dtype);
         if (!es_s || e->ndim < 0 || e->ndim > CFA_MAX_DIMS ||
-            (e->flags & ~(CFA_ENTRY_CAST_BF16 | CFA_ENTRY_CKSUM))) {
+            (e->flags & ~(CFA_ENTRY_CAST_BF16 | CFA_ENTRY_CKSUM | CFA_ENTRY_CONVERT))) {
             fail(err, errlen, "entry %zu (%s): bad dtype, ndim or flags", i, ename(e));
             st = CFA_ERR_INVAL;
             goto done;
@@ -370,15 +371,17 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
             goto done;
         }
         const cfa_dst *d = &dsts[e->dst_index];
-        const int cast = (e->flags & CFA_ENTRY_CAST_BF16) != 0;
-        if (cast ? (e->src_dtype != CFA_DTYPE_F32 || d->dtype != CFA_DTYPE_BF16)
-                 : (e->src_dtype != d->dtype)) {
+        const int converts = (e->flags & (CFA_ENTRY_CAST_BF16 | CFA_ENTRY_CONVERT)) != 0;
+        const int conv = converts ? cfa_conversion(e->src_dtype, d->dtype) : CFA_CONV_NONE;
+        if (converts ? (conv == CFA_CONV_NONE ||
+                        ((e->flags & CFA_ENTRY_CAST_BF16) && conv != CFA_CONV_F32_BF16))
+                     : (e->src_dtype != d->dtype)) {
             fail(err, errlen, "entry %zu (%s): dtype does not match its destination", i,
                  ename(e));
             st = CFA_ERR_DTYPE;
             goto done;
         }
-        const int es_d = cast ? 2 : es_s;
+        const int es_d = cfa_dtype_size(d->dtype);
         uint64_t n = 1;
         for (int k = 0; k < e->ndim; ++k) {
             if (e->shape[k] < 0 || mul_overflows(n, (uint64_t)e->shape[k], &n)) {
@@ -434,6 +437,7 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         info[i].n = n;
         info[i].es_s = es_s;
         info[i].es_d = es_d;
+        info[i].conv = conv;
         info[i].dst_off = first * (uint64_t)es_d;
         info[i].cols = cols;
         info[i].stride = stride;
@@ -492,7 +496,7 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
             memset(&pc, 0, sizeof pc);
             pc.entry = (uint32_t)i;
             pc.dst_index = (uint32_t)entries[i].dst_index;
-            pc.cast = (entries[i].flags & CFA_ENTRY_CAST_BF16) ? 1u : 0u;
+            pc.conv = (uint32_t)in->conv;
             pc.rows = 1;
             const uint64_t es_s = (uint64_t)in->es_s, es_d = (uint64_t)in->es_d;
             const uint64_t a0 = entries[i].blob_offset;
@@ -570,8 +574,9 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
             const ent_info *in = &info[pc->entry];
             const cfa_tensor_entry *e = &entries[pc->entry];
             const uint32_t ck = (e->flags & CFA_ENTRY_CKSUM) ? pc->entry : CFA_NO_CK;
-            const uint32_t mode = CFA_MODE(log2_small(in->es_s), log2_small(in->es_d), pc->cast);
-            const uint32_t cls = pc->cast ? CFA_CLASS_CAST : (uint32_t)log2_small(in->es_s);
+            const uint32_t mode = CFA_MODE(log2_small(in->es_s), log2_small(in->es_d), pc->conv);
+            const uint32_t cls =
+                pc->conv ? CFA_CLASS_OF_CONV(pc->conv) : (uint32_t)log2_small(in->es_s);
             const uint64_t a0 = (uint64_t)(uintptr_t)dsts[pc->dst_index].dev_ptr + pc->dst_offset;
             if (pc->rows > 1) {
                 /* blocks of whole rows, about slab_bytes of destination each */
@@ -617,7 +622,7 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
                 w.src = pc->src_offset + (pos - a0) / (uint64_t)in->es_d * (uint64_t)in->es_s;
                 w.n = (uint32_t)((next - pos) / (uint64_t)in->es_d);
                 const int aligned = ((w.src | w.dst | (next - pos)) & 15u) == 0;
-                if (use_bulk && !pc->cast && aligned) {
+                if (use_bulk && !pc->conv && aligned) {
                     if (vec_push(&bulk, &w)) { st = CFA_ERR_NOMEM; goto done; }
                 } else {
                     if (vec_push(&slabs, &w)) { st = CFA_ERR_NOMEM; goto done; }

@@ -15,7 +15,8 @@
  *     grow with the number of work items;
  *   - source and destination offsets that differ modulo 16 are realigned in registers (two
  *     aligned loads and a funnel shift per 16-byte store), so stores stay 16 bytes wide;
- *   - the fp32 -> bf16 cast rounds to nearest even on the bit pattern with integer operations;
+ *   - dtype conversions (fp32 -> bf16 / fp16, fp16 -> bf16 with round-to-nearest-even;
+ *     bf16 / fp16 -> fp32 exactly) work on bit patterns with integer operations;
  *   - checksums are sums modulo 2^64 of the destination element bit patterns, reduced inside the
  *     CTA or warp and added with one 64-bit atomic per (CTA, run of same-tensor slabs) or per
  *     tiny piece; integer addition is associative, so the result does not depend on the order.
@@ -131,6 +132,58 @@ __device__ __forceinline__ uint32_t bf16_rne(uint32_t u)
     return ((u & 0x7FFFFFFFu) > 0x7F800000u) ? 0x7FC0u : rounded;
 }
 
+/* fp32 bit pattern -> fp16 bit pattern, round to nearest, ties to even.  Magnitudes from
+ * 65520 (the largest half, 65504, plus half its ulp) up become infinity; below 2^-14 the result
+ * is the subnormal m * 2^-24 with m the 24-bit significand shifted right with the same
+ * rounding; NaNs become sign | 0x7E00. */
+__device__ __forceinline__ uint32_t f16_rne(uint32_t u)
+{
+    const uint32_t sign = (u >> 16) & 0x8000u;
+    const uint32_t a = u & 0x7FFFFFFFu;
+    if (a > 0x7F800000u) return sign | 0x7E00u;
+    if (a >= 0x477FF000u) return sign | 0x7C00u;
+    if (a >= 0x38800000u) /* normal: rebias the exponent by 112, keep 10 mantissa bits */
+        return sign | ((a - 0x38000000u + 0xFFFu + ((a >> 13) & 1u)) >> 13);
+    const uint32_t e = a >> 23;
+    if (e < 102) return sign; /* below 2^-25: rounds to zero */
+    const uint32_t sig = (a & 0x7FFFFFu) | 0x800000u;
+    const uint32_t sh = 126u - e; /* 14 .. 24 */
+    const uint32_t q = sig >> sh, rem = sig & ((1u << sh) - 1u), half = 1u << (sh - 1u);
+    return sign | (q + ((rem > half) || (rem == half && (q & 1u)) ? 1u : 0u));
+}
+
+/* fp16 bit pattern -> fp32 bit pattern, exact (subnormals normalised, NaN payloads kept). */
+__device__ __forceinline__ uint32_t f16_to_f32(uint32_t h)
+{
+    const uint32_t sign = (h & 0x8000u) << 16;
+    const uint32_t e = (h >> 10) & 0x1Fu, m = h & 0x3FFu;
+    if (e == 0x1Fu) return sign | 0x7F800000u | (m << 13);
+    if (e != 0) return sign | ((e + 112u) << 23) | (m << 13);
+    if (m == 0) return sign;
+    const uint32_t p = 31u - __clz(m); /* highest set bit, 0 .. 9 */
+    return sign | ((p + 103u) << 23) | ((m << (23u - p)) & 0x7FFFFFu);
+}
+
+template <int CONV> __device__ __forceinline__ uint32_t convert1(uint32_t x)
+{
+    if constexpr (CONV == CFA_CONV_F32_BF16) return bf16_rne(x);
+    else if constexpr (CONV == CFA_CONV_F32_F16) return f16_rne(x);
+    else if constexpr (CONV == CFA_CONV_F16_BF16) return bf16_rne(f16_to_f32(x));
+    else if constexpr (CONV == CFA_CONV_BF16_F32) return x << 16;
+    else return f16_to_f32(x);
+}
+
+/* Source element size, destination element size and conversion of a work class. */
+template <int CLS> struct ClassOf {
+    static constexpr int conv = CLS >= 4 ? CLS - 3 : 0;
+    static constexpr int ses = conv == 0 ? (1 << CLS)
+                               : (conv == CFA_CONV_F32_BF16 || conv == CFA_CONV_F32_F16) ? 4 : 2;
+    static constexpr int des = conv == 0 ? (1 << CLS)
+                               : (conv == CFA_CONV_BF16_F32 || conv == CFA_CONV_F16_F32) ? 4 : 2;
+    static constexpr int log2(int x) { return x == 1 ? 0 : x == 2 ? 1 : x == 4 ? 2 : 3; }
+    static constexpr uint32_t mode = CFA_MODE(log2(ses), log2(des), conv);
+};
+
 /* ---- copy of one contiguous run --------------------------------------------------------- */
 
 template <int ES>
@@ -201,75 +254,77 @@ __device__ uint64_t copy_run(const uint8_t *__restrict__ src, uint8_t *__restric
     return acc;
 }
 
-/* n fp32 elements at src -> n bf16 elements at dst. */
-template <int U>
-__device__ uint64_t cast_run(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst,
-                             uint64_t n, uint32_t tid, uint32_t nthr)
+/* n elements of SES bytes at src -> n converted elements of DES bytes at dst.  Destination
+ * stores are 16 bytes wide; eight elements form a group (32 or 16 source bytes, 16 or 32
+ * destination bytes), loaded as 16-byte vectors when the source is aligned, else one by one. */
+template <int SES, int DES, int CONV, int U>
+__device__ uint64_t convert_run(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst,
+                                uint64_t n, uint32_t tid, uint32_t nthr)
 {
+    typedef typename Elem<SES>::T ST;
+    typedef typename Elem<DES>::T DT;
     uint64_t acc = 0;
-    uint32_t h = (uint32_t)(((16u - ((uintptr_t)dst & 15u)) & 15u) >> 1);
+    uint32_t h = (uint32_t)(((16u - ((uintptr_t)dst & 15u)) & 15u) / DES);
     if (h > n) h = (uint32_t)n;
     for (uint32_t e = tid; e < h; e += nthr) {
-        const uint32_t y = bf16_rne(reinterpret_cast<const uint32_t *>(src)[e]);
-        reinterpret_cast<uint16_t *>(dst)[e] = (uint16_t)y;
+        const uint32_t y = convert1<CONV>(reinterpret_cast<const ST *>(src)[e]);
+        reinterpret_cast<DT *>(dst)[e] = (DT)y;
         acc += y;
     }
-    src += 4u * h;
-    dst += 2u * h;
+    src += (uint64_t)SES * h;
+    dst += (uint64_t)DES * h;
     n -= h;
 
-    const uint32_t ng = (uint32_t)(n >> 3); /* groups of 8: 32 source bytes, one 16-byte store */
+    const uint32_t ng = (uint32_t)(n >> 3);
     uint4 *d = reinterpret_cast<uint4 *>(dst);
-    if (((uintptr_t)src & 15u) == 0) {
-        const uint4 *s = reinterpret_cast<const uint4 *>(src);
-        const uint32_t step = nthr * U;
-        for (uint32_t base = 0; base < ng; base += step) {
-            uint4 a[U], b[U];
+    const bool vec = ((uintptr_t)src & 15u) == 0;
+    const uint32_t step = nthr * U;
+    for (uint32_t base = 0; base < ng; base += step) {
+        uint32_t x[U][8];
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const uint32_t g = base + u * nthr + tid;
-                if (g < ng) {
-                    a[u] = ld_stream(s + 2 * g);
-                    b[u] = ld_stream(s + 2 * g + 1);
-                }
-            }
+        for (int u = 0; u < U; ++u) {
+            const uint32_t g = base + u * nthr + tid;
+            if (g >= ng) continue;
+            if (vec && SES == 4) {
+                const uint4 a = ld_stream(src + 32ull * g), b = ld_stream(src + 32ull * g + 16);
+                x[u][0] = a.x; x[u][1] = a.y; x[u][2] = a.z; x[u][3] = a.w;
+                x[u][4] = b.x; x[u][5] = b.y; x[u][6] = b.z; x[u][7] = b.w;
+            } else if (vec && SES == 2) {
+                const uint4 a = ld_stream(src + 16ull * g);
+                x[u][0] = a.x & 0xFFFFu; x[u][1] = a.x >> 16; x[u][2] = a.y & 0xFFFFu;
+                x[u][3] = a.y >> 16; x[u][4] = a.z & 0xFFFFu; x[u][5] = a.z >> 16;
+                x[u][6] = a.w & 0xFFFFu; x[u][7] = a.w >> 16;
+            } else {
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const uint32_t g = base + u * nthr + tid;
-                if (g < ng) {
-                    const uint32_t r0 = bf16_rne(a[u].x), r1 = bf16_rne(a[u].y);
-                    const uint32_t r2 = bf16_rne(a[u].z), r3 = bf16_rne(a[u].w);
-                    const uint32_t r4 = bf16_rne(b[u].x), r5 = bf16_rne(b[u].y);
-                    const uint32_t r6 = bf16_rne(b[u].z), r7 = bf16_rne(b[u].w);
-                    uint4 o;
-                    o.x = r0 | (r1 << 16);
-                    o.y = r2 | (r3 << 16);
-                    o.z = r4 | (r5 << 16);
-                    o.w = r6 | (r7 << 16);
-                    st_stream(d + g, o);
-                    acc += (uint64_t)(r0 + r1 + r2 + r3) + (r4 + r5 + r6 + r7);
-                }
+                for (int q = 0; q < 8; ++q)
+                    x[u][q] = reinterpret_cast<const ST *>(src)[8ull * g + q];
             }
         }
-    } else {
-        const uint32_t *s = reinterpret_cast<const uint32_t *>(src);
-        for (uint32_t g = tid; g < ng; g += nthr) {
-            uint32_t r[8];
 #pragma unroll
-            for (int q = 0; q < 8; ++q) r[q] = bf16_rne(s[8 * g + q]);
-            uint4 o;
-            o.x = r[0] | (r[1] << 16);
-            o.y = r[2] | (r[3] << 16);
-            o.z = r[4] | (r[5] << 16);
-            o.w = r[6] | (r[7] << 16);
-            st_stream(d + g, o);
-            acc += (uint64_t)(r[0] + r[1] + r[2] + r[3]) + (r[4] + r[5] + r[6] + r[7]);
+        for (int u = 0; u < U; ++u) {
+            const uint32_t g = base + u * nthr + tid;
+            if (g >= ng) continue;
+            uint32_t r[8];
+            uint64_t sum = 0;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                r[q] = convert1<CONV>(x[u][q]);
+                sum += r[q];
+            }
+            if constexpr (DES == 2) {
+                st_stream(d + g, make_uint4(r[0] | (r[1] << 16), r[2] | (r[3] << 16),
+                                            r[4] | (r[5] << 16), r[6] | (r[7] << 16)));
+            } else {
+                st_stream(d + 2ull * g, make_uint4(r[0], r[1], r[2], r[3]));
+                st_stream(d + 2ull * g + 1, make_uint4(r[4], r[5], r[6], r[7]));
+            }
+            acc += sum;
         }
     }
     const uint64_t body = (uint64_t)ng << 3;
     for (uint64_t e = body + tid; e < n; e += nthr) {
-        const uint32_t y = bf16_rne(reinterpret_cast<const uint32_t *>(src)[e]);
-        reinterpret_cast<uint16_t *>(dst)[e] = (uint16_t)y;
+        const uint32_t y = convert1<CONV>(reinterpret_cast<const ST *>(src)[e]);
+        reinterpret_cast<DT *>(dst)[e] = (DT)y;
         acc += y;
     }
     return acc;
@@ -281,7 +336,7 @@ __device__ __forceinline__ bool item_ok(const cfa_work &w, const UnpackArgs &a)
 {
     const uint32_t sl = w.mode & 3u;
     const uint64_t src_bytes = (uint64_t)w.n << sl;
-    const uint32_t want_mode = CLS == CFA_CLASS_CAST ? CFA_MODE(2, 1, 1) : CFA_MODE(CLS, CLS, 0);
+    const uint32_t want_mode = ClassOf<CLS>::mode;
     const uint32_t dl = (w.mode >> 2) & 3u;
     return w.mode == want_mode && w.n != 0 && w.src >= a.src_lo && w.src <= a.src_hi &&
            src_bytes <= a.src_hi - w.src && (w.src & ((1ull << sl) - 1)) == 0 &&
@@ -295,8 +350,9 @@ __device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs
     const uint64_t off = a.src_period ? w.src % a.src_period : w.src;
     const uint8_t *src = reinterpret_cast<const uint8_t *>(a.src_base + off);
     uint8_t *dst = reinterpret_cast<uint8_t *>(w.dst);
-    if constexpr (CLS == CFA_CLASS_CAST)
-        return cast_run<(U > 2 ? 2 : U)>(src, dst, w.n, tid, nthr);
+    typedef ClassOf<CLS> C;
+    if constexpr (C::conv != CFA_CONV_NONE)
+        return convert_run<C::ses, C::des, C::conv, (U > 2 ? 2 : U)>(src, dst, w.n, tid, nthr);
     else
         return copy_run<(1 << CLS), U>(src, dst, (uint64_t)w.n << CLS, tid, nthr);
 }
@@ -384,7 +440,7 @@ struct StridedArgs {
 template <int CLS>
 __device__ __forceinline__ bool sitem_ok(const cfa_swork &w, const StridedArgs &a)
 {
-    const uint32_t want_mode = CLS == CFA_CLASS_CAST ? CFA_MODE(2, 1, 1) : CFA_MODE(CLS, CLS, 0);
+    const uint32_t want_mode = ClassOf<CLS>::mode;
     if (w.mode != want_mode || w.rows == 0 || w.cols == 0 || w.stride < w.cols) return false;
     const uint32_t sl = w.mode & 3u, dl = (w.mode >> 2) & 3u;
     const uint64_t extent = ((uint64_t)(w.rows - 1) * w.stride + w.cols) << sl;
@@ -398,8 +454,9 @@ __device__ __forceinline__ bool sitem_ok(const cfa_swork &w, const StridedArgs &
 template <int CLS>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_strided_kernel(const StridedArgs a)
 {
-    constexpr int SES = CLS == CFA_CLASS_CAST ? 4 : (1 << CLS);
-    constexpr int DES = CLS == CFA_CLASS_CAST ? 2 : (1 << CLS);
+    typedef ClassOf<CLS> C;
+    constexpr int SES = C::ses;
+    constexpr int DES = C::des;
     __shared__ unsigned long long red[kWarps];
     const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
     uint64_t acc = 0;
@@ -421,8 +478,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_strided_kernel(const
         for (uint32_t r = warp; r < w.rows; r += kWarps) {
             const uint8_t *s = src + (uint64_t)r * w.stride * SES;
             uint8_t *d = dst + (uint64_t)r * w.cols * DES;
-            if constexpr (CLS == CFA_CLASS_CAST)
-                acc += cast_run<2>(s, d, w.cols, lane, 32u);
+            if constexpr (C::conv != CFA_CONV_NONE)
+                acc += convert_run<SES, DES, C::conv, 2>(s, d, w.cols, lane, 32u);
             else
                 acc += copy_run<DES, kUnroll>(s, d, (uint64_t)w.cols * DES, lane, 32u);
         }
@@ -431,14 +488,16 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_strided_kernel(const
 }
 
 typedef void (*strided_fn)(const StridedArgs);
-const strided_fn kStrided[CFA_N_CLASSES] = {cfa_strided_kernel<0>, cfa_strided_kernel<1>,
-                                            cfa_strided_kernel<2>, cfa_strided_kernel<3>,
-                                            cfa_strided_kernel<CFA_CLASS_CAST>};
+const strided_fn kStrided[CFA_N_CLASSES] = {
+    cfa_strided_kernel<0>, cfa_strided_kernel<1>, cfa_strided_kernel<2>,
+    cfa_strided_kernel<3>, cfa_strided_kernel<4>, cfa_strided_kernel<5>,
+    cfa_strided_kernel<6>, cfa_strided_kernel<7>, cfa_strided_kernel<8>};
 
 typedef void (*kernel_fn)(const UnpackArgs);
-const kernel_fn kKernels[CFA_N_CLASSES] = {cfa_unpack_kernel<0>, cfa_unpack_kernel<1>,
-                                           cfa_unpack_kernel<2>, cfa_unpack_kernel<3>,
-                                           cfa_unpack_kernel<CFA_CLASS_CAST>};
+const kernel_fn kKernels[CFA_N_CLASSES] = {
+    cfa_unpack_kernel<0>, cfa_unpack_kernel<1>, cfa_unpack_kernel<2>,
+    cfa_unpack_kernel<3>, cfa_unpack_kernel<4>, cfa_unpack_kernel<5>,
+    cfa_unpack_kernel<6>, cfa_unpack_kernel<7>, cfa_unpack_kernel<8>};
 
 } // namespace
 

@@ -21,6 +21,11 @@ def rne_cases():
     return [(int(t[0], 16), int(t[1], 16)) for t in _lines("rne_cases.txt")]
 
 
+def f16_cases():
+    """[(direction, input bits, expected bits)] from f16_cases.txt."""
+    return [(t[0], int(t[1], 16), int(t[2], 16)) for t in _lines("f16_cases.txt")]
+
+
 def manifest_case(name):
     """(Manifest, blob uint8 array, {dst: expected bytes}, expected checksums)."""
     blob, dsts, entries, exp_dst, exp_ck, blob_bytes = None, [], [], {}, None, None

@@ -16,6 +16,10 @@ What pins what:
   tp_shards           tensor-parallel shards: each equals numpy slicing of the full tensor, and
                       the shards of all ranks reassemble (numpy concatenate) into the unsharded
                       load
+  f16_golden          hand-derived binary16 conversion cases (tests/golden/f16_cases.txt)
+  convert_vs_torch    torch's CPU conversions float16 <-> float32, float16 / float32 ->
+                      bfloat16, bfloat16 -> float32 (exhaustive over 16-bit inputs)
+  f16_vs_nearest      the definition of round-to-nearest-even into binary16, in fp64
 """
 import numpy as np
 import torch
@@ -23,7 +27,7 @@ import torch
 import oracle
 from workloads import DTYPE_SIZE, Manifest, dense_config, moe_config, tiny_config
 
-from _golden import manifest_case, rne_cases
+from _golden import f16_cases, manifest_case, rne_cases
 
 
 # ---------------------------------------------------------------------------------------------
@@ -32,6 +36,43 @@ from _golden import manifest_case, rne_cases
 def _torch_bf16_bits(u32):
     f = torch.from_numpy(np.ascontiguousarray(u32, dtype=np.uint32).view(np.float32))
     return f.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+
+
+_TORCH = {"f32": torch.float32, "bf16": torch.bfloat16, "f16": torch.float16}
+_BITS = {"f32": (np.uint32, torch.int32), "bf16": (np.uint16, torch.int16),
+         "f16": (np.uint16, torch.int16)}
+
+
+def torch_convert_bits(src, dst, bits):
+    """torch's CPU conversion of src-dtype bit patterns to dst-dtype bit patterns."""
+    np_s, t_s = _BITS[src]
+    np_d, t_d = _BITS[dst]
+    t = torch.from_numpy(np.ascontiguousarray(bits, dtype=np_s).view(
+        {np.uint32: np.int32, np.uint16: np.int16}[np_s])).view(_TORCH[src])
+    return t.to(_TORCH[dst]).view(t_d).numpy().view(np_d)
+
+
+def _nan_mask(dtype, bits):
+    bits = np.asarray(bits)
+    if dtype == "f32":
+        b = bits.astype(np.uint32)
+        return ((b & 0x7F800000) == 0x7F800000) & ((b & 0x7FFFFF) != 0)
+    b = bits.astype(np.uint32)
+    if dtype == "bf16":
+        return ((b & 0x7F80) == 0x7F80) & ((b & 0x7F) != 0)
+    return ((b & 0x7C00) == 0x7C00) & ((b & 0x3FF) != 0)
+
+
+def check_convert_block(src, dst, bits, lib=None):
+    """Oracle conversion vs torch: bit-equal unless the input is NaN; then both are NaN."""
+    got = oracle.convert(src, dst, bits, lib=lib)
+    ref = torch_convert_bits(src, dst, bits)
+    nan = _nan_mask(src, bits)
+    bad = (~nan) & (got != ref)
+    assert not bad.any(), f"{src}->{dst}({int(np.asarray(bits)[bad][0]):#x}): " \
+                          f"{int(got[bad][0]):#x} vs torch {int(ref[bad][0]):#x}"
+    if nan.any():
+        assert _nan_mask(dst, got[nan]).all() and _nan_mask(dst, ref[nan]).all()
 
 
 def _is_nan32(u32):
@@ -158,7 +199,8 @@ def _expected_by_concat(m, blob):
         for i in sorted(m.entries_of_dst(j), key=lambda i: int(m.e_row[i])):
             sl = _source_elements(m, blob, i)
             if m.e_cast[i]:
-                sl = _torch_bf16_bits(sl.view(np.uint32)).view(np.uint8)
+                src, dst = str(m.e_dtype[i]), str(m.d_dtype[j])
+                sl = torch_convert_bits(src, dst, sl.view(_BITS[src][0])).view(np.uint8)
             parts.append(sl)
         out[j] = np.concatenate(parts) if parts else np.zeros(0, np.uint8)
         assert out[j].size == m.d_nbytes(j)
@@ -234,6 +276,11 @@ def cast_reference(lib=None):
     m = _mini_dense("f32", seed=32)
     assert m.e_cast.all()
     _check_against_concat(m, lib)
+    # the other conversions: fp32 -> fp16, fp16 -> bf16 with fp32 norms, bf16 -> fp32 norms
+    for src, dst, norm in (("f32", "f16", None), ("f16", "bf16", "f32"), ("bf16", "bf16", "f32")):
+        m = _mini_dense(src, seed=33, dst_dtype=dst, norm_dtype=norm)
+        assert m.e_cast.any()
+        _check_against_concat(m, lib)
 
 
 def invariants(lib=None):
@@ -422,5 +469,66 @@ def _kv_rows(full, qkv_name):
     return int(full.e_shape[i, 0])
 
 
+def f16_golden(lib=None):
+    for direction, x, want in f16_cases():
+        if direction == "f32>f16":
+            got = oracle.f32_to_f16_scalar(x, lib=lib)
+        else:
+            got = int(oracle.convert("f16", "f32", np.array([x], np.uint16), lib=lib)[0])
+        assert got == want, f"{direction}({x:#x}) = {got:#x}, want {want:#x}"
+
+
+def convert_vs_torch(lib=None):
+    all16 = np.arange(1 << 16, dtype=np.uint32).astype(np.uint16)
+    for src, dst in (("f16", "f32"), ("f16", "bf16"), ("bf16", "f32")):
+        check_convert_block(src, dst, all16, lib)
+    # f32 -> f16: every sign/exponent/upper fraction pattern with the low 13 bits that decide
+    # the rounding, plus random patterns (all 2^32 in test_convert_exhaustive_vs_torch)
+    hi = np.arange(1 << 19, dtype=np.uint32) << 13
+    lows = np.array([0, 1, 0xFFF, 0x1000, 0x1001, 0x1FFF], dtype=np.uint32)
+    check_convert_block("f32", "f16", (hi[:, None] | lows[None, :]).ravel(), lib)
+    rng = np.random.default_rng(13)
+    check_convert_block("f32", "f16",
+                        rng.integers(0, 1 << 32, size=1 << 20, dtype=np.uint64).astype(np.uint32),
+                        lib)
+
+
+def _f16_value(b16):
+    b = np.asarray(b16, dtype=np.uint32)
+    e = (b >> 10) & 31
+    m = (b & 1023).astype(np.float64)
+    v = np.where(e == 0, np.ldexp(m, -24), np.ldexp(1024.0 + m, e.astype(np.int64) - 25))
+    return np.where(b & 0x8000, -v, v)
+
+
+def f16_vs_nearest(lib=None):
+    """For finite x below the overflow threshold the result must be the nearer of the two
+    binary16 values bracketing x (candidates from a sorted table of all finite halves), the
+    one with an even last fraction bit on a tie."""
+    rng = np.random.default_rng(14)
+    u = rng.integers(0, 1 << 32, size=1 << 18, dtype=np.uint64).astype(np.uint32)
+    mant = rng.integers(0, 1 << 23, size=1 << 18, dtype=np.uint64).astype(np.uint32)
+    expo = rng.integers(100, 145, size=1 << 18, dtype=np.uint64).astype(np.uint32)
+    u = np.concatenate([u, (expo << 23) | mant, ((expo << 23) | (mant & ~np.uint32(0x1FFF)) |
+                                                 0x1000)])
+    x = u.view(np.float32).astype(np.float64)
+    keep = np.isfinite(x) & (np.abs(x) < 65520.0)
+    u, x = u[keep], x[keep]
+    pos = np.arange(0x7C00, dtype=np.uint32)            # every finite non-negative half
+    vals = _f16_value(pos)                               # increasing
+    ax = np.abs(x)
+    k = np.searchsorted(vals, ax, side="right") - 1      # vals[k] <= ax < vals[k + 1]
+    lo = pos[k]
+    hi_v = np.where(k + 1 < pos.size, vals[np.minimum(k + 1, pos.size - 1)], 65536.0)
+    dlo, dhi = ax - vals[k], hi_v - ax
+    pick = np.where(dlo < dhi, lo, np.where(dhi < dlo, lo + 1, np.where(lo & 1, lo + 1, lo)))
+    want = (pick | np.where(np.signbit(x), 0x8000, 0)).astype(np.uint32)
+    got = oracle.convert("f32", "f16", u, lib=lib).astype(np.uint32)
+    bad = got != want
+    assert not bad.any(), f"f16({int(u[bad][0]):#010x}) = {int(got[bad][0]):#06x}, " \
+                          f"nearest-even gives {int(want[bad][0]):#06x}"
+
+
 ALL_PINS = [rne_golden, rne_vs_torch, rne_vs_nearest, golden_manifests, one_to_one,
-            concat_reference, cast_reference, invariants, validation, tp_shards]
+            concat_reference, cast_reference, invariants, validation, tp_shards, f16_golden,
+            convert_vs_torch, f16_vs_nearest]

@@ -132,8 +132,30 @@ def cfg_moe_tp():
                       tp=2, rank=0)
 
 
+def cfg_f32_to_f16():
+    return dense_config("f32_to_f16", 71, layers=2, hidden=512, n_q=8, n_kv=2, head_dim=64,
+                        inter=1536, vocab=1000, src_dtype="f32", dst_dtype="f16", align=4,
+                        jitter=3)
+
+
+def cfg_f16_bits_to_bf16():
+    # random 16-bit patterns: every NaN, infinity and subnormal of binary16 occurs; the norms
+    # are widened to fp32
+    return dense_config("f16bits_to_bf16", 72, layers=2, hidden=512, n_q=8, n_kv=2,
+                        head_dim=64, inter=1536, vocab=1000, src_dtype="f16", norm_dtype="f32",
+                        blob_kind="bits", align=2, jitter=5)
+
+
+def cfg_bf16_f32_norms_tp():
+    return dense_config("bf16_f32norm_tp2r0", 73, layers=2, hidden=512, n_q=8, n_kv=2,
+                        head_dim=64, inter=1536, vocab=1000, norm_dtype="f32", align=2,
+                        jitter=5, tp=2, rank=0)
+
+
 CONFIGS = {"tiny": cfg_tiny, "dense": cfg_dense, "dense_f32": cfg_dense_f32, "moe": cfg_moe,
-           "dense_tp": cfg_dense_tp, "f32_tp": cfg_f32_tp, "moe_tp": cfg_moe_tp}
+           "dense_tp": cfg_dense_tp, "f32_tp": cfg_f32_tp, "moe_tp": cfg_moe_tp,
+           "f32_f16": cfg_f32_to_f16, "f16_bf16": cfg_f16_bits_to_bf16,
+           "bf16_f32norm_tp": cfg_bf16_f32_norms_tp}
 
 
 @pytest.mark.parametrize("cfg", list(CONFIGS))
@@ -156,7 +178,7 @@ def test_parity_chunk_sizes(cfg, chunk):
 
 @pytest.mark.parametrize("misalign", [2, 6, 14])
 def test_parity_misaligned_destinations(misalign):
-    for cfg in ("dense", "moe", "dense_f32"):
+    for cfg in ("dense", "moe", "dense_f32", "f32_f16", "f16_bf16", "dense_tp"):
         m = CONFIGS[cfg]()
         load_and_compare(m, "device", chunk=1 << 20, misalign=misalign)
 
@@ -176,8 +198,8 @@ def test_parity_bulk_path(cfg, kind, chunk):
     """With CFA_OPT_BULK the aligned cast-free slabs go through the TMA bulk kernel."""
     m = CONFIGS[cfg]()
     st = load_and_compare(m, kind, chunk=chunk, bulk=True)
-    if cfg == "dense_f32":
-        assert st["n_bulk"] == 0  # casts never take the bulk path
+    if cfg in ("dense_f32", "f32_f16"):
+        assert st["n_bulk"] == 0  # conversions never take the bulk path
 
 
 def test_bulk_path_takes_every_aligned_slab():

@@ -80,9 +80,10 @@ def execute_pieces_on_cpu(m, pieces, blob):
         for k in range(rows):
             a = int(pc["src_offset"]) + k * step
             src = blob[a:a + cols * es_s]
-            if pc["cast"]:
-                f = torch.from_numpy(src.view(np.float32).copy())
-                src = f.to(torch.bfloat16).view(torch.int16).numpy().view(np.uint8)
+            if pc["conv"]:
+                s_dt, d_dt = str(m.e_dtype[i]), str(m.d_dtype[int(pc["dst_index"])])
+                src = _pins.torch_convert_bits(s_dt, d_dt,
+                                               src.view(_pins._BITS[s_dt][0])).view(np.uint8)
             out[int(pc["dst_index"])][o:o + src.size] = src
             o += src.size
     return out
@@ -100,6 +101,11 @@ def mini_configs():
                      jitter=2, tp=4, rank=2),
         moe_config("m_tp2r0", 57, 2, 32, 4, 2, 8, 48, 3, 52, n_extra=30, align=2, jitter=3,
                    tp=2, rank=0),
+        # dtype conversions
+        dense_config("f32_f16", 58, 2, 64, 4, 2, 16, 96, 100, src_dtype="f32", dst_dtype="f16",
+                     align=4, jitter=2),
+        dense_config("f16_bf16", 59, 2, 64, 4, 2, 16, 96, 100, src_dtype="f16",
+                     norm_dtype="f32", align=2, jitter=3, tp=2, rank=1),
     ]
 
 
@@ -196,6 +202,23 @@ def test_bad_options_and_misaligned_destination():
     with pytest.raises(cfa.CfaError) as e:
         cfa.Plan(entries_for(m), d, m.blob_bytes, host_only=True)
     assert e.value.name == "CFA_ERR_ALIGN"
+
+
+def test_conversion_flags():
+    """CFA_ENTRY_CAST_BF16 accepts only fp32 -> bf16; CFA_ENTRY_CONVERT any listed pair."""
+    m = dense_config("conv", 60, 1, 64, 4, 2, 16, 96, 100, src_dtype="f32", dst_dtype="f16",
+                     align=4)
+    ents = entries_for(m)
+    ok = cfa.Plan(ents, fake_dsts(m), m.blob_bytes, host_only=True)
+    ok.close()
+    ents.arr["flags"] = (ents.arr["flags"] & ~np.uint32(_lib.ENTRY_CONVERT)) | _lib.ENTRY_CAST_BF16
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Plan(ents, fake_dsts(m), m.blob_bytes, host_only=True)
+    assert e.value.name == "CFA_ERR_DTYPE"
+    # an unsupported pair (bf16 -> f16) is refused by both sides
+    mb = dense_config("conv2", 61, 1, 64, 4, 2, 16, 96, 100, src_dtype="bf16", dst_dtype="f16")
+    assert _plan_status(mb) == "CFA_ERR_DTYPE"
+    assert oracle.unpack(mb, mb.blob_range(0, mb.blob_bytes)).status == oracle.ORC_E_DTYPE
 
 
 def test_strided_entries_are_validated_like_the_oracle():

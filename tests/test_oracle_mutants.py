@@ -44,12 +44,22 @@ MUTANTS = [
     ("dst_stride_wrong", "dst + i * (uint64_t)es_d", "dst + i * (uint64_t)es_s"),
     ("checksum_of_source", "ck += y;", "ck += x;"),
     ("checksum_misses_last", "ck += y;", "if (i + 1 < n) ck += y;"),
-    ("cast_ignored", "const uint64_t y = cast ? (uint64_t)oracle_rne_bf16((uint32_t)x) : x;",
+    ("cast_ignored", "const uint64_t y = converts ? orc_convert(conv, x) : x;",
      "const uint64_t y = x;"),
     ("oob_check_off_by_elem", "if (base_elem + n > d_numel)", "if (base_elem + n > d_numel + 1)"),
     ("cover_not_counted", "+= 1u;", "+= 0u;"),
     ("stride_ignored", "const uint64_t src_i = (i / C) * stride + (i % C);",
      "const uint64_t src_i = i;"),
+    ("f16_truncates", "double m = nearbyint(ldexp(v, 10 - E));",
+     "double m = floor(ldexp(v, 10 - E));"),
+    ("f16_subnormal_scale", "const double m = nearbyint(ldexp(v, 24));",
+     "const double m = nearbyint(ldexp(v, 23));"),
+    ("f16_to_f32_bias", "ldexp(1024.0 + (double)m, (int)e - 25)",
+     "ldexp(1024.0 + (double)m, (int)e - 24)"),
+    ("f16_nan_drops_sign", "return sign | 0x7E00u;", "return 0x7E00u;"),
+    ("bf16_to_f32_shift", "return (uint32_t)b << 16;", "return (uint32_t)b << 15;"),
+    ("f16_to_bf16_skips_rounding", "return oracle_rne_bf16(oracle_f16_to_f32(h));",
+     "return (uint16_t)(oracle_f16_to_f32(h) >> 16);"),
     ("stride_uses_row_length", "const uint64_t stride = given ? given : C;",
      "const uint64_t stride = C;"),
 ]
@@ -68,7 +78,8 @@ def test_pins_catch_mutant(name, old, new, mutant_dir):
     so = os.path.join(mutant_dir, f"{name}.so")
     with open(c, "w") as f:
         f.write(src.replace(old, new))
-    subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", c, "-o", so], check=True)
+    subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", c, "-o", so, "-lm"],
+                   check=True)
     root = os.path.dirname(HERE)
     r = subprocess.run([sys.executable, "-c", _RUNNER, HERE, root, so],
                        capture_output=True, text=True, timeout=600)

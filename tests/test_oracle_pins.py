@@ -12,8 +12,8 @@ def test_pin(pin):
 
 
 def test_rne_exhaustive_vs_torch():
-    """All 2^32 fp32 bit patterns: the oracle's cast equals torch's CPU conversion (NaNs as a
-    class, the oracle's NaN being 0x7FC0)."""
+    """All 2^32 fp32 bit patterns: the oracle's fp32 -> bf16 and fp32 -> fp16 conversions equal
+    torch's CPU conversions (NaNs as a class; the oracle's NaNs are 0x7FC0 and sign | 0x7E00)."""
     import os
     from concurrent.futures import ThreadPoolExecutor
     step = 1 << 24
@@ -21,6 +21,7 @@ def test_rne_exhaustive_vs_torch():
     def block(start):
         u = np.arange(start, start + step, dtype=np.uint32)
         _pins.check_rne_block(u)
+        _pins.check_convert_block("f32", "f16", u)
 
     workers = min(8, len(os.sched_getaffinity(0)))
     with ThreadPoolExecutor(workers) as ex:

@@ -25,6 +25,9 @@
  *            non-zero 23-bit mantissa, a quarter of them with low half 0x8000);
  *            656 <= c < 660 -> a signed zero.  That is about 0.5 % ties, 0.5 % subnormals and
  *            a few zeros, and never NaN or Inf.
+ *   f16fin : 2-byte little-endian binary16 patterns that are always finite: element j (blob byte
+ *            2j) takes 16 bits of word j div 4; its exponent field, 5 bits that would be 31 for
+ *            infinities and NaNs, is replaced by those bits mod 31 (so 0, subnormals, .. 30).
  */
 #define _POSIX_C_SOURCE 200809L
 #include <math.h>
@@ -121,6 +124,22 @@ int wl_fill_f32mix(uint64_t seed, uint64_t off, uint64_t len, uint8_t *out)
     return 0;
 }
 
+/* Blob bytes [off, off + len) of kind "f16fin" into out; off and len multiples of 2. */
+int wl_fill_f16fin(uint64_t seed, uint64_t off, uint64_t len, uint8_t *out)
+{
+    if ((off & 1u) || (len & 1u)) return -1;
+    const uint64_t j0 = off >> 1, n = len >> 1;
+    for (uint64_t i = 0; i < n; ++i) {
+        const uint64_t j = j0 + i;
+        const uint32_t bits = (uint32_t)(wl_word(seed, j >> 2) >> (16 * (j & 3u))) & 0xFFFFu;
+        const uint32_t e = ((bits >> 10) & 31u) % 31u;
+        const uint32_t v = (bits & 0x83FFu) | (e << 10);
+        out[2 * i] = (uint8_t)v;
+        out[2 * i + 1] = (uint8_t)(v >> 8);
+    }
+    return 0;
+}
+
 /*
  * A fill callback with the loader's source signature, so that tests and the benchmark can
  * stream a blob that exists only as its generator definition.  `user` points to a
@@ -128,7 +147,7 @@ int wl_fill_f32mix(uint64_t seed, uint64_t off, uint64_t len, uint8_t *out)
  * reaching that blob offset) and delay_us (sleep before every call).
  */
 typedef struct wl_cb_source {
-    int32_t kind; /* 0 = bits, 1 = f32mix */
+    int32_t kind; /* 0 = bits, 1 = f32mix, 2 = f16fin */
     int32_t reserved;
     uint64_t seed;
     uint64_t period;    /* 0 = none */
@@ -152,7 +171,9 @@ int wl_fill_cb(void *user, uint64_t off, void *dst, uint64_t len)
         uint64_t take = s->period ? s->period - o : len;
         if (take > len) take = len;
         if (s->kind == 0) wl_fill_bits(s->seed, o, take, out);
-        else if (wl_fill_f32mix(s->seed, o, take, out) != 0) return 2;
+        else if (s->kind == 1 ? wl_fill_f32mix(s->seed, o, take, out) != 0
+                              : wl_fill_f16fin(s->seed, o, take, out) != 0)
+            return 2;
         out += take;
         off += take;
         len -= take;

@@ -20,7 +20,7 @@ _LIB_PATH = os.path.join(_HERE, "libwlgen.so")
 _lock = threading.Lock()
 _lib = None
 
-KINDS = ("bits", "f32mix")
+KINDS = ("bits", "f32mix", "f16fin")
 
 
 def build(force=False):
@@ -48,6 +48,9 @@ def _load():
             lib.wl_fill_f32mix.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64,
                                            ctypes.c_void_p]
             lib.wl_fill_f32mix.restype = ctypes.c_int
+            lib.wl_fill_f16fin.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64,
+                                           ctypes.c_void_p]
+            lib.wl_fill_f16fin.restype = ctypes.c_int
             lib.wl_splitmix64_word.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
             lib.wl_splitmix64_word.restype = ctypes.c_uint64
             _lib = lib
@@ -65,6 +68,9 @@ def _fill_one(kind, seed, off, length, ptr):
     elif kind == "f32mix":
         if lib.wl_fill_f32mix(seed, off, length, ptr) != 0:
             raise ValueError("f32mix ranges must start and end on 4-byte boundaries")
+    elif kind == "f16fin":
+        if lib.wl_fill_f16fin(seed, off, length, ptr) != 0:
+            raise ValueError("f16fin ranges must start and end on 2-byte boundaries")
     else:
         raise ValueError(f"unknown blob kind {kind!r}")
 

@@ -82,7 +82,7 @@ class CallbackSource:
     def __init__(self, m, fail_from=None, delay_us=0):
         lib = gen._load()
         self.c = self._C()
-        self.c.kind = 0 if m.blob_kind == "bits" else 1
+        self.c.kind = {"bits": 0, "f32mix": 1, "f16fin": 2}[m.blob_kind]
         self.c.seed = m.seed & 0xFFFFFFFFFFFFFFFF
         self.c.period = m.period or 0
         self.c.fail_from = 0xFFFFFFFFFFFFFFFF if fail_from is None else int(fail_from)
