@@ -221,6 +221,8 @@ typedef struct cfa_stats {
     uint64_t bytes_read;      /* algorithmic bytes one load reads from staging */
     uint64_t bytes_written;   /* algorithmic bytes one load writes into destinations */
     uint64_t descriptor_bytes;
+    uint64_t staged_bytes;    /* blob bytes one staged load copies to the device: the byte
+                                 ranges the chunks' pieces read, not whole chunks */
     uint64_t loads;           /* loads enqueued on this plan */
     uint64_t kernel_launches; /* unpack kernel launches enqueued by the last load */
     double plan_ms;           /* host time spent in cfa_plan_create */
@@ -268,9 +270,12 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
 /*
  * Enqueues one complete load of the blob into the destinations and returns without waiting.
  * Every chunk goes through: host staging (HOST: copied by the plan's fill threads; CALLBACK:
- * written by src->fill; PINNED and DEVICE: none), a host->device copy on the plan's copy
- * stream (none for DEVICE), and one unpack kernel on `stream` that writes all pieces of the
- * chunk (DEVICE sources merge contiguous chunks into one launch).  The load is ordered after
+ * written by src->fill; PINNED, DEVICE and HOST_DIRECT: none), a host->device copy on the
+ * plan's copy stream (none for DEVICE and HOST_DIRECT), and the unpack kernels on `stream`
+ * that write all pieces of the chunk (DEVICE sources merge all chunks into one launch per work
+ * class).  Staging and copies move only the byte ranges the chunk's pieces read (strided 2-D
+ * copies for column slices), so a tensor-parallel rank moves about its share of the
+ * checkpoint; cfa_stats.staged_bytes gives the total.  The load is ordered after
  * all work enqueued on `stream` before this call, and work enqueued on `stream` after this
  * call sees every destination written.  Per-layer readiness is published through
  * cfa_wait_layer.  Loads on one plan run in the order they were enqueued; the checksums and

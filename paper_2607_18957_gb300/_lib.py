@@ -49,7 +49,8 @@ class Source(ctypes.Structure):
 class Stats(ctypes.Structure):
     _fields_ = [(n, ctypes.c_uint64) for n in (
         "blob_bytes", "n_entries", "n_dsts", "n_chunks", "n_layers", "n_pieces", "n_slabs",
-        "n_bulk", "n_tiny", "n_strided", "bytes_read", "bytes_written", "descriptor_bytes", "loads",
+        "n_bulk", "n_tiny", "n_strided", "bytes_read", "bytes_written", "descriptor_bytes",
+        "staged_bytes", "loads",
         "kernel_launches")] + [(n, ctypes.c_double) for n in (
             "plan_ms", "load_ms", "h2d_ms", "unpack_ms")]
 

@@ -28,7 +28,8 @@ def _nvcc():
 
 
 def _sources():
-    return [os.path.join(CSRC, f) for f in CU_SOURCES + C_SOURCES + ["cfa_internal.h"]] + \
+    return [os.path.join(CSRC, f) for f in CU_SOURCES + C_SOURCES +
+            ["cfa_internal.h", "cfa_pool.h"]] + \
         [os.path.join(INCLUDE, "cfa.h")]
 
 

@@ -49,6 +49,17 @@ typedef struct cfa_swork {
     uint32_t cls;    /* work class, used while the plan is built */
 } cfa_swork;
 
+/*
+ * A host->device copy of one chunk: `rows` runs of `width` bytes, `pitch` bytes apart, the first
+ * at blob offset `src`; it lands at the same offset inside the chunk's device slot.
+ */
+typedef struct cfa_copy {
+    uint64_t src;
+    uint64_t width;
+    uint64_t pitch;
+    uint64_t rows;
+} cfa_copy;
+
 #define CFA_NO_CK 0xFFFFFFFFu
 
 /* Element conversions (cfa_work.mode bits 4-7, cfa_piece.conv). */
@@ -108,6 +119,11 @@ typedef struct cfa_host_plan {
     size_t n_strided;
     uint32_t *strided_first;
     int64_t *layer_last_chunk; /* n_layers; -1 = the group has no bytes */
+    cfa_copy *copies;          /* what each chunk's pieces read: chunk c owns
+                                  [copy_first[c], copy_first[c + 1]) */
+    size_t n_copies;
+    uint32_t *copy_first;
+    uint64_t staged_bytes;
     uint64_t bytes_read, bytes_written;
     int any_cksum;
 } cfa_host_plan;

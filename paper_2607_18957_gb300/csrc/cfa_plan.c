@@ -230,6 +230,8 @@ void cfa_host_plan_free(cfa_host_plan *hp)
     free(hp->tiny_first);
     free(hp->strided);
     free(hp->strided_first);
+    free(hp->copies);
+    free(hp->copy_first);
     free(hp->layer_last_chunk);
     memset(hp, 0, sizeof *hp);
 }
@@ -636,6 +638,65 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         if ((st = partition_by_class(&tiny, out->tiny_first, n_chunks, S, err, errlen))) goto done;
         if ((st = partition_by_class(&strided, out->strided_first, n_chunks, S, err, errlen)))
             goto done;
+    }
+
+    /* 4b. what each chunk's pieces read: contiguous ranges merged across gaps of at most
+     * kCopyGap bytes, and column slices that would move more than twice their bytes as
+     * strided 2-D copies */
+    out->copy_first = (uint32_t *)calloc((size_t)n_chunks + 1, sizeof(uint32_t));
+    if (!out->copy_first) { st = CFA_ERR_NOMEM; goto done; }
+    {
+        const uint64_t kCopyGap = 1ull << 20;
+        vec cv = {0};
+        cv.elem = sizeof(cfa_copy);
+        size_t p = 0;
+        for (uint32_t c = 0; c < n_chunks; ++c) {
+            out->copy_first[c] = (uint32_t)cv.n;
+            cfa_copy open;
+            int have = 0;
+            for (; p < n_pieces && out->pieces[p].chunk == c; ++p) {
+                const cfa_piece *pc = &out->pieces[p];
+                const uint64_t es = (uint64_t)info[pc->entry].es_s;
+                cfa_copy seg;
+                memset(&seg, 0, sizeof seg);
+                seg.src = pc->src_offset;
+                seg.rows = 1;
+                if (pc->rows > 1) {
+                    const uint64_t width = pc->n_elems / pc->rows * es;
+                    const uint64_t pitch = (uint64_t)pc->src_row_stride * es;
+                    if (2 * width < pitch) {
+                        seg.width = width;
+                        seg.pitch = pitch;
+                        seg.rows = pc->rows;
+                        if (have && vec_push(&cv, &open)) { free(cv.p); st = CFA_ERR_NOMEM; goto done; }
+                        have = 0;
+                        if (vec_push(&cv, &seg)) { free(cv.p); st = CFA_ERR_NOMEM; goto done; }
+                        continue;
+                    }
+                    seg.width = (pc->rows - 1) * pitch + width;
+                } else {
+                    seg.width = pc->n_elems * es;
+                }
+                seg.pitch = seg.width;
+                if (have && seg.src <= open.src + open.width + kCopyGap) {
+                    const uint64_t end = seg.src + seg.width > open.src + open.width
+                                             ? seg.src + seg.width
+                                             : open.src + open.width;
+                    open.width = end - open.src;
+                    open.pitch = open.width;
+                } else {
+                    if (have && vec_push(&cv, &open)) { free(cv.p); st = CFA_ERR_NOMEM; goto done; }
+                    open = seg;
+                    have = 1;
+                }
+            }
+            if (have && vec_push(&cv, &open)) { free(cv.p); st = CFA_ERR_NOMEM; goto done; }
+        }
+        out->copy_first[n_chunks] = (uint32_t)cv.n;
+        out->copies = (cfa_copy *)cv.p;
+        out->n_copies = cv.n;
+        for (size_t k = 0; k < cv.n; ++k)
+            out->staged_bytes += out->copies[k].width * out->copies[k].rows;
     }
 
     /* 5. readiness groups: last chunk carrying one of their bytes */

@@ -38,6 +38,7 @@
 #include <vector>
 
 #include "cfa_internal.h"
+#include "cfa_pool.h"
 
 extern "C" int cfa_unpack_blocks_per_sm(int cls);
 extern "C" int cfa_bulk_blocks_per_sm(int log2es);
@@ -63,84 +64,13 @@ namespace {
 
 thread_local char g_create_err[512];
 
-/* ---- a small thread pool for host staging copies ---------------------------------------- */
-class Pool {
-  public:
-    explicit Pool(int n)
-    {
-        for (int i = 0; i < n; ++i) threads_.emplace_back([this] { loop(); });
-    }
-    ~Pool()
-    {
-        {
-            std::lock_guard<std::mutex> g(mu_);
-            stop_ = true;
-        }
-        cv_.notify_all();
-        for (auto &t : threads_) t.join();
-    }
-    /* Runs f(0 .. nparts-1) on the pool and the calling thread; returns when all are done. */
-    void run(int nparts, const std::function<void(int)> &f)
-    {
-        if (threads_.empty() || nparts <= 1) {
-            for (int k = 0; k < nparts; ++k) f(k);
-            return;
-        }
-        {
-            std::lock_guard<std::mutex> g(mu_);
-            fn_.store(&f);
-            total_.store(nparts);
-            pending_.store(nparts);
-            next_.store(0);
-            ++gen_;
-        }
-        cv_.notify_all();
-        work();
-        std::unique_lock<std::mutex> lk(mu_);
-        done_.wait(lk, [this] { return pending_.load() == 0; });
-    }
-
-  private:
-    void work()
-    {
-        for (;;) {
-            const int k = next_.fetch_add(1);
-            if (k >= total_.load()) return;
-            (*fn_.load())(k);
-            if (pending_.fetch_sub(1) == 1) {
-                std::lock_guard<std::mutex> g(mu_);
-                done_.notify_all();
-            }
-        }
-    }
-    void loop()
-    {
-        uint64_t seen = 0;
-        for (;;) {
-            {
-                std::unique_lock<std::mutex> lk(mu_);
-                cv_.wait(lk, [&] { return stop_ || gen_ != seen; });
-                if (stop_) return;
-                seen = gen_;
-            }
-            work();
-        }
-    }
-    std::vector<std::thread> threads_;
-    std::mutex mu_;
-    std::condition_variable cv_, done_;
-    std::atomic<const std::function<void(int)> *> fn_{nullptr};
-    std::atomic<int> total_{0}, pending_{0}, next_{0};
-    uint64_t gen_ = 0;
-    bool stop_ = false;
-};
-
 struct LoadCtx;
 
 struct FillJob {
     LoadCtx *ctx;
     uint32_t chunk;
     int host_slot;
+    std::vector<std::pair<uint64_t, uint64_t>> ranges; /* built by the first fill */
 };
 
 struct LoadCtx {
@@ -190,7 +120,7 @@ struct cfa_plan {
     std::vector<cudaEvent_t> t_h2d0, t_h2d1, t_k0, t_k1;
     std::vector<std::vector<uint32_t>> layers_ending; /* per chunk */
     std::vector<uint32_t> layers_empty;
-    std::unique_ptr<Pool> pool;
+    std::unique_ptr<cfa::Pool> pool;
     std::vector<std::unique_ptr<LoadCtx>> loads;
     LoadCtx *last = nullptr;
     std::mutex mu;
@@ -222,28 +152,45 @@ void set_err(cfa_plan *p, const char *fmt, ...)
         }                                                                                  \
     } while (0)
 
+/* InDisk -> InMem for one chunk: puts the byte ranges the chunk's pieces read (its copy
+ * segments; the rest of the slot is never read) into pinned slot `host_slot`, split over the
+ * plan's fill threads in parts of at most 16 MiB. */
 void CUDART_CB fill_host_fn(void *arg)
 {
     FillJob *j = static_cast<FillJob *>(arg);
     LoadCtx *ctx = j->ctx;
     cfa_plan *p = ctx->plan;
     if (ctx->error.load()) return;
-    const uint64_t S = p->hp.chunk_bytes;
+    const cfa_host_plan &hp = p->hp;
+    const uint64_t S = hp.chunk_bytes;
     const uint64_t off = (uint64_t)j->chunk * S;
-    const uint64_t len = std::min<uint64_t>(S, p->hp.blob_bytes - off);
     uint8_t *dst = p->h_slots + (uint64_t)j->host_slot * S;
-    const uint64_t part = 16ull << 20;
-    const int nparts = (int)((len + part - 1) / part);
     const cfa_source &src = ctx->src;
+    /* the byte ranges, as (offset in chunk, length): a 2-D segment gives one per row */
+    std::vector<std::pair<uint64_t, uint64_t>> &ranges = j->ranges;
+    if (ranges.empty()) {
+        const uint64_t part = 16ull << 20;
+        for (uint32_t k = hp.copy_first[j->chunk]; k < hp.copy_first[j->chunk + 1]; ++k) {
+            const cfa_copy &cp = hp.copies[k];
+            for (uint64_t r = 0; r < cp.rows; ++r)
+                for (uint64_t a = 0; a < cp.width; a += part)
+                    ranges.emplace_back(cp.src - off + r * cp.pitch + a,
+                                        std::min<uint64_t>(part, cp.width - a));
+        }
+    }
+    const int nparts = (int)std::min<size_t>(ranges.size(), 4096);
+    const size_t per = (ranges.size() + (size_t)nparts - 1) / (size_t)(nparts ? nparts : 1);
     p->pool->run(nparts, [&](int k) {
-        const uint64_t a = (uint64_t)k * part;
-        const uint64_t b = std::min<uint64_t>(len, a + part);
-        if (src.kind == CFA_SRC_HOST) {
-            const uint64_t so = src.period_bytes ? (off % src.period_bytes) : off;
-            std::memcpy(dst + a, static_cast<const uint8_t *>(src.base) + so + a, b - a);
-        } else if (src.fill(src.user, off + a, dst + a, b - a) != 0) {
-            int zero = 0;
-            ctx->error.compare_exchange_strong(zero, CFA_ERR_SOURCE);
+        for (size_t q = (size_t)k * per; q < ranges.size() && q < (size_t)(k + 1) * per; ++q) {
+            const uint64_t a = ranges[q].first, len = ranges[q].second;
+            if (src.kind == CFA_SRC_HOST) {
+                const uint64_t so = src.period_bytes ? (off % src.period_bytes) : off;
+                std::memcpy(dst + a, static_cast<const uint8_t *>(src.base) + so + a, len);
+            } else if (src.fill(src.user, off + a, dst + a, len) != 0) {
+                int zero = 0;
+                ctx->error.compare_exchange_strong(zero, CFA_ERR_SOURCE);
+                return;
+            }
         }
     });
 }
@@ -469,8 +416,8 @@ cfa_status setup_device(cfa_plan *p)
         if ((st = events(p->t_k0, nk, true))) return st;
         if ((st = events(p->t_k1, nk, true))) return st;
     }
-    if (o.fill_threads > 1) p->pool.reset(new Pool(o.fill_threads - 1));
-    else p->pool.reset(new Pool(0));
+    if (o.fill_threads > 1) p->pool.reset(new cfa::Pool(o.fill_threads - 1));
+    else p->pool.reset(new cfa::Pool(0));
     return CFA_OK;
 }
 
@@ -642,7 +589,7 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
     if (staged) {
         ctx->jobs.resize(hp.n_chunks);
         for (uint32_t c = 0; c < hp.n_chunks; ++c)
-            ctx->jobs[c] = FillJob{ctx.get(), c, (int)(c % (uint32_t)p->n_host_slots)};
+            ctx->jobs[c] = FillJob{ctx.get(), c, (int)(c % (uint32_t)p->n_host_slots), {}};
     }
     LoadCtx *cx = ctx.get();
     p->loads.push_back(std::move(ctx));
@@ -681,7 +628,6 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
         for (uint32_t c = 0; c < hp.n_chunks; ++c) {
             const int ds = (int)(c % (uint32_t)p->n_dev_slots);
             const uint64_t off = (uint64_t)c * S;
-            const uint64_t len = std::min<uint64_t>(S, hp.blob_bytes - off);
             const void *hsrc;
             int hs = -1;
             if (staged) {
@@ -698,7 +644,19 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             uint8_t *dslot = p->d_slots + (uint64_t)ds * p->slot_bytes;
             CK(p, cudaStreamWaitEvent(p->copy_stream, p->ev_dev_free[ds], 0));
             if (timing) CK(p, cudaEventRecord(p->t_h2d0[c], p->copy_stream));
-            CK(p, cudaMemcpyAsync(dslot, hsrc, len, cudaMemcpyHostToDevice, p->copy_stream));
+            /* InMem -> InGPU: only the ranges the chunk's pieces read */
+            for (uint32_t k = hp.copy_first[c]; k < hp.copy_first[c + 1]; ++k) {
+                const cfa_copy &cp = hp.copies[k];
+                const uint64_t at = cp.src - off;
+                if (cp.rows == 1)
+                    CK(p, cudaMemcpyAsync(dslot + at, static_cast<const uint8_t *>(hsrc) + at,
+                                          cp.width, cudaMemcpyHostToDevice, p->copy_stream));
+                else
+                    CK(p, cudaMemcpy2DAsync(dslot + at, cp.pitch,
+                                            static_cast<const uint8_t *>(hsrc) + at, cp.pitch,
+                                            cp.width, cp.rows, cudaMemcpyHostToDevice,
+                                            p->copy_stream));
+            }
             if (timing) CK(p, cudaEventRecord(p->t_h2d1[c], p->copy_stream));
             p->last_h2d++;
             if (staged) CK(p, cudaEventRecord(p->ev_host_free[hs], p->copy_stream));
@@ -782,6 +740,7 @@ cfa_status cfa_get_stats(cfa_plan *p, cfa_stats *s)
     s->bytes_written = hp.bytes_written;
     s->descriptor_bytes = (hp.n_slabs + hp.n_bulk + hp.n_tiny) * sizeof(cfa_work) +
                           hp.n_strided * sizeof(cfa_swork);
+    s->staged_bytes = hp.staged_bytes;
     s->loads = p->n_loads;
     s->kernel_launches = p->last_launches;
     s->plan_ms = p->plan_ms;

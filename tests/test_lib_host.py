@@ -253,6 +253,20 @@ def test_host_only_plan_refuses_to_load():
         assert e.value.name == "CFA_ERR_INVAL"
 
 
+def test_staged_bytes_cover_exactly_what_pieces_read():
+    """Staged loads copy only the byte ranges pieces read: the whole checkpoint for a 1:1 model,
+    about one eighth of it for a tensor-parallel rank of eight."""
+    import workloads
+    m = workloads.named_config("llama3_8b_bf16")
+    with host_plan(m, chunk_bytes=m.chunk_bytes) as p:
+        st = p.stats()
+    assert m.total_src_bytes() <= st["staged_bytes"] <= m.blob_bytes
+    m = workloads.named_config("llama3_70b_bf16_tp8r3")
+    with host_plan(m, chunk_bytes=m.chunk_bytes) as p:
+        st = p.stats()
+    assert st["bytes_read"] <= st["staged_bytes"] < 0.2 * m.blob_bytes
+
+
 def test_full_size_manifests_plan_on_the_host():
     import workloads
     for name in ("llama3_8b_bf16", "llama3_70b_bf16"):

@@ -65,17 +65,14 @@ MUTANTS = [
 ]
 
 
-@pytest.fixture(scope="module")
-def mutant_dir(tmp_path_factory):
-    return tmp_path_factory.mktemp("oracle_mutants")
-
-
-@pytest.mark.parametrize("name,old,new", MUTANTS, ids=[m[0] for m in MUTANTS])
-def test_pins_catch_mutant(name, old, new, mutant_dir):
+def _run_mutant(name, old, new, workdir):
+    """Compiles one mutant and runs every pin against it in a child process; returns the pins
+    that failed, or None if the mutant crashed the child (which also counts as caught)."""
     src = open(oracle.SOURCE_PATH).read()
-    assert src.count(old) == 1, f"mutation site for {name} not unique"
-    c = os.path.join(mutant_dir, f"{name}.c")
-    so = os.path.join(mutant_dir, f"{name}.so")
+    if src.count(old) != 1:
+        return f"mutation site for {name} not unique"
+    c = os.path.join(workdir, f"{name}.c")
+    so = os.path.join(workdir, f"{name}.so")
     with open(c, "w") as f:
         f.write(src.replace(old, new))
     subprocess.run(["gcc", "-O1", "-std=c11", "-shared", "-fPIC", c, "-o", so, "-lm"],
@@ -84,7 +81,25 @@ def test_pins_catch_mutant(name, old, new, mutant_dir):
     r = subprocess.run([sys.executable, "-c", _RUNNER, HERE, root, so],
                        capture_output=True, text=True, timeout=600)
     if r.returncode != 0:
-        return  # the mutant crashed the pins' process: caught
+        return None
     line = [ln for ln in r.stdout.splitlines() if ln.startswith("FAILED:")][-1]
-    failed = [x for x in line[len("FAILED:"):].split(",") if x]
-    assert failed, f"no pin caught mutant {name}"
+    return [x for x in line[len("FAILED:"):].split(",") if x]
+
+
+@pytest.fixture(scope="module")
+def mutant_results(tmp_path_factory):
+    """All mutants compiled and checked concurrently, one child process each."""
+    from concurrent.futures import ThreadPoolExecutor
+    workdir = str(tmp_path_factory.mktemp("oracle_mutants"))
+    workers = max(1, min(8, len(os.sched_getaffinity(0))))
+    ex = ThreadPoolExecutor(workers)
+    futs = {name: ex.submit(_run_mutant, name, old, new, workdir) for name, old, new in MUTANTS}
+    yield futs
+    ex.shutdown(wait=True)
+
+
+@pytest.mark.parametrize("name", [m[0] for m in MUTANTS])
+def test_pins_catch_mutant(name, mutant_results):
+    failed = mutant_results[name].result()
+    assert not isinstance(failed, str), failed
+    assert failed is None or failed, f"no pin caught mutant {name}"
