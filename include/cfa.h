@@ -26,8 +26,8 @@
  *   - The return value is a cfa_status: CFA_OK (0) on success, a negative CFA_ERR_* code
  *     otherwise.  No function aborts, throws, traps the GPU or spins without a bound.
  *   - cfa_last_error(plan) gives a human-readable detail of the last failure on that plan;
- *     cfa_last_error(NULL) gives the detail of the last failure of cfa_plan_create on the
- *     calling thread.
+ *     cfa_last_error(NULL) gives the detail of the last failure of cfa_plan_create or of the
+ *     checkpoint-file functions on the calling thread.
  *   - "device pointer" means an address in the global memory of the plan's CUDA device;
  *     "host pointer" means ordinary process memory.
  *   - Streams are CUDA runtime streams (cudaStream_t); NULL is the legacy default stream.
@@ -72,6 +72,7 @@ typedef int cfa_status;
 #define CFA_DTYPE_I32   5
 #define CFA_DTYPE_I64   6
 #define CFA_DTYPE_F64   7
+#define CFA_DTYPE_I16   8
 
 #define CFA_MAX_DIMS    8
 #define CFA_MAX_LAYERS  65536
@@ -371,6 +372,54 @@ cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t n_entries,
                               uint64_t blob_bytes, uint64_t *cksum_dev, cfa_stream stream,
                               char *err, size_t err_len);
 
+/* ---- checkpoint files (the InDisk end of section 4.2's chunk automaton) ------------------- */
+
+/*
+ * A parsed safetensors header.  The file is an 8-byte little-endian length N, N bytes of JSON
+ * mapping each tensor name to {"dtype", "shape", "data_offsets": [begin, end]} (plus an
+ * optional "__metadata__" object), then the data section, which is the loader's blob:
+ * data_offsets are blob offsets.  The paper loads checkpoints of this format (section 5).
+ */
+typedef struct cfa_safetensors cfa_safetensors;
+
+typedef struct cfa_st_tensor {
+    const char *name;      /* owned by the cfa_safetensors handle */
+    int32_t dtype;         /* CFA_DTYPE_* (int8, uint8, bool and fp8 read as U8, uint16 as I16,
+                              uint32 as I32, uint64 as I64) */
+    int32_t ndim;
+    int64_t shape[CFA_MAX_DIMS];
+    uint64_t blob_offset;  /* byte offset of the tensor in the data section */
+    uint64_t nbytes;
+} cfa_st_tensor;
+
+/* Reads and validates the header of `path` (not the data).  Every tensor's data_offsets must
+ * match its shape and dtype and lie inside the file.  Errors: CFA_ERR_INVAL (malformed header,
+ * unknown dtype, more than 8 dimensions), CFA_ERR_SOURCE (cannot read), CFA_ERR_NOMEM. */
+cfa_status cfa_safetensors_open(const char *path, cfa_safetensors **out);
+
+/* The same from a header already in memory (the N JSON bytes); file_bytes is the file's size. */
+cfa_status cfa_safetensors_parse(const void *header, uint64_t header_len, uint64_t file_bytes,
+                                 cfa_safetensors **out);
+
+/* Tensor count, file offset of the data section (8 + N) and its length. */
+cfa_status cfa_safetensors_info(const cfa_safetensors *st, size_t *n_tensors,
+                                uint64_t *data_offset, uint64_t *data_bytes);
+
+/* Tensor i (header order), 0 <= i < n_tensors. */
+cfa_status cfa_safetensors_tensor(const cfa_safetensors *st, size_t i, cfa_st_tensor *out);
+
+/* Frees the handle (and the names it owns).  Accepts NULL. */
+cfa_status cfa_safetensors_close(cfa_safetensors *st);
+
+/*
+ * Fills *out with a CALLBACK source that reads blob byte o from file byte data_offset + o with
+ * pread (several fill threads may read at once).  The file stays open until
+ * cfa_file_source_close(out), which must come after every load using it has completed.
+ * Errors: CFA_ERR_SOURCE (cannot open), CFA_ERR_INVAL, CFA_ERR_NOMEM.
+ */
+cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, cfa_source *out);
+cfa_status cfa_file_source_close(cfa_source *src);
+
 /* Zeroes the plan's checksum buffer on `stream`. */
 cfa_status cfa_reset_checksums(cfa_plan *plan, cfa_stream stream);
 
@@ -388,7 +437,7 @@ const char *cfa_last_error(const cfa_plan *plan);
 const char *cfa_status_name(cfa_status st);
 
 /* sizeof of the ABI struct with this name ("cfa_tensor_entry", "cfa_dst", "cfa_plan_opts",
- * "cfa_source", "cfa_stats", "cfa_piece"), or 0 for an unknown name; lets a binding check its
+ * "cfa_source", "cfa_stats", "cfa_piece", "cfa_st_tensor"), or 0 for an unknown name; lets a binding check its
  * own copies of the layouts.  Host-only. */
 size_t cfa_abi_sizeof(const char *type_name);
 

@@ -27,8 +27,8 @@ _lock = threading.Lock()
 _lib = None
 
 # The oracle's own dtype codes (cfa_oracle.c); dtype names are the manifest's.
-_DTYPE_CODE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7}
-_ELEM = {"u8": 1, "bf16": 2, "f16": 2, "f32": 4, "i32": 4, "i64": 8, "f64": 8}
+_DTYPE_CODE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7, "i16": 8}
+_ELEM = {"u8": 1, "bf16": 2, "f16": 2, "f32": 4, "i32": 4, "i64": 8, "f64": 8, "i16": 2}
 _CONVERT, _CKSUM = 1, 2
 # conversion ids of oracle_convert_array
 CONV = {("f32", "bf16"): 1, ("f32", "f16"): 2, ("f16", "bf16"): 3, ("bf16", "f32"): 4,

@@ -49,7 +49,8 @@
 #include <string.h>
 
 /* The oracle's own dtype codes (its Python wrapper maps dtype names onto these). */
-enum { ORC_U8 = 1, ORC_BF16 = 2, ORC_F16 = 3, ORC_F32 = 4, ORC_I32 = 5, ORC_I64 = 6, ORC_F64 = 7 };
+enum { ORC_U8 = 1, ORC_BF16 = 2, ORC_F16 = 3, ORC_F32 = 4, ORC_I32 = 5, ORC_I64 = 6, ORC_F64 = 7,
+       ORC_I16 = 8 };
 
 /* Entry flags as the wrapper passes them. */
 enum { ORC_CONVERT = 1, ORC_CKSUM = 2 };
@@ -85,6 +86,7 @@ static int orc_elem_size(int32_t dt)
     case ORC_U8: return 1;
     case ORC_BF16: return 2;
     case ORC_F16: return 2;
+    case ORC_I16: return 2;
     case ORC_F32: return 4;
     case ORC_I32: return 4;
     case ORC_I64: return 8;

@@ -20,7 +20,8 @@ import numpy as np
 from . import _lib
 from ._lib import ALL, DTYPE, ENTRY_DTYPE, DST_DTYPE, PIECE_DTYPE  # noqa: F401
 
-__all__ = ["Plan", "Source", "CfaError", "make_entries", "make_dsts", "ALL", "library_path"]
+__all__ = ["Plan", "Source", "FileSource", "Safetensors", "StTensor", "CfaError", "make_entries",
+           "make_dsts", "ALL", "library_path"]
 
 
 class CfaError(RuntimeError):
@@ -168,6 +169,141 @@ class Source:
         s.fill = self.fill or None
         s.user = self.user or None
         return s
+
+
+class FileSource(Source):
+    """A checkpoint file read with pread by the plan's fill threads (cfa_file_source_open):
+    blob byte o is file byte data_offset + o.  Close it after the last load that uses it has
+    completed (the context manager does)."""
+
+    def __init__(self, path, data_offset=0):
+        lib = _lib.load()
+        self._lib = lib
+        self._c = _lib.Source()
+        st = lib.cfa_file_source_open(str(path).encode(), int(data_offset), ctypes.byref(self._c))
+        _check(st)
+        super().__init__(_lib.SRC_CALLBACK, 0, 0, self._c.fill, self._c.user)
+        self.path, self.data_offset = str(path), int(data_offset)
+
+    def to_c(self):
+        if not self._c.user:
+            raise CfaError(-1, "file source is closed")
+        return self._c
+
+    def close(self):
+        if self._c.user:
+            _check(self._lib.cfa_file_source_close(ctypes.byref(self._c)))
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+
+Source.file = staticmethod(lambda path, data_offset=0: FileSource(path, data_offset))
+
+
+class StTensor(tuple):
+    """(name, dtype, shape, offset, nbytes) of one safetensors tensor; offset is a blob offset
+    into the data section."""
+    __slots__ = ()
+    name = property(lambda s: s[0])
+    dtype = property(lambda s: s[1])
+    shape = property(lambda s: s[2])
+    offset = property(lambda s: s[3])
+    nbytes = property(lambda s: s[4])
+
+
+class Safetensors:
+    """A parsed safetensors header (cfa_safetensors).  The file's data section is the loader's
+    blob: `tensors[i].offset` is a blob offset, `data_offset` is where the data section starts in
+    the file and `data_bytes` its length."""
+
+    def __init__(self, handle):
+        lib = _lib.load()
+        n, off, nb = ctypes.c_size_t(), ctypes.c_uint64(), ctypes.c_uint64()
+        try:
+            _check(lib.cfa_safetensors_info(handle, ctypes.byref(n), ctypes.byref(off),
+                                            ctypes.byref(nb)))
+            names = {v: k for k, v in DTYPE.items()}
+            t = _lib.StTensor()
+            out = []
+            for i in range(n.value):
+                _check(lib.cfa_safetensors_tensor(handle, i, ctypes.byref(t)))
+                out.append(StTensor((t.name.decode("utf-8"), names[t.dtype],
+                                     tuple(int(t.shape[k]) for k in range(t.ndim)),
+                                     int(t.blob_offset), int(t.nbytes))))
+        finally:
+            lib.cfa_safetensors_close(handle)
+        self.tensors = out
+        self.data_offset, self.data_bytes = off.value, nb.value
+
+    @classmethod
+    def open(cls, path):
+        """Reads and validates the header of a safetensors file."""
+        lib = _lib.load()
+        h = ctypes.c_void_p()
+        _check(lib.cfa_safetensors_open(str(path).encode(), ctypes.byref(h)))
+        return cls(h)
+
+    @classmethod
+    def parse(cls, header, file_bytes):
+        """Parses the JSON header bytes of a file of `file_bytes` bytes."""
+        lib = _lib.load()
+        h = ctypes.c_void_p()
+        buf = ctypes.create_string_buffer(bytes(header), len(header))
+        _check(lib.cfa_safetensors_parse(buf, len(header), int(file_bytes), ctypes.byref(h)))
+        return cls(h)
+
+    def entries(self, targets, whole_file=False):
+        """Manifest entries for the tensors named in `targets`, in the order of `targets` (a
+        name the file does not hold raises KeyError).  A target is
+        (dst, row) or (dst, row, layer), or a dict with keys dst, row, layer, cast, cksum and at
+        most one of rows=(r0, r1) (a range of the tensor's first dimension) or cols=(c0, c1) (a
+        range of its last dimension, read with a source row stride: a tensor-parallel column
+        shard).  With whole_file the blob is the whole file (offsets shifted by data_offset), so
+        that a mapping of the file from its first byte can serve as the source."""
+        cols = {k: [] for k in ("dtype", "shape", "offset", "dst", "row", "layer", "cast",
+                                 "cksum", "names", "src_row_stride")}
+        shift = self.data_offset if whole_file else 0
+        by_name = {t.name: t for t in self.tensors}
+        for name, v in targets.items():
+            if name not in by_name:
+                raise KeyError(f"the file holds no tensor named {name!r}")
+            t = by_name[name]
+            if not isinstance(v, dict):
+                v = dict(zip(("dst", "row", "layer"), v))
+            es = _lib.DTYPE_SIZE[t.dtype]
+            shape, off, stride = t.shape, t.offset + shift, 0
+            if "rows" in v and "cols" in v:
+                raise ValueError(f"{t.name}: give rows or cols, not both")
+            if "rows" in v:
+                r0, r1 = v["rows"]
+                if not (len(shape) >= 1 and 0 <= r0 <= r1 <= shape[0]):
+                    raise ValueError(f"{t.name}: rows {r0}:{r1} outside shape {shape}")
+                per_row = int(np.prod(shape[1:], dtype=np.int64))
+                off += r0 * per_row * es
+                shape = (r1 - r0,) + tuple(shape[1:])
+            elif "cols" in v:
+                c0, c1 = v["cols"]
+                if not (len(shape) >= 1 and 0 <= c0 <= c1 <= shape[-1]):
+                    raise ValueError(f"{t.name}: cols {c0}:{c1} outside shape {shape}")
+                off += c0 * es
+                if int(np.prod(shape[:-1], dtype=np.int64)) > 1:
+                    stride = shape[-1]
+                shape = tuple(shape[:-1]) + (c1 - c0,)
+            cols["dtype"].append(t.dtype)
+            cols["shape"].append(shape)
+            cols["offset"].append(off)
+            cols["dst"].append(v["dst"])
+            cols["row"].append(v.get("row", 0))
+            cols["layer"].append(v.get("layer", 0))
+            cols["cast"].append(bool(v.get("cast", False)))
+            cols["cksum"].append(bool(v.get("cksum", True)))
+            cols["names"].append(t.name)
+            cols["src_row_stride"].append(stride)
+        return make_entries(**cols)
 
 
 class Plan:

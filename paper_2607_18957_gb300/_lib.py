@@ -13,7 +13,8 @@ STATUS = {0: "CFA_OK", -1: "CFA_ERR_INVAL", -2: "CFA_ERR_OVERLAP", -3: "CFA_ERR_
           -4: "CFA_ERR_COVERAGE", -5: "CFA_ERR_CUDA", -6: "CFA_ERR_SOURCE", -7: "CFA_ERR_TIMEOUT",
           -8: "CFA_ERR_BUSY", -9: "CFA_ERR_NOMEM", -10: "CFA_ERR_DTYPE", -11: "CFA_ERR_ALIGN",
           -12: "CFA_ERR_DEVICE", -13: "CFA_ERR_SHAPE"}
-DTYPE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7}
+DTYPE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7, "i16": 8}
+DTYPE_SIZE = {"u8": 1, "bf16": 2, "f16": 2, "f32": 4, "i32": 4, "i64": 8, "f64": 8, "i16": 2}
 ENTRY_CAST_BF16, ENTRY_CKSUM, ENTRY_CONVERT = 0x1, 0x2, 0x4
 OPT_STRICT_COVERAGE, OPT_HOST_ONLY, OPT_TIMING, OPT_BULK, OPT_NO_MERGE = 0x1, 0x2, 0x4, 0x8, 0x10
 SRC_HOST, SRC_PINNED, SRC_CALLBACK, SRC_DEVICE, SRC_HOST_DIRECT = 1, 2, 3, 4, 5
@@ -63,6 +64,12 @@ class Piece(ctypes.Structure):
                 ("src_row_stride", ctypes.c_uint32)]
 
 
+class StTensor(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char_p), ("dtype", ctypes.c_int32), ("ndim", ctypes.c_int32),
+                ("shape", ctypes.c_int64 * 8), ("blob_offset", ctypes.c_uint64),
+                ("nbytes", ctypes.c_uint64)]
+
+
 PIECE_DTYPE = np.dtype([("chunk", "<u4"), ("entry", "<u4"), ("src_offset", "<u8"),
                         ("dst_index", "<u4"), ("conv", "<u4"), ("dst_offset", "<u8"),
                         ("n_elems", "<u8"), ("rows", "<u4"), ("src_row_stride", "<u4")])
@@ -87,6 +94,13 @@ SIGNATURES = {
     "cfa_abi_sizeof": (_SZ, [ctypes.c_char_p]),
     "cfa_unpack_noalloc": (ctypes.c_int, [_P, _SZ, _P, _SZ, _P, _U64, _P, _P, ctypes.c_char_p,
                                           _SZ]),
+    "cfa_safetensors_open": (ctypes.c_int, [ctypes.c_char_p, _P]),
+    "cfa_safetensors_parse": (ctypes.c_int, [_P, _U64, _U64, _P]),
+    "cfa_safetensors_info": (ctypes.c_int, [_P, _P, _P, _P]),
+    "cfa_safetensors_tensor": (ctypes.c_int, [_P, _SZ, _P]),
+    "cfa_safetensors_close": (ctypes.c_int, [_P]),
+    "cfa_file_source_open": (ctypes.c_int, [ctypes.c_char_p, _U64, _P]),
+    "cfa_file_source_close": (ctypes.c_int, [_P]),
 }
 
 _lib = None
@@ -115,7 +129,8 @@ def load():
 def _check_layouts(lib):
     want = {"cfa_tensor_entry": ENTRY_DTYPE.itemsize, "cfa_dst": DST_DTYPE.itemsize,
             "cfa_plan_opts": ctypes.sizeof(PlanOpts), "cfa_source": ctypes.sizeof(Source),
-            "cfa_stats": ctypes.sizeof(Stats), "cfa_piece": ctypes.sizeof(Piece)}
+            "cfa_stats": ctypes.sizeof(Stats), "cfa_piece": ctypes.sizeof(Piece),
+            "cfa_st_tensor": ctypes.sizeof(StTensor)}
     for name, size in want.items():
         got = lib.cfa_abi_sizeof(name.encode())
         if got != size:

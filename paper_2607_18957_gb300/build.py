@@ -19,7 +19,7 @@ LIB = os.path.join(PKG, "libcfa.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 CU_SOURCES = ["cfa_unpack.cu", "cfa_bulk.cu", "cfa_runtime.cu", "cfa_noalloc.cu"]
-C_SOURCES = ["cfa_plan.c"]
+C_SOURCES = ["cfa_plan.c", "cfa_files.c"]
 
 
 def _nvcc():

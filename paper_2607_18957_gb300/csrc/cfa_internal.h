@@ -128,6 +128,9 @@ typedef struct cfa_host_plan {
     int any_cksum;
 } cfa_host_plan;
 
+/* Sets the calling thread's detail string returned by cfa_last_error(NULL). */
+void cfa_internal_set_error(const char *msg);
+
 cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries,
                                const cfa_dst *dsts, size_t n_dsts, uint64_t blob_bytes,
                                const cfa_plan_opts *opts, cfa_host_plan *out, char *err,

@@ -74,7 +74,8 @@ int dtype_size(int32_t dt)
     switch (dt) {
     case CFA_DTYPE_U8: return 1;
     case CFA_DTYPE_BF16:
-    case CFA_DTYPE_F16: return 2;
+    case CFA_DTYPE_F16:
+    case CFA_DTYPE_I16: return 2;
     case CFA_DTYPE_F32:
     case CFA_DTYPE_I32: return 4;
     case CFA_DTYPE_I64:

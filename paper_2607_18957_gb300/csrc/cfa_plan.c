@@ -38,6 +38,7 @@ int cfa_dtype_size(int32_t dt)
     case CFA_DTYPE_I32: return 4;
     case CFA_DTYPE_I64: return 8;
     case CFA_DTYPE_F64: return 8;
+    case CFA_DTYPE_I16: return 2;
     default: return 0;
     }
 }

@@ -838,6 +838,11 @@ cfa_status cfa_plan_destroy(cfa_plan *p)
 
 const char *cfa_last_error(const cfa_plan *p) { return p ? p->err : g_create_err; }
 
+void cfa_internal_set_error(const char *msg)
+{
+    std::snprintf(g_create_err, sizeof g_create_err, "%s", msg ? msg : "");
+}
+
 const char *cfa_status_name(cfa_status st)
 {
     switch (st) {
@@ -868,6 +873,7 @@ size_t cfa_abi_sizeof(const char *type_name)
     if (!std::strcmp(type_name, "cfa_source")) return sizeof(cfa_source);
     if (!std::strcmp(type_name, "cfa_stats")) return sizeof(cfa_stats);
     if (!std::strcmp(type_name, "cfa_piece")) return sizeof(cfa_piece);
+    if (!std::strcmp(type_name, "cfa_st_tensor")) return sizeof(cfa_st_tensor);
     return 0;
 }
 

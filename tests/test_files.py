@@ -1,0 +1,252 @@
+"""Checkpoint files on the host (no GPU): the safetensors header parser against Python's json
+module, the format's corner cases and malformed headers, manifests rebuilt from a file (whole
+tensors, row and column shards), and the pread file source's fill function."""
+import ctypes
+import json
+import os
+import struct
+
+import numpy as np
+import pytest
+
+import paper_2607_18957_gb300 as cfa
+from paper_2607_18957_gb300 import _lib
+from workloads import dense_config, moe_config
+from workloads.harness import entries_for
+from workloads.stfile import ST_DTYPE, file_tensors, header_bytes, targets_for, write_safetensors
+
+ST_NAME = {v: k for k, v in ST_DTYPE.items()}
+ST_NAME.update({"BOOL": "u8", "I8": "u8", "F8_E4M3": "u8", "F8_E5M2": "u8", "U16": "i16",
+                "U32": "i32", "U64": "i64"})
+
+
+def configs():
+    return [
+        dense_config("st_dense", 81, layers=2, hidden=256, n_q=4, n_kv=2, head_dim=64, inter=640,
+                     vocab=512, align=2, jitter=5),
+        dense_config("st_f32_tp4r1", 82, layers=2, hidden=256, n_q=4, n_kv=2, head_dim=64,
+                     inter=640, vocab=512, src_dtype="f32", align=4, jitter=3, tp=4, rank=1),
+        moe_config("st_moe_tp2r1", 83, layers=1, hidden=128, n_q=2, n_kv=2, head_dim=64,
+                   inter=256, n_experts=4, vocab=256, n_extra=200, align=2, jitter=3, tp=2,
+                   rank=1),
+    ]
+
+
+def write_file(path, header, data=b""):
+    with open(path, "wb") as f:
+        f.write(struct.pack("<Q", len(header)))
+        f.write(header)
+        f.write(data)
+
+
+def expect_from_json(raw, file_bytes):
+    """The tensor list by Python's json module (an independent reading of the header)."""
+    h = json.loads(raw)
+    out = []
+    for name, v in h.items():
+        if name == "__metadata__":
+            continue
+        b, e = v["data_offsets"]
+        out.append((name, ST_NAME[v["dtype"]], tuple(v["shape"]), b, e - b))
+    return out, 8 + len(raw), file_bytes - 8 - len(raw)
+
+
+@pytest.mark.parametrize("idx", [0, 1, 2])
+def test_parse_matches_json_and_the_manifest(tmp_path, idx):
+    m = configs()[idx]
+    p = tmp_path / "model.safetensors"
+    off = write_safetensors(m, p)
+    raw = p.read_bytes()
+    (n,) = struct.unpack("<Q", raw[:8])
+    assert off == 8 + n and off % 8 == 0
+    st = cfa.Safetensors.open(p)
+    want, data_off, data_bytes = expect_from_json(raw[8:8 + n], len(raw))
+    assert [tuple(t) for t in st.tensors] == want
+    assert (st.data_offset, st.data_bytes) == (data_off, data_bytes) == (off, m.blob_bytes)
+    assert [tuple(t) for t in st.tensors] == file_tensors(m)
+    # the same bytes through the in-memory parser
+    st2 = cfa.Safetensors.parse(raw[8:8 + n], len(raw))
+    assert st2.tensors == st.tensors
+    # the data section is the manifest's blob
+    assert np.array_equal(np.frombuffer(raw, np.uint8, offset=off), m.blob_range(0, m.blob_bytes))
+
+
+@pytest.mark.parametrize("idx", [0, 1, 2])
+def test_entries_from_a_file_equal_the_manifest(tmp_path, idx):
+    """Whole tensors, row shards and column shards (source row stride) rebuilt from the header
+    equal the entries the manifest builder made, field by field."""
+    m = configs()[idx]
+    p = tmp_path / "model.safetensors"
+    off = write_safetensors(m, p)
+    st = cfa.Safetensors.open(p)
+    ref = entries_for(m).arr
+    for whole, shift in ((False, 0), (True, off)):
+        got = st.entries(targets_for(m), whole_file=whole).arr
+        for f in ("src_dtype", "ndim", "shape", "dst_index", "layer", "dst_row_offset", "flags",
+                  "src_row_stride"):
+            assert np.array_equal(got[f], ref[f]), f
+        assert np.array_equal(got["blob_offset"], ref["blob_offset"] + np.uint64(shift))
+    if idx:
+        assert (ref["src_row_stride"] > 0).any(), "the shard config has no column slices"
+
+
+def test_entry_slices_are_checked():
+    hdr = header_bytes([("w", "bf16", (4, 6), 0, 48)])
+    st = cfa.Safetensors.parse(hdr, 8 + len(hdr) + 48)
+    e = st.entries({"w": {"dst": 0, "cols": (2, 5)}}).arr
+    assert (e["blob_offset"][0], tuple(e["shape"][0, :2]), e["src_row_stride"][0]) == (4, (4, 3), 6)
+    e = st.entries({"w": {"dst": 0, "rows": (1, 3)}}).arr
+    assert (e["blob_offset"][0], tuple(e["shape"][0, :2]), e["src_row_stride"][0]) == (12, (2, 6), 0)
+    with pytest.raises(ValueError):
+        st.entries({"w": {"dst": 0, "cols": (5, 7)}})
+    with pytest.raises(ValueError):
+        st.entries({"w": {"dst": 0, "rows": (0, 1), "cols": (0, 1)}})
+    with pytest.raises(KeyError):
+        st.entries({"missing": (0, 0)})
+
+
+def test_format_corner_cases():
+    """Keys in any order, unknown keys, nested metadata, escapes and non-ASCII names, scalars,
+    zero-size tensors, every dtype name, whitespace around tokens."""
+    names = ["café.weight", "emoji\U0001F600", 'quote"d', "back\\slash", "tab\tname", "/"]
+    h = {"__metadata__": {"a": [1, 2.5e3, -3, {"b": None}], "c": True, "d": False, "e": "x"}}
+    off = 0
+    dts = ["BOOL", "U8", "I8", "F8_E4M3", "F8_E5M2", "I16", "U16", "F16", "BF16", "I32", "U32",
+           "F32", "I64", "U64", "F64"]
+    size = {"BOOL": 1, "U8": 1, "I8": 1, "F8_E4M3": 1, "F8_E5M2": 1, "I16": 2, "U16": 2,
+            "F16": 2, "BF16": 2, "I32": 4, "U32": 4, "F32": 4, "I64": 8, "U64": 8, "F64": 8}
+    for k, dt in enumerate(dts):
+        shape = [[], [0], [3], [2, 3], [1, 1, 1, 1, 1, 1, 1, 5]][k % 5]
+        nb = size[dt] * int(np.prod(shape, dtype=np.int64))
+        name = names[k] if k < len(names) else f"t{k}"
+        v = {"shape": shape, "data_offsets": [off, off + nb], "extra": {"x": [1]}, "dtype": dt}
+        if k % 2:
+            v = dict(reversed(list(v.items())))
+        h[name] = v
+        off += nb
+    for raw in (json.dumps(h).encode(), json.dumps(h, indent=3).encode(),
+                json.dumps(h, ensure_ascii=False).encode()):
+        st = cfa.Safetensors.parse(raw, 8 + len(raw) + off)
+        want, _, _ = expect_from_json(raw, 8 + len(raw) + off)
+        assert [tuple(t) for t in st.tensors] == want
+    empty = cfa.Safetensors.parse(b"{}", 10)
+    assert empty.tensors == [] and empty.data_bytes == 0
+    meta_only = cfa.Safetensors.parse(b' {"__metadata__" : {} }   ', 8 + 26)
+    assert meta_only.tensors == []
+
+
+BAD_HEADERS = [
+    b"",
+    b"{",
+    b"[]",
+    b'{"a": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]}} x',
+    b'{"a": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]},}',
+    b'{"a": {"dtype": "F4", "shape": [2], "data_offsets": [0, 1]}}',
+    b'{"a": {"dtype": "F32", "shape": [2], "data_offsets": [0, 12]}}',
+    b'{"a": {"dtype": "F32", "shape": [2], "data_offsets": [8, 0]}}',
+    b'{"a": {"dtype": "F32", "shape": [2], "data_offsets": [64, 72]}}',
+    b'{"a": {"dtype": "F32", "shape": [-2], "data_offsets": [0, 8]}}',
+    b'{"a": {"dtype": "F32", "shape": [2.0], "data_offsets": [0, 8]}}',
+    b'{"a": {"dtype": "F32", "shape": [1,1,1,1,1,1,1,1,2], "data_offsets": [0, 8]}}',
+    b'{"a": {"dtype": "F32", "data_offsets": [0, 8]}}',
+    b'{"a": {"dtype": "F32", "shape": [2]}}',
+    b'{"a": {"shape": [2], "data_offsets": [0, 8]}}',
+    b'{"a": {}}',
+    b'{"a": 3}',
+    b'{"a\\x": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]}}',
+    b'{"\\ud800": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]}}',
+    b'{"a": {"dtype": "F32", "shape": [99999999999999999999], "data_offsets": [0, 8]}}',
+    b'{"a": {"dtype": "U8", "shape": [4294967296, 4294967296], "data_offsets": [0, 8]}}',
+    b'{"__metadata__": ' + b"[" * 100 + b"]" * 100 + b"}",
+    b'{"a": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]}',
+]
+
+
+@pytest.mark.parametrize("k", range(len(BAD_HEADERS)))
+def test_malformed_headers_are_rejected(k):
+    raw = BAD_HEADERS[k]
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Safetensors.parse(raw, 8 + len(raw) + 16)
+    assert e.value.name == "CFA_ERR_INVAL"
+
+
+def test_malformed_files_are_rejected(tmp_path):
+    p = tmp_path / "x.safetensors"
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Safetensors.open(tmp_path / "missing.safetensors")
+    assert e.value.name == "CFA_ERR_SOURCE"
+    p.write_bytes(b"\x05\x00")  # shorter than the length word
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Safetensors.open(p)
+    assert e.value.name == "CFA_ERR_SOURCE"
+    p.write_bytes(struct.pack("<Q", 100) + b"{}")  # length past the end of the file
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Safetensors.open(p)
+    assert e.value.name == "CFA_ERR_INVAL"
+    # a tensor running past the end of a truncated file
+    hdr = header_bytes([("w", "f32", (4,), 0, 16)])
+    write_file(p, hdr, b"\0" * 12)
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Safetensors.open(p)
+    assert e.value.name == "CFA_ERR_INVAL" and "data_offsets" in str(e.value)
+    write_file(p, hdr, b"\0" * 16)
+    assert cfa.Safetensors.open(p).tensors[0] == ("w", "f32", (4,), 0, 16)
+
+
+FillFn = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_uint64, ctypes.c_void_p,
+                          ctypes.c_uint64)
+
+
+def test_file_source_fill_reads_the_data_section(tmp_path):
+    m = configs()[0]
+    p = tmp_path / "model.safetensors"
+    off = write_safetensors(m, p)
+    blob = m.blob_range(0, m.blob_bytes)
+    rng = np.random.default_rng(5)
+    with cfa.Source.file(p, off) as src:
+        c = src.to_c()
+        assert c.kind == _lib.SRC_CALLBACK and c.fill and c.user
+        fill = FillFn(c.fill)
+        for _ in range(50):
+            a = int(rng.integers(0, m.blob_bytes))
+            n = int(rng.integers(0, min(1 << 20, m.blob_bytes - a) + 1))
+            buf = np.full(n + 16, 0xAB, dtype=np.uint8)
+            assert fill(c.user, a, buf.ctypes.data + 8, n) == 0
+            assert np.array_equal(buf[8:8 + n], blob[a:a + n])
+            assert (buf[:8] == 0xAB).all() and (buf[8 + n:] == 0xAB).all()
+        buf = np.zeros(16, dtype=np.uint8)
+        assert fill(c.user, m.blob_bytes - 8, buf.ctypes.data, 16) != 0  # past the end
+        assert fill(c.user, (1 << 64) - 4, buf.ctypes.data, 8) != 0    # offset wraps
+    with pytest.raises(cfa.CfaError):
+        src.to_c()  # closed
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Source.file(tmp_path / "missing")
+    assert e.value.name == "CFA_ERR_SOURCE"
+
+
+def test_host_only_plan_from_a_file_matches_the_manifest_plan(tmp_path):
+    """The plan built from the file's entries (pieces, work split, staged bytes) is the plan
+    built from the manifest's."""
+    m = configs()[1]
+    p = tmp_path / "model.safetensors"
+    write_safetensors(m, p)
+    st = cfa.Safetensors.open(p)
+    dsts = [(0x10000 * (j + 1) << 12, str(m.d_dtype[j]), tuple(m.d_shape[j, :m.d_ndim[j]]))
+            for j in range(m.n_dsts)]
+    kw = dict(chunk_bytes=64 << 10, host_only=True)
+    with cfa.Plan(st.entries(targets_for(m)), dsts, st.data_bytes, **kw) as a, \
+            cfa.Plan(entries_for(m), dsts, m.blob_bytes, **kw) as b:
+        assert np.array_equal(a.pieces(), b.pieces())
+        sa, sb = a.stats(), b.stats()
+        for f in ("n_pieces", "n_slabs", "n_tiny", "n_strided", "staged_bytes", "bytes_written"):
+            assert sa[f] == sb[f], f
+
+
+def test_file_abi_is_exported():
+    lib = _lib.load()
+    for name in ("cfa_safetensors_open", "cfa_safetensors_parse", "cfa_safetensors_info",
+                 "cfa_safetensors_tensor", "cfa_safetensors_close", "cfa_file_source_open",
+                 "cfa_file_source_close"):
+        assert hasattr(lib, name)
+    assert lib.cfa_abi_sizeof(b"cfa_st_tensor") == ctypes.sizeof(_lib.StTensor) == 96
+    assert os.path.basename(cfa.library_path()) == "libcfa.so"

@@ -1,0 +1,140 @@
+"""GPU parity for checkpoint files: a safetensors file written from a seeded manifest is loaded
+through its header (Safetensors.entries) and compared byte for byte, checksum for checksum,
+with the oracle on the manifest.  Sources: the pread file source (data section staged through
+the pinned ring), and the whole file read into page-locked or pageable memory with the blob
+being the whole file.  Whole tensors, row and column shards, conversions; a file that shrinks
+under a load is reported as a source error and the plan recovers."""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2607_18957_gb300 as cfa
+from workloads import dense_config, moe_config
+from workloads.harness import DeviceDsts
+from workloads.stfile import targets_for, write_safetensors
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def cuda_device():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.set_device(0)
+
+
+def cfg(name):
+    if name == "dense":
+        return dense_config("file_dense", 91, layers=2, hidden=512, n_q=8, n_kv=2, head_dim=64,
+                            inter=1536, vocab=1000, align=2, jitter=5)
+    if name == "f32_tp":
+        return dense_config("file_f32_tp4r2", 92, layers=2, hidden=512, n_q=8, n_kv=2,
+                            head_dim=64, inter=1536, vocab=1000, src_dtype="f32", align=4,
+                            jitter=3, tp=4, rank=2)
+    if name == "moe_tp":
+        return moe_config("file_moe_tp2r1", 93, layers=2, hidden=256, n_q=4, n_kv=2,
+                          head_dim=64, inter=512, n_experts=4, vocab=500, n_extra=500, align=2,
+                          jitter=3, tp=2, rank=1)
+    if name == "f32_f16":
+        return dense_config("file_f32_f16", 94, layers=2, hidden=512, n_q=8, n_kv=2,
+                            head_dim=64, inter=1536, vocab=1000, src_dtype="f32",
+                            dst_dtype="f16", align=4, jitter=3)
+    raise ValueError(name)
+
+
+_CACHE = {}
+
+
+def prepared(name, tmp_path_factory):
+    """(manifest, file path, data offset, oracle result) for config `name`."""
+    if name not in _CACHE:
+        m = cfg(name)
+        path = tmp_path_factory.mktemp("ckpt") / f"{m.name}.safetensors"
+        off = write_safetensors(m, path)
+        r = oracle.unpack(m, m.blob_range(0, m.blob_bytes))
+        assert r.status == 0, r.status_name
+        _CACHE[name] = (m, str(path), off, r)
+    return _CACHE[name]
+
+
+def aligned_pageable(nbytes, align=256):
+    buf = np.empty(nbytes + align, dtype=np.uint8)
+    off = (-buf.ctypes.data) % align
+    return buf[off:off + nbytes]
+
+
+def compare(m, d, ck, ref, what):
+    for j in range(m.n_dsts):
+        got = d.host_bytes(j)
+        if not np.array_equal(got, ref.dst[j]):
+            bad = np.nonzero(got != ref.dst[j])[0]
+            raise AssertionError(f"{what} {m.d_name[j]}: {bad.size} bytes differ, first at "
+                                 f"{bad[0]}")
+    assert np.array_equal(ck, ref.cksum), f"{what}: checksums differ"
+    assert d.guards_intact(), f"{what}: wrote outside a destination"
+
+
+@pytest.mark.parametrize("chunk", [64 << 10, 1 << 20])
+@pytest.mark.parametrize("kind", ["file", "whole_pinned", "whole_direct_pageable"])
+@pytest.mark.parametrize("name", ["dense", "f32_tp", "moe_tp", "f32_f16"])
+def test_parity_from_a_safetensors_file(tmp_path_factory, name, kind, chunk):
+    m, path, off, ref = prepared(name, tmp_path_factory)
+    st = cfa.Safetensors.open(path)
+    whole = kind != "file"
+    entries = st.entries(targets_for(m), whole_file=whole)
+    keep = []
+    if kind == "file":
+        src = cfa.Source.file(path, st.data_offset)
+        keep.append(src)
+        blob_bytes = st.data_bytes
+    else:
+        data = np.fromfile(path, dtype=np.uint8)
+        blob_bytes = data.size
+        if kind == "whole_pinned":
+            h = torch.from_numpy(data).pin_memory()
+            src = cfa.Source.pinned(h.data_ptr())
+        else:
+            h = aligned_pageable(data.size)
+            h[:] = data
+            src = cfa.Source.host_direct(h.ctypes.data)
+        keep.append(h)
+    d = DeviceDsts(m)
+    with cfa.Plan(entries, d.cfa_dsts, blob_bytes, chunk_bytes=chunk) as plan:
+        plan.load_async(src)
+        plan.wait_layer()
+        ck = plan.checksums()
+        stats = plan.stats()
+    torch.cuda.synchronize()
+    if kind == "file":
+        src.close()
+    compare(m, d, ck, ref, f"{m.name} [{kind}, chunk {chunk}]")
+    if kind == "file":
+        # only the byte ranges the pieces read are read from the file
+        assert stats["staged_bytes"] <= st.data_bytes
+
+
+def test_file_that_shrinks_is_reported_and_the_plan_recovers(tmp_path_factory, tmp_path):
+    m, path, off, ref = prepared("dense", tmp_path_factory)
+    st = cfa.Safetensors.open(path)
+    victim = str(tmp_path / "shrinking.safetensors")
+    with open(path, "rb") as f:
+        whole = f.read()
+    with open(victim, "wb") as f:
+        f.write(whole)
+    entries = st.entries(targets_for(m))
+    d = DeviceDsts(m)
+    with cfa.Plan(entries, d.cfa_dsts, st.data_bytes, chunk_bytes=256 << 10) as plan:
+        with cfa.Source.file(victim, st.data_offset) as src:
+            os.truncate(victim, off + st.data_bytes // 2)
+            plan.load_async(src)
+            with pytest.raises(cfa.CfaError) as e:
+                plan.wait_layer()
+            assert e.value.name == "CFA_ERR_SOURCE"
+        with cfa.Source.file(path, st.data_offset) as src:
+            plan.load_async(src)
+            plan.wait_layer()
+        ck = plan.checksums()
+    compare(m, d, ck, ref, "after a failed file load")
