@@ -237,7 +237,9 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
 def file_attribution(m, pageable, dsts, stream, args, threads):
     """A load from a safetensors file of the checkpoint (its header read by the library, the
     data section read with pread by the fill threads into the pinned ring).  The file is
-    written just before, so it is read from the page cache; it is removed afterwards."""
+    written just before, so buffered reads come from the page cache; O_DIRECT reads (data
+    section at a 4 KiB boundary, so whole blocks land in the pinned slots) come from the
+    storage under the temporary directory.  The file is removed afterwards."""
     import shutil
     import struct
     import tempfile
@@ -251,12 +253,14 @@ def file_attribution(m, pageable, dsts, stream, args, threads):
         if shutil.disk_usage(d).free < m.blob_bytes * 1.2:
             return {"e2e_file": f"not measured: under {m.blob_bytes * 1.2 / 1e9:.0f} GB free"}
         path = os.path.join(d, "model.safetensors")
-        hdr = header_bytes(file_tensors(m))
+        hdr = header_bytes(file_tensors(m), data_align=4096)
         t0 = time.perf_counter()
         with open(path, "wb") as f:
             f.write(struct.pack("<Q", len(hdr)))
             f.write(hdr)
             f.write(memoryview(pageable))
+            f.flush()
+            os.fsync(f.fileno())
         write_s = time.perf_counter() - t0
         st = cfa.Safetensors.open(path)
         plan = cfa.Plan(st.entries(targets_for(m)), dsts.cfa_dsts, st.data_bytes,
@@ -267,13 +271,52 @@ def file_attribution(m, pageable, dsts, stream, args, threads):
             plan.checksums()
             ms = min(_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
                      for _ in range(2))
+        out = {"e2e_file_s_per_model": round(ms / 1e3, 4),
+               "e2e_file_gbs": round(m.blob_bytes / ms / 1e6, 2),
+               "file": f"safetensors, {len(st.tensors)} tensors, page cache (written and "
+                       f"synced in {write_s:.1f} s just before)"}
+        try:
+            with cfa.Source.file(path, st.data_offset, direct=True) as src:
+                plan.load_async(src, stream)
+                plan.checksums()
+                ms = _timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
+            out["e2e_file_direct_s_per_model"] = round(ms / 1e3, 4)
+            out["e2e_file_direct_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
+        except cfa.CfaError as e:
+            out["e2e_file_direct"] = f"unavailable: {e}"
         plan.close()
-        return {"e2e_file_s_per_model": round(ms / 1e3, 4),
-                "e2e_file_gbs": round(m.blob_bytes / ms / 1e6, 2),
-                "file": f"safetensors, {len(st.tensors)} tensors, page cache (written in "
-                        f"{write_s:.1f} s just before)"}
+        return out
     finally:
         shutil.rmtree(d, ignore_errors=True)
+
+
+_COPY = {1: "u8", 2: "u16", 4: "u32", 8: "u64"}
+_CONV_CLASS = {("f32", "bf16"): 4, ("f32", "f16"): 5, ("f16", "bf16"): 6, ("bf16", "f32"): 7,
+               ("f16", "f32"): 8}
+_BLOB_KIND = {"bits": "random bit patterns",
+              "f32mix": "fp32 normal(0, 0.02) with ties and subnormals",
+              "f16fin": "finite fp16 values"}
+
+
+def path_types(m):
+    """(dtype string, dominant work class, its description) of a manifest: the element types
+    the unpack moves (copies by size, conversions by name) and the class with the most bytes."""
+    from workloads import DTYPE_SIZE
+    kinds, by_class = set(), {}
+    for i in range(m.n_entries):
+        s, d = str(m.e_dtype[i]), str(m.d_dtype[int(m.e_dst[i])])
+        n = m.e_numel(i)
+        if m.e_cast[i]:
+            kinds.add(f"{s}->{d}")
+            cls, desc = _CONV_CLASS[(s, d)], f"{s} -> {d} conversion class"
+        else:
+            es = DTYPE_SIZE[s]
+            kinds.add(_COPY[es])
+            cls, desc = es.bit_length() - 1, f"{8 * es}-bit copy class"
+        b = by_class.setdefault(cls, [0, desc])
+        b[0] += n * (DTYPE_SIZE[s] + DTYPE_SIZE[d])
+    cls = max(by_class, key=lambda c: by_class[c][0])
+    return "+".join(sorted(kinds)), cls, by_class[cls][1]
 
 
 def _timed(fn, stream):
@@ -339,7 +382,8 @@ def run_reference(args):
         "impl": "reference", "metric": METRIC, "value": round(gbs, 4), "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(ms, 3), "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "u16", "data": "synthetic (seeded generator)",
+        "vs_baseline": None, "dtype": path_types(m)[0],
+        "data": f"synthetic (seeded counter-based generator; {_BLOB_KIND[m.blob_kind]})",
         "config": {"workload": m.name, "step": "one destination tensor per step, in blob order",
                    "parallelism": "replicas"},
         "cpu_baseline": {"value": round(gbs, 4), "unit": UNIT, "cores": cores, "kind": "oracle",
@@ -503,12 +547,11 @@ def run_ours(args):
         if world > 1:
             dist.destroy_process_group()
         return
+    dtype, cls, cls_desc = path_types(m)
     if st["n_bulk"]:
         kernel_name = "cfa_bulk_kernel (TMA bulk copies) + cfa_unpack_kernel (heads, tails, tiny)"
-    elif bool(m.e_cast.any()):
-        kernel_name = "cfa_unpack_kernel<4> (fp32 -> bf16 cast class)"
     else:
-        kernel_name = "cfa_unpack_kernel (16-byte vector copy)"
+        kernel_name = f"cfa_unpack_kernel<{cls}> ({cls_desc}; 16-byte vectors)"
     peaks, peak_kind = measured_peaks()
     peak = float(peaks.get("hbm_gbs", HBM_FALLBACK_GBS))
     avg_launch_ms = statistics.mean(per_load)
@@ -517,8 +560,8 @@ def run_ours(args):
         "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "u16",
-        "data": "synthetic (seeded counter-based generator; random bf16 bit patterns)",
+        "scaling": "weak", "vs_baseline": None, "dtype": dtype,
+        "data": f"synthetic (seeded counter-based generator; {_BLOB_KIND[m.blob_kind]})",
         "config": {"workload": m.name, "blob_bytes": m.blob_bytes, "tensors": m.n_entries,
                    "destinations": m.n_dsts, "algorithmic_bytes_per_step": algo_bytes,
                    "chunk_bytes": m.chunk_bytes, "kernel_source": "device-resident blob",

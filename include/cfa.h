@@ -411,13 +411,22 @@ cfa_status cfa_safetensors_tensor(const cfa_safetensors *st, size_t i, cfa_st_te
 /* Frees the handle (and the names it owns).  Accepts NULL. */
 cfa_status cfa_safetensors_close(cfa_safetensors *st);
 
+/* cfa_file_source_open flags. */
+#define CFA_FILE_DIRECT 0x1u /* O_DIRECT reads that bypass the page cache (storage bandwidth) */
+
 /*
  * Fills *out with a CALLBACK source that reads blob byte o from file byte data_offset + o with
- * pread (several fill threads may read at once).  The file stays open until
- * cfa_file_source_close(out), which must come after every load using it has completed.
- * Errors: CFA_ERR_SOURCE (cannot open), CFA_ERR_INVAL, CFA_ERR_NOMEM.
+ * pread (several fill threads may read at once).  With CFA_FILE_DIRECT the file is opened with
+ * O_DIRECT: reads move whole 4 KiB blocks; where a destination range and its file range start
+ * at the same offset within a block (data_offset a multiple of 4 KiB and a chunk length that is
+ * too) the middle blocks land in the pinned slot directly, the rest passes through 4 MiB
+ * bounce buffers owned by the source.  The file stays open until cfa_file_source_close(out),
+ * which must come after every load using it has completed.
+ * Errors: CFA_ERR_SOURCE (cannot open; for CFA_FILE_DIRECT also a file system without
+ * O_DIRECT), CFA_ERR_INVAL (unknown flag), CFA_ERR_NOMEM.
  */
-cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, cfa_source *out);
+cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t flags,
+                                cfa_source *out);
 cfa_status cfa_file_source_close(cfa_source *src);
 
 /* Zeroes the plan's checksum buffer on `stream`. */

@@ -173,17 +173,19 @@ class Source:
 
 class FileSource(Source):
     """A checkpoint file read with pread by the plan's fill threads (cfa_file_source_open):
-    blob byte o is file byte data_offset + o.  Close it after the last load that uses it has
-    completed (the context manager does)."""
+    blob byte o is file byte data_offset + o; direct=True reads with O_DIRECT, past the page
+    cache.  Close it after the last load that uses it has completed (the context manager
+    does)."""
 
-    def __init__(self, path, data_offset=0):
+    def __init__(self, path, data_offset=0, direct=False):
         lib = _lib.load()
         self._lib = lib
         self._c = _lib.Source()
-        st = lib.cfa_file_source_open(str(path).encode(), int(data_offset), ctypes.byref(self._c))
+        st = lib.cfa_file_source_open(str(path).encode(), int(data_offset),
+                                      _lib.FILE_DIRECT if direct else 0, ctypes.byref(self._c))
         _check(st)
         super().__init__(_lib.SRC_CALLBACK, 0, 0, self._c.fill, self._c.user)
-        self.path, self.data_offset = str(path), int(data_offset)
+        self.path, self.data_offset, self.direct = str(path), int(data_offset), bool(direct)
 
     def to_c(self):
         if not self._c.user:
@@ -201,7 +203,8 @@ class FileSource(Source):
         self.close()
 
 
-Source.file = staticmethod(lambda path, data_offset=0: FileSource(path, data_offset))
+Source.file = staticmethod(lambda path, data_offset=0, direct=False:
+                           FileSource(path, data_offset, direct))
 
 
 class StTensor(tuple):

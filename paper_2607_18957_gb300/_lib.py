@@ -18,6 +18,7 @@ DTYPE_SIZE = {"u8": 1, "bf16": 2, "f16": 2, "f32": 4, "i32": 4, "i64": 8, "f64":
 ENTRY_CAST_BF16, ENTRY_CKSUM, ENTRY_CONVERT = 0x1, 0x2, 0x4
 OPT_STRICT_COVERAGE, OPT_HOST_ONLY, OPT_TIMING, OPT_BULK, OPT_NO_MERGE = 0x1, 0x2, 0x4, 0x8, 0x10
 SRC_HOST, SRC_PINNED, SRC_CALLBACK, SRC_DEVICE, SRC_HOST_DIRECT = 1, 2, 3, 4, 5
+FILE_DIRECT = 0x1
 ALL = -1
 
 # cfa_tensor_entry and cfa_dst as numpy records (fast for 10^5 entries)
@@ -99,7 +100,7 @@ SIGNATURES = {
     "cfa_safetensors_info": (ctypes.c_int, [_P, _P, _P, _P]),
     "cfa_safetensors_tensor": (ctypes.c_int, [_P, _SZ, _P]),
     "cfa_safetensors_close": (ctypes.c_int, [_P]),
-    "cfa_file_source_open": (ctypes.c_int, [ctypes.c_char_p, _U64, _P]),
+    "cfa_file_source_open": (ctypes.c_int, [ctypes.c_char_p, _U64, ctypes.c_uint32, _P]),
     "cfa_file_source_close": (ctypes.c_int, [_P]),
 }
 

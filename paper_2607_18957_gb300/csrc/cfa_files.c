@@ -14,6 +14,7 @@
 #define _GNU_SOURCE
 #include <errno.h>
 #include <fcntl.h>
+#include <pthread.h>
 #include <stdarg.h>
 #include <stdio.h>
 #include <stdlib.h>
@@ -465,19 +466,31 @@ cfa_status cfa_safetensors_close(cfa_safetensors *st)
 
 /* ---- a file source --------------------------------------------------------------------- */
 
+/* Direct reads: file offsets, lengths and buffer addresses in multiples of this. */
+#define FD_BLOCK 4096u
+/* Bounce buffer size of one direct read. */
+#define FD_BOUNCE (4u << 20)
+
+typedef struct bounce {
+    struct bounce *next;
+    uint8_t *buf; /* FD_BOUNCE bytes, FD_BLOCK-aligned */
+} bounce;
+
 typedef struct {
     int fd;
+    int direct;
     uint64_t data_offset;
     uint64_t file_bytes;
+    pthread_mutex_t mu; /* guards `free_list` */
+    bounce *free_list;  /* bounce buffers not in use (direct reads only) */
 } file_src;
 
-static int file_fill(void *user, uint64_t off, void *dst, uint64_t len)
+/* Reads exactly len bytes at file offset fo into d (buffered, or direct when every one of d,
+ * fo and len is a multiple of FD_BLOCK, except that a direct read may end at end of file). */
+static int read_full(int fd, uint8_t *d, uint64_t len, uint64_t fo)
 {
-    const file_src *f = (const file_src *)user;
-    if (off + len < off || f->data_offset + off + len > f->file_bytes) return 1;
-    uint8_t *d = (uint8_t *)dst;
     for (uint64_t got = 0; got < len;) {
-        const ssize_t k = pread(f->fd, d + got, len - got, (off_t)(f->data_offset + off + got));
+        const ssize_t k = pread(fd, d + got, len - got, (off_t)(fo + got));
         if (k < 0 && errno == EINTR) continue;
         if (k <= 0) return 2;
         got += (uint64_t)k;
@@ -485,21 +498,123 @@ static int file_fill(void *user, uint64_t off, void *dst, uint64_t len)
     return 0;
 }
 
-cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, cfa_source *out)
+static bounce *take_bounce(file_src *f)
+{
+    pthread_mutex_lock(&f->mu);
+    bounce *b = f->free_list;
+    if (b) f->free_list = b->next;
+    pthread_mutex_unlock(&f->mu);
+    if (b) return b;
+    b = (bounce *)calloc(1, sizeof *b);
+    if (!b) return NULL;
+    if (posix_memalign((void **)&b->buf, FD_BLOCK, FD_BOUNCE) != 0) {
+        free(b);
+        return NULL;
+    }
+    return b;
+}
+
+static void give_bounce(file_src *f, bounce *b)
+{
+    pthread_mutex_lock(&f->mu);
+    b->next = f->free_list;
+    f->free_list = b;
+    pthread_mutex_unlock(&f->mu);
+}
+
+/* Direct read of file bytes [fo, fo + len) into d through a bounce buffer: whole blocks are
+ * read into the buffer (the last one may stop at end of file) and the wanted bytes copied out. */
+static int bounce_read(file_src *f, uint8_t *d, uint64_t len, uint64_t fo)
+{
+    bounce *b = take_bounce(f);
+    if (!b) return 3;
+    int rc = 0;
+    while (len && !rc) {
+        const uint64_t a = fo & ~(uint64_t)(FD_BLOCK - 1);
+        const uint64_t head = fo - a;
+        uint64_t want = head + len;
+        if (want > FD_BOUNCE) want = FD_BOUNCE;
+        uint64_t span = (want + FD_BLOCK - 1) & ~(uint64_t)(FD_BLOCK - 1);
+        if (a + span > f->file_bytes) { /* the file's last block: read up to its end */
+            const uint64_t tail = f->file_bytes - a;
+            span = (tail + FD_BLOCK - 1) & ~(uint64_t)(FD_BLOCK - 1);
+            if (want > tail) want = tail;
+        }
+        uint64_t got = 0;
+        while (got < want) {
+            const ssize_t k = pread(f->fd, b->buf + got, span - got, (off_t)(a + got));
+            if (k < 0 && errno == EINTR) continue;
+            if (k <= 0) break;
+            got += (uint64_t)k;
+        }
+        if (got < want || want <= head) {
+            rc = 2;
+            break;
+        }
+        const uint64_t n = want - head;
+        memcpy(d, b->buf + head, n);
+        d += n;
+        fo += n;
+        len -= n;
+    }
+    give_bounce(f, b);
+    return rc;
+}
+
+/* O_DIRECT fill: when the destination and the file offset share their position within a
+ * block, the whole blocks in the middle are read straight into the destination and only the
+ * partial first and last blocks go through a bounce buffer; otherwise everything bounces. */
+static int direct_fill(file_src *f, uint8_t *d, uint64_t len, uint64_t fo)
+{
+    const uint64_t B = FD_BLOCK;
+    if (((uintptr_t)d & (B - 1)) == (fo & (B - 1))) {
+        const uint64_t lo = (fo + B - 1) & ~(B - 1);
+        const uint64_t hi = (fo + len) & ~(B - 1);
+        if (hi > lo) {
+            int rc = 0;
+            if (lo > fo) rc = bounce_read(f, d, lo - fo, fo);
+            if (!rc) rc = read_full(f->fd, d + (lo - fo), hi - lo, lo);
+            if (!rc && fo + len > hi) rc = bounce_read(f, d + (hi - fo), fo + len - hi, hi);
+            return rc;
+        }
+    }
+    return bounce_read(f, d, len, fo);
+}
+
+static int file_fill(void *user, uint64_t off, void *dst, uint64_t len)
+{
+    file_src *f = (file_src *)user;
+    if (off + len < off || f->data_offset + off < off ||
+        f->data_offset + off + len > f->file_bytes)
+        return 1;
+    if (!len) return 0;
+    if (f->direct) return direct_fill(f, (uint8_t *)dst, len, f->data_offset + off);
+    return read_full(f->fd, (uint8_t *)dst, len, f->data_offset + off);
+}
+
+cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t flags,
+                                cfa_source *out)
 {
     g_files_err[0] = 0;
-    if (!path || !out) return CFA_ERR_INVAL;
+    if (!path || !out || (flags & ~(uint32_t)CFA_FILE_DIRECT)) return CFA_ERR_INVAL;
     memset(out, 0, sizeof *out);
     file_src *f = (file_src *)calloc(1, sizeof *f);
     if (!f) return CFA_ERR_NOMEM;
-    f->fd = open(path, O_RDONLY | O_CLOEXEC);
+    f->direct = (flags & CFA_FILE_DIRECT) != 0;
+    f->fd = open(path, O_RDONLY | O_CLOEXEC | (f->direct ? O_DIRECT : 0));
     struct stat sb;
     if (f->fd < 0 || fstat(f->fd, &sb) != 0) {
-        ferr("cannot open %s: %s", path, strerror(errno));
+        if (f->direct && errno == EINVAL)
+            ferr("cannot open %s for direct reads: the file system does not support O_DIRECT",
+                 path);
+        else
+            ferr("cannot open %s: %s", path, strerror(errno));
         if (f->fd >= 0) close(f->fd);
         free(f);
         return CFA_ERR_SOURCE;
     }
+    if (!f->direct) posix_fadvise(f->fd, 0, 0, POSIX_FADV_SEQUENTIAL);
+    pthread_mutex_init(&f->mu, NULL);
     f->data_offset = data_offset;
     f->file_bytes = (uint64_t)sb.st_size;
     out->kind = CFA_SRC_CALLBACK;
@@ -514,6 +629,13 @@ cfa_status cfa_file_source_close(cfa_source *src)
     if (src->kind == CFA_SRC_CALLBACK && src->fill == file_fill && src->user) {
         file_src *f = (file_src *)src->user;
         close(f->fd);
+        for (bounce *b = f->free_list; b;) {
+            bounce *n = b->next;
+            free(b->buf);
+            free(b);
+            b = n;
+        }
+        pthread_mutex_destroy(&f->mu);
         free(f);
         src->user = NULL;
         return CFA_OK;

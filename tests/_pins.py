@@ -9,6 +9,7 @@ What pins what:
   golden_manifests    hand-written manifests with their loaded bytes typed out by hand
   one_to_one          closed form: a 1:1 cast-free load copies blob slices (numpy sum checksums)
   concat_reference    fused layouts equal numpy/torch concatenation and stacking of the parts
+                      (bf16, MoE expert stacks, 8-bit weights with per-block fp32 scales)
   cast_reference      cast entries equal torch's conversion of the source values
   invariants          exact-once coverage, byte conservation, repack(unpack(blob)) == blob,
                       entry-order invariance (Theorem 2), padding independence
@@ -16,6 +17,8 @@ What pins what:
   tp_shards           tensor-parallel shards: each equals numpy slicing of the full tensor, and
                       the shards of all ranks reassemble (numpy concatenate) into the unsharded
                       load
+  ep_shards           expert-parallel ranks: whole experts of the unchanged blob; the ranks'
+                      expert stacks concatenate into the unsharded ones, the rest is replicated
   f16_golden          hand-derived binary16 conversion cases (tests/golden/f16_cases.txt)
   convert_vs_torch    torch's CPU conversions float16 <-> float32, float16 / float32 ->
                       bfloat16, bfloat16 -> float32 (exhaustive over 16-bit inputs)
@@ -25,7 +28,8 @@ import numpy as np
 import torch
 
 import oracle
-from workloads import DTYPE_SIZE, Manifest, dense_config, moe_config, tiny_config
+from workloads import (DTYPE_SIZE, Manifest, dense_config, fp8_block_config, moe_config,
+                       tiny_config)
 
 from _golden import f16_cases, manifest_case, rne_cases
 
@@ -214,11 +218,11 @@ def _mini_dense(src="bf16", seed=31, **kw):
                         inter=96, vocab=100, src_dtype=src, **kw)
 
 
-def _mini_moe(seed=41, **kw):
+def _mini_moe(seed=41, n_experts=3, **kw):
     kw.setdefault("align", 2)
     kw.setdefault("jitter", 3)
     return moe_config("mini_moe", seed, layers=2, hidden=32, n_q=4, n_kv=2, head_dim=8,
-                      inter=48, n_experts=3, vocab=52, n_extra=25, **kw)
+                      inter=48, n_experts=n_experts, vocab=52, n_extra=25, **kw)
 
 
 def _check_against_concat(m, lib):
@@ -270,6 +274,18 @@ def concat_reference(lib=None):
                 off = int(mm.e_offset[i])
                 parts.append(blob[off:off + mm.e_nbytes(i)].view(np.uint16).reshape(I2 // 2, H))
             assert np.array_equal(w13[e], np.concatenate(parts, axis=0)), (j, e)
+    # 8-bit weights with per-block fp32 scales: both passed through; fused weights and fused
+    # scales keep the same part order, one scale row per `block` weight rows
+    for fuse in (True, False):
+        m8 = fp8_block_config("mini_fp8", 37, layers=2, hidden=48, n_q=4, n_kv=2, head_dim=16,
+                              inter=80, vocab=30, block=16, fuse=fuse, align=1, jitter=5)
+        _check_against_concat(m8, lib)
+        for j, name in enumerate(m8.d_name):
+            if name.endswith("_scale_inv"):
+                jw = m8.d_name.index(name[:-len("_scale_inv")])
+                rw, cw = m8.d_shape_tuple(jw)
+                assert m8.d_shape_tuple(j) == (-(-rw // 16), -(-cw // 16)), name
+                assert str(m8.d_dtype[j]) == "f32" and str(m8.d_dtype[jw]) == "u8"
 
 
 def cast_reference(lib=None):
@@ -463,6 +479,41 @@ def _check_reassembly(full, rf, ranks, tp):
     del m0
 
 
+def ep_shards(lib=None):
+    """Expert-parallel ranks read whole experts out of the unchanged blob: each rank's
+    destinations equal concatenation of its parts, and the ranks' w13 / w2 stacked along the
+    expert axis give the unsharded ones; every other destination equals the unsharded load."""
+    full = _mini_moe(seed=36, n_experts=4)
+    blob = _blob(full)
+    rf = oracle.unpack(full, blob, lib=lib)
+    assert rf.status == 0
+    for ep in (2, 4):
+        ranks = []
+        for rank in range(ep):
+            m = _mini_moe(seed=36, n_experts=4, ep=ep, rank=rank)
+            assert m.blob_bytes == full.blob_bytes
+            for i, name in enumerate(m.e_name):
+                assert m.e_offset[i] == full.e_offset[full.e_name.index(name)], name
+            r = oracle.unpack(m, blob, lib=lib)
+            assert r.status == 0, (ep, rank, r.status_name)
+            exp = _expected_by_concat(m, blob)
+            for j in range(m.n_dsts):
+                assert np.array_equal(r.dst[j], exp[j]), (ep, rank, m.d_name[j])
+            ranks.append((m, r))
+        for jf, name in enumerate(full.d_name):
+            want = rf.dst[jf].view(np.uint16).reshape(full.d_shape_tuple(jf))
+            parts = []
+            for m, r in ranks:
+                j = m.d_name.index(name)
+                parts.append(r.dst[j].view(np.uint16).reshape(m.d_shape_tuple(j)))
+            if name.endswith(("w13_weight", "w2_weight")):
+                assert all(p.shape[0] == want.shape[0] // ep for p in parts), name
+                assert np.array_equal(np.concatenate(parts, axis=0), want), name
+            else:
+                for p in parts:
+                    assert np.array_equal(p, want), name
+
+
 def _kv_rows(full, qkv_name):
     prefix = qkv_name.rsplit("qkv_proj", 1)[0]
     i = full.e_name.index(prefix + "k_proj.weight")
@@ -530,5 +581,5 @@ def f16_vs_nearest(lib=None):
 
 
 ALL_PINS = [rne_golden, rne_vs_torch, rne_vs_nearest, golden_manifests, one_to_one,
-            concat_reference, cast_reference, invariants, validation, tp_shards, f16_golden,
-            convert_vs_torch, f16_vs_nearest]
+            concat_reference, cast_reference, invariants, validation, tp_shards, ep_shards,
+            f16_golden, convert_vs_torch, f16_vs_nearest]

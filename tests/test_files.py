@@ -197,23 +197,50 @@ FillFn = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_uint64, ctypes
                           ctypes.c_uint64)
 
 
-def test_file_source_fill_reads_the_data_section(tmp_path):
+def _direct_supported(path):
+    try:
+        fd = os.open(path, os.O_RDONLY | os.O_DIRECT)
+    except OSError:
+        return False
+    os.close(fd)
+    return True
+
+
+@pytest.mark.parametrize("direct,data_align", [(False, 8), (True, 8), (True, 4096)])
+def test_file_source_fill_reads_the_data_section(tmp_path, direct, data_align):
+    """Random ranges, destinations at every offset class within a 4 KiB block (for direct
+    reads: bounced, and block-congruent with the file so the middle blocks land in place),
+    ranges ending at the end of the file, and nothing written outside the range."""
     m = configs()[0]
     p = tmp_path / "model.safetensors"
-    off = write_safetensors(m, p)
+    off = write_safetensors(m, p, data_align=data_align)
+    assert off % data_align == 0
+    if direct and not _direct_supported(p):
+        pytest.skip("the file system has no O_DIRECT")
     blob = m.blob_range(0, m.blob_bytes)
     rng = np.random.default_rng(5)
-    with cfa.Source.file(p, off) as src:
+    B = 4096
+    with cfa.Source.file(p, off, direct=direct) as src:
         c = src.to_c()
         assert c.kind == _lib.SRC_CALLBACK and c.fill and c.user
         fill = FillFn(c.fill)
-        for _ in range(50):
+        cases = []
+        for k in range(60):
             a = int(rng.integers(0, m.blob_bytes))
-            n = int(rng.integers(0, min(1 << 20, m.blob_bytes - a) + 1))
-            buf = np.full(n + 16, 0xAB, dtype=np.uint8)
-            assert fill(c.user, a, buf.ctypes.data + 8, n) == 0
-            assert np.array_equal(buf[8:8 + n], blob[a:a + n])
-            assert (buf[:8] == 0xAB).all() and (buf[8 + n:] == 0xAB).all()
+            n = int(rng.integers(0, min(9 << 20, m.blob_bytes - a) + 1))
+            cases.append((a, n))
+        cases += [(m.blob_bytes - 5, 5), (m.blob_bytes - (3 << 20) - 7, (3 << 20) + 7),
+                  (0, m.blob_bytes), (B - off % B, 5 * B), (0, 1)]
+        for k, (a, n) in enumerate(cases):
+            raw = np.full(n + 3 * B, 0xAB, dtype=np.uint8)
+            base = raw.ctypes.data
+            if k % 2:  # block-congruent with the file offset
+                lead = ((off + a) - (base + 64)) % B + 64
+            else:
+                lead = 64 + 7 * k % B
+            assert fill(c.user, a, base + lead, n) == 0, (a, n)
+            assert np.array_equal(raw[lead:lead + n], blob[a:a + n]), (a, n, lead)
+            assert (raw[:lead] == 0xAB).all() and (raw[lead + n:] == 0xAB).all()
         buf = np.zeros(16, dtype=np.uint8)
         assert fill(c.user, m.blob_bytes - 8, buf.ctypes.data, 16) != 0  # past the end
         assert fill(c.user, (1 << 64) - 4, buf.ctypes.data, 8) != 0    # offset wraps

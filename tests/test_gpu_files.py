@@ -1,8 +1,8 @@
 """GPU parity for checkpoint files: a safetensors file written from a seeded manifest is loaded
 through its header (Safetensors.entries) and compared byte for byte, checksum for checksum,
 with the oracle on the manifest.  Sources: the pread file source (data section staged through
-the pinned ring), and the whole file read into page-locked or pageable memory with the blob
-being the whole file.  Whole tensors, row and column shards, conversions; a file that shrinks
+the pinned ring, buffered or O_DIRECT), and the whole file read into page-locked or pageable
+memory with the blob being the whole file.  Whole tensors, row and column shards, conversions; a file that shrinks
 under a load is reported as a source error and the plan recovers."""
 import os
 
@@ -114,6 +114,28 @@ def test_parity_from_a_safetensors_file(tmp_path_factory, name, kind, chunk):
     if kind == "file":
         # only the byte ranges the pieces read are read from the file
         assert stats["staged_bytes"] <= st.data_bytes
+
+
+@pytest.mark.parametrize("data_align", [8, 4096])
+@pytest.mark.parametrize("name", ["dense", "f32_tp", "moe_tp"])
+def test_parity_from_a_file_with_direct_reads(tmp_path_factory, tmp_path, name, data_align):
+    """O_DIRECT reads: through bounce buffers (data section at an 8-byte boundary), or for the
+    most part straight into the pinned slots (data section at a 4 KiB boundary)."""
+    m, _, _, ref = prepared(name, tmp_path_factory)
+    path = str(tmp_path / "direct.safetensors")
+    off = write_safetensors(m, path, data_align=data_align)
+    try:
+        src = cfa.Source.file(path, off, direct=True)
+    except cfa.CfaError as e:
+        pytest.skip(f"no O_DIRECT here: {e}")
+    st = cfa.Safetensors.open(path)
+    d = DeviceDsts(m)
+    with src, cfa.Plan(st.entries(targets_for(m)), d.cfa_dsts, st.data_bytes,
+                       chunk_bytes=1 << 20) as plan:
+        plan.load_async(src)
+        plan.wait_layer()
+        ck = plan.checksums()
+    compare(m, d, ck, ref, f"{m.name} [direct, data at {data_align}]")
 
 
 def test_file_that_shrinks_is_reported_and_the_plan_recovers(tmp_path_factory, tmp_path):

@@ -1,5 +1,6 @@
-"""GPU parity at the full sizes of the five workloads, in the launch configurations the
-benchmark times: every destination byte and every checksum against the oracle (run per batch of
+"""GPU parity at the full sizes of the five workloads (plus a tensor-parallel rank of the 70B
+one, an expert-parallel rank of the MoE one and an 8-bit block-scaled 8B checkpoint), in the
+launch configurations the benchmark times: every destination byte and every checksum against the oracle (run per batch of
 destinations on regenerated blob windows, on all host cores).  Also the per-layer readiness
 times of the 70B-shaped streaming load."""
 import os
@@ -151,6 +152,46 @@ def test_full_mixtral_8x7b_bf16():
     d.buf.fill_(0xA5)
     cb = CallbackSource(m)
     ck2, _, _ = _load(m, d, cb.source(), fill_threads=16)
+    assert np.array_equal(ck, ck2)
+    verify_all(m, d, ck2)
+
+
+def test_full_mixtral_8x7b_bf16_expert_parallel_rank():
+    """Rank 3 of 8 experts-wise: expert 3 of every layer plus the replicated attention, router,
+    norms, vocabulary and 200k extras, read from the whole checkpoint (device-resident, then
+    staged from the callback source, which fills only the rank's byte ranges)."""
+    m = workloads.named_config("mixtral_8x7b_bf16_ep8r3")
+    assert len(m.unread) == 32 * 7 * 3
+    d = DeviceDsts(m)
+    blob = device_source_blob(m)
+    ck, st, _ = _load(m, d, cfa.Source.device(blob.data_ptr()), dev_slots=0, host_slots=0)
+    assert st["bytes_read"] < m.blob_bytes // 4
+    verify_all(m, d, ck)
+    assert d.guards_intact()
+    del blob
+    torch.cuda.empty_cache()
+    d.buf.fill_(0xA5)
+    cb = CallbackSource(m)
+    ck2, st2, _ = _load(m, d, cb.source(), fill_threads=16)
+    assert st2["staged_bytes"] < m.blob_bytes // 4
+    assert np.array_equal(ck, ck2)
+    verify_all(m, d, ck2)
+
+
+def test_full_llama3_8b_fp8_block128():
+    """8-bit weights with fp32 per-128x128-block scales (fused like the weights), bf16
+    embedding, norms and head: device-resident and pinned-host loads."""
+    m = workloads.named_config("llama3_8b_fp8_block128")
+    d = DeviceDsts(m)
+    blob = device_source_blob(m)
+    ck, st, _ = _load(m, d, cfa.Source.device(blob.data_ptr()), dev_slots=0, host_slots=0)
+    verify_all(m, d, ck)
+    assert d.guards_intact()
+    del blob
+    host = torch.empty(m.blob_bytes, dtype=torch.uint8, pin_memory=True)
+    m.fill_source_ptr(host.data_ptr())
+    d.buf.fill_(0xA5)
+    ck2, _, _ = _load(m, d, cfa.Source.pinned(host.data_ptr()), host_slots=0)
     assert np.array_equal(ck, ck2)
     verify_all(m, d, ck2)
 

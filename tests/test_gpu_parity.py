@@ -11,7 +11,7 @@ import torch
 
 import oracle
 import paper_2607_18957_gb300 as cfa
-from workloads import dense_config, moe_config, tiny_config
+from workloads import dense_config, fp8_block_config, moe_config, tiny_config
 from workloads.harness import CallbackSource, DeviceDsts, entries_for, pinned_blob
 
 pytestmark = pytest.mark.gpu
@@ -152,10 +152,23 @@ def cfg_bf16_f32_norms_tp():
                         jitter=5, tp=2, rank=0)
 
 
+def cfg_moe_ep():
+    return moe_config("moe_ep4r2", 74, layers=2, hidden=256, n_q=4, n_kv=2, head_dim=64,
+                      inter=512, n_experts=8, vocab=500, n_extra=300, align=2, jitter=3, ep=4,
+                      rank=2)
+
+
+def cfg_fp8_block():
+    # 8-bit weights at odd byte offsets with fp32 block scales (scales fused like the weights)
+    return fp8_block_config("fp8_block", 75, layers=2, hidden=512, n_q=8, n_kv=2, head_dim=64,
+                            inter=1536, vocab=1000, block=128, align=1, jitter=7)
+
+
 CONFIGS = {"tiny": cfg_tiny, "dense": cfg_dense, "dense_f32": cfg_dense_f32, "moe": cfg_moe,
            "dense_tp": cfg_dense_tp, "f32_tp": cfg_f32_tp, "moe_tp": cfg_moe_tp,
            "f32_f16": cfg_f32_to_f16, "f16_bf16": cfg_f16_bits_to_bf16,
-           "bf16_f32norm_tp": cfg_bf16_f32_norms_tp}
+           "bf16_f32norm_tp": cfg_bf16_f32_norms_tp, "moe_ep": cfg_moe_ep,
+           "fp8_block": cfg_fp8_block}
 
 
 @pytest.mark.parametrize("cfg", list(CONFIGS))

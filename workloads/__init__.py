@@ -10,6 +10,7 @@ from .manifests import (  # noqa: F401
     Manifest,
     tiny_config,
     dense_config,
+    fp8_block_config,
     moe_config,
     named_config,
     NAMED_CONFIGS,

@@ -30,6 +30,11 @@ def file_tensors(m):
         if name in seen and seen[name] != key:
             raise ValueError(f"two different tensors named {name}")
         seen[name] = key
+    for name, dt, full, off in m.unread:
+        nb = DTYPE_SIZE[dt] * int(np.prod(full, dtype=np.int64))
+        if name in seen:
+            raise ValueError(f"two different tensors named {name}")
+        seen[name] = (name, dt, tuple(int(x) for x in full), int(off), nb)
     ts = sorted(seen.values(), key=lambda t: t[3])
     out, pos, k = [], 0, 0
     for t in ts:
@@ -45,20 +50,22 @@ def file_tensors(m):
     return out
 
 
-def header_bytes(tensors, metadata=None):
-    """The JSON header (padded with spaces to a multiple of 8 bytes, counting the length word)."""
+def header_bytes(tensors, metadata=None, data_align=8):
+    """The JSON header, padded with spaces so that the data section (after the 8-byte length
+    word and the header) starts at a multiple of data_align bytes."""
     h = {}
     if metadata is not None:
         h["__metadata__"] = metadata
     for name, dt, shape, off, nb in tensors:
         h[name] = {"dtype": ST_DTYPE[dt], "shape": list(shape), "data_offsets": [off, off + nb]}
     raw = json.dumps(h, separators=(",", ":")).encode()
-    return raw + b" " * ((-len(raw)) % 8)
+    return raw + b" " * ((-(8 + len(raw))) % data_align)
 
 
-def write_safetensors(m, path, piece=64 << 20):
+def write_safetensors(m, path, piece=64 << 20, data_align=8):
     """Writes m's blob as a safetensors file at `path`; returns the data section's file offset."""
-    hdr = header_bytes(file_tensors(m), metadata={"format": "pt", "source": m.name})
+    hdr = header_bytes(file_tensors(m), metadata={"format": "pt", "source": m.name},
+                       data_align=data_align)
     tmp = str(path) + ".part"
     with open(tmp, "wb") as f:
         f.write(struct.pack("<Q", len(hdr)))
