@@ -382,20 +382,40 @@ __device__ __forceinline__ void block_flush(uint64_t &acc, uint32_t ck, unsigned
     acc = 0;
 }
 
-/* One launch: the block-level items of one class (first), then its warp-level items. */
+/* One launch: the block-level items (slabs) and the warp-level items (tiny pieces, in groups of
+ * one per warp) of one class.  The groups are spread evenly among the slabs: a tiny piece is
+ * bound by memory latency, a slab by bandwidth, so a CTA working on tiny pieces overlaps with
+ * its SM neighbours streaming slabs instead of all of them running at the end of the launch.
+ * Item i of the first n_groups * (q + 1) items (q = n_slabs / n_groups) is group i / (q + 1)
+ * when i mod (q + 1) == q, else slab (i / (q + 1)) * q + i mod (q + 1); the items after those
+ * are the remaining slabs in order. */
 template <int CLS>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_unpack_kernel(const UnpackArgs a)
 {
     __shared__ unsigned long long red[kWarps];
     const uint32_t n_groups = (a.n_tiny + kWarps - 1) / kWarps;
     const uint32_t n_items = a.n_slabs + n_groups;
+    const uint32_t q = n_groups ? a.n_slabs / n_groups : 0;
+    const uint32_t mixed = n_groups * (q + 1); /* items in the interleaved prefix */
     const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
     uint64_t acc = 0;
     uint32_t acc_ck = CFA_NO_CK;
 
     for (uint32_t item = blockIdx.x; item < n_items; item += gridDim.x) {
-        if (item < a.n_slabs) {
-            const cfa_work w = a.slabs[item]; /* the same 32 bytes for every thread */
+        uint32_t slab, group;
+        bool is_slab;
+        if (item < mixed) {
+            const uint32_t p = item / (q + 1), r = item - p * (q + 1);
+            is_slab = r != q;
+            slab = p * q + r;
+            group = p;
+        } else {
+            is_slab = true;
+            slab = n_groups * q + (item - mixed);
+            group = 0;
+        }
+        if (is_slab) {
+            const cfa_work w = a.slabs[slab]; /* the same 32 bytes for every thread */
             if (!item_ok<CLS>(w, a)) {
                 if (threadIdx.x == 0) atomicCAS(a.status, 0, 1);
                 continue;
@@ -409,7 +429,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_unpack_kernel(const 
         } else {
             if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
             acc_ck = CFA_NO_CK;
-            const uint32_t t = (item - a.n_slabs) * kWarps + warp;
+            const uint32_t t = group * kWarps + warp;
             if (t < a.n_tiny) {
                 const cfa_work w = a.tiny[t];
                 if (!item_ok<CLS>(w, a)) {
