@@ -210,7 +210,7 @@ static int jskip(jrd *r)
         }
     } else if (c == '-' || (c >= '0' && c <= '9')) {
         r->p++;
-        while (r->p < r->end && strchr("0123456789.eE+-", *r->p)) r->p++;
+        while (r->p < r->end && *r->p && strchr("0123456789.eE+-", *r->p)) r->p++;
     } else if (r->end - r->p >= 4 && !memcmp(r->p, "true", 4)) {
         r->p += 4;
     } else if (r->end - r->p >= 5 && !memcmp(r->p, "false", 5)) {

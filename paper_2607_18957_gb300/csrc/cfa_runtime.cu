@@ -96,6 +96,9 @@ struct DeviceGuard {
 
 } // namespace
 
+/* Kernels of one launch group beyond the first run on up to this many side streams. */
+constexpr int kSideStreams = 2;
+
 struct cfa_plan {
     cfa_host_plan hp{};
     bool host_only = false;
@@ -115,6 +118,9 @@ struct cfa_plan {
     uint8_t *h_slots = nullptr;
     int n_host_slots = 0;
     cudaStream_t fill_stream = nullptr, copy_stream = nullptr, aux_stream = nullptr;
+    /* side streams that run a launch group's other kernels beside the caller's stream */
+    cudaStream_t side_stream[kSideStreams] = {nullptr};
+    cudaEvent_t ev_fork = nullptr, ev_join[kSideStreams] = {nullptr};
     std::vector<cudaEvent_t> ev_dev_free, ev_h2d, ev_host_free, ev_filled, ev_layer;
     cudaEvent_t ev_begin = nullptr, ev_all = nullptr;
     std::vector<cudaEvent_t> t_h2d0, t_h2d1, t_k0, t_k1;
@@ -197,8 +203,12 @@ void CUDART_CB fill_host_fn(void *arg)
 
 /* Unpacks chunks [c0, c1), whose blob byte o sits at device address src_base + o (or
  * src_base + (o mod period) for a periodic source): per work class present in those chunks
- * (normally one), a TMA bulk launch for its aligned cast-free slabs and a vector launch for
- * everything else. */
+ * (normally one), a TMA bulk launch for its aligned cast-free slabs, a launch for its column
+ * slices and a vector launch for everything else.  The kernels of one group write disjoint
+ * destination bytes and add their checksums atomically, so they are independent: the first
+ * runs on `s`, the others on side streams forked from `s` and joined back into it, so that
+ * one kernel's last CTAs overlap the next kernel's first instead of the GPU draining between
+ * them. */
 cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint64_t period,
                   cudaStream_t s)
 {
@@ -207,36 +217,53 @@ cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint
     const uint64_t hi = std::min<uint64_t>(hp.blob_bytes, (uint64_t)c1 * hp.chunk_bytes);
     const size_t row = (size_t)hp.n_chunks + 1;
     const bool timing_on = (hp.opts.flags & CFA_OPT_TIMING) != 0;
+    enum { BULK, STRIDED, VECTOR };
+    struct Job {
+        int type, k;
+        uint32_t a0, a1, b0, b1;
+    };
+    Job jobs[3 * CFA_N_CLASSES];
+    int n = 0;
     for (int k = 0; k < CFA_N_CLASSES && hp.n_bulk; ++k) {
         const uint32_t b0 = hp.bulk_first[k * row + c0], b1 = hp.bulk_first[k * row + c1];
-        if (b1 == b0) continue;
-        const bool timing = timing_on && p->last_launches < p->t_k0.size();
-        if (timing) CK(p, cudaEventRecord(p->t_k0[p->last_launches], s));
-        CK(p, cfa_launch_bulk(k, p->d_bulk + b0, b1 - b0, src_base, period, lo, hi, p->d_ck,
-                              p->d_status, p->bulk_grid_cap[k], s));
-        if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], s));
-        p->last_launches++;
+        if (b1 != b0) jobs[n++] = Job{BULK, k, b0, b1, 0, 0};
     }
     for (int k = 0; k < CFA_N_CLASSES && hp.n_strided; ++k) {
         const uint32_t r0 = hp.strided_first[k * row + c0], r1 = hp.strided_first[k * row + c1];
-        if (r1 == r0) continue;
-        const bool timing = timing_on && p->last_launches < p->t_k0.size();
-        if (timing) CK(p, cudaEventRecord(p->t_k0[p->last_launches], s));
-        CK(p, cfa_launch_strided(k, p->d_strided + r0, r1 - r0, src_base, period, lo, hi,
-                                 p->d_ck, p->d_status, p->strided_grid_cap[k], s));
-        if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], s));
-        p->last_launches++;
+        if (r1 != r0) jobs[n++] = Job{STRIDED, k, r0, r1, 0, 0};
     }
     for (int k = 0; k < CFA_N_CLASSES; ++k) {
         const uint32_t s0 = hp.slab_first[k * row + c0], s1 = hp.slab_first[k * row + c1];
         const uint32_t t0 = hp.tiny_first[k * row + c0], t1 = hp.tiny_first[k * row + c1];
-        if (s1 == s0 && t1 == t0) continue;
+        if (s1 != s0 || t1 != t0) jobs[n++] = Job{VECTOR, k, s0, s1, t0, t1};
+    }
+    const int n_side = std::min(n - 1, kSideStreams);
+    if (n_side > 0) {
+        CK(p, cudaEventRecord(p->ev_fork, s));
+        for (int j = 0; j < n_side; ++j) CK(p, cudaStreamWaitEvent(p->side_stream[j], p->ev_fork, 0));
+    }
+    for (int i = 0; i < n; ++i) {
+        const Job &J = jobs[i];
+        const int k = J.k;
+        cudaStream_t ls = i == 0 ? s : p->side_stream[(i - 1) % kSideStreams];
         const bool timing = timing_on && p->last_launches < p->t_k0.size();
-        if (timing) CK(p, cudaEventRecord(p->t_k0[p->last_launches], s));
-        CK(p, cfa_launch_unpack(k, p->d_slabs + s0, s1 - s0, p->d_tiny + t0, t1 - t0, src_base,
-                                period, lo, hi, p->d_ck, p->d_status, p->grid_cap[k], s));
-        if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], s));
+        if (timing) CK(p, cudaEventRecord(p->t_k0[p->last_launches], ls));
+        if (J.type == BULK)
+            CK(p, cfa_launch_bulk(k, p->d_bulk + J.a0, J.a1 - J.a0, src_base, period, lo, hi,
+                                  p->d_ck, p->d_status, p->bulk_grid_cap[k], ls));
+        else if (J.type == STRIDED)
+            CK(p, cfa_launch_strided(k, p->d_strided + J.a0, J.a1 - J.a0, src_base, period, lo,
+                                     hi, p->d_ck, p->d_status, p->strided_grid_cap[k], ls));
+        else
+            CK(p, cfa_launch_unpack(k, p->d_slabs + J.a0, J.a1 - J.a0, p->d_tiny + J.b0,
+                                    J.b1 - J.b0, src_base, period, lo, hi, p->d_ck, p->d_status,
+                                    p->grid_cap[k], ls));
+        if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], ls));
         p->last_launches++;
+    }
+    for (int j = 0; j < n_side; ++j) {
+        CK(p, cudaEventRecord(p->ev_join[j], p->side_stream[j]));
+        CK(p, cudaStreamWaitEvent(s, p->ev_join[j], 0));
     }
     return CFA_OK;
 }
@@ -279,6 +306,12 @@ void release(cfa_plan *p)
         kill(p->t_k1);
         if (p->ev_begin) cudaEventDestroy(p->ev_begin);
         if (p->ev_all) cudaEventDestroy(p->ev_all);
+        if (p->ev_fork) cudaEventDestroy(p->ev_fork);
+        for (int j = 0; j < kSideStreams; ++j) {
+            if (p->side_stream[j]) cudaStreamSynchronize(p->side_stream[j]);
+            if (p->ev_join[j]) cudaEventDestroy(p->ev_join[j]);
+            if (p->side_stream[j]) cudaStreamDestroy(p->side_stream[j]);
+        }
         if (p->fill_stream) cudaStreamDestroy(p->fill_stream);
         if (p->copy_stream) cudaStreamDestroy(p->copy_stream);
         if (p->aux_stream) cudaStreamDestroy(p->aux_stream);
@@ -393,6 +426,11 @@ cfa_status setup_device(cfa_plan *p)
     CK(nullptr, cudaStreamCreateWithFlags(&p->fill_stream, cudaStreamNonBlocking));
     CK(nullptr, cudaStreamCreateWithFlags(&p->copy_stream, cudaStreamNonBlocking));
     CK(nullptr, cudaStreamCreateWithFlags(&p->aux_stream, cudaStreamNonBlocking));
+    for (int j = 0; j < kSideStreams; ++j) {
+        CK(nullptr, cudaStreamCreateWithFlags(&p->side_stream[j], cudaStreamNonBlocking));
+        if ((st = make_event(nullptr, &p->ev_join[j], false))) return st;
+    }
+    if ((st = make_event(nullptr, &p->ev_fork, false))) return st;
     const bool timing = (o.flags & CFA_OPT_TIMING) != 0;
     auto events = [&](std::vector<cudaEvent_t> &v, size_t n, bool t) -> cfa_status {
         v.assign(n, nullptr);

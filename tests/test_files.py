@@ -159,6 +159,8 @@ BAD_HEADERS = [
     b'{"a": {"dtype": "U8", "shape": [4294967296, 4294967296], "data_offsets": [0, 8]}}',
     b'{"__metadata__": ' + b"[" * 100 + b"]" * 100 + b"}",
     b'{"a": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]}',
+    b'{"__metadata__": {"x": 1\x002}}',
+    b'{"a\x00": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]}}',
 ]
 
 
