@@ -395,38 +395,62 @@ def run_reference(args):
 
 
 # ------------------------------------------------------------------------------------------
+class Ranks:
+    """The job's processes: one per GPU under torchrun (RANK / LOCAL_RANK / WORLD_SIZE /
+    MASTER_* from the environment), each loading its own replica of the checkpoint.  The
+    collectives only serve the timing: a barrier on both sides of the timed region, the maximum
+    of the ranks' times and the sum of their units.  NCCL on GPUs; gloo on the host (tests)."""
+
+    def __init__(self, backend="nccl", device="cuda"):
+        import torch.distributed as dist
+        self.dist = dist
+        self.world = int(os.environ.get("WORLD_SIZE", "1"))
+        self.rank = int(os.environ.get("RANK", "0"))
+        self.local = int(os.environ.get("LOCAL_RANK", "0"))
+        self.device = device
+        if self.world > 1:
+            dist.init_process_group(backend)
+
+    def _reduce(self, x, op):
+        if self.world == 1:
+            return float(x)
+        import torch
+        t = torch.tensor([float(x)], dtype=torch.float64, device=self.device)
+        self.dist.all_reduce(t, op=op)
+        return float(t.item())
+
+    def barrier(self):
+        if self.world > 1:
+            self.dist.barrier()
+
+    def max(self, x):
+        return self._reduce(x, self.dist.ReduceOp.MAX)
+
+    def sum(self, x):
+        return self._reduce(x, self.dist.ReduceOp.SUM)
+
+    def close(self):
+        if self.world > 1:
+            self.dist.destroy_process_group()
+
+
+def whole_job_gbs(ranks, bytes_this_rank, ms_this_rank):
+    """Whole-job throughput: the bytes all ranks moved over the slowest rank's time."""
+    return ranks.sum(bytes_this_rank) / (ranks.max(ms_this_rank) / 1e3) / 1e9
+
+
 def run_ours(args):
     import numpy as np
     import torch
-    import torch.distributed as dist
 
     import paper_2607_18957_gb300 as cfa
     from workloads.harness import DeviceDsts, entries_for, pinned_blob
 
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     torch.cuda.set_device(local)
-    if world > 1:
-        dist.init_process_group("nccl")
-
-    def barrier():
-        if world > 1:
-            dist.barrier()
-
-    def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
-
-    def sum_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        return float(t.item())
+    ranks = Ranks("nccl", "cuda")
+    world, rank = ranks.world, ranks.rank
+    barrier, max_over_ranks, sum_over_ranks = ranks.barrier, ranks.max, ranks.sum
 
     m = make_workload(args.workload)
     t_setup = time.time()
@@ -475,7 +499,7 @@ def run_ours(args):
     ck_dev = plan.checksums()
     plan.close()
     total_ms = max_over_ranks(kernel_ms)
-    value = sum_over_ranks(algo_bytes * args.steps) / (total_ms / 1e3) / 1e9
+    value = whole_job_gbs(ranks, algo_bytes * args.steps, kernel_ms)
 
     # ---------------- end to end: pinned host blob -> final layout through the C ABI ---------
     e2e = None
@@ -544,8 +568,7 @@ def run_ours(args):
                "sample": desc}
 
     if rank != 0:
-        if world > 1:
-            dist.destroy_process_group()
+        ranks.close()
         return
     dtype, cls, cls_desc = path_types(m)
     if st["n_bulk"]:
@@ -580,8 +603,7 @@ def run_ours(args):
         "setup_s": round(setup_s, 2),
     }
     print(json.dumps(line), flush=True)
-    if world > 1:
-        dist.destroy_process_group()
+    ranks.close()
 
 
 def main():
