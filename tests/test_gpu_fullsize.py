@@ -217,6 +217,54 @@ def test_full_llama3_70b_bf16_tensor_parallel_rank():
     verify_all(m, d, ck2)
 
 
+def _past_4gib_manifest():
+    """Tensors with more than 2^32 bytes and elements, at blob offsets and destination offsets
+    beyond 4 GiB, source offsets off the 16-byte grid, and an fp32 -> bf16 conversion of
+    1.1 G elements (random fp32 bit patterns: NaNs, infinities and subnormals included)."""
+    nb = 2_300_000_001        # bf16 elements (4.6 GB)
+    nu = 4_400_000_003        # u8 elements (4.4 GB)
+    nc = 1_100_000_000        # fp32 elements converted to bf16
+    o_small, o_bf, o_u8 = 0, 2050, 2050 + 2 * nb + 13
+    o_f32 = (o_u8 + nu + 3) // 4 * 4 + 4
+    blob = o_f32 + 4 * nc + 100
+    entries = [
+        {"name": "small", "dtype": "bf16", "shape": (777,), "offset": o_small, "dst": 0},
+        {"name": "big_bf16", "dtype": "bf16", "shape": (nb,), "offset": o_bf, "dst": 1},
+        {"name": "big_u8", "dtype": "u8", "shape": (nu,), "offset": o_u8, "dst": 2},
+        {"name": "big_cast", "dtype": "f32", "shape": (nc,), "offset": o_f32, "dst": 3,
+         "cast": True},
+    ]
+    dsts = [{"name": "small", "dtype": "bf16", "shape": (777,)},
+            {"name": "big_bf16", "dtype": "bf16", "shape": (nb,)},
+            {"name": "big_u8", "dtype": "u8", "shape": (nu,)},
+            {"name": "big_cast", "dtype": "bf16", "shape": (nc,)}]
+    return workloads.Manifest("past_4gib", entries, dsts, blob, "bits", 77,
+                              chunk_bytes=1 << 30)
+
+
+def test_tensors_past_4_gib():
+    m = _past_4gib_manifest()
+    d = DeviceDsts(m)
+    assert d.offsets[-1] > (1 << 32)
+    blob = device_source_blob(m)
+    ck, st, _ = _load(m, d, cfa.Source.device(blob.data_ptr()), dev_slots=0, host_slots=0)
+    verify_all(m, d, ck)
+    assert d.guards_intact()
+    del blob
+    torch.cuda.empty_cache()
+    # staged through pinned slots of 512 MiB from the callback source
+    d.buf.fill_(0xA5)
+    cb = CallbackSource(m)
+    with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=512 << 20,
+                  fill_threads=16) as plan:
+        plan.load_async(cb.source())
+        plan.wait_layer()
+        ck2 = plan.checksums()
+    assert np.array_equal(ck, ck2)
+    verify_all(m, d, ck2)
+    assert d.guards_intact()
+
+
 def test_full_llama3_70b_bf16_streamed():
     m = workloads.named_config("llama3_70b_bf16")
     d = DeviceDsts(m)
