@@ -151,8 +151,9 @@ typedef struct cfa_dst {
 #define CFA_OPT_TIMING          0x4u  /* record per-chunk timing events (cfa_get_stats, timeline) */
 #define CFA_OPT_BULK            0x8u  /* copy cast-free slabs whose source, destination and
                                          length are multiples of 16 bytes with the TMA bulk-copy
-                                         kernel instead of the 16-byte vector kernel (off by
-                                         default: the vector kernel is 1-2 % faster on GB300) */
+                                         kernel; without it every slab takes the 16-byte vector
+                                         kernel.  Set by cfa_plan_opts_default: the bulk kernel
+                                         is 1-4 % faster on GB300 */
 #define CFA_OPT_NO_MERGE        0x10u /* DEVICE sources: one launch per chunk instead of one
                                          launch per contiguous run of chunks */
 
@@ -187,7 +188,9 @@ void cfa_plan_opts_default(cfa_plan_opts *opts);
                                  Page-locked memory always qualifies; pageable memory needs a
                                  device that can access it (cudaDevAttrPageableMemoryAccess:
                                  Grace-Blackwell and Grace-Hopper over NVLink-C2C), otherwise
-                                 the load is refused with CFA_ERR_INVAL before any GPU work */
+                                 the load is refused with CFA_ERR_INVAL before any GPU work.
+                                 Host memory is read by the vector kernel only: the TMA bulk
+                                 path is kept for device memory */
 
 /* Writes blob bytes [blob_offset, blob_offset + len) to host memory dst and returns 0, or
  * returns non-zero on failure.  It runs on a CUDA host-function thread and must not call CUDA. */

@@ -315,7 +315,7 @@ class Plan:
 
     def __init__(self, entries, dsts, blob_bytes, chunk_bytes=512 << 20, host_slots=2,
                  dev_slots=2, fill_threads=8, slab_bytes=65536, tiny_bytes=8192, strict=True,
-                 host_only=False, timing=False, bulk=False, no_merge=False, device=-1,
+                 host_only=False, timing=False, bulk=True, no_merge=False, device=-1,
                  workspace=0, workspace_bytes=0):
         lib = _lib.load()
         self._lib = lib

@@ -1,19 +1,24 @@
 /*
  * TMA bulk-copy unpack: the "InGPU -> Loaded" copy of InstantInfer section 4.2 for large
  * contiguous runs that need no cast and whose source, destination and length are multiples of
- * 16 bytes.  Instead of every thread moving 16-byte vectors through registers, one thread per
- * CTA drives the Tensor Memory Accelerator with non-tensor bulk copies:
+ * 16 bytes.  Instead of every thread moving 16-byte vectors through registers, the Tensor
+ * Memory Accelerator moves the bytes with non-tensor bulk copies:
  *
  *     global (staging) --cp.async.bulk--> shared stage --cp.async.bulk--> global (destination)
  *
- * through a ring of shared-memory stages.  Loads run kStages - 1 sub-blocks ahead of the
- * stores; completion of a load is signalled on the stage's mbarrier (complete_tx); a stage is
- * reloaded only after the bulk store that read it has finished reading (bulk_group wait).  The
- * other threads only sum the stage for the per-tensor checksum while the store drains it.  Plain
- * cp.async.bulk only: no tensor maps, no multicast, one CTA's own shared memory.
+ * Each CTA is two warps over a ring of two 32 KiB stages, three CTAs per SM:
+ *   - warp 0 (one lane) loads: it waits until a stage is empty, then issues the bulk load of the
+ *     next sub-block into it, completing on the stage's `full` mbarrier (complete_tx);
+ *   - warp 1 consumes: it waits on `full`, sums the stage for the per-tensor checksum (all 32
+ *     lanes), and one lane issues the bulk store; once the store of the previous sub-block has
+ *     finished reading its stage (bulk_group read wait), that stage is released on its `empty`
+ *     mbarrier.
+ * No block-wide barrier runs inside the loop.  Plain cp.async.bulk only: no tensor maps, no
+ * multicast, one CTA's own shared memory.
  *
- * Every wait is bounded: a wait that runs out sets the status word, the CTA waits (again
- * bounded) for its own copies still in flight, and returns.
+ * Every wait is bounded: a wait that runs out sets the status word and ends both loops; the CTA
+ * then waits (again bounded) for the loads it issued but did not consume, and for its stores,
+ * and returns.
  */
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -22,11 +27,10 @@
 
 namespace {
 
-constexpr int kThreads = 128;
-constexpr int kWarps = kThreads / 32;
-constexpr int kStages = 4;
-constexpr uint32_t kStageBytes = 24 * 1024;
-constexpr uint32_t kSmemBytes = kStages * kStageBytes; /* 96 KiB: two CTAs per SM */
+constexpr int kThreads = 64; /* warp 0 loads, warp 1 checksums and stores */
+constexpr int kStages = 2;
+constexpr uint32_t kStageBytes = 32 * 1024;
+constexpr uint32_t kSmemBytes = kStages * kStageBytes; /* 64 KiB: three CTAs per SM */
 constexpr uint32_t kSpinLimit = 1u << 20;              /* try_wait polls before giving up */
 
 struct BulkArgs {
@@ -131,20 +135,17 @@ __device__ __forceinline__ uint64_t warp_sum(uint64_t v)
     return v;
 }
 
-__device__ __forceinline__ void block_flush(uint64_t &acc, uint32_t ck, unsigned long long *out,
-                                            unsigned long long *red)
+/* Adds the consumer warp's checksum to slot ck; all 32 lanes call it. */
+__device__ __forceinline__ void warp_flush(uint64_t &acc, uint32_t ck, unsigned long long *out)
 {
     const uint64_t v = warp_sum(acc);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        unsigned long long t = 0;
-#pragma unroll
-        for (int q = 0; q < kWarps; ++q) t += red[q];
-        atomicAdd(out + ck, t);
-    }
-    __syncthreads();
+    if ((threadIdx.x & 31) == 0) atomicAdd(out + ck, v);
     acc = 0;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 
 /* A bulk item is sound if its source lies inside the launch's readable range and source,
@@ -158,20 +159,12 @@ __device__ __forceinline__ bool bulk_item_ok(const cfa_work &w, const BulkArgs &
            ((w.src | w.dst | bytes | a.src_base | a.src_period) & 15u) == 0;
 }
 
-/* Walks the sub-blocks of this CTA's items (items blockIdx.x, + gridDim.x, ...), each at most
- * kStageBytes long. */
-struct Cursor {
-    uint32_t item, off, count;
-    __device__ Cursor() : item(blockIdx.x), off(0), count(0) {}
-    __device__ void advance(uint32_t len, uint32_t total)
-    {
-        off += len;
-        ++count;
-        if (off >= total) {
-            off = 0;
-            item += gridDim.x;
-        }
-    }
+/* What the consumer needs of a staged sub-block; written by the producer before the load is
+ * issued, published to the consumer by the stage's `full` barrier.  len == 0 ends the stream. */
+struct StageMeta {
+    uint64_t dst;
+    uint32_t len;
+    uint32_t ck;
 };
 
 template <int LOG2ES>
@@ -179,83 +172,138 @@ __global__ void __launch_bounds__(kThreads) cfa_bulk_kernel(const BulkArgs a)
 {
     extern __shared__ __align__(128) uint8_t stage[];
     __shared__ __align__(8) uint64_t full[kStages];
-    __shared__ unsigned long long red[kWarps];
-    __shared__ int aborted;
+    __shared__ __align__(8) uint64_t empty[kStages];
+    __shared__ StageMeta meta[kStages];
+    __shared__ volatile int aborted;
+    __shared__ uint32_t n_issued, n_consumed;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) mbar_init(&full[s], 1);
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], 1);
+        }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         aborted = 0;
+        n_issued = 0;
+        n_consumed = 0;
     }
     __syncthreads();
+    const uint32_t lane = threadIdx.x & 31u;
 
-    /* producer (thread 0): issues the load of the next sub-block, if any */
-    Cursor prod;
-    auto issue = [&]() {
-        while (prod.item < a.n_items && !bulk_item_ok<LOG2ES>(a.items[prod.item], a))
-            prod.item += gridDim.x;
-        if (prod.item >= a.n_items) return;
-        const cfa_work w = a.items[prod.item];
-        const uint32_t total = w.n << LOG2ES;
-        const uint32_t len = min(kStageBytes, total - prod.off);
-        const int s = prod.count % kStages;
-        mbar_expect_tx(&full[s], len);
-        const uint64_t off = a.src_period ? w.src % a.src_period : w.src;
-        bulk_load(stage + s * kStageBytes,
-                  reinterpret_cast<const uint8_t *>(a.src_base + off) + prod.off, len, &full[s]);
-        prod.advance(len, total);
-    };
-    if (threadIdx.x == 0)
-        for (int k = 0; k < kStages - 1; ++k) issue();
-
-    uint64_t acc = 0;
-    uint32_t acc_ck = CFA_NO_CK;
-    Cursor cons;
-    while (cons.item < a.n_items) {
-        const cfa_work w = a.items[cons.item];
-        if (!bulk_item_ok<LOG2ES>(w, a)) { /* skipped by the producer too */
-            if (threadIdx.x == 0) atomicCAS(a.status, 0, 1);
-            cons.item += gridDim.x;
-            continue;
+    if (threadIdx.x < 32) {
+        /* producer: sub-block p goes to stage p mod kStages once sub-block p - kStages, the
+         * stage's previous tenant, has been released.  The next item's descriptor is fetched
+         * while the current item's sub-blocks are issued. */
+        if (lane == 0) {
+            /* item `it` is being issued from w; item it + gridDim.x is in flight into nxt */
+            uint32_t it = blockIdx.x, p = 0, off = 0;
+            bool have = it < a.n_items;
+            cfa_work w{}, nxt{};
+            if (have) w = a.items[it];
+            uint32_t it_n = it + gridDim.x;
+            if (it_n < a.n_items) nxt = a.items[it_n];
+            auto step = [&]() { /* move to the next item of this CTA */
+                it = it_n;
+                have = it < a.n_items;
+                if (have) {
+                    w = nxt;
+                    it_n = it + gridDim.x;
+                    if (it_n < a.n_items) nxt = a.items[it_n];
+                }
+            };
+            auto settle = [&]() { /* skip items that fail the checks */
+                while (have && !bulk_item_ok<LOG2ES>(w, a)) {
+                    atomicCAS(a.status, 0, 1);
+                    step();
+                }
+            };
+            settle();
+            for (;;) {
+                const int s = p % kStages;
+                if (p >= kStages && !mbar_wait(&empty[s], ((p / kStages) - 1u) & 1u)) {
+                    aborted = 1;
+                    break;
+                }
+                if (!have || aborted) { /* end marker: a plain arrive completes the phase */
+                    meta[s].len = 0;
+                    mbar_arrive(&full[s]);
+                    break;
+                }
+                const uint32_t total = w.n << LOG2ES;
+                const uint32_t len = min(kStageBytes, total - off);
+                meta[s].dst = w.dst + off;
+                meta[s].len = len;
+                meta[s].ck = w.ck;
+                mbar_expect_tx(&full[s], len);
+                const uint64_t so = a.src_period ? w.src % a.src_period : w.src;
+                bulk_load(stage + s * kStageBytes,
+                          reinterpret_cast<const uint8_t *>(a.src_base + so) + off, len,
+                          &full[s]);
+                ++p;
+                n_issued = p;
+                off += len;
+                if (off >= total) {
+                    off = 0;
+                    step();
+                    settle();
+                }
+            }
         }
-        const uint32_t total = w.n << LOG2ES;
-        const uint32_t len = min(kStageBytes, total - cons.off);
-        const int s = cons.count % kStages;
-        if (!mbar_wait(&full[s], (cons.count / kStages) & 1u)) aborted = 1;
-        __syncthreads();
-        if (aborted) break;
-        if (w.ck != acc_ck) {
-            if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
-            acc_ck = w.ck;
+    } else {
+        /* consumer: checksum and store sub-block c, then release the stage of c - 1 */
+        uint64_t acc = 0;
+        uint32_t acc_ck = CFA_NO_CK;
+        uint32_t c = 0;
+        for (;; ++c) {
+            const int s = c % kStages;
+            const bool ok = mbar_wait(&full[s], (c / kStages) & 1u);
+            if (__any_sync(0xFFFFFFFFu, !ok)) {
+                if (lane == 0) aborted = 1;
+                break;
+            }
+            const StageMeta m = meta[s];
+            if (m.len == 0) break;
+            if (m.ck != acc_ck) {
+                if (acc_ck != CFA_NO_CK) warp_flush(acc, acc_ck, a.ck);
+                acc_ck = m.ck;
+            }
+            if (m.ck != CFA_NO_CK) {
+                /* eight independent shared loads per lane in flight, then the ragged rest */
+                const uint4 *v = reinterpret_cast<const uint4 *>(stage + s * kStageBytes);
+                const uint32_t nv = m.len >> 4;
+                uint32_t i = lane;
+                for (; i + 7 * 32 < nv; i += 8 * 32) {
+                    uint4 x[8];
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) x[u] = v[i + u * 32];
+#pragma unroll
+                    for (int u = 0; u < 8; ++u) acc += vsum<1 << LOG2ES>(x[u]);
+                }
+                for (; i < nv; i += 32) acc += vsum<1 << LOG2ES>(v[i]);
+            }
+            if (lane == 0) {
+                bulk_store(reinterpret_cast<uint8_t *>(m.dst), stage + s * kStageBytes, m.len);
+                bulk_commit();
+                /* the store of c - 1 has read its stage, and every lane finished summing it
+                 * before the __syncwarp that ended iteration c - 1 */
+                bulk_wait_read_all_but_one();
+                if (c >= 1) mbar_arrive(&empty[(c - 1) % kStages]);
+            }
+            __syncwarp();
         }
-        if (w.ck != CFA_NO_CK) {
-            const uint4 *v = reinterpret_cast<const uint4 *>(stage + s * kStageBytes);
-            for (uint32_t i = threadIdx.x; i < (len >> 4); i += kThreads) acc += vsum<1 << LOG2ES>(v[i]);
-        }
-        if (threadIdx.x == 0) {
-            bulk_store(reinterpret_cast<uint8_t *>(w.dst) + cons.off, stage + s * kStageBytes,
-                       len);
-            bulk_commit();
-            /* the stage loaded next is the one the previous store read from */
-            bulk_wait_read_all_but_one();
-        }
-        /* every thread has finished reading stage s (checksum) before it can be reloaded */
-        __syncthreads();
-        if (threadIdx.x == 0) issue();
-        cons.advance(len, total);
-    }
-    if (aborted) {
-        if (threadIdx.x == 0) {
-            atomicCAS(a.status, 0, 2);
-            /* loads issued but not consumed: wait for them (bounded) before shared memory goes */
-            for (uint32_t c = cons.count; c < prod.count; ++c)
-                mbar_wait(&full[c % kStages], (c / kStages) & 1u);
+        if (acc_ck != CFA_NO_CK) warp_flush(acc, acc_ck, a.ck);
+        if (lane == 0) {
             bulk_wait_all();
+            n_consumed = c;
         }
-        return;
     }
-    if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
-    if (threadIdx.x == 0) bulk_wait_all();
+    __syncthreads();
+    if (aborted && threadIdx.x == 0) {
+        atomicCAS(a.status, 0, 2);
+        /* loads issued but not consumed: wait for them (bounded) before shared memory goes */
+        for (uint32_t k = n_consumed; k < n_issued; ++k)
+            mbar_wait(&full[k % kStages], (k / kStages) & 1u);
+    }
 }
 
 typedef void (*bulk_fn)(const BulkArgs);

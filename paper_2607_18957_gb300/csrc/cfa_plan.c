@@ -56,7 +56,7 @@ void cfa_plan_opts_default(cfa_plan_opts *o)
     o->device = -1;
     o->slab_bytes = 65536;
     o->tiny_bytes = 8192;
-    o->flags = CFA_OPT_STRICT_COVERAGE;
+    o->flags = CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK;
 }
 
 static void fail(char *err, size_t n, const char *fmt, ...)

@@ -208,16 +208,18 @@ void CUDART_CB fill_host_fn(void *arg)
  * destination bytes and add their checksums atomically, so they are independent: the first
  * runs on `s`, the others on side streams forked from `s` and joined back into it, so that
  * one kernel's last CTAs overlap the next kernel's first instead of the GPU draining between
- * them. */
+ * them.  With tma = false (a source in host memory, read over the host link) the aligned slabs
+ * planned for the TMA kernel are copied by the vector kernel instead: bulk copies are for
+ * device memory. */
 cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint64_t period,
-                  cudaStream_t s)
+                  cudaStream_t s, bool tma = true)
 {
     const cfa_host_plan &hp = p->hp;
     const uint64_t lo = (uint64_t)c0 * hp.chunk_bytes;
     const uint64_t hi = std::min<uint64_t>(hp.blob_bytes, (uint64_t)c1 * hp.chunk_bytes);
     const size_t row = (size_t)hp.n_chunks + 1;
     const bool timing_on = (hp.opts.flags & CFA_OPT_TIMING) != 0;
-    enum { BULK, STRIDED, VECTOR };
+    enum { BULK, BULK_AS_VECTOR, STRIDED, VECTOR };
     struct Job {
         int type, k;
         uint32_t a0, a1, b0, b1;
@@ -226,7 +228,7 @@ cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint
     int n = 0;
     for (int k = 0; k < CFA_N_CLASSES && hp.n_bulk; ++k) {
         const uint32_t b0 = hp.bulk_first[k * row + c0], b1 = hp.bulk_first[k * row + c1];
-        if (b1 != b0) jobs[n++] = Job{BULK, k, b0, b1, 0, 0};
+        if (b1 != b0) jobs[n++] = Job{tma ? BULK : BULK_AS_VECTOR, k, b0, b1, 0, 0};
     }
     for (int k = 0; k < CFA_N_CLASSES && hp.n_strided; ++k) {
         const uint32_t r0 = hp.strided_first[k * row + c0], r1 = hp.strided_first[k * row + c1];
@@ -251,6 +253,9 @@ cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint
         if (J.type == BULK)
             CK(p, cfa_launch_bulk(k, p->d_bulk + J.a0, J.a1 - J.a0, src_base, period, lo, hi,
                                   p->d_ck, p->d_status, p->bulk_grid_cap[k], ls));
+        else if (J.type == BULK_AS_VECTOR) /* bulk items are copy-class slabs of class k */
+            CK(p, cfa_launch_unpack(k, p->d_bulk + J.a0, J.a1 - J.a0, nullptr, 0, src_base,
+                                    period, lo, hi, p->d_ck, p->d_status, p->grid_cap[k], ls));
         else if (J.type == STRIDED)
             CK(p, cfa_launch_strided(k, p->d_strided + J.a0, J.a1 - J.a0, src_base, period, lo,
                                      hi, p->d_ck, p->d_status, p->strided_grid_cap[k], ls));
@@ -466,7 +471,10 @@ cfa_status check_status_word(cfa_plan *p)
     CK(p, cudaMemcpyAsync(&h, p->d_status, sizeof(int), cudaMemcpyDeviceToHost, p->aux_stream));
     CK(p, cudaStreamSynchronize(p->aux_stream));
     if (h) {
-        set_err(p, "the unpack kernel rejected a work item outside its chunk");
+        set_err(p, h == 2 ? "a TMA bulk-copy wait ran out (status word 2)"
+                          : "the unpack kernel rejected a work item outside its chunk or of the "
+                            "wrong class (status word %d)",
+                h);
         return CFA_ERR_DEVICE;
     }
     return CFA_OK;
@@ -657,7 +665,8 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
                                                                                  : hp.n_chunks;
         for (uint32_t c0 = 0; c0 < hp.n_chunks;) {
             const uint32_t c1 = std::min<uint32_t>(hp.n_chunks, c0 + per_run);
-            cfa_status st = launch(p, c0, c1, base, src->period_bytes, cs);
+            cfa_status st =
+                launch(p, c0, c1, base, src->period_bytes, cs, kind == CFA_SRC_DEVICE);
             if (st) return st;
             if ((st = record_layers(p, c0, c1, cs))) return st;
             c0 = c1;

@@ -66,7 +66,7 @@ def test_random_manifest_on_the_gpu(seed):
     kw = dict(chunk_bytes=256 * int(rng.choice([1, 3, 17, 256, 4096])),
               slab_bytes=int(rng.choice([4096, 65536])),
               tiny_bytes=int(rng.choice([0, 256, 8192])),
-              bulk=bool(rng.random() < 0.4))
+              bulk=bool(rng.random() < 0.6))
     with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, **kw) as plan:
         for rep in range(2):  # twice: plan reuse must give the same state
             plan.load_async(src)

@@ -207,21 +207,34 @@ def test_parity_work_splits(slab, tiny):
 @pytest.mark.parametrize("cfg", list(CONFIGS))
 @pytest.mark.parametrize("kind", ["device", "pinned", "callback"])
 @pytest.mark.parametrize("chunk", [4096 + 256, 1 << 20])
-def test_parity_bulk_path(cfg, kind, chunk):
-    """With CFA_OPT_BULK the aligned cast-free slabs go through the TMA bulk kernel."""
+def test_parity_vector_only_path(cfg, kind, chunk):
+    """Without CFA_OPT_BULK every slab, aligned or not, goes through the vector kernel."""
     m = CONFIGS[cfg]()
-    st = load_and_compare(m, kind, chunk=chunk, bulk=True)
-    if cfg in ("dense_f32", "f32_f16"):
-        assert st["n_bulk"] == 0  # conversions never take the bulk path
+    st = load_and_compare(m, kind, chunk=chunk, bulk=False)
+    assert st["n_bulk"] == 0
 
 
 def test_bulk_path_takes_every_aligned_slab():
     m = dense_config("dense_aligned", 67, layers=2, hidden=512, n_q=8, n_kv=2, head_dim=64,
                      inter=1536, vocab=1000, align=256)
-    st = load_and_compare(m, "device", chunk=1 << 20, bulk=True)
-    assert st["n_bulk"] > 0 and st["n_slabs"] == 0
     st = load_and_compare(m, "device", chunk=1 << 20)
+    assert st["n_bulk"] > 0 and st["n_slabs"] == 0
+    st = load_and_compare(m, "device", chunk=1 << 20, bulk=False)
     assert st["n_bulk"] == 0 and st["n_slabs"] > 0
+    # conversions never take the bulk path
+    st = load_and_compare(CONFIGS["dense_f32"](), "device", chunk=1 << 20)
+    assert st["n_bulk"] == 0
+
+
+@pytest.mark.parametrize("kind", ["direct_pageable", "direct_pinned", "device", "pinned"])
+def test_aligned_slabs_from_host_memory(kind):
+    """A 16-byte-aligned checkpoint (every slab a bulk item) of about 200 MB read in place from
+    host memory takes the vector kernel for its bulk items; from device memory and staging slots
+    the TMA kernel."""
+    m = dense_config("aligned_200mb", 76, layers=2, hidden=2048, n_q=16, n_kv=4, head_dim=128,
+                     inter=6144, vocab=8000, align=256)
+    st = load_and_compare(m, kind, chunk=16 << 20)
+    assert st["n_bulk"] > 0 and st["n_slabs"] == 0
 
 
 def test_parity_aligned_full_tiny_workload():

@@ -278,3 +278,22 @@ def test_full_size_manifests_plan_on_the_host():
             assert st["n_layers"] == m.n_groups()
             pcs = p.pieces()
             assert int(pcs["n_elems"].sum()) == sum(m.e_numel(i) for i in range(m.n_entries))
+
+
+def test_default_options_take_the_bulk_path():
+    """cfa_plan_opts_default turns the TMA bulk path on; the binding's default follows it."""
+    import ctypes
+    lib = _lib.load()
+    o = _lib.PlanOpts()
+    lib.cfa_plan_opts_default(ctypes.byref(o))
+    assert o.flags & _lib.OPT_BULK and o.flags & _lib.OPT_STRICT_COVERAGE
+    import inspect
+    assert inspect.signature(cfa.Plan).parameters["bulk"].default is True
+    # aligned cast-free slabs become bulk items by default, and never with bulk=False
+    m = dense_config("d_aligned", 52, 2, 64, 4, 2, 16, 96, 100, align=256)
+    with host_plan(m, chunk_bytes=1 << 20, tiny_bytes=0) as p:
+        st = p.stats()
+        assert st["n_bulk"] > 0 and st["n_slabs"] == 0
+    with host_plan(m, chunk_bytes=1 << 20, tiny_bytes=0, bulk=False) as p:
+        st = p.stats()
+        assert st["n_bulk"] == 0 and st["n_slabs"] > 0
