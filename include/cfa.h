@@ -442,6 +442,17 @@ cfa_status cfa_reset_checksums(cfa_plan *plan, cfa_stream stream);
  */
 cfa_status cfa_plan_destroy(cfa_plan *plan);
 
+/*
+ * Self-test of the loader's only device-side waits, the TMA kernel's bounded mbarrier waits
+ * (no counterpart in the paper): on `device` (-1 = current) one CTA of the TMA kernel is given a
+ * valid 16-byte item, a short wait limit and a loader that issues nothing, so its first wait for
+ * a staged sub-block runs out.  *status_word receives the status word the kernel left: 2 when
+ * the expired wait ended the kernel cleanly.  The CUDA context stays usable.  Allocates and
+ * frees a few hundred bytes of device memory; synchronizes the device.
+ * Errors: CFA_ERR_INVAL (status_word NULL), CFA_ERR_CUDA.
+ */
+cfa_status cfa_selftest_wait_timeout(int device, int *status_word);
+
 /* Detail of the last failure (see the conventions above).  Never NULL. */
 const char *cfa_last_error(const cfa_plan *plan);
 

@@ -102,6 +102,7 @@ SIGNATURES = {
     "cfa_safetensors_close": (ctypes.c_int, [_P]),
     "cfa_file_source_open": (ctypes.c_int, [ctypes.c_char_p, _U64, ctypes.c_uint32, _P]),
     "cfa_file_source_close": (ctypes.c_int, [_P]),
+    "cfa_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_int, _P]),
 }
 
 _lib = None

@@ -32,11 +32,13 @@ constexpr int kStages = 2;
 constexpr uint32_t kStageBytes = 32 * 1024;
 constexpr uint32_t kSmemBytes = kStages * kStageBytes; /* 64 KiB: three CTAs per SM */
 constexpr uint32_t kSpinLimit = 1u << 20;              /* try_wait polls before giving up */
+constexpr uint32_t kLoseLoads = 1u << 31;              /* self-test: the loader issues nothing */
 
 struct BulkArgs {
     const cfa_work *items;
     uint32_t n_items;
-    uint32_t pad;
+    uint32_t spin_limit; /* try_wait polls before a wait gives up; the self-test sets a short one
+                            and tells the loader to issue nothing (spin_limit | kLoseLoads) */
     uint64_t src_base;
     uint64_t src_period; /* 0, or P: blob byte o sits at src_base + (o mod P) */
     uint64_t src_lo, src_hi;
@@ -75,9 +77,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
 }
 
 /* Waits for phase `parity` of the barrier to complete; false if the spin limit ran out. */
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity)
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity, uint32_t limit)
 {
-    for (uint32_t k = 0; k < kSpinLimit; ++k)
+    for (uint32_t k = 0; k < limit; ++k)
         if (mbar_try_wait(bar, parity)) return true;
     return false;
 }
@@ -189,6 +191,7 @@ __global__ void __launch_bounds__(kThreads) cfa_bulk_kernel(const BulkArgs a)
     }
     __syncthreads();
     const uint32_t lane = threadIdx.x & 31u;
+    const uint32_t limit = a.spin_limit & ~kLoseLoads;
 
     if (threadIdx.x < 32) {
         /* producer: sub-block p goes to stage p mod kStages once sub-block p - kStages, the
@@ -220,7 +223,8 @@ __global__ void __launch_bounds__(kThreads) cfa_bulk_kernel(const BulkArgs a)
             settle();
             for (;;) {
                 const int s = p % kStages;
-                if (p >= kStages && !mbar_wait(&empty[s], ((p / kStages) - 1u) & 1u)) {
+                if (a.spin_limit & kLoseLoads) break; /* self-test: nothing arrives on full */
+                if (p >= kStages && !mbar_wait(&empty[s], ((p / kStages) - 1u) & 1u, limit)) {
                     aborted = 1;
                     break;
                 }
@@ -256,7 +260,7 @@ __global__ void __launch_bounds__(kThreads) cfa_bulk_kernel(const BulkArgs a)
         uint32_t c = 0;
         for (;; ++c) {
             const int s = c % kStages;
-            const bool ok = mbar_wait(&full[s], (c / kStages) & 1u);
+            const bool ok = mbar_wait(&full[s], (c / kStages) & 1u, limit);
             if (__any_sync(0xFFFFFFFFu, !ok)) {
                 if (lane == 0) aborted = 1;
                 break;
@@ -302,7 +306,7 @@ __global__ void __launch_bounds__(kThreads) cfa_bulk_kernel(const BulkArgs a)
         atomicCAS(a.status, 0, 2);
         /* loads issued but not consumed: wait for them (bounded) before shared memory goes */
         for (uint32_t k = n_consumed; k < n_issued; ++k)
-            mbar_wait(&full[k % kStages], (k / kStages) & 1u);
+            mbar_wait(&full[k % kStages], (k / kStages) & 1u, limit);
     }
 }
 
@@ -339,7 +343,7 @@ extern "C" cudaError_t cfa_launch_bulk(int log2es, const cfa_work *items, uint32
     BulkArgs a;
     a.items = items;
     a.n_items = n_items;
-    a.pad = 0;
+    a.spin_limit = kSpinLimit;
     a.src_base = src_base;
     a.src_period = src_period;
     a.src_lo = src_lo;
@@ -349,4 +353,56 @@ extern "C" cudaError_t cfa_launch_bulk(int log2es, const cfa_work *items, uint32
     const uint32_t grid = n_items < (uint32_t)grid_cap ? n_items : (uint32_t)grid_cap;
     kBulk[log2es]<<<grid, kThreads, kSmemBytes, stream>>>(a);
     return cudaGetLastError();
+}
+
+/* Self-test of the bounded waits: one CTA of the TMA kernel over one valid 16-byte item, with a
+ * short wait limit and its loader told to issue nothing, so the consumer's first wait on `full`
+ * runs out.  The kernel must flag the status word (2) and return; the context stays usable. */
+extern "C" cudaError_t cfa_bulk_selftest_timeout(int *status_host)
+{
+    cfa_work *d_item = nullptr;
+    uint8_t *d_buf = nullptr;
+    unsigned long long *d_ck = nullptr;
+    int *d_status = nullptr;
+    cudaError_t e = cudaSuccess;
+    if (!status_host) return cudaErrorInvalidValue;
+    *status_host = -1;
+    if ((e = cudaFuncSetAttribute(kBulk[1], cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)kSmemBytes)) != cudaSuccess)
+        return e;
+    if ((e = cudaMalloc(&d_item, sizeof(cfa_work))) != cudaSuccess) goto out;
+    if ((e = cudaMalloc(&d_buf, 512)) != cudaSuccess) goto out;
+    if ((e = cudaMalloc(&d_ck, sizeof(unsigned long long))) != cudaSuccess) goto out;
+    if ((e = cudaMalloc(&d_status, sizeof(int))) != cudaSuccess) goto out;
+    {
+        cfa_work w{};
+        w.src = 0;
+        w.dst = (uint64_t)(uintptr_t)(d_buf + 256);
+        w.n = 8; /* 16 bytes of 16-bit elements */
+        w.ck = 0;
+        w.mode = CFA_MODE(1, 1, 0);
+        if ((e = cudaMemcpy(d_item, &w, sizeof w, cudaMemcpyHostToDevice)) != cudaSuccess) goto out;
+        if ((e = cudaMemset(d_status, 0, sizeof(int))) != cudaSuccess) goto out;
+        if ((e = cudaMemset(d_ck, 0, sizeof(unsigned long long))) != cudaSuccess) goto out;
+        BulkArgs a;
+        a.items = d_item;
+        a.n_items = 1;
+        a.spin_limit = 256u | kLoseLoads;
+        a.src_base = (uint64_t)(uintptr_t)d_buf;
+        a.src_period = 0;
+        a.src_lo = 0;
+        a.src_hi = 256;
+        a.ck = d_ck;
+        a.status = d_status;
+        kBulk[1]<<<1, kThreads, kSmemBytes>>>(a);
+        if ((e = cudaGetLastError()) != cudaSuccess) goto out;
+        if ((e = cudaDeviceSynchronize()) != cudaSuccess) goto out;
+        e = cudaMemcpy(status_host, d_status, sizeof(int), cudaMemcpyDeviceToHost);
+    }
+out:
+    if (d_item) cudaFree(d_item);
+    if (d_buf) cudaFree(d_buf);
+    if (d_ck) cudaFree(d_ck);
+    if (d_status) cudaFree(d_status);
+    return e;
 }

@@ -53,6 +53,7 @@ extern "C" cudaError_t cfa_launch_bulk(int log2es, const cfa_work *items, uint32
                                        uint64_t src_lo, uint64_t src_hi,
                                        unsigned long long *ck, int *status, int grid_cap,
                                        cudaStream_t stream);
+extern "C" cudaError_t cfa_bulk_selftest_timeout(int *status_host);
 extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_t n_slabs,
                                          const cfa_work *tiny, uint32_t n_tiny,
                                          uint64_t src_base, uint64_t src_period,
@@ -922,6 +923,21 @@ size_t cfa_abi_sizeof(const char *type_name)
     if (!std::strcmp(type_name, "cfa_piece")) return sizeof(cfa_piece);
     if (!std::strcmp(type_name, "cfa_st_tensor")) return sizeof(cfa_st_tensor);
     return 0;
+}
+
+cfa_status cfa_selftest_wait_timeout(int device, int *status_word)
+{
+    if (!status_word) return CFA_ERR_INVAL;
+    int prev = 0;
+    CK(nullptr, cudaGetDevice(&prev));
+    if (device >= 0) CK(nullptr, cudaSetDevice(device));
+    const cudaError_t e = cfa_bulk_selftest_timeout(status_word);
+    if (device >= 0) cudaSetDevice(prev);
+    if (e != cudaSuccess) {
+        set_err(nullptr, "TMA wait self-test failed: %s", cudaGetErrorString(e));
+        return CFA_ERR_CUDA;
+    }
+    return CFA_OK;
 }
 
 } /* extern "C" */

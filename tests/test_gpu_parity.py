@@ -397,3 +397,16 @@ def test_empty_plan_loads():
         plan.load_async(cfa.Source.device(0))
         plan.wait_layer()
         assert plan.checksums().size == 0
+
+
+def test_tma_wait_that_runs_out_ends_the_kernel_cleanly():
+    """The TMA kernel's waits are bounded: with its loader issuing nothing, the first wait for a
+    staged sub-block runs out, the kernel flags status 2 and returns, and the context loads
+    correctly afterwards."""
+    import ctypes
+    lib = cfa._lib.load()
+    word = ctypes.c_int(-1)
+    assert lib.cfa_selftest_wait_timeout(-1, ctypes.byref(word)) == 0
+    assert word.value == 2
+    torch.cuda.synchronize()
+    load_and_compare(CONFIGS["dense"](), "device", chunk=1 << 20)
