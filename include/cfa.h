@@ -166,10 +166,10 @@ typedef struct cfa_plan_opts {
     int32_t fill_threads;     /* host threads copying pageable sources into pinned slots; default 8 */
     int32_t device;           /* CUDA device ordinal; -1 = the current device */
     uint32_t slab_bytes;      /* destination bytes per block-level work item, a multiple of 4096;
-                                 default 65536 */
+                                 default 262144 */
     uint32_t tiny_bytes;      /* pieces with fewer destination bytes go warp-per-descriptor;
                                  default 8192 */
-    uint32_t flags;           /* CFA_OPT_*; default CFA_OPT_STRICT_COVERAGE */
+    uint32_t flags;           /* CFA_OPT_*; default CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK */
     uint32_t reserved;        /* must be 0 */
     void *workspace;          /* optional device memory for the staging slots (NULL = plan allocates) */
     uint64_t workspace_bytes; /* must be >= dev_slots * chunk_bytes when workspace is given */

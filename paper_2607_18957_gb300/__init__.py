@@ -14,6 +14,7 @@ memory and streams only, and is imported lazily.
     ck = plan.checksums()
 """
 import ctypes
+import itertools
 
 import numpy as np
 
@@ -51,6 +52,27 @@ def _stream_handle(stream):
     return stream.cuda_stream
 
 
+def _shape_columns(shapes, n):
+    """Shapes (sequences of ints) -> ([n, 8] int64 array, [n] int32 ndim), without a Python loop
+    per element."""
+    if not isinstance(shapes, (list, tuple)):
+        shapes = list(shapes)
+    if len(shapes) != n:
+        raise ValueError(f"{len(shapes)} shapes for {n} entries")
+    nd = np.fromiter((len(s) for s in shapes), dtype=np.int32, count=n)
+    if n and int(nd.max()) > 8:
+        raise ValueError("more than 8 dimensions")
+    out = np.zeros((n, 8), dtype=np.int64)
+    total = int(nd.sum())
+    if total:
+        flat = np.fromiter((int(x) for x in itertools.chain.from_iterable(shapes)),
+                           dtype=np.int64, count=total)
+        rows = np.repeat(np.arange(n), nd)
+        starts = np.repeat(np.cumsum(nd) - nd, nd)
+        out[rows, np.arange(total) - starts] = flat
+    return out, nd
+
+
 def make_entries(dtype, shape, offset, dst, row=None, cast=None, cksum=None, layer=None,
                  names=None, src_row_stride=None):
     """Builds the cfa_tensor_entry array from columns.
@@ -67,16 +89,13 @@ def make_entries(dtype, shape, offset, dst, row=None, cast=None, cksum=None, lay
     """
     n = len(dst)
     e = np.zeros(n, dtype=ENTRY_DTYPE)
-    codes = [DTYPE[str(x)] if not isinstance(x, (int, np.integer)) else int(x) for x in dtype]
-    e["src_dtype"] = np.asarray(codes, dtype=np.int32) if n else 0
+    codes = _dtype_codes(dtype)
+    e["src_dtype"] = codes if n else 0
     if isinstance(shape, tuple) and len(shape) == 2 and isinstance(shape[0], np.ndarray):
         e["shape"] = shape[0]
         e["ndim"] = shape[1]
     else:
-        for i, s in enumerate(shape):
-            s = tuple(int(x) for x in s)
-            e["ndim"][i] = len(s)
-            e["shape"][i, :len(s)] = s
+        e["shape"], e["ndim"] = _shape_columns(shape, n)
     e["blob_offset"] = np.asarray(offset, dtype=np.uint64) if n else 0
     e["dst_index"] = np.asarray(dst, dtype=np.int32) if n else 0
     if row is not None:
@@ -116,15 +135,29 @@ class _Entries:
         return len(self.arr)
 
 
+def _dtype_codes(dtypes):
+    """dtype names or CFA_DTYPE_* codes -> int32 array of codes."""
+    memo = {}
+
+    def code(x):
+        if isinstance(x, (int, np.integer)):
+            return int(x)
+        k = str(x)
+        if k not in memo:
+            memo[k] = DTYPE[k]
+        return memo[k]
+    return np.fromiter((code(x) for x in dtypes), dtype=np.int32)
+
+
 def make_dsts(dsts):
     """[(device pointer, dtype name or code, shape), ...] -> cfa_dst array."""
-    d = np.zeros(len(dsts), dtype=DST_DTYPE)
-    for j, (ptr, dt, shape) in enumerate(dsts):
-        s = tuple(int(x) for x in shape)
-        d["dev_ptr"][j] = int(ptr)
-        d["dtype"][j] = DTYPE[str(dt)] if not isinstance(dt, (int, np.integer)) else int(dt)
-        d["ndim"][j] = len(s)
-        d["shape"][j, :len(s)] = s
+    n = len(dsts)
+    d = np.zeros(n, dtype=DST_DTYPE)
+    if n:
+        ptrs, dts, shapes = zip(*dsts)
+        d["dev_ptr"] = np.fromiter((int(x) for x in ptrs), dtype=np.uint64, count=n)
+        d["dtype"] = _dtype_codes(dts)
+        d["shape"], d["ndim"] = _shape_columns(shapes, n)
     return d
 
 
@@ -314,7 +347,7 @@ class Plan:
     staging slots, streams and events."""
 
     def __init__(self, entries, dsts, blob_bytes, chunk_bytes=512 << 20, host_slots=2,
-                 dev_slots=2, fill_threads=8, slab_bytes=65536, tiny_bytes=8192, strict=True,
+                 dev_slots=2, fill_threads=8, slab_bytes=262144, tiny_bytes=8192, strict=True,
                  host_only=False, timing=False, bulk=True, no_merge=False, device=-1,
                  workspace=0, workspace_bytes=0):
         lib = _lib.load()

@@ -54,7 +54,7 @@ void cfa_plan_opts_default(cfa_plan_opts *o)
     o->dev_slots = 2;
     o->fill_threads = 8;
     o->device = -1;
-    o->slab_bytes = 65536;
+    o->slab_bytes = 262144;
     o->tiny_bytes = 8192;
     o->flags = CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK;
 }
