@@ -32,6 +32,10 @@ constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kUnroll = 4;
 constexpr int kMinBlocks = 4; /* 64 registers per thread at most */
+/* Rounds of 32-vector loads in flight per warp on the realigning path: two for slabs (one or
+ * four are slower: too little in flight, or spills), one for column-slice rows. */
+constexpr int kRealignRounds = 2;
+constexpr int kRealignRoundsRows = 1;
 
 struct UnpackArgs {
     const cfa_work *slabs;
@@ -202,7 +206,7 @@ __device__ __forceinline__ uint64_t copy_elems(const uint8_t *src, uint8_t *dst,
 
 /* Copies nbytes (a multiple of ES) from src to dst; thread tid of nthr.  Returns this thread's
  * share of the checksum. */
-template <int ES, int U>
+template <int ES, int U, int UR>
 __device__ uint64_t copy_run(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst,
                              uint64_t nbytes, uint32_t tid, uint32_t nthr)
 {
@@ -240,12 +244,52 @@ __device__ uint64_t copy_run(const uint8_t *__restrict__ src, uint8_t *__restric
         }
     } else {
         /* source off by k bytes: every 16-byte store takes bytes k..k+15 of two aligned
-         * vectors, both of which hold needed bytes, so nothing outside the run is read */
+         * vectors s[i] and s[i + 1], both of which hold needed bytes, so nothing outside the
+         * run is read.  Each warp takes UR * 32 consecutive vectors per round (lane l, round
+         * u: vector w0 + 32u + l) and loads each once; s[i + 1] comes by shuffle from the
+         * next lane, or for lane 31 from lane 0 of the next round.  The one vector per warp
+         * that has no loaded neighbour (lane 31's last one, or the run's last vector) is loaded
+         * by its lane in the same round of loads. */
         const uint4 *s = reinterpret_cast<const uint4 *>(src - k);
-        for (uint32_t i = tid; i < nvec; i += nthr) {
-            const uint4 o = funnel16(ld_shared_line(s + i), ld_shared_line(s + i + 1), k);
-            st_stream(d + i, o);
-            acc += vsum<ES>(o);
+        const uint32_t lane = tid & 31u, wid = tid >> 5;
+        const uint32_t step = nthr * UR;
+        for (uint32_t base = 0; base < nvec; base += step) {
+            const uint32_t w0 = base + wid * 32u * UR;
+            uint4 a[UR];
+            int own = -1; /* the round whose neighbour this lane loads itself */
+#pragma unroll
+            for (int u = 0; u < UR; ++u) {
+                const uint32_t i = w0 + 32u * u + lane;
+                a[u] = make_uint4(0u, 0u, 0u, 0u);
+                if (i < nvec) {
+                    a[u] = ld_shared_line(s + i);
+                    if (i + 1 == nvec || (lane == 31u && u == UR - 1)) own = u;
+                }
+            }
+            uint4 c = make_uint4(0u, 0u, 0u, 0u);
+            if (own >= 0) c = ld_shared_line(s + w0 + 32u * own + lane + 1);
+#pragma unroll
+            for (int u = 0; u < UR; ++u) {
+                const uint32_t i = w0 + 32u * u + lane;
+                uint4 b, n0;
+                b.x = __shfl_down_sync(0xFFFFFFFFu, a[u].x, 1);
+                b.y = __shfl_down_sync(0xFFFFFFFFu, a[u].y, 1);
+                b.z = __shfl_down_sync(0xFFFFFFFFu, a[u].z, 1);
+                b.w = __shfl_down_sync(0xFFFFFFFFu, a[u].w, 1);
+                if (u + 1 < UR) {
+                    n0.x = __shfl_sync(0xFFFFFFFFu, a[u + 1].x, 0);
+                    n0.y = __shfl_sync(0xFFFFFFFFu, a[u + 1].y, 0);
+                    n0.z = __shfl_sync(0xFFFFFFFFu, a[u + 1].z, 0);
+                    n0.w = __shfl_sync(0xFFFFFFFFu, a[u + 1].w, 0);
+                    if (lane == 31u) b = n0;
+                }
+                if (i < nvec) {
+                    if (own == u) b = c;
+                    const uint4 o = funnel16(a[u], b, k);
+                    st_stream(d + i, o);
+                    acc += vsum<ES>(o);
+                }
+            }
         }
     }
     /* tail */
@@ -354,7 +398,8 @@ __device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs
     if constexpr (C::conv != CFA_CONV_NONE)
         return convert_run<C::ses, C::des, C::conv, (U > 2 ? 2 : U)>(src, dst, w.n, tid, nthr);
     else
-        return copy_run<(1 << CLS), U>(src, dst, (uint64_t)w.n << CLS, tid, nthr);
+        return copy_run<(1 << CLS), U, (U > 1 ? kRealignRounds : 1)>(src, dst,
+                                                                    (uint64_t)w.n << CLS, tid, nthr);
 }
 
 __device__ __forceinline__ uint64_t warp_sum(uint64_t v)
@@ -501,7 +546,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_strided_kernel(const
             if constexpr (C::conv != CFA_CONV_NONE)
                 acc += convert_run<SES, DES, C::conv, 2>(s, d, w.cols, lane, 32u);
             else
-                acc += copy_run<DES, kUnroll>(s, d, (uint64_t)w.cols * DES, lane, 32u);
+                acc += copy_run<DES, kUnroll, kRealignRoundsRows>(s, d, (uint64_t)w.cols * DES,
+                                                                  lane, 32u);
         }
     }
     if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
