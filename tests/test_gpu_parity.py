@@ -410,3 +410,44 @@ def test_tma_wait_that_runs_out_ends_the_kernel_cleanly():
     assert word.value == 2
     torch.cuda.synchronize()
     load_and_compare(CONFIGS["dense"](), "device", chunk=1 << 20)
+
+
+def test_two_plans_load_at_once_from_two_threads():
+    """Two plans (different checkpoints, sources and destinations) loading at the same time on
+    their own streams from their own host threads: each matches the oracle."""
+    import threading
+    cases = []
+    for name, kind in (("moe", "callback"), ("f32_tp", "pinned")):
+        m = CONFIGS[name]()
+        blob, ref = reference(m)
+        keep = []
+        src = make_source(kind, m, blob, keep)
+        d = DeviceDsts(m)
+        plan = cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=256 << 10)
+        cases.append((m, ref, src, d, plan, keep, torch.cuda.Stream()))
+    errors, results = [], {}
+
+    def run(k):
+        m, ref, src, d, plan, keep, stream = cases[k]
+        try:
+            torch.cuda.set_device(0)
+            for _ in range(3):
+                plan.load_async(src, stream)
+                plan.wait_layer()
+            results[k] = plan.checksums()
+        except Exception as e:  # reported below
+            errors.append(e)
+
+    threads = [threading.Thread(target=run, args=(k,)) for k in range(len(cases))]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join(timeout=300)
+    assert not errors, errors
+    torch.cuda.synchronize()
+    for k, (m, ref, src, d, plan, keep, stream) in enumerate(cases):
+        for j in range(m.n_dsts):
+            assert np.array_equal(d.host_bytes(j), ref.dst[j]), (m.name, m.d_name[j])
+        assert np.array_equal(results[k], ref.cksum), m.name
+        assert d.guards_intact()
+        plan.close()
