@@ -319,6 +319,18 @@ cfa_status cfa_get_stats(cfa_plan *plan, cfa_stats *out);
  */
 cfa_status cfa_get_layer_times(cfa_plan *plan, float *ms_out, size_t n);
 
+/* One chunk of the last load on the timeline, in milliseconds from its first operation; -1 where
+ * the step did not run (no host->device copy for in-place sources).  A merged launch over several
+ * chunks gives each of them the launch's interval. */
+typedef struct cfa_chunk_times {
+    float h2d_begin_ms, h2d_end_ms;       /* the chunk's copies into its device slot */
+    float unpack_begin_ms, unpack_end_ms; /* first start and last end of the kernels reading it */
+} cfa_chunk_times;
+
+/* Per-chunk timeline of the last load, chunks 0 .. n-1 (n <= n_chunks; CFA_OPT_TIMING plans;
+ * blocks until the load completes).  Errors: CFA_ERR_INVAL (no timing, no load, n too large). */
+cfa_status cfa_get_timeline(cfa_plan *plan, cfa_chunk_times *out, size_t n);
+
 /*
  * Number of readiness groups and pieces of the plan; then the pieces themselves, in chunk order
  * (at most cap of them into out).  Host-only; works on CFA_OPT_HOST_ONLY plans.
@@ -460,7 +472,8 @@ const char *cfa_last_error(const cfa_plan *plan);
 const char *cfa_status_name(cfa_status st);
 
 /* sizeof of the ABI struct with this name ("cfa_tensor_entry", "cfa_dst", "cfa_plan_opts",
- * "cfa_source", "cfa_stats", "cfa_piece", "cfa_st_tensor"), or 0 for an unknown name; lets a binding check its
+ * "cfa_source", "cfa_stats", "cfa_piece", "cfa_st_tensor", "cfa_chunk_times"), or 0 for an
+ * unknown name; lets a binding check its
  * own copies of the layouts.  Host-only. */
 size_t cfa_abi_sizeof(const char *type_name);
 

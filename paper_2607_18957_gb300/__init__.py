@@ -421,6 +421,16 @@ class Plan:
         _check(self._lib.cfa_get_stats(self._handle, ctypes.byref(s)), self._handle)
         return {name: getattr(s, name) for name, _ in _lib.Stats._fields_}
 
+    def timeline(self):
+        """Per-chunk timeline of the last load (CFA_OPT_TIMING plans): a float32 array [n_chunks,
+        4] of h2d begin/end and unpack begin/end in ms from the load's first operation (-1 where
+        the step did not run)."""
+        n = self.info()["n_chunks"]
+        out = np.zeros((n, 4), dtype=np.float32)
+        _check(self._lib.cfa_get_timeline(self._handle, out.ctypes.data if n else None, n),
+               self._handle)
+        return out
+
     def layer_times(self, n=None):
         if n is None:
             n = self.info()["n_layers"]

@@ -103,6 +103,7 @@ SIGNATURES = {
     "cfa_file_source_open": (ctypes.c_int, [ctypes.c_char_p, _U64, ctypes.c_uint32, _P]),
     "cfa_file_source_close": (ctypes.c_int, [_P]),
     "cfa_selftest_wait_timeout": (ctypes.c_int, [ctypes.c_int, _P]),
+    "cfa_get_timeline": (ctypes.c_int, [_P, _P, _SZ]),
 }
 
 _lib = None
@@ -132,7 +133,8 @@ def _check_layouts(lib):
     want = {"cfa_tensor_entry": ENTRY_DTYPE.itemsize, "cfa_dst": DST_DTYPE.itemsize,
             "cfa_plan_opts": ctypes.sizeof(PlanOpts), "cfa_source": ctypes.sizeof(Source),
             "cfa_stats": ctypes.sizeof(Stats), "cfa_piece": ctypes.sizeof(Piece),
-            "cfa_st_tensor": ctypes.sizeof(StTensor)}
+            "cfa_st_tensor": ctypes.sizeof(StTensor),
+            "cfa_chunk_times": 16}
     for name, size in want.items():
         got = lib.cfa_abi_sizeof(name.encode())
         if got != size:

@@ -28,6 +28,7 @@
 #include <chrono>
 #include <condition_variable>
 #include <cstdarg>
+#include <cstdlib>
 #include <cstdio>
 #include <cstring>
 #include <functional>
@@ -125,6 +126,7 @@ struct cfa_plan {
     std::vector<cudaEvent_t> ev_dev_free, ev_h2d, ev_host_free, ev_filled, ev_layer;
     cudaEvent_t ev_begin = nullptr, ev_all = nullptr;
     std::vector<cudaEvent_t> t_h2d0, t_h2d1, t_k0, t_k1;
+    std::vector<uint32_t> t_k_c0, t_k_c1; /* chunk range of each timed launch */
     std::vector<std::vector<uint32_t>> layers_ending; /* per chunk */
     std::vector<uint32_t> layers_empty;
     std::unique_ptr<cfa::Pool> pool;
@@ -140,6 +142,27 @@ struct cfa_plan {
 
 namespace {
 
+/* CFA_LOG=1 in the environment: one line per plan, per load and per error on stderr. */
+bool log_on()
+{
+    static const bool on = [] {
+        const char *v = std::getenv("CFA_LOG");
+        return v && *v && std::strcmp(v, "0") != 0;
+    }();
+    return on;
+}
+
+void logf(const char *fmt, ...)
+{
+    if (!log_on()) return;
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    std::fprintf(stderr, "cfa: %s\n", buf);
+}
+
 void set_err(cfa_plan *p, const char *fmt, ...)
 {
     char *buf = p ? p->err : g_create_err;
@@ -148,6 +171,7 @@ void set_err(cfa_plan *p, const char *fmt, ...)
     va_start(ap, fmt);
     vsnprintf(buf, n, fmt, ap);
     va_end(ap);
+    logf("error: %s", buf);
 }
 
 #define CK(p, call)                                                                        \
@@ -250,7 +274,11 @@ cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint
         const int k = J.k;
         cudaStream_t ls = i == 0 ? s : p->side_stream[(i - 1) % kSideStreams];
         const bool timing = timing_on && p->last_launches < p->t_k0.size();
-        if (timing) CK(p, cudaEventRecord(p->t_k0[p->last_launches], ls));
+        if (timing) {
+            CK(p, cudaEventRecord(p->t_k0[p->last_launches], ls));
+            p->t_k_c0[p->last_launches] = c0;
+            p->t_k_c1[p->last_launches] = c1;
+        }
         if (J.type == BULK)
             CK(p, cfa_launch_bulk(k, p->d_bulk + J.a0, J.a1 - J.a0, src_base, period, lo, hi,
                                   p->d_ck, p->d_status, p->bulk_grid_cap[k], ls));
@@ -459,6 +487,8 @@ cfa_status setup_device(cfa_plan *p)
         const size_t nk = 3 * CFA_N_CLASSES * ((size_t)hp.n_chunks + 1);
         if ((st = events(p->t_k0, nk, true))) return st;
         if ((st = events(p->t_k1, nk, true))) return st;
+        p->t_k_c0.assign(nk, 0);
+        p->t_k_c1.assign(nk, 0);
     }
     if (o.fill_threads > 1) p->pool.reset(new cfa::Pool(o.fill_threads - 1));
     else p->pool.reset(new cfa::Pool(0));
@@ -528,6 +558,7 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
     cfa_status st = cfa_host_plan_build(entries, n_entries, dsts, n_dsts, blob_bytes, opts,
                                         &p->hp, g_create_err, sizeof(g_create_err));
     if (st) {
+        logf("error: %s", g_create_err);
         delete p;
         return st;
     }
@@ -550,6 +581,12 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
     }
     p->plan_ms = std::chrono::duration<double, std::milli>(std::chrono::steady_clock::now() - t0)
                      .count();
+    logf("plan: %zu entries, %zu destinations, %llu blob bytes in %u chunks of %llu; pieces %zu, "
+         "TMA items %zu, vector slabs %zu, tiny %zu, column blocks %zu; staged bytes %llu; "
+         "%.1f ms",
+         hp.n_entries, hp.n_dsts, (unsigned long long)hp.blob_bytes, hp.n_chunks,
+         (unsigned long long)hp.chunk_bytes, hp.n_pieces, hp.n_bulk, hp.n_slabs, hp.n_tiny,
+         hp.n_strided, (unsigned long long)hp.staged_bytes, p->plan_ms);
     *out = p;
     return CFA_OK;
 }
@@ -717,6 +754,8 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
         }
     }
     CK(p, cudaEventRecord(p->ev_all, cs));
+    logf("load %llu enqueued: source kind %d, %llu kernel launches, %u staged chunks",
+         (unsigned long long)p->n_loads, kind, (unsigned long long)p->last_launches, p->last_h2d);
     return CFA_OK;
 }
 
@@ -824,6 +863,33 @@ cfa_status cfa_get_layer_times(cfa_plan *p, float *ms_out, size_t n)
     return CFA_OK;
 }
 
+cfa_status cfa_get_timeline(cfa_plan *p, cfa_chunk_times *out, size_t n)
+{
+    if (!p || p->host_only || (n && !out) || n > p->hp.n_chunks) return CFA_ERR_INVAL;
+    if (!(p->hp.opts.flags & CFA_OPT_TIMING) || !p->last) {
+        set_err(p, "the timeline needs a CFA_OPT_TIMING plan and a load");
+        return CFA_ERR_INVAL;
+    }
+    DeviceGuard g(p->device);
+    CK(p, cudaEventSynchronize(p->ev_all));
+    for (size_t c = 0; c < n; ++c) out[c] = cfa_chunk_times{-1.f, -1.f, -1.f, -1.f};
+    for (uint32_t c = 0; c < p->last_h2d && c < n && c < p->t_h2d0.size(); ++c) {
+        CK(p, cudaEventElapsedTime(&out[c].h2d_begin_ms, p->ev_begin, p->t_h2d0[c]));
+        CK(p, cudaEventElapsedTime(&out[c].h2d_end_ms, p->ev_begin, p->t_h2d1[c]));
+    }
+    for (uint64_t k = 0; k < p->last_launches && k < p->t_k0.size(); ++k) {
+        float b = 0, e = 0;
+        CK(p, cudaEventElapsedTime(&b, p->ev_begin, p->t_k0[k]));
+        CK(p, cudaEventElapsedTime(&e, p->ev_begin, p->t_k1[k]));
+        for (uint32_t c = p->t_k_c0[k]; c < p->t_k_c1[k] && c < n; ++c) {
+            if (out[c].unpack_begin_ms < 0 || b < out[c].unpack_begin_ms)
+                out[c].unpack_begin_ms = b;
+            if (e > out[c].unpack_end_ms) out[c].unpack_end_ms = e;
+        }
+    }
+    return CFA_OK;
+}
+
 cfa_status cfa_plan_info(const cfa_plan *p, uint64_t *n_layers, uint64_t *n_pieces,
                          uint64_t *n_chunks)
 {
@@ -922,6 +988,7 @@ size_t cfa_abi_sizeof(const char *type_name)
     if (!std::strcmp(type_name, "cfa_stats")) return sizeof(cfa_stats);
     if (!std::strcmp(type_name, "cfa_piece")) return sizeof(cfa_piece);
     if (!std::strcmp(type_name, "cfa_st_tensor")) return sizeof(cfa_st_tensor);
+    if (!std::strcmp(type_name, "cfa_chunk_times")) return sizeof(cfa_chunk_times);
     return 0;
 }
 

@@ -451,3 +451,50 @@ def test_two_plans_load_at_once_from_two_threads():
         assert np.array_equal(results[k], ref.cksum), m.name
         assert d.guards_intact()
         plan.close()
+
+
+def test_timeline_orders_copies_before_unpacks():
+    m = CONFIGS["dense"]()
+    blob, ref = reference(m)
+    keep = []
+    d = DeviceDsts(m)
+    with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=1 << 20,
+                  timing=True) as plan:
+        plan.load_async(make_source("pinned", m, blob, keep))
+        plan.wait_layer()
+        t = plan.timeline()
+        n = plan.stats()["n_chunks"]
+        assert t.shape == (n, 4)
+        assert (t[:, 0] >= 0).all() and (t[:, 1] >= t[:, 0]).all()
+        ran = t[:, 2] >= 0
+        assert ran.sum() >= n - 1
+        # a chunk is unpacked only after its copy into the device slot has finished
+        assert (t[ran, 2] >= t[ran, 1] - 1e-3).all() and (t[ran, 3] >= t[ran, 2]).all()
+        # with two device slots, chunk c + 2's copy waits for chunk c's unpack
+        assert (t[2:, 0] >= t[:-2, 3] - 1e-3)[ran[:-2]].all()
+        # a device-resident source: no copies, one merged launch over every chunk
+        plan.load_async(make_source("device", m, blob, keep))
+        plan.wait_layer()
+        t = plan.timeline()
+        assert (t[:, 0] == -1).all() and (t[:, 1] == -1).all()
+        assert len(set(t[:, 2].tolist())) == 1 and (t[:, 3] > t[:, 2]).all()
+        ck = plan.checksums()
+    assert np.array_equal(ck, ref.cksum)
+
+
+def test_destroy_while_a_load_is_in_flight():
+    """Closing a plan with a load still running (a slow callback source) waits for the load and
+    frees everything; the destinations hold the complete load."""
+    m = CONFIGS["moe"]()
+    blob, ref = reference(m)
+    cb = CallbackSource(m, delay_us=300)
+    d = DeviceDsts(m)
+    plan = cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=256 << 10)
+    plan.load_async(cb.source())
+    timeout = {v: k for k, v in cfa._lib.STATUS.items()}["CFA_ERR_TIMEOUT"]
+    assert plan.try_wait_layer(timeout_ns=0) == timeout
+    plan.close()
+    torch.cuda.synchronize()
+    for j in range(m.n_dsts):
+        assert np.array_equal(d.host_bytes(j), ref.dst[j]), m.d_name[j]
+    assert d.guards_intact()

@@ -297,3 +297,29 @@ def test_default_options_take_the_bulk_path():
     with host_plan(m, chunk_bytes=1 << 20, tiny_bytes=0, bulk=False) as p:
         st = p.stats()
         assert st["n_bulk"] == 0 and st["n_slabs"] > 0
+
+
+def test_log_lines_on_request():
+    """CFA_LOG=1 prints one line per plan and per error on stderr (a child process, so the
+    variable is read fresh)."""
+    import subprocess
+    import sys
+    code = ("import paper_2607_18957_gb300 as cfa\n"
+            "e = cfa.make_entries(dtype=['bf16'], shape=[(1024,)], offset=[0], dst=[0])\n"
+            "cfa.Plan(e, [(0x100000, 'bf16', (1024,))], 2048, host_only=True).close()\n"
+            "try:\n"
+            "    cfa.Plan(e, [(0x100000, 'bf16', (1000,))], 2048, host_only=True)\n"
+            "except cfa.CfaError:\n"
+            "    pass\n")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    env = dict(os.environ, CFA_LOG="1", PYTHONPATH=root)
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                       timeout=120)
+    assert r.returncode == 0, r.stderr
+    lines = [x for x in r.stderr.splitlines() if x.startswith("cfa: ")]
+    assert any(x.startswith("cfa: plan: 1 entries") for x in lines), r.stderr
+    assert any("rows fall outside the destination" in x for x in lines), r.stderr
+    env["CFA_LOG"] = "0"
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                       timeout=120)
+    assert "cfa: " not in r.stderr
