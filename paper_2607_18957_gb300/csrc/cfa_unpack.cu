@@ -31,11 +31,12 @@ namespace {
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kUnroll = 4;
-constexpr int kMinBlocks = 4; /* 64 registers per thread at most */
-/* Rounds of 32-vector loads in flight per warp on the realigning path: two for slabs (one or
- * four are slower: too little in flight, or spills), one for column-slice rows. */
-constexpr int kRealignRounds = 2;
-constexpr int kRealignRoundsRows = 1;
+constexpr int kMinBlocks = 4;     /* conversion classes: 64 registers per thread at most */
+constexpr int kCopyMinBlocks = 3; /* copy classes: 80 registers, room for the realigning path */
+/* Rounds of 32-vector loads in flight per warp on the realigning path: four for slabs (with
+ * three CTAs per SM the copy kernels hold them without spilling), two for column-slice rows. */
+constexpr int kRealignRounds = 4;
+constexpr int kRealignRoundsRows = 2;
 
 struct UnpackArgs {
     const cfa_work *slabs;
@@ -435,7 +436,8 @@ __device__ __forceinline__ void block_flush(uint64_t &acc, uint32_t ck, unsigned
  * when i mod (q + 1) == q, else slab (i / (q + 1)) * q + i mod (q + 1); the items after those
  * are the remaining slabs in order. */
 template <int CLS>
-__global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_unpack_kernel(const UnpackArgs a)
+__global__ void __launch_bounds__(kThreads, (CLS < 4 ? kCopyMinBlocks : kMinBlocks))
+    cfa_unpack_kernel(const UnpackArgs a)
 {
     __shared__ unsigned long long red[kWarps];
     const uint32_t n_groups = (a.n_tiny + kWarps - 1) / kWarps;
@@ -517,7 +519,8 @@ __device__ __forceinline__ bool sitem_ok(const cfa_swork &w, const StridedArgs &
  * like a contiguous run (16-byte vectors, realigned when source and destination disagree mod
  * 16, four vectors in flight per lane). */
 template <int CLS>
-__global__ void __launch_bounds__(kThreads, kMinBlocks) cfa_strided_kernel(const StridedArgs a)
+__global__ void __launch_bounds__(kThreads, (CLS < 4 ? kCopyMinBlocks : kMinBlocks))
+    cfa_strided_kernel(const StridedArgs a)
 {
     typedef ClassOf<CLS> C;
     constexpr int SES = C::ses;
