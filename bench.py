@@ -82,7 +82,7 @@ def measured_peaks():
 
 def kernel_source_hash():
     h = hashlib.sha256()
-    for f in ("cfa_unpack.cu", "cfa_bulk.cu"):
+    for f in ("cfa_unpack.cu", "cfa_bulk.cu", "cfa_device.cuh"):
         with open(os.path.join(ROOT, "paper_2607_18957_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()

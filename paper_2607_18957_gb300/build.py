@@ -29,7 +29,7 @@ def _nvcc():
 
 def _sources():
     return [os.path.join(CSRC, f) for f in CU_SOURCES + C_SOURCES +
-            ["cfa_internal.h", "cfa_pool.h"]] + \
+            ["cfa_internal.h", "cfa_pool.h", "cfa_device.cuh"]] + \
         [os.path.join(INCLUDE, "cfa.h")]
 
 

@@ -23,9 +23,13 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "cfa_device.cuh"
 #include "cfa_internal.h"
 
 namespace {
+
+using cfa_dev::vsum;
+using cfa_dev::warp_sum;
 
 constexpr int kThreads = 64; /* warp 0 loads, warp 1 checksums and stores */
 constexpr int kStages = 2;
@@ -108,34 +112,6 @@ __device__ __forceinline__ void bulk_wait_read_all_but_one()
 }
 
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-
-template <int ES> __device__ __forceinline__ uint64_t vsum(uint4 v);
-template <> __device__ __forceinline__ uint64_t vsum<1>(uint4 v)
-{
-    return (uint64_t)(__vsadu4(v.x, 0u) + __vsadu4(v.y, 0u) + __vsadu4(v.z, 0u) +
-                      __vsadu4(v.w, 0u));
-}
-template <> __device__ __forceinline__ uint64_t vsum<2>(uint4 v)
-{
-    const uint32_t lo = (v.x & 0xFFFFu) + (v.y & 0xFFFFu) + (v.z & 0xFFFFu) + (v.w & 0xFFFFu);
-    const uint32_t hi = (v.x >> 16) + (v.y >> 16) + (v.z >> 16) + (v.w >> 16);
-    return (uint64_t)lo + hi;
-}
-template <> __device__ __forceinline__ uint64_t vsum<4>(uint4 v)
-{
-    return (uint64_t)v.x + v.y + v.z + v.w;
-}
-template <> __device__ __forceinline__ uint64_t vsum<8>(uint4 v)
-{
-    return (((uint64_t)v.y << 32) | v.x) + (((uint64_t)v.w << 32) | v.z);
-}
-
-__device__ __forceinline__ uint64_t warp_sum(uint64_t v)
-{
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, o);
-    return v;
-}
 
 /* Adds the consumer warp's checksum to slot ck; all 32 lanes call it. */
 __device__ __forceinline__ void warp_flush(uint64_t &acc, uint32_t ck, unsigned long long *out)

@@ -24,9 +24,13 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "cfa_device.cuh"
 #include "cfa_internal.h"
 
 namespace {
+
+using cfa_dev::vsum;
+using cfa_dev::warp_sum;
 
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
@@ -88,27 +92,6 @@ template <> struct Elem<4> { typedef uint32_t T; };
 template <> struct Elem<8> { typedef unsigned long long T; };
 
 /* Sum of the ES-byte little-endian integers in a 16-byte vector. */
-template <int ES> __device__ __forceinline__ uint64_t vsum(uint4 v);
-template <> __device__ __forceinline__ uint64_t vsum<1>(uint4 v)
-{
-    return (uint64_t)(__vsadu4(v.x, 0u) + __vsadu4(v.y, 0u) + __vsadu4(v.z, 0u) +
-                      __vsadu4(v.w, 0u));
-}
-template <> __device__ __forceinline__ uint64_t vsum<2>(uint4 v)
-{
-    const uint32_t lo = (v.x & 0xFFFFu) + (v.y & 0xFFFFu) + (v.z & 0xFFFFu) + (v.w & 0xFFFFu);
-    const uint32_t hi = (v.x >> 16) + (v.y >> 16) + (v.z >> 16) + (v.w >> 16);
-    return (uint64_t)lo + hi;
-}
-template <> __device__ __forceinline__ uint64_t vsum<4>(uint4 v)
-{
-    return (uint64_t)v.x + v.y + v.z + v.w;
-}
-template <> __device__ __forceinline__ uint64_t vsum<8>(uint4 v)
-{
-    return (((uint64_t)v.y << 32) | v.x) + (((uint64_t)v.w << 32) | v.z);
-}
-
 /* Bytes k .. k+15 of the 32-byte concatenation a:b (little-endian), 0 < k < 16. */
 __device__ __forceinline__ uint4 funnel16(uint4 a, uint4 b, uint32_t k)
 {
@@ -401,13 +384,6 @@ __device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs
     else
         return copy_run<(1 << CLS), U, (U > 1 ? kRealignRounds : 1)>(src, dst,
                                                                     (uint64_t)w.n << CLS, tid, nthr);
-}
-
-__device__ __forceinline__ uint64_t warp_sum(uint64_t v)
-{
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_down_sync(0xFFFFFFFFu, v, o);
-    return v;
 }
 
 /* Adds the CTA's accumulated checksum to slot ck; every thread of the CTA must call it. */
