@@ -38,6 +38,10 @@ typedef struct cfa_work {
  * starts at source blob offset src + k * stride * (source element size) and lands at
  * dst + k * cols * (destination element size).  40 bytes.
  */
+/* Tiny pieces with at most this many destination bytes are copied by 8-lane warp segments; the
+ * plan orders them ahead of the larger tiny pieces of the same (class, chunk). */
+#define CFA_TINY_SEG_BYTES 512u
+
 typedef struct cfa_swork {
     uint64_t src;
     uint64_t dst;

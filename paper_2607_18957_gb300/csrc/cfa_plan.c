@@ -213,6 +213,31 @@ static cfa_status partition_by_class(vec *v, uint32_t *first, uint32_t n_chunks,
     return CFA_OK;
 }
 
+/* Within each (class, chunk) range of tiny items, the pieces of at most CFA_TINY_SEG_BYTES
+ * destination bytes first (stable), so the kernel's warps mostly get pieces of one kind. */
+static cfa_status order_tiny(vec *v, const uint32_t *first, uint32_t n_chunks)
+{
+    if (v->n == 0) return CFA_OK;
+    cfa_work *w = (cfa_work *)v->p;
+    cfa_work *tmp = (cfa_work *)malloc(v->n * sizeof(cfa_work));
+    if (!tmp) return CFA_ERR_NOMEM;
+    const size_t row = (size_t)n_chunks + 1;
+    for (size_t k = 0; k < CFA_N_CLASSES; ++k) {
+        for (size_t c = 0; c < n_chunks; ++c) {
+            const uint32_t a = first[k * row + c], b = first[k * row + c + 1];
+            size_t o = a;
+            for (int pass = 0; pass < 2; ++pass)
+                for (uint32_t q = a; q < b; ++q) {
+                    const uint64_t bytes = (uint64_t)w[q].n << ((w[q].mode >> 2) & 3u);
+                    if ((bytes <= CFA_TINY_SEG_BYTES) == (pass == 0)) tmp[o++] = w[q];
+                }
+        }
+    }
+    memcpy(w, tmp, v->n * sizeof(cfa_work));
+    free(tmp);
+    return CFA_OK;
+}
+
 void cfa_host_plan_free(cfa_host_plan *hp)
 {
     if (!hp) return;
@@ -637,6 +662,7 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         if ((st = partition_by_class(&slabs, out->slab_first, n_chunks, S, err, errlen))) goto done;
         if ((st = partition_by_class(&bulk, out->bulk_first, n_chunks, S, err, errlen))) goto done;
         if ((st = partition_by_class(&tiny, out->tiny_first, n_chunks, S, err, errlen))) goto done;
+        if ((st = order_tiny(&tiny, out->tiny_first, n_chunks))) goto done;
         if ((st = partition_by_class(&strided, out->strided_first, n_chunks, S, err, errlen)))
             goto done;
     }

@@ -190,7 +190,7 @@ __device__ __forceinline__ uint64_t copy_elems(const uint8_t *src, uint8_t *dst,
 
 /* Copies nbytes (a multiple of ES) from src to dst; thread tid of nthr.  Returns this thread's
  * share of the checksum. */
-template <int ES, int U, int UR>
+template <int ES, int U, int UR, int W = 32>
 __device__ uint64_t copy_run(const uint8_t *__restrict__ src, uint8_t *__restrict__ dst,
                              uint64_t nbytes, uint32_t tid, uint32_t nthr)
 {
@@ -234,38 +234,41 @@ __device__ uint64_t copy_run(const uint8_t *__restrict__ src, uint8_t *__restric
          * next lane, or for lane 31 from lane 0 of the next round.  The one vector per warp
          * that has no loaded neighbour (lane 31's last one, or the run's last vector) is loaded
          * by its lane in the same round of loads. */
+        /* W = 32: whole warps; W = 8: the run belongs to one 8-lane segment of a warp (the
+         * sub-warp path for tiny pieces), and every shuffle stays inside the segment */
         const uint4 *s = reinterpret_cast<const uint4 *>(src - k);
-        const uint32_t lane = tid & 31u, wid = tid >> 5;
+        const uint32_t lane = tid & (W - 1u), wid = tid / W;
+        const uint32_t mask = W == 32 ? 0xFFFFFFFFu : (((1u << W) - 1u) << (threadIdx.x & 31u & ~(W - 1u)));
         const uint32_t step = nthr * UR;
         for (uint32_t base = 0; base < nvec; base += step) {
-            const uint32_t w0 = base + wid * 32u * UR;
+            const uint32_t w0 = base + wid * W * UR;
             uint4 a[UR];
             int own = -1; /* the round whose neighbour this lane loads itself */
 #pragma unroll
             for (int u = 0; u < UR; ++u) {
-                const uint32_t i = w0 + 32u * u + lane;
+                const uint32_t i = w0 + W * u + lane;
                 a[u] = make_uint4(0u, 0u, 0u, 0u);
                 if (i < nvec) {
                     a[u] = ld_shared_line(s + i);
-                    if (i + 1 == nvec || (lane == 31u && u == UR - 1)) own = u;
+                    if (i + 1 == nvec || (lane == W - 1u && u == UR - 1)) own = u;
                 }
             }
             uint4 c = make_uint4(0u, 0u, 0u, 0u);
-            if (own >= 0) c = ld_shared_line(s + w0 + 32u * own + lane + 1);
+            if (own >= 0) c = ld_shared_line(s + w0 + W * own + lane + 1);
 #pragma unroll
             for (int u = 0; u < UR; ++u) {
-                const uint32_t i = w0 + 32u * u + lane;
+                const uint32_t i = w0 + W * u + lane;
                 uint4 b, n0;
-                b.x = __shfl_down_sync(0xFFFFFFFFu, a[u].x, 1);
-                b.y = __shfl_down_sync(0xFFFFFFFFu, a[u].y, 1);
-                b.z = __shfl_down_sync(0xFFFFFFFFu, a[u].z, 1);
-                b.w = __shfl_down_sync(0xFFFFFFFFu, a[u].w, 1);
+                b.x = __shfl_down_sync(mask, a[u].x, 1, W);
+                b.y = __shfl_down_sync(mask, a[u].y, 1, W);
+                b.z = __shfl_down_sync(mask, a[u].z, 1, W);
+                b.w = __shfl_down_sync(mask, a[u].w, 1, W);
                 if (u + 1 < UR) {
-                    n0.x = __shfl_sync(0xFFFFFFFFu, a[u + 1].x, 0);
-                    n0.y = __shfl_sync(0xFFFFFFFFu, a[u + 1].y, 0);
-                    n0.z = __shfl_sync(0xFFFFFFFFu, a[u + 1].z, 0);
-                    n0.w = __shfl_sync(0xFFFFFFFFu, a[u + 1].w, 0);
-                    if (lane == 31u) b = n0;
+                    n0.x = __shfl_sync(mask, a[u + 1].x, 0, W);
+                    n0.y = __shfl_sync(mask, a[u + 1].y, 0, W);
+                    n0.z = __shfl_sync(mask, a[u + 1].z, 0, W);
+                    n0.w = __shfl_sync(mask, a[u + 1].w, 0, W);
+                    if (lane == W - 1u) b = n0;
                 }
                 if (i < nvec) {
                     if (own == u) b = c;
@@ -371,7 +374,7 @@ __device__ __forceinline__ bool item_ok(const cfa_work &w, const UnpackArgs &a)
            (w.dst & ((1ull << dl) - 1)) == 0;
 }
 
-template <int CLS, int U>
+template <int CLS, int U, int W = 32>
 __device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs &a, uint32_t tid,
                                              uint32_t nthr)
 {
@@ -382,8 +385,9 @@ __device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs
     if constexpr (C::conv != CFA_CONV_NONE)
         return convert_run<C::ses, C::des, C::conv, (U > 2 ? 2 : U)>(src, dst, w.n, tid, nthr);
     else
-        return copy_run<(1 << CLS), U, (U > 1 ? kRealignRounds : 1)>(src, dst,
-                                                                    (uint64_t)w.n << CLS, tid, nthr);
+        return copy_run<(1 << CLS), U, (U > 1 ? kRealignRounds : 1), W>(src, dst,
+                                                                       (uint64_t)w.n << CLS, tid,
+                                                                       nthr);
 }
 
 /* Adds the CTA's accumulated checksum to slot ck; every thread of the CTA must call it. */
@@ -411,12 +415,61 @@ __device__ __forceinline__ void block_flush(uint64_t &acc, uint32_t ck, unsigned
  * Item i of the first n_groups * (q + 1) items (q = n_slabs / n_groups) is group i / (q + 1)
  * when i mod (q + 1) == q, else slab (i / (q + 1)) * q + i mod (q + 1); the items after those
  * are the remaining slabs in order. */
+/* Tiny pieces: a group is kSegs pieces per warp.  When every piece of a warp's share has at most
+ * kSegMaxBytes destination bytes, each 8-lane segment copies one piece on its own (four pieces in
+ * flight per warp); otherwise the whole warp copies the pieces one after the other.  The plan
+ * puts the small pieces of each (class, chunk) first, so most warps see one kind. */
+constexpr int kSegLanes = 8;
+constexpr int kSegs = 32 / kSegLanes;
+constexpr uint32_t kSegMaxBytes = CFA_TINY_SEG_BYTES;
+constexpr uint32_t kTinyPerGroup = kWarps * kSegs;
+
+template <int CLS>
+__device__ __forceinline__ void run_tiny(const UnpackArgs &a, uint32_t group, uint32_t warp,
+                                         uint32_t lane)
+{
+    const uint32_t seg = lane / kSegLanes, sub = lane % kSegLanes;
+    const uint32_t t = (group * kWarps + warp) * kSegs + seg;
+    cfa_work w{};
+    bool ok = false;
+    uint32_t bytes = 0;
+    if (t < a.n_tiny) {
+        w = a.tiny[t]; /* the same 32 bytes for the segment's lanes */
+        ok = item_ok<CLS>(w, a);
+        if (!ok && sub == 0) atomicCAS(a.status, 0, 1);
+        if (ok) bytes = w.n << ((w.mode >> 2) & 3u);
+    }
+    if (!__any_sync(0xFFFFFFFFu, bytes > kSegMaxBytes)) {
+        if (ok) {
+            const uint32_t mask = 0xFFu << (seg * kSegLanes);
+            uint64_t v = run_item<CLS, 1, kSegLanes>(w, a, sub, kSegLanes);
+#pragma unroll
+            for (int o = kSegLanes / 2; o > 0; o >>= 1) v += __shfl_down_sync(mask, v, o, kSegLanes);
+            if (sub == 0 && w.ck != CFA_NO_CK) atomicAdd(a.ck + w.ck, v);
+        }
+        return;
+    }
+    for (int k = 0; k < kSegs; ++k) {
+        const int src_lane = k * kSegLanes;
+        if (!__shfl_sync(0xFFFFFFFFu, (int)ok, src_lane)) continue;
+        cfa_work wk;
+        wk.src = __shfl_sync(0xFFFFFFFFu, (unsigned long long)w.src, src_lane);
+        wk.dst = __shfl_sync(0xFFFFFFFFu, (unsigned long long)w.dst, src_lane);
+        wk.n = __shfl_sync(0xFFFFFFFFu, w.n, src_lane);
+        wk.ck = __shfl_sync(0xFFFFFFFFu, w.ck, src_lane);
+        wk.mode = __shfl_sync(0xFFFFFFFFu, w.mode, src_lane);
+        wk.pad = __shfl_sync(0xFFFFFFFFu, w.pad, src_lane);
+        const uint64_t v = warp_sum(run_item<CLS, 1>(wk, a, lane, 32u));
+        if (lane == 0 && wk.ck != CFA_NO_CK) atomicAdd(a.ck + wk.ck, v);
+    }
+}
+
 template <int CLS>
 __global__ void __launch_bounds__(kThreads, (CLS < 4 ? kCopyMinBlocks : kMinBlocks))
     cfa_unpack_kernel(const UnpackArgs a)
 {
     __shared__ unsigned long long red[kWarps];
-    const uint32_t n_groups = (a.n_tiny + kWarps - 1) / kWarps;
+    const uint32_t n_groups = (a.n_tiny + kTinyPerGroup - 1) / kTinyPerGroup;
     const uint32_t n_items = a.n_slabs + n_groups;
     const uint32_t q = n_groups ? a.n_slabs / n_groups : 0;
     const uint32_t mixed = n_groups * (q + 1); /* items in the interleaved prefix */
@@ -452,16 +505,7 @@ __global__ void __launch_bounds__(kThreads, (CLS < 4 ? kCopyMinBlocks : kMinBloc
         } else {
             if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
             acc_ck = CFA_NO_CK;
-            const uint32_t t = group * kWarps + warp;
-            if (t < a.n_tiny) {
-                const cfa_work w = a.tiny[t];
-                if (!item_ok<CLS>(w, a)) {
-                    if (lane == 0) atomicCAS(a.status, 0, 1);
-                } else {
-                    const uint64_t v = warp_sum(run_item<CLS, 1>(w, a, lane, 32u));
-                    if (lane == 0 && w.ck != CFA_NO_CK) atomicAdd(a.ck + w.ck, v);
-                }
-            }
+            run_tiny<CLS>(a, group, warp, lane);
         }
     }
     if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
@@ -568,7 +612,7 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
                                          cudaStream_t stream)
 {
     if (cls < 0 || cls >= CFA_N_CLASSES || grid_cap <= 0) return cudaErrorInvalidValue;
-    const uint64_t items = (uint64_t)n_slabs + (n_tiny + kWarps - 1) / kWarps;
+    const uint64_t items = (uint64_t)n_slabs + (n_tiny + kTinyPerGroup - 1) / kTinyPerGroup;
     if (items == 0) return cudaSuccess;
     UnpackArgs a;
     a.slabs = slabs;
