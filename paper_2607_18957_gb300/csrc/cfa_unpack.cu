@@ -36,9 +36,12 @@ constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kUnroll = 4;
 constexpr int kMinBlocks = 4;     /* conversion classes: 64 registers per thread at most */
-constexpr int kCopyMinBlocks = 3; /* copy classes: 80 registers, room for the realigning path */
+constexpr int kCopyMinBlocks = 3; /* 2-8-byte copy classes: 80 registers, room for the
+                                     realigning path; the 1-byte class keeps 4 CTAs (its byte-wise
+                                     checksum wants the warps: 0.96 vs 0.92 of the roofline) */
 /* Rounds of 32-vector loads in flight per warp on the realigning path: four for slabs (with
- * three CTAs per SM the copy kernels hold them without spilling), two for column-slice rows. */
+ * three CTAs per SM the copy kernels hold them without spilling; two for the 1-byte class at
+ * four CTAs), two for column-slice rows. */
 constexpr int kRealignRounds = 4;
 constexpr int kRealignRoundsRows = 2;
 
@@ -385,7 +388,7 @@ __device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs
     if constexpr (C::conv != CFA_CONV_NONE)
         return convert_run<C::ses, C::des, C::conv, (U > 2 ? 2 : U)>(src, dst, w.n, tid, nthr);
     else
-        return copy_run<(1 << CLS), U, (U > 1 ? kRealignRounds : 1), W>(src, dst,
+        return copy_run<(1 << CLS), U, (U > 1 ? (CLS >= 1 ? kRealignRounds : 2) : 1), W>(src, dst,
                                                                        (uint64_t)w.n << CLS, tid,
                                                                        nthr);
 }
@@ -465,7 +468,7 @@ __device__ __forceinline__ void run_tiny(const UnpackArgs &a, uint32_t group, ui
 }
 
 template <int CLS>
-__global__ void __launch_bounds__(kThreads, (CLS < 4 ? kCopyMinBlocks : kMinBlocks))
+__global__ void __launch_bounds__(kThreads, (CLS >= 1 && CLS < 4 ? kCopyMinBlocks : kMinBlocks))
     cfa_unpack_kernel(const UnpackArgs a)
 {
     __shared__ unsigned long long red[kWarps];
