@@ -51,6 +51,9 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--no-attribution", action="store_true",
                     help="skip the end-to-end attribution measurements")
+    ap.add_argument("--timeline", default=None, metavar="PATH",
+                    help="write the per-chunk timeline (copy and unpack intervals) of the timed "
+                         "pinned load of the attribution to PATH as JSON")
     ap.add_argument("--vector-only", dest="bulk", action="store_false",
                     help="copy every slab with the 16-byte vector kernel instead of the TMA bulk "
                          "kernel (for comparison)")
@@ -223,6 +226,15 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
     plan.wait_layer()
     t = plan.layer_times()
     st = plan.stats()
+    if args.timeline:
+        tl = plan.timeline()
+        with open(args.timeline, "w") as f:
+            json.dump({"workload": m.name, "chunk_bytes": m.chunk_bytes,
+                       "source": "pinned host blob, 2 device staging slots",
+                       "columns": ["h2d_begin_ms", "h2d_end_ms", "unpack_begin_ms",
+                                   "unpack_end_ms"],
+                       "chunks": [[round(float(x), 4) for x in row] for row in tl],
+                       "layer_ready_ms": [round(float(x), 4) for x in t]}, f)
     plan.close()
     out["layer_ready_ms"] = {"first_group": round(float(t[0]), 2),
                              "median_group": round(float(np.median(t)), 2),

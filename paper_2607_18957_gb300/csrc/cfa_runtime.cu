@@ -22,6 +22,7 @@
  * sit in device memory, and contiguous chunks are unpacked by one launch.
  */
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h> /* header-only; ranges show in profilers that attach to NVTX */
 
 #include <algorithm>
 #include <atomic>
@@ -186,12 +187,19 @@ void set_err(cfa_plan *p, const char *fmt, ...)
 /* InDisk -> InMem for one chunk: puts the byte ranges the chunk's pieces read (its copy
  * segments; the rest of the slot is never read) into pinned slot `host_slot`, split over the
  * plan's fill threads in parts of at most 16 MiB. */
+/* NVTX range for the lifetime of a scope. */
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+};
+
 void CUDART_CB fill_host_fn(void *arg)
 {
     FillJob *j = static_cast<FillJob *>(arg);
     LoadCtx *ctx = j->ctx;
     cfa_plan *p = ctx->plan;
     if (ctx->error.load()) return;
+    NvtxRange range("cfa fill chunk (InDisk -> InMem)");
     const cfa_host_plan &hp = p->hp;
     const uint64_t S = hp.chunk_bytes;
     const uint64_t off = (uint64_t)j->chunk * S;
@@ -549,6 +557,7 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
         return CFA_ERR_INVAL;
     }
     *out = nullptr;
+    NvtxRange range("cfa plan create");
     const auto t0 = std::chrono::steady_clock::now();
     cfa_plan *p = new (std::nothrow) cfa_plan();
     if (!p) {
@@ -594,6 +603,7 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
 cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_)
 {
     if (!p || !src) return CFA_ERR_INVAL;
+    NvtxRange range("cfa enqueue load");
     if (p->host_only) {
         set_err(p, "host-only plan cannot load");
         return CFA_ERR_INVAL;
