@@ -232,16 +232,17 @@ __device__ uint64_t copy_run(const uint8_t *__restrict__ src, uint8_t *__restric
     } else {
         /* source off by k bytes: every 16-byte store takes bytes k..k+15 of two aligned
          * vectors s[i] and s[i + 1], both of which hold needed bytes, so nothing outside the
-         * run is read.  Each warp takes UR * 32 consecutive vectors per round (lane l, round
-         * u: vector w0 + 32u + l) and loads each once; s[i + 1] comes by shuffle from the
-         * next lane, or for lane 31 from lane 0 of the next round.  The one vector per warp
-         * that has no loaded neighbour (lane 31's last one, or the run's last vector) is loaded
-         * by its lane in the same round of loads. */
-        /* W = 32: whole warps; W = 8: the run belongs to one 8-lane segment of a warp (the
-         * sub-warp path for tiny pieces), and every shuffle stays inside the segment */
+         * run is read.  A group of W lanes (a warp, W = 32, or an 8-lane segment of one on the
+         * sub-warp path for tiny pieces, W = 8) takes UR * W consecutive vectors at a time
+         * (lane l, round u: vector w0 + W u + l) and loads each once; s[i + 1] comes by shuffle
+         * from the next lane, or for the group's last lane from lane 0 of the next round.  The
+         * one vector per group that has no loaded neighbour (the last lane's last one, or the
+         * run's last vector) is loaded by its lane in the same round of loads.  Every shuffle
+         * stays inside the group. */
         const uint4 *s = reinterpret_cast<const uint4 *>(src - k);
         const uint32_t lane = tid & (W - 1u), wid = tid / W;
-        const uint32_t mask = W == 32 ? 0xFFFFFFFFu : (((1u << W) - 1u) << (threadIdx.x & 31u & ~(W - 1u)));
+        const uint32_t mask =
+            W == 32 ? 0xFFFFFFFFu : (((1u << W) - 1u) << (threadIdx.x & 31u & ~(W - 1u)));
         const uint32_t step = nthr * UR;
         for (uint32_t base = 0; base < nvec; base += step) {
             const uint32_t w0 = base + wid * W * UR;
