@@ -88,3 +88,22 @@ def test_reference_arm_under_torchrun_prints_one_line():
     d = lines[0]
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["steps"] == 2
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["cpu_baseline"]["kind"] == "oracle"
+
+
+def test_bench_labels_and_traffic_record(monkeypatch):
+    """The benchmark's dtype label and dominant work class come from the workload; the recorded
+    ncu traffic is reported only while the kernel sources match the capture."""
+    sys.path.insert(0, ROOT)
+    import bench
+    import workloads
+    assert bench.path_types(workloads.named_config("llama3_8b_bf16"))[:2] == ("u16", 1)
+    assert bench.path_types(workloads.named_config("llama3_8b_f32_rne"))[:2] == ("f32->bf16", 4)
+    dt, cls, _ = bench.path_types(workloads.named_config("llama3_8b_fp8_block128"))
+    assert dt == "u16+u32+u8" and cls == 0
+    with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+        rec = json.load(f)["llama3_8b_bf16"]
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda: rec["kernel_sha256"])
+    assert bench.recorded_traffic("llama3_8b_bf16") == rec["dram_bytes_per_launch"]
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda: "0" * 64)
+    assert bench.recorded_traffic("llama3_8b_bf16") is None
+    assert bench.recorded_traffic("no_such_workload") is None
