@@ -12,15 +12,17 @@
  *   - each chunk moves InDisk -> InMem -> InGPU -> Destroyed through a two-stage pipeline
  *     (section 4.2, dependency (i)): host staging into a pinned slot, then a host->device copy
  *     into a device staging slot;
- *   - once a chunk is InGPU, one batched GPU kernel copies and assembles every tensor piece
+ *   - once a chunk is InGPU, one batched launch group copies and assembles every tensor piece
  *     that lies in it into its destination (dependency (ii)), which moves those tensors from
- *     Alloc to Loaded;
+ *     Alloc to Loaded: a TMA bulk-copy kernel for 16-byte-aligned runs, 16-byte vector kernels
+ *     for the rest (realigning unaligned runs in registers), and a kernel for column slices;
  *   - the chunk's staging slot is released once all its pieces are written (dependency (iii)).
  *
- * Beyond what the paper states, the kernel also fuses the serving engine's layout transforms
+ * Beyond what the paper states, the kernels also fuse the serving engine's layout transforms
  * (several checkpoint tensors written at row offsets of one fused destination, e.g. q/k/v into
- * one qkv weight), an optional fp32 -> bf16 round-to-nearest-even cast, and an optional
- * per-tensor 64-bit additive checksum of the destination element bits.
+ * one qkv weight; tensor- and expert-parallel shards), optional dtype conversions (fp32 -> bf16
+ * and fp32 -> fp16 with round-to-nearest-even, fp16 -> bf16, bf16 / fp16 -> fp32), and an
+ * optional per-tensor 64-bit additive checksum of the destination element bits.
  *
  * Conventions for every function below:
  *   - The return value is a cfa_status: CFA_OK (0) on success, a negative CFA_ERR_* code
@@ -134,8 +136,8 @@ typedef struct cfa_tensor_entry {
 /*
  * One destination parameter of the serving engine (a Loaded tensor of section 4.2).
  * dev_ptr is a device pointer owned by the caller, aligned to its element size (16-byte
- * alignment is what makes the vector path apply), and it must stay valid for every load that
- * uses the plan.  Destinations must not overlap one another in memory.
+ * alignment of destination and source lets whole slabs take the TMA kernel), and it must stay
+ * valid for every load that uses the plan.  Destinations must not overlap one another in memory.
  */
 typedef struct cfa_dst {
     void *dev_ptr;
@@ -167,7 +169,8 @@ typedef struct cfa_plan_opts {
     int32_t device;           /* CUDA device ordinal; -1 = the current device */
     uint32_t slab_bytes;      /* destination bytes per block-level work item, a multiple of 4096;
                                  default 262144 */
-    uint32_t tiny_bytes;      /* pieces with fewer destination bytes go warp-per-descriptor;
+    uint32_t tiny_bytes;      /* pieces with fewer destination bytes are warp-level items (four
+                                 per warp; those of at most 512 bytes in 8-lane segments);
                                  default 8192 */
     uint32_t flags;           /* CFA_OPT_*; default CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK */
     uint32_t reserved;        /* must be 0 */
@@ -193,15 +196,16 @@ void cfa_plan_opts_default(cfa_plan_opts *opts);
                                  path is kept for device memory */
 
 /* Writes blob bytes [blob_offset, blob_offset + len) to host memory dst and returns 0, or
- * returns non-zero on failure.  It runs on a CUDA host-function thread and must not call CUDA. */
+ * returns non-zero on failure.  It is called from the plan's fill threads, several at once for
+ * disjoint ranges, so it must be thread-safe; it must not call CUDA. */
 typedef int (*cfa_fill_fn)(void *user, uint64_t blob_offset, void *dst, uint64_t len);
 
 /*
  * Where the blob's bytes come from.  With period_bytes == 0, blob byte o is base[o].  With
  * period_bytes > 0 (a multiple of chunk_bytes), the blob is periodic and byte o is
  * base[o % period_bytes]; this streams a blob larger than memory from a smaller pool.  base must
- * be 256-byte aligned for PINNED, DEVICE and HOST_DIRECT sources.  The source must stay valid until the load
- * has completed (cfa_wait_layer(CFA_ALL) returned CFA_OK).
+ * be 256-byte aligned for PINNED, DEVICE and HOST_DIRECT sources.  The source must stay valid
+ * until the load has completed (cfa_wait_layer(CFA_ALL) returned).
  */
 typedef struct cfa_source {
     int32_t kind;
