@@ -54,6 +54,9 @@ def parse_args():
     ap.add_argument("--timeline", default=None, metavar="PATH",
                     help="write the per-chunk timeline (copy and unpack intervals) of the timed "
                          "pinned load of the attribution to PATH as JSON")
+    ap.add_argument("--stage-slices", action="store_true",
+                    help="pinned sources: copy column slices through the device slots instead of "
+                         "reading them in place (for comparison)")
     ap.add_argument("--vector-only", dest="bulk", action="store_false",
                     help="copy every slab with the 16-byte vector kernel instead of the TMA bulk "
                          "kernel (for comparison)")
@@ -176,7 +179,8 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
     out = {"h2d_pinned_gbs": round(h2d_gbs, 2)}
     # first, next to the end-to-end steps: per-layer readiness of one timed pinned load
     plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                    dev_slots=2, host_slots=0, timing=True, bulk=args.bulk)
+                    dev_slots=2, host_slots=0, timing=True, bulk=args.bulk,
+                    stage_slices=args.stage_slices)
     plan.load_async(cfa.Source.pinned(host.data_ptr(), period=m.period or 0), stream)
     plan.wait_layer()
     t = plan.layer_times()
@@ -539,7 +543,8 @@ def run_ours(args):
         del dtmp
         e2e_steps = args.e2e_steps or min(args.steps, 20)
         plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                        dev_slots=2, host_slots=0, bulk=args.bulk)
+                        dev_slots=2, host_slots=0, bulk=args.bulk,
+                        stage_slices=args.stage_slices)
         hsrc_all = cfa.Source.pinned(host.data_ptr(), period=m.period or 0)
         for _ in range(min(args.warmup, 3)):
             plan.load_async(hsrc_all, stream)

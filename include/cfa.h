@@ -158,6 +158,10 @@ typedef struct cfa_dst {
                                          is 1-4 % faster on GB300 */
 #define CFA_OPT_NO_MERGE        0x10u /* DEVICE sources: one launch per chunk instead of one
                                          launch per contiguous run of chunks */
+#define CFA_OPT_STAGE_SLICES    0x20u /* PINNED sources: copy column slices through the device
+                                         slots as strided 2-D copies; without it (the default)
+                                         the column-slice kernel reads them in place from the
+                                         pinned memory over the host link, beside the copy ring */
 
 typedef struct cfa_plan_opts {
     uint64_t chunk_bytes;     /* chunk length S, a multiple of 256; default 512 MiB */

@@ -348,7 +348,8 @@ class Plan:
 
     def __init__(self, entries, dsts, blob_bytes, chunk_bytes=512 << 20, host_slots=2,
                  dev_slots=2, fill_threads=8, slab_bytes=262144, tiny_bytes=8192, strict=True,
-                 host_only=False, timing=False, bulk=True, no_merge=False, device=-1,
+                 host_only=False, timing=False, bulk=True, no_merge=False, stage_slices=False,
+                 device=-1,
                  workspace=0, workspace_bytes=0):
         lib = _lib.load()
         self._lib = lib
@@ -372,7 +373,8 @@ class Plan:
                    (_lib.OPT_HOST_ONLY if host_only else 0) |
                    (_lib.OPT_TIMING if timing else 0) |
                    (_lib.OPT_BULK if bulk else 0) |
-                   (_lib.OPT_NO_MERGE if no_merge else 0))
+                   (_lib.OPT_NO_MERGE if no_merge else 0) |
+                   (_lib.OPT_STAGE_SLICES if stage_slices else 0))
         o.workspace = workspace or None
         o.workspace_bytes = workspace_bytes
         h = ctypes.c_void_p()

@@ -17,6 +17,7 @@ DTYPE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7, "
 DTYPE_SIZE = {"u8": 1, "bf16": 2, "f16": 2, "f32": 4, "i32": 4, "i64": 8, "f64": 8, "i16": 2}
 ENTRY_CAST_BF16, ENTRY_CKSUM, ENTRY_CONVERT = 0x1, 0x2, 0x4
 OPT_STRICT_COVERAGE, OPT_HOST_ONLY, OPT_TIMING, OPT_BULK, OPT_NO_MERGE = 0x1, 0x2, 0x4, 0x8, 0x10
+OPT_STAGE_SLICES = 0x20
 SRC_HOST, SRC_PINNED, SRC_CALLBACK, SRC_DEVICE, SRC_HOST_DIRECT = 1, 2, 3, 4, 5
 FILE_DIRECT = 0x1
 ALL = -1

@@ -124,6 +124,9 @@ struct cfa_plan {
     /* side streams that run a launch group's other kernels beside the caller's stream */
     cudaStream_t side_stream[kSideStreams] = {nullptr};
     cudaEvent_t ev_fork = nullptr, ev_join[kSideStreams] = {nullptr};
+    /* pinned sources: column slices read in place over the host link, beside the copy ring */
+    cudaStream_t direct_stream = nullptr;
+    cudaEvent_t ev_direct = nullptr;
     std::vector<cudaEvent_t> ev_dev_free, ev_h2d, ev_host_free, ev_filled, ev_layer;
     cudaEvent_t ev_begin = nullptr, ev_all = nullptr;
     std::vector<cudaEvent_t> t_h2d0, t_h2d1, t_k0, t_k1;
@@ -244,8 +247,10 @@ void CUDART_CB fill_host_fn(void *arg)
  * them.  With tma = false (a source in host memory, read over the host link) the aligned slabs
  * planned for the TMA kernel are copied by the vector kernel instead: bulk copies are for
  * device memory. */
+enum { LAUNCH_CONTIG = 1, LAUNCH_STRIDED = 2, LAUNCH_ALL = 3 };
+
 cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint64_t period,
-                  cudaStream_t s, bool tma = true)
+                  cudaStream_t s, bool tma = true, int what = LAUNCH_ALL)
 {
     const cfa_host_plan &hp = p->hp;
     const uint64_t lo = (uint64_t)c0 * hp.chunk_bytes;
@@ -259,15 +264,15 @@ cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint
     };
     Job jobs[3 * CFA_N_CLASSES];
     int n = 0;
-    for (int k = 0; k < CFA_N_CLASSES && hp.n_bulk; ++k) {
+    for (int k = 0; k < CFA_N_CLASSES && hp.n_bulk && (what & LAUNCH_CONTIG); ++k) {
         const uint32_t b0 = hp.bulk_first[k * row + c0], b1 = hp.bulk_first[k * row + c1];
         if (b1 != b0) jobs[n++] = Job{tma ? BULK : BULK_AS_VECTOR, k, b0, b1, 0, 0};
     }
-    for (int k = 0; k < CFA_N_CLASSES && hp.n_strided; ++k) {
+    for (int k = 0; k < CFA_N_CLASSES && hp.n_strided && (what & LAUNCH_STRIDED); ++k) {
         const uint32_t r0 = hp.strided_first[k * row + c0], r1 = hp.strided_first[k * row + c1];
         if (r1 != r0) jobs[n++] = Job{STRIDED, k, r0, r1, 0, 0};
     }
-    for (int k = 0; k < CFA_N_CLASSES; ++k) {
+    for (int k = 0; k < CFA_N_CLASSES && (what & LAUNCH_CONTIG); ++k) {
         const uint32_t s0 = hp.slab_first[k * row + c0], s1 = hp.slab_first[k * row + c1];
         const uint32_t t0 = hp.tiny_first[k * row + c0], t1 = hp.tiny_first[k * row + c1];
         if (s1 != s0 || t1 != t0) jobs[n++] = Job{VECTOR, k, s0, s1, t0, t1};
@@ -349,6 +354,9 @@ void release(cfa_plan *p)
         if (p->ev_begin) cudaEventDestroy(p->ev_begin);
         if (p->ev_all) cudaEventDestroy(p->ev_all);
         if (p->ev_fork) cudaEventDestroy(p->ev_fork);
+        if (p->direct_stream) cudaStreamSynchronize(p->direct_stream);
+        if (p->ev_direct) cudaEventDestroy(p->ev_direct);
+        if (p->direct_stream) cudaStreamDestroy(p->direct_stream);
         for (int j = 0; j < kSideStreams; ++j) {
             if (p->side_stream[j]) cudaStreamSynchronize(p->side_stream[j]);
             if (p->ev_join[j]) cudaEventDestroy(p->ev_join[j]);
@@ -473,6 +481,8 @@ cfa_status setup_device(cfa_plan *p)
         if ((st = make_event(nullptr, &p->ev_join[j], false))) return st;
     }
     if ((st = make_event(nullptr, &p->ev_fork, false))) return st;
+    CK(nullptr, cudaStreamCreateWithFlags(&p->direct_stream, cudaStreamNonBlocking));
+    if ((st = make_event(nullptr, &p->ev_direct, false))) return st;
     const bool timing = (o.flags & CFA_OPT_TIMING) != 0;
     auto events = [&](std::vector<cudaEvent_t> &v, size_t n, bool t) -> cfa_status {
         v.assign(n, nullptr);
@@ -720,6 +730,20 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             c0 = c1;
         }
     } else {
+        /* A pinned source is readable by the GPU in place, so its column slices need not go
+         * through the slots as strided 2-D copies (slower than plain copies on the copy engine):
+         * the column-slice kernels read them over the host link on the direct stream, in chunk
+         * order and ahead of the copy ring, and each chunk's readiness also waits for them. */
+        const bool slices_in_place = kind == CFA_SRC_PINNED && hp.n_strided &&
+                                     !(hp.opts.flags & CFA_OPT_STAGE_SLICES);
+        const size_t row = (size_t)hp.n_chunks + 1;
+        auto has_slices = [&](uint32_t c) {
+            for (int k = 0; k < CFA_N_CLASSES; ++k)
+                if (hp.strided_first[k * row + c + 1] != hp.strided_first[k * row + c])
+                    return true;
+            return false;
+        };
+        if (slices_in_place) CK(p, cudaStreamWaitEvent(p->direct_stream, p->ev_begin, 0));
         for (uint32_t c = 0; c < hp.n_chunks; ++c) {
             const int ds = (int)(c % (uint32_t)p->n_dev_slots);
             const uint64_t off = (uint64_t)c * S;
@@ -743,6 +767,7 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             for (uint32_t k = hp.copy_first[c]; k < hp.copy_first[c + 1]; ++k) {
                 const cfa_copy &cp = hp.copies[k];
                 const uint64_t at = cp.src - off;
+                if (slices_in_place && cp.rows > 1) continue; /* read in place instead */
                 if (cp.rows == 1)
                     CK(p, cudaMemcpyAsync(dslot + at, static_cast<const uint8_t *>(hsrc) + at,
                                           cp.width, cudaMemcpyHostToDevice, p->copy_stream));
@@ -756,10 +781,19 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             p->last_h2d++;
             if (staged) CK(p, cudaEventRecord(p->ev_host_free[hs], p->copy_stream));
             CK(p, cudaEventRecord(p->ev_h2d[ds], p->copy_stream));
+            const bool direct_c = slices_in_place && has_slices(c);
+            if (direct_c) {
+                cfa_status st = launch(p, c, c + 1, (uint64_t)(uintptr_t)src->base,
+                                       src->period_bytes, p->direct_stream, false, LAUNCH_STRIDED);
+                if (st) return st;
+                CK(p, cudaEventRecord(p->ev_direct, p->direct_stream));
+            }
             CK(p, cudaStreamWaitEvent(cs, p->ev_h2d[ds], 0));
-            cfa_status st = launch(p, c, c + 1, (uint64_t)(uintptr_t)dslot - off, 0, cs);
+            cfa_status st = launch(p, c, c + 1, (uint64_t)(uintptr_t)dslot - off, 0, cs, true,
+                                   slices_in_place ? LAUNCH_CONTIG : LAUNCH_ALL);
             if (st) return st;
             CK(p, cudaEventRecord(p->ev_dev_free[ds], cs));
+            if (direct_c) CK(p, cudaStreamWaitEvent(cs, p->ev_direct, 0));
             if ((st = record_layers(p, c, c + 1, cs))) return st;
         }
     }

@@ -498,3 +498,42 @@ def test_destroy_while_a_load_is_in_flight():
     for j in range(m.n_dsts):
         assert np.array_equal(d.host_bytes(j), ref.dst[j]), m.d_name[j]
     assert d.guards_intact()
+
+
+@pytest.mark.parametrize("stage_slices", [False, True])
+@pytest.mark.parametrize("chunk", [256, 64 << 10, 1 << 20])
+@pytest.mark.parametrize("cfg", ["dense_tp", "f32_tp", "moe_tp", "bf16_f32norm_tp"])
+def test_column_slices_from_pinned_memory(cfg, chunk, stage_slices):
+    """Pinned sources read column slices in place beside the copy ring (default), or copy them
+    through the slots as strided 2-D copies (stage_slices)."""
+    m = CONFIGS[cfg]()
+    st = load_and_compare(m, "pinned", chunk=chunk, stage_slices=stage_slices)
+    if chunk >= 64 << 10:  # with 256-byte chunks every slice row is cut into contiguous pieces
+        assert st["n_strided"] > 0
+
+
+def test_layer_readiness_waits_for_column_slices_read_in_place():
+    """A readiness group of a tensor-parallel rank is signalled only after its column slices,
+    read in place on their own stream, are written: snapshots taken on a consumer stream right
+    after each group's event equal the oracle."""
+    m = dense_config("tp_layers", 66, layers=4, hidden=512, n_q=8, n_kv=2, head_dim=64,
+                     inter=1536, vocab=1000, tp=2, rank=1)
+    blob, ref = reference(m)
+    h = torch.from_numpy(blob).pin_memory()
+    d = DeviceDsts(m)
+    consumer = torch.cuda.Stream()
+    with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=256 << 10) as plan:
+        groups = plan.info()["n_layers"]
+        for rep in range(3):
+            d.buf.fill_(0xA5)
+            plan.load_async(cfa.Source.pinned(h.data_ptr()))
+            snaps = {}
+            for g in range(groups):
+                plan.wait_layer(g, stream=consumer)
+                with torch.cuda.stream(consumer):
+                    for j in sorted(set(int(m.e_dst[i]) for i in np.nonzero(m.e_layer == g)[0])):
+                        snaps[j] = d.view(j).clone()
+            consumer.synchronize()
+            for j, t in snaps.items():
+                assert np.array_equal(t.cpu().numpy(), ref.dst[j]), (rep, m.d_name[j])
+            assert len(snaps) == m.n_dsts
