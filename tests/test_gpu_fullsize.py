@@ -215,6 +215,16 @@ def test_full_llama3_70b_bf16_tensor_parallel_rank():
                       dev_slots=0, host_slots=0)
     assert np.array_equal(ck, ck2)
     verify_all(m, d, ck2)
+    # and staged from the pinned pool: contiguous ranges through the copy ring, column slices
+    # read in place beside it
+    del dpool
+    torch.cuda.empty_cache()
+    d.buf.fill_(0xA5)
+    ck3, st3, _ = _load(m, d, cfa.Source.pinned(pool.data_ptr(), period=m.period),
+                        host_slots=0)
+    assert np.array_equal(ck, ck3)
+    verify_all(m, d, ck3)
+    assert d.guards_intact()
 
 
 def _past_4gib_manifest():
