@@ -256,10 +256,11 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
 
 def file_attribution(m, pageable, dsts, stream, args, threads):
     """A load from a safetensors file of the checkpoint (its header read by the library, the
-    data section read with pread by the fill threads into the pinned ring).  The file is
-    written just before, so buffered reads come from the page cache; O_DIRECT reads (data
-    section at a 4 KiB boundary, so whole blocks land in the pinned slots) come from the
-    storage under the temporary directory.  The file is removed afterwards."""
+    data section read by the fill threads into the pinned ring: with pread, or copied from a
+    read-only mapping of the file).  The file is written just before, so buffered reads come
+    from the page cache; O_DIRECT reads (data section at a 4 KiB boundary, so whole blocks land
+    in the pinned slots) come from the storage under the temporary directory.  The file is
+    removed afterwards."""
     import shutil
     import struct
     import tempfile
@@ -295,6 +296,13 @@ def file_attribution(m, pageable, dsts, stream, args, threads):
                "e2e_file_gbs": round(m.blob_bytes / ms / 1e6, 2),
                "file": f"safetensors, {len(st.tensors)} tensors, page cache (written and "
                        f"synced in {write_s:.1f} s just before)"}
+        with cfa.Source.file(path, st.data_offset, mapped=True) as src:
+            plan.load_async(src, stream)
+            plan.checksums()
+            ms = min(_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
+                     for _ in range(2))
+        out["e2e_file_mapped_s_per_model"] = round(ms / 1e3, 4)
+        out["e2e_file_mapped_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
         try:
             with cfa.Source.file(path, st.data_offset, direct=True) as src:
                 plan.load_async(src, stream)

@@ -436,6 +436,12 @@ cfa_status cfa_safetensors_close(cfa_safetensors *st);
 
 /* cfa_file_source_open flags. */
 #define CFA_FILE_DIRECT 0x1u /* O_DIRECT reads that bypass the page cache (storage bandwidth) */
+#define CFA_FILE_MMAP   0x2u /* map the file read-only and fill with memcpy from the mapping:
+                                 no system call per range (page-cache-resident files: 1.2x on
+                                 large ranges, 2-5x on the rows of column slices, on Grace).
+                                 The file must not shrink while mapped: reading a page past its
+                                 end raises SIGBUS instead of CFA_ERR_SOURCE.  Not combinable
+                                 with CFA_FILE_DIRECT. */
 
 /*
  * Fills *out with a CALLBACK source that reads blob byte o from file byte data_offset + o with

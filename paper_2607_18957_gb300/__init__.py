@@ -207,15 +207,17 @@ class Source:
 class FileSource(Source):
     """A checkpoint file read with pread by the plan's fill threads (cfa_file_source_open):
     blob byte o is file byte data_offset + o; direct=True reads with O_DIRECT, past the page
-    cache.  Close it after the last load that uses it has completed (the context manager
+    cache; mapped=True copies from a read-only mapping of the file (faster for page-cache-
+    resident files; the file must not shrink while mapped).  Close it after the last load that uses it has completed (the context manager
     does)."""
 
-    def __init__(self, path, data_offset=0, direct=False):
+    def __init__(self, path, data_offset=0, direct=False, mapped=False):
         lib = _lib.load()
         self._lib = lib
         self._c = _lib.Source()
-        st = lib.cfa_file_source_open(str(path).encode(), int(data_offset),
-                                      _lib.FILE_DIRECT if direct else 0, ctypes.byref(self._c))
+        flags = (_lib.FILE_DIRECT if direct else 0) | (_lib.FILE_MMAP if mapped else 0)
+        st = lib.cfa_file_source_open(str(path).encode(), int(data_offset), flags,
+                                      ctypes.byref(self._c))
         _check(st)
         super().__init__(_lib.SRC_CALLBACK, 0, 0, self._c.fill, self._c.user)
         self.path, self.data_offset, self.direct = str(path), int(data_offset), bool(direct)
@@ -236,8 +238,8 @@ class FileSource(Source):
         self.close()
 
 
-Source.file = staticmethod(lambda path, data_offset=0, direct=False:
-                           FileSource(path, data_offset, direct))
+Source.file = staticmethod(lambda path, data_offset=0, direct=False, mapped=False:
+                           FileSource(path, data_offset, direct, mapped))
 
 
 class StTensor(tuple):

@@ -19,6 +19,7 @@
 #include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
+#include <sys/mman.h>
 #include <sys/stat.h>
 #include <unistd.h>
 
@@ -479,6 +480,7 @@ typedef struct bounce {
 typedef struct {
     int fd;
     int direct;
+    const uint8_t *map; /* CFA_FILE_MMAP: the whole file, mapped read-only */
     uint64_t data_offset;
     uint64_t file_bytes;
     pthread_mutex_t mu; /* guards `free_list` */
@@ -588,6 +590,10 @@ static int file_fill(void *user, uint64_t off, void *dst, uint64_t len)
         f->data_offset + off + len > f->file_bytes)
         return 1;
     if (!len) return 0;
+    if (f->map) {
+        memcpy(dst, f->map + f->data_offset + off, len);
+        return 0;
+    }
     if (f->direct) return direct_fill(f, (uint8_t *)dst, len, f->data_offset + off);
     return read_full(f->fd, (uint8_t *)dst, len, f->data_offset + off);
 }
@@ -596,7 +602,9 @@ cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t
                                 cfa_source *out)
 {
     g_files_err[0] = 0;
-    if (!path || !out || (flags & ~(uint32_t)CFA_FILE_DIRECT)) return CFA_ERR_INVAL;
+    if (!path || !out || (flags & ~(uint32_t)(CFA_FILE_DIRECT | CFA_FILE_MMAP)) ||
+        ((flags & CFA_FILE_DIRECT) && (flags & CFA_FILE_MMAP)))
+        return CFA_ERR_INVAL;
     memset(out, 0, sizeof *out);
     file_src *f = (file_src *)calloc(1, sizeof *f);
     if (!f) return CFA_ERR_NOMEM;
@@ -617,6 +625,17 @@ cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t
     pthread_mutex_init(&f->mu, NULL);
     f->data_offset = data_offset;
     f->file_bytes = (uint64_t)sb.st_size;
+    if ((flags & CFA_FILE_MMAP) && f->file_bytes) {
+        void *m = mmap(NULL, (size_t)f->file_bytes, PROT_READ, MAP_SHARED, f->fd, 0);
+        if (m == MAP_FAILED) {
+            ferr("cannot map %s: %s", path, strerror(errno));
+            pthread_mutex_destroy(&f->mu);
+            close(f->fd);
+            free(f);
+            return CFA_ERR_SOURCE;
+        }
+        f->map = (const uint8_t *)m;
+    }
     out->kind = CFA_SRC_CALLBACK;
     out->fill = file_fill;
     out->user = f;
@@ -628,6 +647,7 @@ cfa_status cfa_file_source_close(cfa_source *src)
     if (!src) return CFA_ERR_INVAL;
     if (src->kind == CFA_SRC_CALLBACK && src->fill == file_fill && src->user) {
         file_src *f = (file_src *)src->user;
+        if (f->map) munmap((void *)f->map, (size_t)f->file_bytes);
         close(f->fd);
         for (bounce *b = f->free_list; b;) {
             bounce *n = b->next;

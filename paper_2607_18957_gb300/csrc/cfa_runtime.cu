@@ -208,10 +208,12 @@ void CUDART_CB fill_host_fn(void *arg)
     const uint64_t off = (uint64_t)j->chunk * S;
     uint8_t *dst = p->h_slots + (uint64_t)j->host_slot * S;
     const cfa_source &src = ctx->src;
-    /* the byte ranges, as (offset in chunk, length): a 2-D segment gives one per row */
+    /* the byte ranges, as (offset in chunk, length): a 2-D segment gives one per row, and
+     * long ranges are cut into 1 MiB pieces so that every fill thread gets a share even when a
+     * chunk holds only a few of them (a tensor-parallel shard) */
     std::vector<std::pair<uint64_t, uint64_t>> &ranges = j->ranges;
     if (ranges.empty()) {
-        const uint64_t part = 16ull << 20;
+        const uint64_t part = 1ull << 20;
         for (uint32_t k = hp.copy_first[j->chunk]; k < hp.copy_first[j->chunk + 1]; ++k) {
             const cfa_copy &cp = hp.copies[k];
             for (uint64_t r = 0; r < cp.rows; ++r)

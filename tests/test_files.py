@@ -208,8 +208,9 @@ def _direct_supported(path):
     return True
 
 
-@pytest.mark.parametrize("direct,data_align", [(False, 8), (True, 8), (True, 4096)])
-def test_file_source_fill_reads_the_data_section(tmp_path, direct, data_align):
+@pytest.mark.parametrize("mode,data_align", [("pread", 8), ("direct", 8), ("direct", 4096),
+                                             ("mmap", 8), ("mmap", 4096)])
+def test_file_source_fill_reads_the_data_section(tmp_path, mode, data_align):
     """Random ranges, destinations at every offset class within a 4 KiB block (for direct
     reads: bounced, and block-congruent with the file so the middle blocks land in place),
     ranges ending at the end of the file, and nothing written outside the range."""
@@ -217,12 +218,13 @@ def test_file_source_fill_reads_the_data_section(tmp_path, direct, data_align):
     p = tmp_path / "model.safetensors"
     off = write_safetensors(m, p, data_align=data_align)
     assert off % data_align == 0
+    direct = mode == "direct"
     if direct and not _direct_supported(p):
         pytest.skip("the file system has no O_DIRECT")
     blob = m.blob_range(0, m.blob_bytes)
     rng = np.random.default_rng(5)
     B = 4096
-    with cfa.Source.file(p, off, direct=direct) as src:
+    with cfa.Source.file(p, off, direct=direct, mapped=mode == "mmap") as src:
         c = src.to_c()
         assert c.kind == _lib.SRC_CALLBACK and c.fill and c.user
         fill = FillFn(c.fill)
@@ -279,3 +281,20 @@ def test_file_abi_is_exported():
         assert hasattr(lib, name)
     assert lib.cfa_abi_sizeof(b"cfa_st_tensor") == ctypes.sizeof(_lib.StTensor) == 96
     assert os.path.basename(cfa.library_path()) == "libcfa.so"
+
+
+def test_file_source_flags_are_checked(tmp_path):
+    p = tmp_path / "f.bin"
+    p.write_bytes(b"\0" * 4096)
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Source.file(p, 0, direct=True, mapped=True)
+    assert e.value.name == "CFA_ERR_INVAL"
+    lib = _lib.load()
+    c = _lib.Source()
+    assert lib.cfa_file_source_open(str(p).encode(), 0, 0x80, ctypes.byref(c)) == -1
+    empty = tmp_path / "empty.bin"
+    empty.write_bytes(b"")
+    with cfa.Source.file(empty, 0, mapped=True) as src:  # nothing to map, nothing to read
+        fill = FillFn(src.to_c().fill)
+        assert fill(src.to_c().user, 0, None, 0) == 0
+        assert fill(src.to_c().user, 0, None, 1) != 0

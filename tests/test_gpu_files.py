@@ -78,16 +78,16 @@ def compare(m, d, ck, ref, what):
 
 
 @pytest.mark.parametrize("chunk", [64 << 10, 1 << 20])
-@pytest.mark.parametrize("kind", ["file", "whole_pinned", "whole_direct_pageable"])
+@pytest.mark.parametrize("kind", ["file", "file_mapped", "whole_pinned", "whole_direct_pageable"])
 @pytest.mark.parametrize("name", ["dense", "f32_tp", "moe_tp", "f32_f16"])
 def test_parity_from_a_safetensors_file(tmp_path_factory, name, kind, chunk):
     m, path, off, ref = prepared(name, tmp_path_factory)
     st = cfa.Safetensors.open(path)
-    whole = kind != "file"
+    whole = kind.startswith("whole")
     entries = st.entries(targets_for(m), whole_file=whole)
     keep = []
-    if kind == "file":
-        src = cfa.Source.file(path, st.data_offset)
+    if not whole:
+        src = cfa.Source.file(path, st.data_offset, mapped=kind == "file_mapped")
         keep.append(src)
         blob_bytes = st.data_bytes
     else:
@@ -108,10 +108,10 @@ def test_parity_from_a_safetensors_file(tmp_path_factory, name, kind, chunk):
         ck = plan.checksums()
         stats = plan.stats()
     torch.cuda.synchronize()
-    if kind == "file":
+    if not whole:
         src.close()
     compare(m, d, ck, ref, f"{m.name} [{kind}, chunk {chunk}]")
-    if kind == "file":
+    if not whole:
         # only the byte ranges the pieces read are read from the file
         assert stats["staged_bytes"] <= st.data_bytes
 
