@@ -287,7 +287,9 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
  * that write all pieces of the chunk (DEVICE sources merge all chunks into one launch per work
  * class).  Staging and copies move only the byte ranges the chunk's pieces read (strided 2-D
  * copies for column slices), so a tensor-parallel rank moves about its share of the
- * checkpoint; cfa_stats.staged_bytes gives the total.  The load is ordered after
+ * checkpoint; cfa_stats.staged_bytes gives the total.  A chunk no piece reads (an
+ * expert-parallel rank's view of other ranks' experts) is skipped altogether: no fill, no copy,
+ * no launch, and it takes no staging slot.  The load is ordered after
  * all work enqueued on `stream` before this call, and work enqueued on `stream` after this
  * call sees every destination written.  Per-layer readiness is published through
  * cfa_wait_layer.  Loads on one plan run in the order they were enqueued; the checksums and
@@ -328,7 +330,8 @@ cfa_status cfa_get_stats(cfa_plan *plan, cfa_stats *out);
 cfa_status cfa_get_layer_times(cfa_plan *plan, float *ms_out, size_t n);
 
 /* One chunk of the last load on the timeline, in milliseconds from its first operation; -1 where
- * the step did not run (no host->device copy for in-place sources).  A merged launch over several
+ * the step did not run (no host->device copy for in-place sources, nothing for a chunk no piece
+ * reads).  A merged launch over several
  * chunks gives each of them the launch's interval. */
 typedef struct cfa_chunk_times {
     float h2d_begin_ms, h2d_end_ms;       /* the chunk's copies into its device slot */

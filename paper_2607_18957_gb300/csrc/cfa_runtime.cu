@@ -132,6 +132,10 @@ struct cfa_plan {
     std::vector<cudaEvent_t> t_h2d0, t_h2d1, t_k0, t_k1;
     std::vector<uint32_t> t_k_c0, t_k_c1; /* chunk range of each timed launch */
     std::vector<std::vector<uint32_t>> layers_ending; /* per chunk */
+    /* per chunk: some piece reads it.  A staged load skips the other chunks (no fill, copy,
+     * slot or launch), so that a rank's plan, which leaves whole chunks of other ranks'
+     * experts unread, keeps its copy stream busy instead of cycling slots through them. */
+    std::vector<uint8_t> chunk_busy;
     std::vector<uint32_t> layers_empty;
     std::unique_ptr<cfa::Pool> pool;
     std::vector<std::unique_ptr<LoadCtx>> loads;
@@ -187,15 +191,15 @@ void set_err(cfa_plan *p, const char *fmt, ...)
         }                                                                                  \
     } while (0)
 
-/* InDisk -> InMem for one chunk: puts the byte ranges the chunk's pieces read (its copy
- * segments; the rest of the slot is never read) into pinned slot `host_slot`, split over the
- * plan's fill threads in parts of at most 16 MiB. */
 /* NVTX range for the lifetime of a scope. */
 struct NvtxRange {
     explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
     ~NvtxRange() { nvtxRangePop(); }
 };
 
+/* InDisk -> InMem for one chunk: puts the byte ranges the chunk's pieces read (its copy
+ * segments; the rest of the slot is never read) into pinned slot `host_slot`, split over the
+ * plan's fill threads in parts of at most 1 MiB. */
 void CUDART_CB fill_host_fn(void *arg)
 {
     FillJob *j = static_cast<FillJob *>(arg);
@@ -590,6 +594,8 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
         if (hp.layer_last_chunk[l] < 0) p->layers_empty.push_back(l);
         else p->layers_ending[(size_t)hp.layer_last_chunk[l]].push_back(l);
     }
+    p->chunk_busy.assign(hp.n_chunks, 0);
+    for (size_t i = 0; i < hp.n_pieces; ++i) p->chunk_busy[hp.pieces[i].chunk] = 1;
     if (!p->host_only) {
         st = setup_device(p);
         if (st) {
@@ -694,8 +700,11 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
     ctx->src = *src;
     if (staged) {
         ctx->jobs.resize(hp.n_chunks);
+        uint32_t k = 0; /* busy chunks take the pinned slots in turn */
         for (uint32_t c = 0; c < hp.n_chunks; ++c)
-            ctx->jobs[c] = FillJob{ctx.get(), c, (int)(c % (uint32_t)p->n_host_slots), {}};
+            ctx->jobs[c] = FillJob{ctx.get(), c,
+                                   p->chunk_busy[c] ? (int)(k++ % (uint32_t)p->n_host_slots) : -1,
+                                   {}};
     }
     LoadCtx *cx = ctx.get();
     p->loads.push_back(std::move(ctx));
@@ -746,13 +755,19 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             return false;
         };
         if (slices_in_place) CK(p, cudaStreamWaitEvent(p->direct_stream, p->ev_begin, 0));
+        uint32_t k = 0; /* busy chunks so far: they take the slots in turn */
         for (uint32_t c = 0; c < hp.n_chunks; ++c) {
-            const int ds = (int)(c % (uint32_t)p->n_dev_slots);
+            if (!p->chunk_busy[c]) {
+                cfa_status st = record_layers(p, c, c + 1, cs);
+                if (st) return st;
+                continue;
+            }
+            const int ds = (int)(k % (uint32_t)p->n_dev_slots);
             const uint64_t off = (uint64_t)c * S;
             const void *hsrc;
             int hs = -1;
             if (staged) {
-                hs = (int)(c % (uint32_t)p->n_host_slots);
+                hs = cx->jobs[c].host_slot;
                 CK(p, cudaStreamWaitEvent(p->fill_stream, p->ev_host_free[hs], 0));
                 CK(p, cudaLaunchHostFunc(p->fill_stream, fill_host_fn, &cx->jobs[c]));
                 CK(p, cudaEventRecord(p->ev_filled[hs], p->fill_stream));
@@ -781,6 +796,7 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             }
             if (timing) CK(p, cudaEventRecord(p->t_h2d1[c], p->copy_stream));
             p->last_h2d++;
+            ++k;
             if (staged) CK(p, cudaEventRecord(p->ev_host_free[hs], p->copy_stream));
             CK(p, cudaEventRecord(p->ev_h2d[ds], p->copy_stream));
             const bool direct_c = slices_in_place && has_slices(c);
@@ -883,7 +899,8 @@ cfa_status cfa_get_stats(cfa_plan *p, cfa_stats *s)
         float ms = 0;
         CK(p, cudaEventElapsedTime(&ms, p->ev_begin, p->ev_all));
         s->load_ms = ms;
-        for (uint32_t c = 0; c < p->last_h2d && c < p->t_h2d0.size(); ++c) {
+        for (uint32_t c = 0; p->last_h2d && c < p->t_h2d0.size(); ++c) {
+            if (!p->chunk_busy[c]) continue;
             CK(p, cudaEventElapsedTime(&ms, p->t_h2d0[c], p->t_h2d1[c]));
             s->h2d_ms += ms;
         }
@@ -919,7 +936,8 @@ cfa_status cfa_get_timeline(cfa_plan *p, cfa_chunk_times *out, size_t n)
     DeviceGuard g(p->device);
     CK(p, cudaEventSynchronize(p->ev_all));
     for (size_t c = 0; c < n; ++c) out[c] = cfa_chunk_times{-1.f, -1.f, -1.f, -1.f};
-    for (uint32_t c = 0; c < p->last_h2d && c < n && c < p->t_h2d0.size(); ++c) {
+    for (uint32_t c = 0; p->last_h2d && c < n && c < p->t_h2d0.size(); ++c) {
+        if (!p->chunk_busy[c]) continue; /* not staged */
         CK(p, cudaEventElapsedTime(&out[c].h2d_begin_ms, p->ev_begin, p->t_h2d0[c]));
         CK(p, cudaEventElapsedTime(&out[c].h2d_end_ms, p->ev_begin, p->t_h2d1[c]));
     }

@@ -482,6 +482,41 @@ def test_timeline_orders_copies_before_unpacks():
     assert np.array_equal(ck, ref.cksum)
 
 
+@pytest.mark.parametrize("kind", ["pinned", "host", "callback"])
+def test_staged_load_skips_chunks_no_piece_reads(kind):
+    """An expert-parallel rank leaves whole chunks of other ranks' experts unread: a staged load
+    neither fills, copies nor unpacks them, and they take no staging slot, so the busy chunks'
+    copies follow one another with the two device slots alternating between busy chunks."""
+    m = cfg_moe_ep()
+    blob, ref = reference(m)
+    keep = []
+    d = DeviceDsts(m)
+    with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=64 << 10,
+                  timing=True, fill_threads=4) as plan:
+        n = plan.info()["n_chunks"]
+        busy = np.zeros(n, dtype=bool)
+        busy[plan.pieces()["chunk"]] = True
+        assert 0 < busy.sum() < n - 8  # whole chunks of other ranks' experts
+        for _ in range(2):
+            plan.load_async(make_source(kind, m, blob, keep))
+            plan.wait_layer()
+            ck = plan.checksums()
+            for j in range(m.n_dsts):
+                assert np.array_equal(d.host_bytes(j), ref.dst[j])
+            assert np.array_equal(ck, ref.cksum)
+            assert d.guards_intact()
+            t = plan.timeline()
+            assert (t[~busy] == -1).all()
+            tb = t[busy]
+            assert (tb[:, 0] >= 0).all() and (tb[:, 1] >= tb[:, 0]).all()
+            assert (tb[:, 2] >= tb[:, 1] - 1e-3).all() and (tb[:, 3] >= tb[:, 2]).all()
+            assert (tb[1:, 0] >= tb[:-1, 1] - 1e-3).all()  # one copy stream, chunk order
+            # the slot of busy chunk k + 2 is the slot of busy chunk k
+            assert (tb[2:, 0] >= tb[:-2, 3] - 1e-3).all()
+            lt = plan.layer_times()
+            assert (lt > 0).all() and (lt <= plan.stats()["load_ms"] + 1e-3).all()
+
+
 def test_destroy_while_a_load_is_in_flight():
     """Closing a plan with a load still running (a slow callback source) waits for the load and
     frees everything; the destinations hold the complete load."""
