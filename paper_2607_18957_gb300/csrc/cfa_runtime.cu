@@ -535,10 +535,16 @@ cfa_status check_status_word(cfa_plan *p)
     return CFA_OK;
 }
 
+/* Polls `ev` from the host, sleeping between queries, until it completes or timeout_ns passes
+ * (timeout_ns < 0: no limit).  The sleep doubles from 2 us up to kPollSleepMaxUs, so a load is
+ * noticed within about that much (plus the thread's timer slack) of its end: a 1 ms cap cost
+ * the end-to-end figure of a 76 ms load a whole millisecond. */
+constexpr int64_t kPollSleepMaxUs = 50;
+
 cfa_status wait_event_host(cfa_plan *p, cudaEvent_t ev, int64_t timeout_ns)
 {
     const auto t0 = std::chrono::steady_clock::now();
-    int64_t sleep_us = 10;
+    int64_t sleep_us = 2;
     for (;;) {
         const cudaError_t q = cudaEventQuery(ev);
         if (q == cudaSuccess) return CFA_OK;
@@ -556,7 +562,7 @@ cfa_status wait_event_host(cfa_plan *p, cudaEvent_t ev, int64_t timeout_ns)
             }
         }
         std::this_thread::sleep_for(std::chrono::microseconds(sleep_us));
-        sleep_us = std::min<int64_t>(sleep_us * 2, 1000);
+        sleep_us = std::min<int64_t>(sleep_us * 2, kPollSleepMaxUs);
     }
 }
 
