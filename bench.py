@@ -167,9 +167,10 @@ class ClockSampler:
 # ------------------------------------------------------------------------------------------
 def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
     """Where end-to-end time goes: (CFA_OPT_TIMING) per-layer readiness of one pinned load, the
-    host link for pinned and pageable memory, host memcpy with the loader's fill threads, a load
-    from a pageable copy of the checkpoint through the pinned staging ring and the same copy read
-    in place, and a load from a safetensors file."""
+    pinned blob read in place by the kernels (no copy engine), the host link for pinned and
+    pageable memory, host memcpy with the loader's fill threads, a load from a pageable copy of
+    the checkpoint through the pinned staging ring and the same copy read in place, and a load
+    from a safetensors file."""
     from concurrent.futures import ThreadPoolExecutor
 
     import numpy as np
@@ -201,6 +202,21 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
                              "groups": int(t.size), "load_ms": round(st["load_ms"], 2),
                              "h2d_ms": round(st["h2d_ms"], 2),
                              "unpack_ms": round(st["unpack_ms"], 2)}
+    # the same pinned blob read in place by the unpack kernels over NVLink-C2C (no copy
+    # engine, no slots): every step, to show step-to-step spread beside the staged steps
+    plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                    dev_slots=0, host_slots=0, bulk=args.bulk)
+    src = cfa.Source.host_direct(host.data_ptr(), period=m.period or 0)
+    try:
+        plan.load_async(src, stream)
+        plan.checksums()
+        steps = [_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
+                 for _ in range(6)]
+        out["e2e_direct_pinned_s_per_model"] = round(statistics.mean(steps) / 1e3, 4)
+        out["e2e_direct_pinned_step_ms"] = [round(x, 1) for x in steps]
+    except cfa.CfaError as e:
+        out["e2e_direct_pinned"] = f"unavailable: {e}"
+    plan.close()
     gib = 1 << 30
     threads = max(1, len(os.sched_getaffinity(0)))
     raw = np.empty(m.source_bytes() + 256, dtype=np.uint8)
@@ -257,7 +273,7 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
 def file_attribution(m, pageable, dsts, stream, args, threads):
     """A load from a safetensors file of the checkpoint (its header read by the library, the
     data section read by the fill threads into the pinned ring: with pread, or copied from a
-    read-only mapping of the file).  The file is written just before, so buffered reads come
+    read-only mapping of the file; or the mapping read in place by the unpack kernels).  The file is written just before, so buffered reads come
     from the page cache; O_DIRECT reads (data section at a 4 KiB boundary, so whole blocks land
     in the pinned slots) come from the storage under the temporary directory.  The file is
     removed afterwards."""
@@ -303,6 +319,16 @@ def file_attribution(m, pageable, dsts, stream, args, threads):
                      for _ in range(2))
         out["e2e_file_mapped_s_per_model"] = round(ms / 1e3, 4)
         out["e2e_file_mapped_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
+        try:  # the mapping read in place by the unpack kernels over the host link
+            with cfa.Source.file(path, st.data_offset, in_place=True) as src:
+                plan.load_async(src, stream)
+                plan.checksums()
+                ms = min(_timed(lambda: (plan.load_async(src, stream), plan.checksums()),
+                                stream) for _ in range(2))
+            out["e2e_file_in_place_s_per_model"] = round(ms / 1e3, 4)
+            out["e2e_file_in_place_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
+        except cfa.CfaError as e:
+            out["e2e_file_in_place"] = f"unavailable: {e}"
         try:
             with cfa.Source.file(path, st.data_offset, direct=True) as src:
                 plan.load_async(src, stream)

@@ -208,8 +208,12 @@ typedef int (*cfa_fill_fn)(void *user, uint64_t blob_offset, void *dst, uint64_t
  * Where the blob's bytes come from.  With period_bytes == 0, blob byte o is base[o].  With
  * period_bytes > 0 (a multiple of chunk_bytes), the blob is periodic and byte o is
  * base[o % period_bytes]; this streams a blob larger than memory from a smaller pool.  base must
- * be 256-byte aligned for PINNED, DEVICE and HOST_DIRECT sources.  The source must stay valid
- * until the load has completed (cfa_wait_layer(CFA_ALL) returned).
+ * be 256-byte aligned for PINNED and DEVICE sources and 8-byte aligned for HOST_DIRECT ones (the
+ * vector kernels that read host memory take any 16-byte phase; 8 keeps every element aligned).
+ * size_bytes, when not 0, is how many bytes can be read at base: a load whose plan would read
+ * past them (blob_bytes, or period_bytes for a periodic source) is refused with CFA_ERR_INVAL
+ * before any GPU work.  The source must stay valid until the load has completed
+ * (cfa_wait_layer(CFA_ALL) returned).
  */
 typedef struct cfa_source {
     int32_t kind;
@@ -218,6 +222,7 @@ typedef struct cfa_source {
     uint64_t period_bytes;
     cfa_fill_fn fill;
     void *user;
+    uint64_t size_bytes; /* 0: not stated */
 } cfa_source;
 
 typedef struct cfa_plan cfa_plan;
@@ -445,6 +450,15 @@ cfa_status cfa_safetensors_close(cfa_safetensors *st);
                                  The file must not shrink while mapped: reading a page past its
                                  end raises SIGBUS instead of CFA_ERR_SOURCE.  Not combinable
                                  with CFA_FILE_DIRECT. */
+#define CFA_FILE_MMAP_IN_PLACE 0x4u /* map the file read-only, populated, and give a HOST_DIRECT
+                                 source over the mapping: the unpack kernels read the file's
+                                 page-cache pages in place over the host link, with no fill
+                                 threads, pinned slots or copies (devices with pageable memory
+                                 access, such as Grace-based GB300: 2x the pread and copy modes
+                                 for a page-cache-resident file).  base = mapping + data_offset,
+                                 so data_offset must be a multiple of 8 (a safetensors data
+                                 section is); size_bytes = file size - data_offset.  Same SIGBUS
+                                 caveat as CFA_FILE_MMAP; not combinable with the other flags. */
 
 /*
  * Fills *out with a CALLBACK source that reads blob byte o from file byte data_offset + o with
@@ -452,10 +466,13 @@ cfa_status cfa_safetensors_close(cfa_safetensors *st);
  * O_DIRECT: reads move whole 4 KiB blocks; where a destination range and its file range start
  * at the same offset within a block (data_offset a multiple of 4 KiB and a chunk length that is
  * too) the middle blocks land in the pinned slot directly, the rest passes through 4 MiB
- * bounce buffers owned by the source.  The file stays open until cfa_file_source_close(out),
- * which must come after every load using it has completed.
- * Errors: CFA_ERR_SOURCE (cannot open; for CFA_FILE_DIRECT also a file system without
- * O_DIRECT), CFA_ERR_INVAL (unknown flag), CFA_ERR_NOMEM.
+ * bounce buffers owned by the source.  With CFA_FILE_MMAP_IN_PLACE *out is a HOST_DIRECT
+ * source instead (its fill pointer is set only to mark it as a file source for
+ * cfa_file_source_close; HOST_DIRECT loads never call it).  The file stays open until
+ * cfa_file_source_close(out), which must come after every load using it has completed.
+ * Errors: CFA_ERR_SOURCE (cannot open or map; for CFA_FILE_DIRECT also a file system without
+ * O_DIRECT; data_offset past the end of the file), CFA_ERR_ALIGN (CFA_FILE_MMAP_IN_PLACE with
+ * data_offset not a multiple of 8), CFA_ERR_INVAL (unknown flag or combination), CFA_ERR_NOMEM.
  */
 cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t flags,
                                 cfa_source *out);

@@ -164,29 +164,30 @@ def make_dsts(dsts):
 class Source:
     """Where the blob comes from (cfa_source)."""
 
-    def __init__(self, kind, base=0, period=0, fill=None, user=None):
+    def __init__(self, kind, base=0, period=0, fill=None, user=None, size=0):
         self.kind, self.base, self.period, self.fill, self.user = kind, base, period, fill, user
+        self.size = size  # bytes readable at base; 0: not stated (a load checks it when stated)
 
     @classmethod
-    def host(cls, ptr, period=0):
+    def host(cls, ptr, period=0, size=0):
         """Pageable host memory, copied into pinned slots by the plan's threads."""
-        return cls(_lib.SRC_HOST, ptr, period)
+        return cls(_lib.SRC_HOST, ptr, period, size=size)
 
     @classmethod
-    def pinned(cls, ptr, period=0):
+    def pinned(cls, ptr, period=0, size=0):
         """Page-locked host memory, copied straight to the device."""
-        return cls(_lib.SRC_PINNED, ptr, period)
+        return cls(_lib.SRC_PINNED, ptr, period, size=size)
 
     @classmethod
-    def device(cls, ptr, period=0):
+    def device(cls, ptr, period=0, size=0):
         """Device memory that already holds the blob (no staging, no copies)."""
-        return cls(_lib.SRC_DEVICE, ptr, period)
+        return cls(_lib.SRC_DEVICE, ptr, period, size=size)
 
     @classmethod
-    def host_direct(cls, ptr, period=0):
-        """Host memory (pageable or page-locked) that the unpack kernel reads in place over the
-        host link; pageable memory needs a device with pageable memory access."""
-        return cls(_lib.SRC_HOST_DIRECT, ptr, period)
+    def host_direct(cls, ptr, period=0, size=0):
+        """Host memory (pageable or page-locked, 8-byte aligned) that the unpack kernel reads in
+        place over the host link; pageable memory needs a device with pageable memory access."""
+        return cls(_lib.SRC_HOST_DIRECT, ptr, period, size=size)
 
     @classmethod
     def callback(cls, fill_fn_ptr, user_ptr=0):
@@ -201,26 +202,33 @@ class Source:
         s.period_bytes = self.period
         s.fill = self.fill or None
         s.user = self.user or None
+        s.size_bytes = self.size
         return s
 
 
 class FileSource(Source):
-    """A checkpoint file read with pread by the plan's fill threads (cfa_file_source_open):
-    blob byte o is file byte data_offset + o; direct=True reads with O_DIRECT, past the page
-    cache; mapped=True copies from a read-only mapping of the file (faster for page-cache-
-    resident files; the file must not shrink while mapped).  Close it after the last load that uses it has completed (the context manager
-    does)."""
+    """A checkpoint file (cfa_file_source_open): blob byte o is file byte data_offset + o.  By
+    default the plan's fill threads read it with pread; direct=True reads with O_DIRECT, past
+    the page cache; mapped=True copies from a read-only mapping of the file (faster for page-
+    cache-resident files); in_place=True maps the file and lets the unpack kernels read the
+    mapping over the host link, with no fill threads, pinned slots or copies (devices with
+    pageable memory access; data_offset a multiple of 8).  A mapped file must not shrink while
+    mapped.  Close the source after the last load that uses it has completed (the context
+    manager does)."""
 
-    def __init__(self, path, data_offset=0, direct=False, mapped=False):
+    def __init__(self, path, data_offset=0, direct=False, mapped=False, in_place=False):
         lib = _lib.load()
         self._lib = lib
         self._c = _lib.Source()
-        flags = (_lib.FILE_DIRECT if direct else 0) | (_lib.FILE_MMAP if mapped else 0)
+        flags = ((_lib.FILE_DIRECT if direct else 0) | (_lib.FILE_MMAP if mapped else 0) |
+                 (_lib.FILE_MMAP_IN_PLACE if in_place else 0))
         st = lib.cfa_file_source_open(str(path).encode(), int(data_offset), flags,
                                       ctypes.byref(self._c))
         _check(st)
-        super().__init__(_lib.SRC_CALLBACK, 0, 0, self._c.fill, self._c.user)
+        super().__init__(self._c.kind, self._c.base or 0, 0, self._c.fill, self._c.user,
+                         size=self._c.size_bytes)
         self.path, self.data_offset, self.direct = str(path), int(data_offset), bool(direct)
+        self.in_place = bool(in_place)
 
     def to_c(self):
         if not self._c.user:
@@ -238,8 +246,9 @@ class FileSource(Source):
         self.close()
 
 
-Source.file = staticmethod(lambda path, data_offset=0, direct=False, mapped=False:
-                           FileSource(path, data_offset, direct, mapped))
+Source.file = staticmethod(lambda path, data_offset=0, direct=False, mapped=False,
+                           in_place=False: FileSource(path, data_offset, direct, mapped,
+                                                      in_place))
 
 
 class StTensor(tuple):

@@ -19,7 +19,7 @@ ENTRY_CAST_BF16, ENTRY_CKSUM, ENTRY_CONVERT = 0x1, 0x2, 0x4
 OPT_STRICT_COVERAGE, OPT_HOST_ONLY, OPT_TIMING, OPT_BULK, OPT_NO_MERGE = 0x1, 0x2, 0x4, 0x8, 0x10
 OPT_STAGE_SLICES = 0x20
 SRC_HOST, SRC_PINNED, SRC_CALLBACK, SRC_DEVICE, SRC_HOST_DIRECT = 1, 2, 3, 4, 5
-FILE_DIRECT, FILE_MMAP = 0x1, 0x2
+FILE_DIRECT, FILE_MMAP, FILE_MMAP_IN_PLACE = 0x1, 0x2, 0x4
 ALL = -1
 
 # cfa_tensor_entry and cfa_dst as numpy records (fast for 10^5 entries)
@@ -46,7 +46,8 @@ class PlanOpts(ctypes.Structure):
 class Source(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int32), ("reserved", ctypes.c_int32),
                 ("base", ctypes.c_void_p), ("period_bytes", ctypes.c_uint64),
-                ("fill", ctypes.c_void_p), ("user", ctypes.c_void_p)]
+                ("fill", ctypes.c_void_p), ("user", ctypes.c_void_p),
+                ("size_bytes", ctypes.c_uint64)]
 
 
 class Stats(ctypes.Structure):

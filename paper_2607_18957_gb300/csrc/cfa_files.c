@@ -480,7 +480,7 @@ typedef struct bounce {
 typedef struct {
     int fd;
     int direct;
-    const uint8_t *map; /* CFA_FILE_MMAP: the whole file, mapped read-only */
+    const uint8_t *map; /* CFA_FILE_MMAP(_IN_PLACE): the whole file, mapped read-only */
     uint64_t data_offset;
     uint64_t file_bytes;
     pthread_mutex_t mu; /* guards `free_list` */
@@ -602,9 +602,15 @@ cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t
                                 cfa_source *out)
 {
     g_files_err[0] = 0;
-    if (!path || !out || (flags & ~(uint32_t)(CFA_FILE_DIRECT | CFA_FILE_MMAP)) ||
-        ((flags & CFA_FILE_DIRECT) && (flags & CFA_FILE_MMAP)))
-        return CFA_ERR_INVAL;
+    const uint32_t modes = flags & (CFA_FILE_DIRECT | CFA_FILE_MMAP | CFA_FILE_MMAP_IN_PLACE);
+    if (!path || !out || modes != flags || (modes & (modes - 1)))
+        return CFA_ERR_INVAL; /* an unknown flag, or more than one mode */
+    const int in_place = (flags & CFA_FILE_MMAP_IN_PLACE) != 0;
+    if (in_place && (data_offset & 7u)) {
+        ferr("in-place reads need the data section at a multiple of 8 bytes in the file (data "
+             "offset %llu)", (unsigned long long)data_offset);
+        return CFA_ERR_ALIGN;
+    }
     memset(out, 0, sizeof *out);
     file_src *f = (file_src *)calloc(1, sizeof *f);
     if (!f) return CFA_ERR_NOMEM;
@@ -625,8 +631,19 @@ cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t
     pthread_mutex_init(&f->mu, NULL);
     f->data_offset = data_offset;
     f->file_bytes = (uint64_t)sb.st_size;
-    if ((flags & CFA_FILE_MMAP) && f->file_bytes) {
-        void *m = mmap(NULL, (size_t)f->file_bytes, PROT_READ, MAP_SHARED, f->fd, 0);
+    if (in_place && data_offset > f->file_bytes) {
+        ferr("data offset %llu is past the end of %s (%llu bytes)",
+             (unsigned long long)data_offset, path, (unsigned long long)f->file_bytes);
+        pthread_mutex_destroy(&f->mu);
+        close(f->fd);
+        free(f);
+        return CFA_ERR_SOURCE;
+    }
+    if ((flags & (CFA_FILE_MMAP | CFA_FILE_MMAP_IN_PLACE)) && f->file_bytes) {
+        /* in place, the pages are mapped up front (read into the page cache if they are not
+         * there yet), so the kernels' first reads do not wait on page faults */
+        void *m = mmap(NULL, (size_t)f->file_bytes, PROT_READ,
+                       MAP_SHARED | (in_place ? MAP_POPULATE : 0), f->fd, 0);
         if (m == MAP_FAILED) {
             ferr("cannot map %s: %s", path, strerror(errno));
             pthread_mutex_destroy(&f->mu);
@@ -636,16 +653,23 @@ cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t
         }
         f->map = (const uint8_t *)m;
     }
-    out->kind = CFA_SRC_CALLBACK;
-    out->fill = file_fill;
+    out->fill = file_fill; /* for a HOST_DIRECT source only a mark: such loads never fill */
     out->user = f;
+    if (in_place) {
+        out->kind = CFA_SRC_HOST_DIRECT;
+        out->base = f->map ? f->map + data_offset : NULL;
+        out->size_bytes = f->file_bytes - data_offset;
+    } else {
+        out->kind = CFA_SRC_CALLBACK;
+    }
     return CFA_OK;
 }
 
 cfa_status cfa_file_source_close(cfa_source *src)
 {
     if (!src) return CFA_ERR_INVAL;
-    if (src->kind == CFA_SRC_CALLBACK && src->fill == file_fill && src->user) {
+    if ((src->kind == CFA_SRC_CALLBACK || src->kind == CFA_SRC_HOST_DIRECT) &&
+        src->fill == file_fill && src->user) {
         file_src *f = (file_src *)src->user;
         if (f->map) munmap((void *)f->map, (size_t)f->file_bytes);
         close(f->fd);

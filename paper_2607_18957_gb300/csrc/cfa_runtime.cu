@@ -652,9 +652,21 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
         set_err(p, "source has no base pointer or fill function");
         return CFA_ERR_INVAL;
     }
-    if ((kind == CFA_SRC_PINNED || kind == CFA_SRC_DEVICE || kind == CFA_SRC_HOST_DIRECT) &&
-        ((uintptr_t)src->base & 255u)) {
-        set_err(p, "pinned, device and direct host sources must be 256-byte aligned");
+    if (kind != CFA_SRC_CALLBACK && src->size_bytes) {
+        const uint64_t need = src->period_bytes ? std::min(src->period_bytes, hp.blob_bytes)
+                                                : hp.blob_bytes;
+        if (need > src->size_bytes) {
+            set_err(p, "the plan reads %llu bytes of the source, which holds %llu",
+                    (unsigned long long)need, (unsigned long long)src->size_bytes);
+            return CFA_ERR_INVAL;
+        }
+    }
+    if (kind == CFA_SRC_HOST_DIRECT && ((uintptr_t)src->base & 7u)) {
+        set_err(p, "direct host sources must be 8-byte aligned");
+        return CFA_ERR_ALIGN;
+    }
+    if ((kind == CFA_SRC_PINNED || kind == CFA_SRC_DEVICE) && ((uintptr_t)src->base & 255u)) {
+        set_err(p, "pinned and device sources must be 256-byte aligned");
         return CFA_ERR_ALIGN;
     }
     const bool staged = kind == CFA_SRC_HOST || kind == CFA_SRC_CALLBACK;

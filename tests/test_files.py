@@ -298,3 +298,52 @@ def test_file_source_flags_are_checked(tmp_path):
         fill = FillFn(src.to_c().fill)
         assert fill(src.to_c().user, 0, None, 0) == 0
         assert fill(src.to_c().user, 0, None, 1) != 0
+
+
+@pytest.mark.parametrize("data_align", [8, 4096])
+def test_in_place_file_source_maps_the_data_section(tmp_path, data_align):
+    """CFA_FILE_MMAP_IN_PLACE gives a HOST_DIRECT source whose base is the data section inside
+    a read-only mapping of the whole file and whose size is the rest of the file; closing it
+    unmaps the file."""
+    m = configs()[0]
+    p = tmp_path / "model.safetensors"
+    off = write_safetensors(m, p, data_align=data_align)
+    size = os.path.getsize(p)
+    with cfa.Source.file(p, off, in_place=True) as src:
+        c = src.to_c()
+        assert c.kind == _lib.SRC_HOST_DIRECT and c.base and c.user and c.fill
+        assert c.base % 8 == 0 and c.size_bytes == size - off == m.blob_bytes
+        assert src.base == c.base and src.size == c.size_bytes
+        got = np.frombuffer(ctypes.string_at(c.base, c.size_bytes), dtype=np.uint8)
+        assert np.array_equal(got, m.blob_range(0, m.blob_bytes))
+    with pytest.raises(cfa.CfaError):
+        src.to_c()  # closed
+
+
+def test_in_place_file_source_rules(tmp_path):
+    p = tmp_path / "f.bin"
+    p.write_bytes(bytes(range(256)) * 16)
+    for kw in (dict(direct=True), dict(mapped=True)):
+        with pytest.raises(cfa.CfaError) as e:
+            cfa.Source.file(p, 0, in_place=True, **kw)
+        assert e.value.name == "CFA_ERR_INVAL"
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Source.file(p, 12, in_place=True)  # elements would not be aligned
+    assert e.value.name == "CFA_ERR_ALIGN" and "multiple of 8" in str(e.value)
+    with pytest.raises(cfa.CfaError) as e:
+        cfa.Source.file(p, 4096 + 8, in_place=True)
+    assert e.value.name == "CFA_ERR_SOURCE" and "past the end" in str(e.value)
+    with cfa.Source.file(p, 4096, in_place=True) as src:  # an empty data section at the end
+        assert src.to_c().size_bytes == 0
+    with cfa.Source.file(p, 8, in_place=True) as src:
+        c = src.to_c()
+        assert c.size_bytes == 4088 and ctypes.string_at(c.base, 4) == bytes([8, 9, 10, 11])
+    empty = tmp_path / "empty.bin"
+    empty.write_bytes(b"")
+    with cfa.Source.file(empty, 0, in_place=True) as src:  # nothing to map
+        assert not src.to_c().base and src.to_c().size_bytes == 0
+    # a HOST_DIRECT source the library did not open is not closed by cfa_file_source_close
+    lib = _lib.load()
+    c = _lib.Source()
+    c.kind, c.user = _lib.SRC_HOST_DIRECT, 1234
+    assert lib.cfa_file_source_close(ctypes.byref(c)) == -1

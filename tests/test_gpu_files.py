@@ -1,8 +1,8 @@
 """GPU parity for checkpoint files: a safetensors file written from a seeded manifest is loaded
 through its header (Safetensors.entries) and compared byte for byte, checksum for checksum,
 with the oracle on the manifest.  Sources: the pread file source (data section staged through
-the pinned ring, buffered or O_DIRECT), and the whole file read into page-locked or pageable
-memory with the blob being the whole file.  Whole tensors, row and column shards, conversions; a file that shrinks
+the pinned ring, buffered or O_DIRECT, or the mapped file read in place by the kernels), and
+the whole file read into page-locked or pageable memory with the blob being the whole file.  Whole tensors, row and column shards, conversions; a file that shrinks
 under a load is reported as a source error and the plan recovers."""
 import os
 
@@ -78,7 +78,8 @@ def compare(m, d, ck, ref, what):
 
 
 @pytest.mark.parametrize("chunk", [64 << 10, 1 << 20])
-@pytest.mark.parametrize("kind", ["file", "file_mapped", "whole_pinned", "whole_direct_pageable"])
+@pytest.mark.parametrize("kind", ["file", "file_mapped", "file_in_place", "whole_pinned",
+                                  "whole_direct_pageable"])
 @pytest.mark.parametrize("name", ["dense", "f32_tp", "moe_tp", "f32_f16"])
 def test_parity_from_a_safetensors_file(tmp_path_factory, name, kind, chunk):
     m, path, off, ref = prepared(name, tmp_path_factory)
@@ -87,7 +88,8 @@ def test_parity_from_a_safetensors_file(tmp_path_factory, name, kind, chunk):
     entries = st.entries(targets_for(m), whole_file=whole)
     keep = []
     if not whole:
-        src = cfa.Source.file(path, st.data_offset, mapped=kind == "file_mapped")
+        src = cfa.Source.file(path, st.data_offset, mapped=kind == "file_mapped",
+                              in_place=kind == "file_in_place")
         keep.append(src)
         blob_bytes = st.data_bytes
     else:
@@ -114,6 +116,74 @@ def test_parity_from_a_safetensors_file(tmp_path_factory, name, kind, chunk):
     if not whole:
         # only the byte ranges the pieces read are read from the file
         assert stats["staged_bytes"] <= st.data_bytes
+
+
+@pytest.mark.parametrize("phase", [0, 8])
+@pytest.mark.parametrize("name", ["dense", "f32_tp", "moe_tp", "f32_f16"])
+def test_parity_from_a_file_read_in_place(tmp_path_factory, tmp_path, name, phase):
+    """CFA_FILE_MMAP_IN_PLACE: the kernels read the mapped file over the host link, with the
+    data section at a 16-byte boundary of the file or 8 bytes past one (header padded with
+    spaces), so that every 16-byte phase of the source reaches the vector kernels."""
+    from workloads.stfile import file_tensors, header_bytes
+    import struct
+    m, _, _, ref = prepared(name, tmp_path_factory)
+    hdr = header_bytes(file_tensors(m), data_align=16) + b" " * phase
+    path = str(tmp_path / "in_place.safetensors")
+    with open(path, "wb") as f:
+        f.write(struct.pack("<Q", len(hdr)))
+        f.write(hdr)
+        f.write(m.blob_range(0, m.blob_bytes).tobytes())
+    st = cfa.Safetensors.open(path)
+    assert st.data_offset % 16 == phase
+    d = DeviceDsts(m)
+    with cfa.Source.file(path, st.data_offset, in_place=True) as src, \
+            cfa.Plan(st.entries(targets_for(m)), d.cfa_dsts, st.data_bytes,
+                     chunk_bytes=256 << 10) as plan:
+        for _ in range(2):
+            plan.load_async(src)
+            plan.wait_layer()
+            ck = plan.checksums()
+            compare(m, d, ck, ref, f"{m.name} [in place, phase {phase}]")
+            d.buf.fill_(0xA5)
+        assert plan.stats()["staged_bytes"] <= st.data_bytes
+    # a plan that reads past the source's stated size is refused before any GPU work
+    with cfa.Source.file(path, st.data_offset, in_place=True) as src, \
+            cfa.Plan(st.entries(targets_for(m), whole_file=True), d.cfa_dsts,
+                     st.data_offset + st.data_bytes, chunk_bytes=256 << 10) as plan:
+        with pytest.raises(cfa.CfaError) as e:
+            plan.load_async(src)
+        assert e.value.name == "CFA_ERR_INVAL" and "holds" in str(e.value)
+    torch.cuda.synchronize()
+    assert (d.buf == 0xA5).all()
+
+
+def test_source_size_and_direct_alignment_rules(tmp_path_factory):
+    """A stated source size smaller than what the plan reads is refused for every in-place
+    kind; a direct host source needs 8-byte alignment only (a pageable copy 8 bytes past a
+    16-byte boundary loads exactly)."""
+    m, path, off, ref = prepared("dense", tmp_path_factory)
+    st = cfa.Safetensors.open(path)
+    data = np.fromfile(path, dtype=np.uint8)[st.data_offset:]
+    h = aligned_pageable(data.size + 16)
+    h8 = h[8:8 + data.size]
+    h8[:] = data
+    pinned = torch.from_numpy(np.ascontiguousarray(data)).pin_memory()
+    d = DeviceDsts(m)
+    with cfa.Plan(st.entries(targets_for(m)), d.cfa_dsts, st.data_bytes,
+                  chunk_bytes=1 << 20) as plan:
+        for src in (cfa.Source.host_direct(h8.ctypes.data, size=st.data_bytes - 1),
+                    cfa.Source.host(h8.ctypes.data, size=100),
+                    cfa.Source.pinned(pinned.data_ptr(), size=st.data_bytes - 2)):
+            with pytest.raises(cfa.CfaError) as e:
+                plan.load_async(src)
+            assert e.value.name == "CFA_ERR_INVAL"
+        with pytest.raises(cfa.CfaError) as e:
+            plan.load_async(cfa.Source.host_direct(h8.ctypes.data + 4))
+        assert e.value.name == "CFA_ERR_ALIGN"
+        plan.load_async(cfa.Source.host_direct(h8.ctypes.data, size=st.data_bytes))
+        plan.wait_layer()
+        ck = plan.checksums()
+    compare(m, d, ck, ref, "direct host source 8 bytes past a 16-byte boundary")
 
 
 @pytest.mark.parametrize("data_align", [8, 4096])
