@@ -457,8 +457,11 @@ cfa_status cfa_safetensors_close(cfa_safetensors *st);
                                  access, such as Grace-based GB300: 2x the pread and copy modes
                                  for a page-cache-resident file).  base = mapping + data_offset,
                                  so data_offset must be a multiple of 8 (a safetensors data
-                                 section is); size_bytes = file size - data_offset.  Same SIGBUS
-                                 caveat as CFA_FILE_MMAP; not combinable with the other flags. */
+                                 section is); size_bytes = file size - data_offset.  The file
+                                 must not shrink or be rewritten while mapped: on the GPU a page
+                                 that cannot be read is a device memory fault that ends the CUDA
+                                 context, not an error code.  Not combinable with the other
+                                 flags. */
 
 /*
  * Fills *out with a CALLBACK source that reads blob byte o from file byte data_offset + o with
