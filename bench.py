@@ -554,6 +554,14 @@ def run_ours(args):
     plan.close()
     total_ms = max_over_ranks(kernel_ms)
     value = whole_job_gbs(ranks, algo_bytes * args.steps, kernel_ms)
+    # context for the roofline: this GPU's own device copy, taken the way the measured peak was
+    # (torch copy_ of 1 Gi bf16 elements, read + write bytes, best of 10)
+    ca = torch.empty(1 << 30, dtype=torch.bfloat16, device="cuda")
+    cb = torch.empty_like(ca)
+    cb.copy_(ca)
+    copy_ms = min(_timed(lambda: cb.copy_(ca), stream) for _ in range(10))
+    same_box_copy_gbs = 2 * ca.numel() * 2 / (copy_ms / 1e3) / 1e9
+    del ca, cb
 
     # ---------------- end to end: pinned host blob -> final layout through the C ABI ---------
     e2e = None
@@ -651,7 +659,9 @@ def run_ours(args):
                      "traffic": recorded_traffic(m.name) if st["n_bulk"] else None,
                      "peak_source": peak_kind,
                      "kernel": kernel_name,
-                     "launch_ms": round(avg_launch_ms, 4)},
+                     "launch_ms": round(avg_launch_ms, 4),
+                     "same_box_copy_gbs": round(same_box_copy_gbs, 1),
+                     "frac_of_same_box_copy": round(achieved / same_box_copy_gbs, 4)},
         "e2e": e2e,
         "cpu_baseline": cpu,
         "gpu_launches": int(launches_per_load * args.steps),
