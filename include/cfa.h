@@ -369,8 +369,8 @@ cfa_status cfa_unpack_chunks_async(cfa_plan *plan, uint32_t chunk_begin, uint32_
  * Unpacks a blob that already sits in device memory into its destinations WITHOUT ALLOCATING
  * ANYTHING -- no cudaMalloc, no cudaFree, no host heap.  The paper has no counterpart: it is for
  * callers that cannot allocate, such as a serving engine whose memory pool already owns the
- * device, code running under CUDA stream capture (where cudaMalloc and cudaFree are not
- * allowed), or a restricted runtime with no allocator.  It is cfa_plan_create +
+ * device, a latency-critical path that cannot afford cudaFree's implicit device-wide
+ * synchronisation, or a restricted runtime with no allocator.  It is cfa_plan_create +
  * cfa_load_async(DEVICE source) + cfa_get_checksums' buffer in one call, with these
  * differences:
  *   - no plan: every entry is validated on its own (dtype, shape, bounds, alignment), but the

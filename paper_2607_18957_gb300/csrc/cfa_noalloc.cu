@@ -4,8 +4,8 @@
  *
  * Who needs it: code that runs where allocating is not allowed or not possible -- inside a
  * serving engine whose memory pool already owns the whole device and forbids side allocations,
- * under CUDA stream capture (cudaMalloc / cudaFree are not capturable), or in a restricted
- * runtime that has no allocator at hand.  cfa_plan_create allocates a device descriptor table,
+ * on a latency-critical path that cannot afford cudaFree's implicit device-wide
+ * synchronisation, or in a restricted runtime that has no allocator at hand.  cfa_plan_create allocates a device descriptor table,
  * a checksum buffer and staging slots; this entry point allocates nothing at all, on the device
  * or on the host.  Its scratch (the work descriptors and a status word) lives in a file-scope
  * device array of fixed size; the host side builds the descriptors in a file-scope host array.
@@ -86,6 +86,14 @@ int dtype_size(int32_t dt)
 
 int log2_es(int es) { return es == 1 ? 0 : es == 2 ? 1 : es == 4 ? 2 : 3; }
 
+/* a * b into *out; false when the product does not fit in 64 bits */
+bool mul_fits(uint64_t a, uint64_t b, uint64_t *out)
+{
+    if (a != 0 && b > UINT64_MAX / a) return false;
+    *out = a * b;
+    return true;
+}
+
 cfa_status fail(cfa_status st, const char *msg, size_t i)
 {
     say("cfa_unpack_noalloc: %s (entry %zu)", msg, i);
@@ -115,28 +123,32 @@ cfa_status place(const cfa_tensor_entry &e, const cfa_dst *dsts, size_t n_dsts,
                  : (e.src_dtype != d.dtype))
         return fail(CFA_ERR_DTYPE, "dtype does not match the destination", i);
     *es_d = es_dst;
-    uint64_t n = 1, d_numel = 1;
+    /* every product is checked: a shape whose size wraps around 64 bits would pass the bounds
+     * checks below with a wrong size */
+    uint64_t n = 1, d_numel = 1, src_len = 0, d_bytes = 0;
     for (int k = 0; k < e.ndim; ++k) {
-        if (e.shape[k] < 0) return fail(CFA_ERR_INVAL, "negative dimension", i);
-        n *= (uint64_t)e.shape[k];
+        if (e.shape[k] < 0 || !mul_fits(n, (uint64_t)e.shape[k], &n))
+            return fail(CFA_ERR_INVAL, "negative or overflowing dimension", i);
     }
     for (int k = 0; k < d.ndim; ++k) {
-        if (d.shape[k] < 0) return fail(CFA_ERR_INVAL, "negative destination dimension", i);
-        d_numel *= (uint64_t)d.shape[k];
+        if (d.shape[k] < 0 || !mul_fits(d_numel, (uint64_t)d.shape[k], &d_numel))
+            return fail(CFA_ERR_INVAL, "negative or overflowing destination dimension", i);
     }
+    if (!mul_fits(d_numel, (uint64_t)es_dst, &d_bytes) || !mul_fits(n, (uint64_t)*es_s, &src_len))
+        return fail(CFA_ERR_INVAL, "tensor or destination too large", i);
     uint64_t row = 1;
     if (d.ndim >= 2) {
         row = (uint64_t)d.shape[d.ndim - 1];
         if (n && (e.ndim == 0 || (uint64_t)e.shape[e.ndim - 1] != row))
             return fail(CFA_ERR_SHAPE, "last dimension differs from the destination row", i);
     }
-    if (e.dst_row_offset < 0) return fail(CFA_ERR_OOB, "negative row offset", i);
-    const uint64_t first = (uint64_t)e.dst_row_offset * row;
-    if (first > d_numel || n > d_numel - first)
+    uint64_t first = 0;
+    if (e.dst_row_offset < 0 || !mul_fits((uint64_t)e.dst_row_offset, row, &first) ||
+        first > d_numel || n > d_numel - first)
         return fail(CFA_ERR_OOB, "rows fall outside the destination", i);
     if (e.blob_offset % (uint64_t)*es_s)
         return fail(CFA_ERR_ALIGN, "blob offset not a multiple of the element size", i);
-    if (e.blob_offset > blob_bytes || n * (uint64_t)*es_s > blob_bytes - e.blob_offset)
+    if (e.blob_offset > blob_bytes || src_len > blob_bytes - e.blob_offset)
         return fail(CFA_ERR_OOB, "reads past the end of the blob", i);
     if (n && ((uintptr_t)d.dev_ptr % (uintptr_t)*es_d || !d.dev_ptr))
         return fail(CFA_ERR_ALIGN, "destination pointer NULL or misaligned", i);

@@ -323,3 +323,57 @@ def test_log_lines_on_request():
     r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
                        timeout=120)
     assert "cfa: " not in r.stderr
+
+
+def _noalloc_status(m, ents=None, blob_ptr=FAKE_BASE, blob_bytes=None):
+    """Calls cfa_unpack_noalloc with fake device pointers; only its validation may run."""
+    import ctypes
+    lib = _lib.load()
+    e = ents if ents is not None else entries_for(m)
+    d = cfa.make_dsts(fake_dsts(m))
+    err = ctypes.create_string_buffer(512)
+    st = lib.cfa_unpack_noalloc(e.arr.ctypes.data, len(e.arr), d.ctypes.data, len(d), blob_ptr,
+                                m.blob_bytes if blob_bytes is None else blob_bytes, None, None,
+                                err, len(err))
+    return _lib.STATUS.get(st, str(st)), err.value.decode()
+
+
+@pytest.mark.skipif(torch.cuda.is_available(),
+                    reason="fake device pointers: run only where no kernel can be launched")
+def test_noalloc_validation_rejects_what_the_planned_path_rejects():
+    # every malformed entry is refused before any CUDA call, with the planned path's status
+    m, blob, _, _ = manifest_case("fused_tiny.txt")
+    cases = [dict(i=0, offset=32), dict(i=0, offset=5), dict(i=0, row=3), dict(i=0, dtype="f16"),
+             dict(i=3, cast=False), dict(i=0, shape=(1, 4)), dict(i=5, row=2),
+             # sizes that wrap around 64 bits must not slip through the bounds checks
+             dict(i=0, shape=(1 << 40, 1 << 40, 2)), dict(i=5, row=(1 << 62) + 1),
+             dict(i=5, shape=(1 << 62,))]
+    for change in cases:
+        i = change.pop("i")
+        mv = _pins._variant(m, i, **change)
+        planned = _plan_status(mv)
+        assert planned != "CFA_OK", change
+        st, msg = _noalloc_status(mv)
+        assert st == planned, (change, st, msg)
+        assert msg.startswith("cfa_unpack_noalloc:"), msg
+
+
+@pytest.mark.skipif(torch.cuda.is_available(),
+                    reason="fake device pointers: run only where no kernel can be launched")
+def test_noalloc_argument_checks():
+    m, _, _, _ = manifest_case("fused_tiny.txt")
+    assert _noalloc_status(m, blob_ptr=FAKE_BASE + 16)[0] == "CFA_ERR_ALIGN"  # blob not 256-aligned
+    assert _noalloc_status(m, blob_ptr=0)[0] == "CFA_ERR_INVAL"               # NULL blob
+    # column slices need the plan's strided pieces
+    mv = _pins._variant(m, 0, stride=3)
+    assert _plan_status(mv) == "CFA_OK"
+    assert _noalloc_status(mv)[0] == "CFA_ERR_INVAL"
+    # more work items than the fixed scratch holds: one per tensor below 8 KiB
+    from workloads import Manifest
+    n = 16385
+    big = Manifest("too_many", [{"name": f"t{k}", "dtype": "bf16", "shape": (4,), "offset": 8 * k,
+                                 "dst": k} for k in range(n)],
+                   [{"name": f"d{k}", "dtype": "bf16", "shape": (4,)} for k in range(n)],
+                   8 * n, "bits", 1)
+    st, msg = _noalloc_status(big)
+    assert st == "CFA_ERR_INVAL" and "16384" in msg

@@ -1,8 +1,8 @@
 """cfa_unpack_noalloc, the entry point that allocates nothing.
 
 It exists for callers that cannot allocate device memory: an engine whose memory pool already
-owns the whole GPU, code running under CUDA stream capture (cudaMalloc/cudaFree are not allowed
-there), or a runtime without an allocator.  Here it is called through the C ABI (ctypes) and its
+owns the whole GPU, a latency-critical path that cannot afford cudaFree's implicit device-wide
+synchronisation, or a runtime without an allocator.  Here it is called through the C ABI (ctypes) and its
 destinations and checksums must equal, bit for bit, those of the planned path (cfa_plan_create
 + cfa_load_async with a device source) -- on two calls in a row, since every call reuses the
 same fixed scratch array.  Collected last on purpose: it runs after every other test, and also
