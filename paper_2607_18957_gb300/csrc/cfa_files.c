@@ -16,6 +16,7 @@
 #include <fcntl.h>
 #include <pthread.h>
 #include <stdarg.h>
+#include <stddef.h>
 #include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
@@ -106,7 +107,35 @@ static int hex4(const char *s, unsigned *v)
     return 1;
 }
 
-/* Reads a string; returns a malloc'd, NUL-terminated UTF-8 copy (NULL on error). */
+/* Length of the well-formed UTF-8 sequence starting at s (at most `left` bytes), 0 if it is
+ * not one: the ranges of the Unicode standard's table of well-formed byte sequences, which
+ * exclude overlong forms, UTF-16 surrogates and code points above U+10FFFF. */
+static int utf8_len(const unsigned char *s, ptrdiff_t left)
+{
+    const unsigned c = s[0];
+    int n;
+    unsigned lo = 0x80, hi = 0xBF; /* range of the second byte */
+    if (c < 0x80) return 1;
+    if (c >= 0xC2 && c <= 0xDF) n = 2;
+    else if (c >= 0xE0 && c <= 0xEF) {
+        n = 3;
+        if (c == 0xE0) lo = 0xA0;
+        if (c == 0xED) hi = 0x9F;
+    } else if (c >= 0xF0 && c <= 0xF4) {
+        n = 4;
+        if (c == 0xF0) lo = 0x90;
+        if (c == 0xF4) hi = 0x8F;
+    } else {
+        return 0;
+    }
+    if (left < n || s[1] < lo || s[1] > hi) return 0;
+    for (int k = 2; k < n; ++k)
+        if (s[k] < 0x80 || s[k] > 0xBF) return 0;
+    return n;
+}
+
+/* Reads a string; returns a malloc'd, NUL-terminated UTF-8 copy (NULL on error, including
+ * control characters and bytes that are not well-formed UTF-8). */
 static char *jstr(jrd *r)
 {
     jws(r);
@@ -119,6 +148,14 @@ static char *jstr(jrd *r)
     char *out = (char *)malloc(n + 1), *o = out;
     if (!out) return NULL;
     while (r->p < r->end && *r->p != '"') {
+        if ((unsigned char)*r->p >= 0x80) {
+            const int len = utf8_len((const unsigned char *)r->p, r->end - r->p);
+            if (!len) goto bad;
+            memcpy(o, r->p, (size_t)len);
+            o += len;
+            r->p += len;
+            continue;
+        }
         char c = *r->p++;
         if ((unsigned char)c < 0x20) goto bad;
         if (c != '\\') {
@@ -177,9 +214,34 @@ static int juint(jrd *r, uint64_t *v)
         x = x * 10 + d;
         r->p++;
     }
-    if (r->p == s) return 0;
+    if (r->p == s || (*s == '0' && r->p - s > 1)) return 0; /* JSON allows no leading zero */
     if (r->p < r->end && (*r->p == '.' || *r->p == 'e' || *r->p == 'E')) return 0;
     *v = x;
+    return 1;
+}
+
+static int jdigits(jrd *r)
+{
+    const char *s = r->p;
+    while (r->p < r->end && *r->p >= '0' && *r->p <= '9') r->p++;
+    return r->p > s;
+}
+
+/* Skips a number of the JSON grammar: -? (0 | [1-9][0-9]*) (. [0-9]+)? ([eE] [+-]? [0-9]+)? */
+static int jnumber(jrd *r)
+{
+    if (r->p < r->end && *r->p == '-') r->p++;
+    if (r->p < r->end && *r->p == '0') r->p++;
+    else if (!jdigits(r)) return 0;
+    if (r->p < r->end && *r->p == '.') {
+        r->p++;
+        if (!jdigits(r)) return 0;
+    }
+    if (r->p < r->end && (*r->p == 'e' || *r->p == 'E')) {
+        r->p++;
+        if (r->p < r->end && (*r->p == '+' || *r->p == '-')) r->p++;
+        if (!jdigits(r)) return 0;
+    }
     return 1;
 }
 
@@ -210,8 +272,7 @@ static int jskip(jrd *r)
             if (ok && !jlit(r, close)) ok = 0;
         }
     } else if (c == '-' || (c >= '0' && c <= '9')) {
-        r->p++;
-        while (r->p < r->end && *r->p && strchr("0123456789.eE+-", *r->p)) r->p++;
+        ok = jnumber(r);
     } else if (r->end - r->p >= 4 && !memcmp(r->p, "true", 4)) {
         r->p += 4;
     } else if (r->end - r->p >= 5 && !memcmp(r->p, "false", 5)) {
@@ -364,12 +425,19 @@ cfa_status cfa_safetensors_parse(const void *header, uint64_t header_len, uint64
                 ok = 0;
                 break;
             }
+            /* the product of the non-zero dimensions must fit in 64 bits, whatever their order */
             uint64_t numel = 1;
+            int zero = 0;
             for (int k = 0; k < t->ndim; ++k) {
                 const uint64_t d = (uint64_t)t->shape[k];
-                if (d && numel > UINT64_MAX / d) { ok = 0; break; }
+                if (!d) {
+                    zero = 1;
+                    continue;
+                }
+                if (numel > UINT64_MAX / d) { ok = 0; break; }
                 numel *= d;
             }
+            if (zero) numel = 0;
             if (!ok || e < b || e > st->data_bytes || (e - b) / (uint64_t)es != numel ||
                 (e - b) % (uint64_t)es) {
                 ferr("tensor %s: data_offsets [%llu, %llu) do not fit its shape and dtype or the "

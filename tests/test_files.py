@@ -4,7 +4,9 @@ tensors, row and column shards), and the pread file source's fill function."""
 import ctypes
 import json
 import os
+import random
 import struct
+import subprocess
 
 import numpy as np
 import pytest
@@ -14,6 +16,8 @@ from paper_2607_18957_gb300 import _lib
 from workloads import dense_config, moe_config
 from workloads.harness import entries_for
 from workloads.stfile import ST_DTYPE, file_tensors, header_bytes, targets_for, write_safetensors
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 ST_NAME = {v: k for k, v in ST_DTYPE.items()}
 ST_NAME.update({"BOOL": "u8", "I8": "u8", "F8_E4M3": "u8", "F8_E5M2": "u8", "U16": "i16",
@@ -170,6 +174,145 @@ def test_malformed_headers_are_rejected(k):
     with pytest.raises(cfa.CfaError) as e:
         cfa.Safetensors.parse(raw, 8 + len(raw) + 16)
     assert e.value.name == "CFA_ERR_INVAL"
+
+
+ST_ES = {"BOOL": 1, "U8": 1, "I8": 1, "F8_E4M3": 1, "F8_E5M2": 1, "I16": 2, "U16": 2, "F16": 2,
+         "BF16": 2, "I32": 4, "U32": 4, "F32": 4, "I64": 8, "U64": 8, "F64": 8}
+
+
+def json_reading(raw, file_bytes):
+    """The tensor list a strict reading of the header by Python's json module gives, or None
+    where the format rejects the header.  The rules: UTF-8 JSON text, no NaN or Infinity; every
+    string a sequence of Unicode scalar values (a lone surrogate escape is rejected); a top-level
+    object whose values other than __metadata__ are objects with a known dtype, a shape of at most
+    8 integers in [0, 2^63) whose non-zero product fits in 64 bits, and data_offsets [b, e] with
+    b <= e <= the data section's size and e - b the shape's byte size.  Repeated names are kept,
+    in order (the parser does not check them)."""
+    def reject_constant(name):
+        raise ValueError(name)
+
+    def scalar_values_only(x):
+        if isinstance(x, str):
+            try:
+                x.encode("utf-8")
+            except UnicodeEncodeError:
+                return False
+            return True
+        if isinstance(x, (list, tuple)):
+            return all(scalar_values_only(y) for y in x)
+        return True
+
+    try:
+        h = json.loads(raw.decode("utf-8"), object_pairs_hook=list,
+                       parse_constant=reject_constant)
+    except ValueError:  # includes UnicodeDecodeError and json.JSONDecodeError
+        return None
+    if not isinstance(h, list) or not scalar_values_only(h):
+        return None
+    data_bytes = file_bytes - 8 - len(raw)
+    out = []
+    for name, v in h:
+        if name == "__metadata__":
+            continue
+        if not isinstance(v, list):
+            return None
+        d = dict(v)
+        if not {"dtype", "shape", "data_offsets"} <= d.keys():
+            return None
+        dt, shape, offs = d["dtype"], d["shape"], d["data_offsets"]
+        if (not isinstance(dt, str) or dt not in ST_ES or not isinstance(shape, list)
+                or len(shape) > 8 or not isinstance(offs, list) or len(offs) != 2):
+            return None
+        if any(type(x) is not int or not 0 <= x < 1 << 63 for x in shape):
+            return None
+        if any(type(x) is not int or not 0 <= x < 1 << 64 for x in offs):
+            return None
+        nz = 1
+        for x in shape:
+            nz *= x or 1
+        if nz >= 1 << 64:
+            return None
+        nbytes = 0 if 0 in shape else ST_ES[dt] * nz
+        b, e = offs
+        if not b <= e <= data_bytes or e - b != nbytes:
+            return None
+        out.append((name, ST_NAME[dt], tuple(shape), b, e - b))
+    return out
+
+
+_FUZZ_TOKENS = [b"{", b"}", b"[", b"]", b",", b":", b'"', b"\\", b"\\u", b"\\u00", b"\\ud800",
+                b"\\udc00", b"\\ud800\\udc00", b"1e999", b"-1", b"-0", b"01", b"1.5", b"2.0", b"1E2",
+                b"18446744073709551615", b"18446744073709551616", b"9223372036854775808",
+                b"99999999999999999999999", b"null", b"true", b"NaN", b"\x00", b"\t", b"\n",
+                b"\xff", b"\xc3\xa9", b"\xe2\x82", b"\xed\xa0\x80", b"\xf4\x90\x80\x80", b"\xc0\xaf",
+                b'"dtype"', b'"shape"', b'"data_offsets"', b'"__metadata__"', b"[[", b"]]"]
+
+
+def mutated_headers(seed, n):
+    """n (header, file size) pairs: valid headers (every dtype, 0-3 dimensions, metadata,
+    non-ASCII names) with up to three random deletions, token insertions, byte changes or
+    truncations each."""
+    rng = random.Random(seed)
+    for _ in range(n):
+        h, off = {}, 0
+        if rng.random() < 0.5:
+            h["__metadata__"] = {"format": "pt", "k": "v\u00e9\"x\\n", "l": [1, 2.5, None, True]}
+        for i in range(rng.randint(0, 5)):
+            dt = rng.choice(sorted(ST_ES))
+            shape = [rng.randint(0, 5) for _ in range(rng.randint(0, 3))]
+            nb = ST_ES[dt] * int(np.prod(shape, dtype=np.int64))
+            h[f"layer.{i}.w\u00e9"] = {"dtype": dt, "shape": shape, "data_offsets": [off, off + nb]}
+            off += nb
+        b = bytearray(json.dumps(h, ensure_ascii=rng.random() < 0.5).encode())
+        for _ in range(rng.randint(0, 3)):
+            r = rng.random()
+            if r < 0.3 and b:
+                i = rng.randrange(len(b))
+                del b[i:i + rng.randint(1, 6)]
+            elif r < 0.7:
+                i = rng.randrange(len(b) + 1)
+                b[i:i] = rng.choice(_FUZZ_TOKENS)
+            elif r < 0.9 and b:
+                b[rng.randrange(len(b))] = rng.randrange(256)
+            else:
+                b = b[:rng.randrange(len(b) + 1)]
+        yield bytes(b), 8 + len(b) + off + rng.choice([0, 0, 0, 1, 1 << 40])
+
+
+@pytest.mark.parametrize("seed", [1, 2])
+def test_mutated_headers_parse_as_python_json_reads_them(seed):
+    accepted = rejected = 0
+    for raw, file_bytes in mutated_headers(seed, 3000):
+        want = json_reading(raw, file_bytes)
+        try:
+            got = [tuple(t) for t in cfa.Safetensors.parse(raw, file_bytes).tensors]
+        except cfa.CfaError as e:
+            assert e.name == "CFA_ERR_INVAL"
+            got = None
+        assert got == want, raw
+        accepted += got is not None
+        rejected += got is None
+    assert accepted > 100 and rejected > 100
+
+
+def test_header_parser_under_address_sanitizer(tmp_path):
+    exe = tmp_path / "st_header_fuzz"
+    csrc = os.path.join(ROOT, "paper_2607_18957_gb300", "csrc")
+    r = subprocess.run(["gcc", "-g", "-O1", "-std=c11", "-fsanitize=address,undefined",
+                        "-fno-sanitize-recover=all", "-I", csrc, "-I", os.path.join(ROOT, "include"),
+                        os.path.join(ROOT, "tests", "st_header_fuzz.c"),
+                        os.path.join(csrc, "cfa_files.c"), "-o", str(exe), "-lpthread"],
+                       capture_output=True, text=True)
+    if r.returncode != 0:
+        pytest.skip("no AddressSanitizer runtime for gcc here: " + r.stderr[-200:])
+    inputs = tmp_path / "headers.bin"
+    with open(inputs, "wb") as f:
+        for raw, file_bytes in mutated_headers(7, 20000):
+            f.write(struct.pack("<IQ", len(raw), file_bytes) + raw)
+        for raw in BAD_HEADERS:
+            f.write(struct.pack("<IQ", len(raw), 8 + len(raw) + 16) + raw)
+    r = subprocess.run([str(exe), str(inputs)], capture_output=True, text=True, timeout=300)
+    assert r.returncode == 0, r.stdout + r.stderr[-2000:]
 
 
 def test_malformed_files_are_rejected(tmp_path):
