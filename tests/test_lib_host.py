@@ -377,3 +377,17 @@ def test_noalloc_argument_checks():
                    8 * n, "bits", 1)
     st, msg = _noalloc_status(big)
     assert st == "CFA_ERR_INVAL" and "16384" in msg
+
+
+def test_plain_c_program_through_the_header(tmp_path):
+    """tests/c_consumer.c: strict C11 against include/cfa.h, linked to libcfa.so; struct sizes
+    agree with the library's, a host-only plan gives hand-computed pieces, errors carry their
+    messages, and a safetensors header parses.  Makes no CUDA call."""
+    import subprocess
+    exe = tmp_path / "c_consumer"
+    pkg = os.path.dirname(_lib.LIB_PATH)
+    subprocess.run(["gcc", "-std=c11", "-pedantic", "-Wall", "-Wextra", "-Werror",
+                    "-I", os.path.join(ROOT, "include"), os.path.join(ROOT, "tests", "c_consumer.c"),
+                    "-L", pkg, "-lcfa", "-Wl,-rpath," + pkg, "-o", str(exe)], check=True)
+    r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert r.returncode == 0 and r.stdout.strip() == "ok", r.stdout + r.stderr

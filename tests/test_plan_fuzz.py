@@ -119,3 +119,85 @@ def test_random_manifest_pieces_reproduce_the_oracle(seed):
             for k in range(int(r)):
                 read[a + k * s * e:a + k * s * e + c * e] = True
         assert int(read.sum()) <= st["staged_bytes"] <= m.blob_bytes
+
+
+def _corrupt(rng, ents, dsts, opts):
+    """One field of one entry or destination, or one option, set to an extreme value."""
+    big = [-1, 0, 1, 3, 1 << 31, (1 << 32) + 1, 1 << 62, (1 << 63) - 1]
+    what = int(rng.integers(0, 14))
+    i = int(rng.integers(0, len(ents))) if len(ents) else 0
+    j = int(rng.integers(0, len(dsts)))
+    pick = lambda vals: vals[int(rng.integers(0, len(vals)))]
+    if what == 0 and len(ents):
+        ents["shape"][i][int(rng.integers(0, 8))] = pick(big)
+    elif what == 1 and len(ents):
+        ents["ndim"][i] = pick([-1, 0, 1, 3, 8, 9])
+    elif what == 2 and len(ents):
+        ents["blob_offset"][i] = pick([1, opts[0] - 1, opts[0], 1 << 40, (1 << 64) - 2])
+    elif what == 3 and len(ents):
+        ents["dst_index"][i] = pick([-1, len(dsts), 1 << 30])
+    elif what == 4 and len(ents):
+        ents["dst_row_offset"][i] = pick(big)
+    elif what == 5 and len(ents):
+        ents["flags"][i] = pick([0, 1, 4, 0xFF, 1 << 31])
+    elif what == 6 and len(ents):
+        ents["src_row_stride"][i] = pick([1, 2, 7, 1 << 20, (1 << 32) - 1])
+    elif what == 7 and len(ents):
+        ents["layer"][i] = pick([-1, 1 << 20, (1 << 31) - 1])
+    elif what == 8 and len(ents):
+        ents["src_dtype"][i] = pick([0, 9, -3, 4])
+    elif what == 9:
+        dsts["dtype"][j] = pick([0, 9, 1, 7])
+    elif what == 10:
+        dsts["ndim"][j] = pick([-1, 0, 1, 3, 9])
+    elif what == 11:
+        dsts["shape"][j][int(rng.integers(0, 2))] = pick(big)
+    elif what == 12:
+        dsts["dev_ptr"][j] = pick([0, 1, int(dsts["dev_ptr"][j]) + 1, int(dsts["dev_ptr"][0])])
+    else:
+        opts[int(rng.integers(0, 4))] = pick([0, 1, 100, 256, 4096, 1 << 20, (1 << 64) - 256])
+
+
+def test_plan_builder_under_address_sanitizer(tmp_path):
+    """The 200 random manifests (several chunk, slab and tiny sizes each) and 1,600 single-field
+    corruptions of them through the plan builder built with AddressSanitizer and UBSan; every
+    accepted plan's pieces and work items are checked to stay inside their chunk, the blob and
+    one destination (tests/plan_fuzz_asan.c)."""
+    import os
+    import struct
+    import subprocess
+
+    from test_lib_host import ROOT
+    exe = tmp_path / "plan_fuzz_asan"
+    csrc = os.path.join(ROOT, "paper_2607_18957_gb300", "csrc")
+    r = subprocess.run(["gcc", "-g", "-O1", "-std=c11", "-fsanitize=address,undefined",
+                        "-fno-sanitize-recover=all", "-I", csrc,
+                        "-I", os.path.join(ROOT, "include"),
+                        os.path.join(ROOT, "tests", "plan_fuzz_asan.c"),
+                        os.path.join(csrc, "cfa_plan.c"), "-o", str(exe)],
+                       capture_output=True, text=True)
+    if r.returncode != 0:
+        pytest.skip("no AddressSanitizer runtime for gcc here: " + r.stderr[-200:])
+    path = tmp_path / "manifests.bin"
+    with open(path, "wb") as f:
+        for seed in range(200):
+            m = random_manifest(seed)
+            rng = np.random.default_rng(10_000 + seed)
+            base_e = entries_for(m).arr.copy()
+            base_e["name"] = 0
+            base_d = cfa.make_dsts(fake_dsts(m))
+            for variant in range(10):
+                ents, dsts = base_e.copy(), base_d.copy()
+                # blob bytes, chunk bytes, slab bytes, tiny bytes
+                opts = [m.blob_bytes, 256 * int(rng.integers(1, 64)),
+                        int(rng.choice([4096, 8192, 65536])), int(rng.choice([0, 64, 8192]))]
+                if variant >= 2:
+                    _corrupt(rng, ents, dsts, opts)
+                flags = 0x1 | 0x8 if variant % 3 else 0x8  # strict coverage on most
+                f.write(struct.pack("<QQQQIIII", len(ents), len(dsts), opts[0] % (1 << 64),
+                                    opts[1] % (1 << 64), opts[2] % (1 << 32),
+                                    opts[3] % (1 << 32), flags, 0))
+                f.write(ents.tobytes())
+                f.write(dsts.tobytes())
+    r = subprocess.run([str(exe), str(path)], capture_output=True, text=True, timeout=600)
+    assert r.returncode == 0, r.stdout + r.stderr[-3000:]
