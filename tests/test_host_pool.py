@@ -3,6 +3,8 @@ once and never after its run returned, over thousands of back-to-back runs."""
 import os
 import subprocess
 
+import pytest
+
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 
@@ -13,3 +15,18 @@ def test_pool_stress(tmp_path):
                     os.path.join(ROOT, "tests", "pool_stress.cpp"), "-o", str(exe)], check=True)
     r = subprocess.run([str(exe), "20000"], capture_output=True, text=True, timeout=120)
     assert r.returncode == 0, r.stdout + r.stderr
+
+
+def test_pool_stress_under_thread_sanitizer(tmp_path):
+    """The same stress run built with ThreadSanitizer: no data race between the caller, the
+    workers and the job they share."""
+    exe = tmp_path / "pool_stress_tsan"
+    r = subprocess.run(["g++", "-O1", "-g", "-std=c++17", "-pthread", "-fsanitize=thread",
+                        "-I", os.path.join(ROOT, "paper_2607_18957_gb300", "csrc"),
+                        os.path.join(ROOT, "tests", "pool_stress.cpp"), "-o", str(exe)],
+                       capture_output=True, text=True)
+    if r.returncode != 0:
+        pytest.skip("no ThreadSanitizer runtime for g++ here: " + r.stderr[-200:])
+    r = subprocess.run([str(exe), "5000"], capture_output=True, text=True, timeout=300,
+                       env={**os.environ, "TSAN_OPTIONS": "halt_on_error=1 exitcode=66"})
+    assert r.returncode == 0, r.stdout + r.stderr[-3000:]
