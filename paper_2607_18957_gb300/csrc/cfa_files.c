@@ -654,16 +654,15 @@ static int direct_fill(file_src *f, uint8_t *d, uint64_t len, uint64_t fo)
 static int file_fill(void *user, uint64_t off, void *dst, uint64_t len)
 {
     file_src *f = (file_src *)user;
-    if (off + len < off || f->data_offset + off < off ||
-        f->data_offset + off + len > f->file_bytes)
-        return 1;
+    const uint64_t fo = f->data_offset + off; /* file offset; every sum checked for wrap-around */
+    if (fo < off || fo + len < fo || fo + len > f->file_bytes) return 1;
     if (!len) return 0;
     if (f->map) {
-        memcpy(dst, f->map + f->data_offset + off, len);
+        memcpy(dst, f->map + fo, len);
         return 0;
     }
-    if (f->direct) return direct_fill(f, (uint8_t *)dst, len, f->data_offset + off);
-    return read_full(f->fd, (uint8_t *)dst, len, f->data_offset + off);
+    if (f->direct) return direct_fill(f, (uint8_t *)dst, len, fo);
+    return read_full(f->fd, (uint8_t *)dst, len, fo);
 }
 
 cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t flags,
@@ -699,7 +698,7 @@ cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t
     pthread_mutex_init(&f->mu, NULL);
     f->data_offset = data_offset;
     f->file_bytes = (uint64_t)sb.st_size;
-    if (in_place && data_offset > f->file_bytes) {
+    if (data_offset > f->file_bytes) {
         ferr("data offset %llu is past the end of %s (%llu bytes)",
              (unsigned long long)data_offset, path, (unsigned long long)f->file_bytes);
         pthread_mutex_destroy(&f->mu);

@@ -490,3 +490,28 @@ def test_in_place_file_source_rules(tmp_path):
     c = _lib.Source()
     c.kind, c.user = _lib.SRC_HOST_DIRECT, 1234
     assert lib.cfa_file_source_close(ctypes.byref(c)) == -1
+
+
+@pytest.mark.parametrize("sanitizer", ["thread", "address,undefined"])
+def test_concurrent_fills_under_sanitizers(tmp_path, sanitizer):
+    """tests/file_fill_stress.c: eight threads fill random ranges of a 24 MiB file at random
+    destination alignments in every read mode, at a block-aligned and an unaligned data offset,
+    with requests past the end and wrapping around 64 bits refused; built with ThreadSanitizer
+    and with AddressSanitizer + UBSan."""
+    exe = tmp_path / "file_fill_stress"
+    csrc = os.path.join(ROOT, "paper_2607_18957_gb300", "csrc")
+    r = subprocess.run(["gcc", "-g", "-O1", "-std=c11", "-pthread", f"-fsanitize={sanitizer}",
+                        "-fno-sanitize-recover=all", "-I", csrc, "-I", os.path.join(ROOT, "include"),
+                        os.path.join(ROOT, "tests", "file_fill_stress.c"),
+                        os.path.join(csrc, "cfa_files.c"), "-o", str(exe)],
+                       capture_output=True, text=True)
+    if r.returncode != 0:
+        pytest.skip(f"no {sanitizer} sanitizer runtime for gcc here: " + r.stderr[-200:])
+    path = tmp_path / "file.bin"
+    path.write_bytes(np.random.default_rng(5).integers(0, 256, (24 << 20) + 777, np.uint8)
+                     .tobytes())
+    for data_offset in (4096, 4104):
+        r = subprocess.run([str(exe), str(path), str(data_offset)], capture_output=True,
+                           text=True, timeout=600,
+                           env={**os.environ, "TSAN_OPTIONS": "halt_on_error=1 exitcode=66"})
+        assert r.returncode == 0, (data_offset, r.stdout + r.stderr[-3000:])
