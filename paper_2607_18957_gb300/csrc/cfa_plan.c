@@ -101,6 +101,73 @@ static int vec_push(vec *v, const void *x)
 }
 
 /* ------------------------------------------------------------------------------------------ */
+/* stable ordering by a 64-bit key                                                              */
+
+/* Reorders the n records of `elem` bytes at `base` by key[i] (the key of record i), stably:
+ * records with equal keys keep their order.  A least-significant-digit radix sort on 11-bit
+ * digits, with only as many passes as the largest key needs, so a few hundred thousand pieces
+ * take a few milliseconds instead of a comparison sort's tens; records already in order are left
+ * alone.  Returns 0, or -1 when out of memory. */
+static int sort_by_key(void *base, size_t n, size_t elem, const uint64_t *key)
+{
+    enum { BITS = 11, RADIX = 1 << BITS };
+    uint64_t maxk = 0;
+    int sorted = 1;
+    for (size_t i = 0; i < n; ++i) {
+        if (key[i] > maxk) maxk = key[i];
+        if (i && key[i] < key[i - 1]) sorted = 0;
+    }
+    if (sorted) return 0;
+    size_t *idx = (size_t *)malloc(n * sizeof(size_t)), *idx2 = (size_t *)malloc(n * sizeof(size_t));
+    uint64_t *k1 = (uint64_t *)malloc(n * sizeof(uint64_t)), *k2 = (uint64_t *)malloc(n * sizeof(uint64_t));
+    size_t *count = (size_t *)malloc((RADIX + 1) * sizeof(size_t));
+    char *tmp = (char *)malloc(n * elem);
+    int rc = -1;
+    if (!idx || !idx2 || !k1 || !k2 || !count || !tmp) goto out;
+    for (size_t i = 0; i < n; ++i) {
+        idx[i] = i;
+        k1[i] = key[i];
+    }
+    for (int shift = 0; shift < 64 && (maxk >> shift); shift += BITS) {
+        memset(count, 0, (RADIX + 1) * sizeof(size_t));
+        for (size_t i = 0; i < n; ++i) count[((k1[i] >> shift) & (RADIX - 1)) + 1]++;
+        for (int d = 0; d < RADIX; ++d) count[d + 1] += count[d];
+        for (size_t i = 0; i < n; ++i) {
+            const size_t to = count[(k1[i] >> shift) & (RADIX - 1)]++;
+            idx2[to] = idx[i];
+            k2[to] = k1[i];
+        }
+        size_t *ti = idx;
+        idx = idx2;
+        idx2 = ti;
+        uint64_t *tk = k1;
+        k1 = k2;
+        k2 = tk;
+    }
+    for (size_t i = 0; i < n; ++i) memcpy(tmp + i * elem, (const char *)base + idx[i] * elem, elem);
+    memcpy(base, tmp, n * elem);
+    rc = 0;
+out:
+    free(idx);
+    free(idx2);
+    free(k1);
+    free(k2);
+    free(count);
+    free(tmp);
+    return rc;
+}
+
+static int bit_width(uint64_t x)
+{
+    int b = 0;
+    while (x) {
+        b++;
+        x >>= 1;
+    }
+    return b;
+}
+
+/* ------------------------------------------------------------------------------------------ */
 
 typedef struct {
     uint64_t n;       /* elements */
@@ -130,21 +197,6 @@ typedef struct {
     uint64_t ptr, len;
     uint32_t idx;
 } dspan;
-
-static int cmp_dspan(const void *a, const void *b)
-{
-    const dspan *x = (const dspan *)a, *y = (const dspan *)b;
-    if (x->ptr != y->ptr) return x->ptr < y->ptr ? -1 : 1;
-    return (x->idx > y->idx) - (x->idx < y->idx);
-}
-
-static int cmp_piece(const void *a, const void *b)
-{
-    const cfa_piece *x = (const cfa_piece *)a, *y = (const cfa_piece *)b;
-    if (x->chunk != y->chunk) return x->chunk < y->chunk ? -1 : 1;
-    if (x->src_offset != y->src_offset) return x->src_offset < y->src_offset ? -1 : 1;
-    return (x->entry > y->entry) - (x->entry < y->entry);
-}
 
 static int mul_overflows(uint64_t a, uint64_t b, uint64_t *out)
 {
@@ -364,7 +416,15 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         ds[j].len = dst_bytes[j];
         ds[j].idx = (uint32_t)j;
     }
-    qsort(ds, n_dsts, sizeof(dspan), cmp_dspan);
+    /* by address; ds[j].idx == j, so the stable order breaks ties by index */
+    {
+        uint64_t *key = (uint64_t *)calloc(n_dsts ? n_dsts : 1, sizeof(uint64_t));
+        if (!key) { st = CFA_ERR_NOMEM; goto done; }
+        for (size_t j = 0; j < n_dsts; ++j) key[j] = ds[j].ptr;
+        const int r = sort_by_key(ds, n_dsts, sizeof(dspan), key);
+        free(key);
+        if (r) { st = CFA_ERR_NOMEM; goto done; }
+    }
     for (size_t j = 1; j < n_dsts; ++j) {
         const dspan *p = &ds[j - 1], *q = &ds[j];
         if (p->len && q->len && q->ptr < p->ptr + p->len) {
@@ -485,7 +545,25 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         spans[n_spans].len = info[i].n * (uint64_t)info[i].es_d;
         n_spans++;
     }
-    qsort(spans, n_spans, sizeof(span), cmp_span);
+    /* by (destination, offset); spans are in entry order, so the stable order breaks ties by
+     * entry.  Both fields go into one key when they fit in 64 bits together. */
+    {
+        uint64_t max_off = 0;
+        for (size_t k = 0; k < n_spans; ++k)
+            if (spans[k].off > max_off) max_off = spans[k].off;
+        const int ob = bit_width(max_off);
+        if (ob + bit_width((uint64_t)n_dsts) <= 64) {
+            uint64_t *key = (uint64_t *)calloc(n_spans ? n_spans : 1, sizeof(uint64_t));
+            if (!key) { st = CFA_ERR_NOMEM; goto done; }
+            for (size_t k = 0; k < n_spans; ++k)
+                key[k] = ob == 64 ? spans[k].off : ((uint64_t)spans[k].dst << ob) | spans[k].off;
+            const int r = sort_by_key(spans, n_spans, sizeof(span), key);
+            free(key);
+            if (r) { st = CFA_ERR_NOMEM; goto done; }
+        } else {
+            qsort(spans, n_spans, sizeof(span), cmp_span);
+        }
+    }
     {
         size_t k = 0;
         for (size_t j = 0; j < n_dsts; ++j) {
@@ -580,7 +658,16 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         }
     }
     const size_t n_pieces = out->n_pieces;
-    qsort(out->pieces, n_pieces, sizeof(cfa_piece), cmp_piece);
+    /* by (chunk, blob offset, entry): a piece's chunk is its blob offset / S and the pieces were
+     * made in entry order, so a stable order by blob offset is that order */
+    {
+        uint64_t *key = (uint64_t *)calloc(n_pieces ? n_pieces : 1, sizeof(uint64_t));
+        if (!key) { st = CFA_ERR_NOMEM; goto done; }
+        for (size_t q = 0; q < n_pieces; ++q) key[q] = out->pieces[q].src_offset;
+        const int r = sort_by_key(out->pieces, n_pieces, sizeof(cfa_piece), key);
+        free(key);
+        if (r) { st = CFA_ERR_NOMEM; goto done; }
+    }
 
     /* 4. work items, ordered by (class, chunk) */
     const uint32_t n_chunks = (uint32_t)n_chunks64;
