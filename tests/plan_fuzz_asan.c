@@ -1,7 +1,8 @@
 /* Replays manifests through the host plan builder (paper_2607_18957_gb300/csrc/cfa_plan.c) built
  * with AddressSanitizer and UBSan, so that an out-of-bounds access, a leak or undefined behaviour
  * aborts the run.  Every accepted plan is checked against its own inputs:
- *   - each piece lies inside its chunk and the blob, and inside its destination;
+ *   - each piece lies inside its chunk and the blob, and inside its destination, and the pieces
+ *     are ordered by (chunk, blob offset, entry);
  *   - each work item reads inside the blob and writes inside exactly one destination;
  *   - each class/chunk range table is monotone and ends at the item count.
  * Input file: records of
@@ -62,6 +63,13 @@ static int check_plan(const cfa_host_plan *hp)
         if (end > blob || (end - 1) / S != p->chunk) return 21;
         const uint64_t base = (uint64_t)(uintptr_t)hp->dsts[p->dst_index].dev_ptr;
         if (owner(base + p->dst_offset, p->n_elems * es_d) != (long)p->dst_index) return 22;
+        if (i) { /* ordered by (chunk, blob offset, entry), as the copy ranges are walked */
+            const cfa_piece *q = p - 1;
+            if (q->chunk > p->chunk ||
+                (q->chunk == p->chunk && (q->src_offset > p->src_offset ||
+                                          (q->src_offset == p->src_offset && q->entry >= p->entry))))
+                return 23;
+        }
     }
     int r;
     if ((r = check_items(hp->slabs, hp->n_slabs, hp->slab_first, hp->n_chunks, blob))) return r;
