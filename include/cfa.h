@@ -439,6 +439,18 @@ cfa_status cfa_safetensors_info(const cfa_safetensors *st, size_t *n_tensors,
 /* Tensor i (header order), 0 <= i < n_tensors. */
 cfa_status cfa_safetensors_tensor(const cfa_safetensors *st, size_t i, cfa_st_tensor *out);
 
+/* Tensors first .. first + count - 1 (header order) into out[0 .. count - 1], in one call (a
+ * header of 10^5 tensors is read in milliseconds instead of one call per tensor).  The names
+ * stay owned by the handle.  CFA_ERR_INVAL if the range is not inside [0, n_tensors). */
+cfa_status cfa_safetensors_tensors(const cfa_safetensors *st, size_t first, size_t count,
+                                   cfa_st_tensor *out);
+
+/* Every tensor name in header order, each followed by a NUL byte, into buf (cap bytes); *bytes
+ * receives the length this takes.  buf = NULL only reports the length.  Names hold no NUL byte
+ * (the parser refuses \u0000).  CFA_ERR_INVAL if cap is smaller than the length. */
+cfa_status cfa_safetensors_names(const cfa_safetensors *st, char *buf, uint64_t cap,
+                                 uint64_t *bytes);
+
 /* Frees the handle (and the names it owns).  Accepts NULL. */
 cfa_status cfa_safetensors_close(cfa_safetensors *st);
 

@@ -13,7 +13,9 @@ memory and streams only, and is imported lazily.
     plan.wait_layer()                        # whole load
     ck = plan.checksums()
 """
+import contextlib
 import ctypes
+import gc
 import itertools
 
 import numpy as np
@@ -59,14 +61,13 @@ def _shape_columns(shapes, n):
         shapes = list(shapes)
     if len(shapes) != n:
         raise ValueError(f"{len(shapes)} shapes for {n} entries")
-    nd = np.fromiter((len(s) for s in shapes), dtype=np.int32, count=n)
+    nd = np.fromiter(map(len, shapes), dtype=np.int32, count=n)
     if n and int(nd.max()) > 8:
         raise ValueError("more than 8 dimensions")
     out = np.zeros((n, 8), dtype=np.int64)
     total = int(nd.sum())
     if total:
-        flat = np.fromiter((int(x) for x in itertools.chain.from_iterable(shapes)),
-                           dtype=np.int64, count=total)
+        flat = np.fromiter(itertools.chain.from_iterable(shapes), dtype=np.int64, count=total)
         rows = np.repeat(np.arange(n), nd)
         starts = np.repeat(np.cumsum(nd) - nd, nd)
         out[rows, np.arange(total) - starts] = flat
@@ -114,16 +115,25 @@ def make_entries(dtype, shape, offset, dst, row=None, cast=None, cksum=None, lay
         e["src_row_stride"] = np.asarray(src_row_stride, dtype=np.uint32)
     keep = None
     if names is not None:
-        blob = b"".join(s.encode() + b"\0" for s in names)
+        enc = [s.encode() for s in names]
+        blob = b"\0".join(enc) + b"\0"
         keep = ctypes.create_string_buffer(blob, len(blob))
-        base = ctypes.addressof(keep)
-        offs = np.zeros(n, dtype=np.uint64)
-        pos = 0
-        for i, s in enumerate(names):
-            offs[i] = base + pos
-            pos += len(s.encode()) + 1
-        e["name"] = offs
+        size = np.fromiter(map(len, enc), dtype=np.uint64, count=n) + np.uint64(1)
+        e["name"] = np.uint64(ctypes.addressof(keep)) + np.cumsum(size, dtype=np.uint64) - size
     return _Entries(e, keep)
+
+
+@contextlib.contextmanager
+def _no_cyclic_gc():
+    """Pauses the cyclic garbage collector while a large table of tuples is built (they form no
+    cycles; with 10^5 of them the collector's repeated scans took half the time)."""
+    was = gc.isenabled()
+    gc.disable()
+    try:
+        yield
+    finally:
+        if was:
+            gc.enable()
 
 
 class _Entries:
@@ -137,6 +147,11 @@ class _Entries:
 
 def _dtype_codes(dtypes):
     """dtype names or CFA_DTYPE_* codes -> int32 array of codes."""
+    if isinstance(dtypes, np.ndarray) and dtypes.dtype.kind in "iu":
+        return dtypes.astype(np.int32)
+    if all(type(x) is str for x in dtypes):  # names: one lookup per distinct name
+        names, inverse = np.unique(np.asarray(dtypes, dtype=str), return_inverse=True)
+        return np.array([DTYPE[k] for k in names.tolist()], dtype=np.int32)[inverse.ravel()]
     memo = {}
 
     def code(x):
@@ -273,14 +288,22 @@ class Safetensors:
         try:
             _check(lib.cfa_safetensors_info(handle, ctypes.byref(n), ctypes.byref(off),
                                             ctypes.byref(nb)))
-            names = {v: k for k, v in DTYPE.items()}
-            t = _lib.StTensor()
-            out = []
-            for i in range(n.value):
-                _check(lib.cfa_safetensors_tensor(handle, i, ctypes.byref(t)))
-                out.append(StTensor((t.name.decode("utf-8"), names[t.dtype],
-                                     tuple(int(t.shape[k]) for k in range(t.ndim)),
-                                     int(t.blob_offset), int(t.nbytes))))
+            # the whole tensor table in one call; names are read before the handle is closed
+            rec = np.zeros(n.value, dtype=_lib.ST_TENSOR_DTYPE)
+            _check(lib.cfa_safetensors_tensors(handle, 0, n.value,
+                                               rec.ctypes.data if n.value else None))
+            nbytes = ctypes.c_uint64()
+            _check(lib.cfa_safetensors_names(handle, None, 0, ctypes.byref(nbytes)))
+            buf = ctypes.create_string_buffer(max(nbytes.value, 1))
+            _check(lib.cfa_safetensors_names(handle, buf, nbytes.value, ctypes.byref(nbytes)))
+            names = buf.raw[:nbytes.value].decode("utf-8").split("\0")[:n.value]
+            dt_name = {v: k for k, v in DTYPE.items()}
+            with _no_cyclic_gc():
+                out = [StTensor((nm, dt_name[c], tuple(sh[:k]), o, b))
+                       for nm, c, sh, k, o, b in zip(names, rec["dtype"].tolist(),
+                                                     rec["shape"].tolist(), rec["ndim"].tolist(),
+                                                     rec["blob_offset"].tolist(),
+                                                     rec["nbytes"].tolist())]
         finally:
             lib.cfa_safetensors_close(handle)
         self.tensors = out
@@ -311,46 +334,52 @@ class Safetensors:
         range of its last dimension, read with a source row stride: a tensor-parallel column
         shard).  With whole_file the blob is the whole file (offsets shifted by data_offset), so
         that a mapping of the file from its first byte can serve as the source."""
-        cols = {k: [] for k in ("dtype", "shape", "offset", "dst", "row", "layer", "cast",
-                                 "cksum", "names", "src_row_stride")}
+        n = len(targets)
+        dtype, shape, names = [None] * n, [None] * n, [None] * n
+        offset, dst, row, layer = [0] * n, [0] * n, [0] * n, [0] * n
+        cast, cksum, stride = [False] * n, [True] * n, [0] * n
         shift = self.data_offset if whole_file else 0
-        by_name = {t.name: t for t in self.tensors}
-        for name, v in targets.items():
-            if name not in by_name:
+        by_name = {t[0]: t for t in self.tensors}
+        size = _lib.DTYPE_SIZE
+        for i, (name, v) in enumerate(targets.items()):
+            t = by_name.get(name)
+            if t is None:
                 raise KeyError(f"the file holds no tensor named {name!r}")
-            t = by_name[name]
-            if not isinstance(v, dict):
-                v = dict(zip(("dst", "row", "layer"), v))
-            es = _lib.DTYPE_SIZE[t.dtype]
-            shape, off, stride = t.shape, t.offset + shift, 0
+            tname, tdt, tshape, toff = t[0], t[1], t[2], t[3]
+            dtype[i], shape[i], names[i], offset[i] = tdt, tshape, tname, toff + shift
+            if not isinstance(v, dict):  # (dst, row) or (dst, row, layer)
+                dst[i] = v[0]
+                if len(v) > 1:
+                    row[i] = v[1]
+                if len(v) > 2:
+                    layer[i] = v[2]
+                continue
+            dst[i] = v["dst"]
+            row[i] = v.get("row", 0)
+            layer[i] = v.get("layer", 0)
+            cast[i] = bool(v.get("cast", False))
+            cksum[i] = bool(v.get("cksum", True))
             if "rows" in v and "cols" in v:
-                raise ValueError(f"{t.name}: give rows or cols, not both")
+                raise ValueError(f"{tname}: give rows or cols, not both")
+            es = size[tdt]
             if "rows" in v:
                 r0, r1 = v["rows"]
-                if not (len(shape) >= 1 and 0 <= r0 <= r1 <= shape[0]):
-                    raise ValueError(f"{t.name}: rows {r0}:{r1} outside shape {shape}")
-                per_row = int(np.prod(shape[1:], dtype=np.int64))
-                off += r0 * per_row * es
-                shape = (r1 - r0,) + tuple(shape[1:])
+                if not (len(tshape) >= 1 and 0 <= r0 <= r1 <= tshape[0]):
+                    raise ValueError(f"{tname}: rows {r0}:{r1} outside shape {tshape}")
+                per_row = int(np.prod(tshape[1:], dtype=np.int64))
+                offset[i] += r0 * per_row * es
+                shape[i] = (r1 - r0,) + tuple(tshape[1:])
             elif "cols" in v:
                 c0, c1 = v["cols"]
-                if not (len(shape) >= 1 and 0 <= c0 <= c1 <= shape[-1]):
-                    raise ValueError(f"{t.name}: cols {c0}:{c1} outside shape {shape}")
-                off += c0 * es
-                if int(np.prod(shape[:-1], dtype=np.int64)) > 1:
-                    stride = shape[-1]
-                shape = tuple(shape[:-1]) + (c1 - c0,)
-            cols["dtype"].append(t.dtype)
-            cols["shape"].append(shape)
-            cols["offset"].append(off)
-            cols["dst"].append(v["dst"])
-            cols["row"].append(v.get("row", 0))
-            cols["layer"].append(v.get("layer", 0))
-            cols["cast"].append(bool(v.get("cast", False)))
-            cols["cksum"].append(bool(v.get("cksum", True)))
-            cols["names"].append(t.name)
-            cols["src_row_stride"].append(stride)
-        return make_entries(**cols)
+                if not (len(tshape) >= 1 and 0 <= c0 <= c1 <= tshape[-1]):
+                    raise ValueError(f"{tname}: cols {c0}:{c1} outside shape {tshape}")
+                offset[i] += c0 * es
+                if int(np.prod(tshape[:-1], dtype=np.int64)) > 1:
+                    stride[i] = tshape[-1]
+                shape[i] = tuple(tshape[:-1]) + (c1 - c0,)
+        return make_entries(dtype=dtype, shape=shape, offset=offset, dst=dst, row=row,
+                            cast=cast, cksum=cksum, layer=layer, names=names,
+                            src_row_stride=stride)
 
 
 class Plan:

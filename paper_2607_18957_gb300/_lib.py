@@ -73,6 +73,12 @@ class StTensor(ctypes.Structure):
                 ("nbytes", ctypes.c_uint64)]
 
 
+# cfa_st_tensor as a numpy record (bulk reads of a header's tensor table)
+ST_TENSOR_DTYPE = np.dtype([("name", "<u8"), ("dtype", "<i4"), ("ndim", "<i4"),
+                            ("shape", "<i8", (8,)), ("blob_offset", "<u8"), ("nbytes", "<u8")])
+
+assert ST_TENSOR_DTYPE.itemsize == ctypes.sizeof(StTensor)
+
 PIECE_DTYPE = np.dtype([("chunk", "<u4"), ("entry", "<u4"), ("src_offset", "<u8"),
                         ("dst_index", "<u4"), ("conv", "<u4"), ("dst_offset", "<u8"),
                         ("n_elems", "<u8"), ("rows", "<u4"), ("src_row_stride", "<u4")])
@@ -101,6 +107,8 @@ SIGNATURES = {
     "cfa_safetensors_parse": (ctypes.c_int, [_P, _U64, _U64, _P]),
     "cfa_safetensors_info": (ctypes.c_int, [_P, _P, _P, _P]),
     "cfa_safetensors_tensor": (ctypes.c_int, [_P, _SZ, _P]),
+    "cfa_safetensors_tensors": (ctypes.c_int, [_P, _SZ, _SZ, _P]),
+    "cfa_safetensors_names": (ctypes.c_int, [_P, _P, _U64, _P]),
     "cfa_safetensors_close": (ctypes.c_int, [_P]),
     "cfa_file_source_open": (ctypes.c_int, [ctypes.c_char_p, _U64, ctypes.c_uint32, _P]),
     "cfa_file_source_close": (ctypes.c_int, [_P]),
@@ -135,7 +143,7 @@ def _check_layouts(lib):
     want = {"cfa_tensor_entry": ENTRY_DTYPE.itemsize, "cfa_dst": DST_DTYPE.itemsize,
             "cfa_plan_opts": ctypes.sizeof(PlanOpts), "cfa_source": ctypes.sizeof(Source),
             "cfa_stats": ctypes.sizeof(Stats), "cfa_piece": ctypes.sizeof(Piece),
-            "cfa_st_tensor": ctypes.sizeof(StTensor),
+            "cfa_st_tensor": ST_TENSOR_DTYPE.itemsize,
             "cfa_chunk_times": 16}
     for name, size in want.items():
         got = lib.cfa_abi_sizeof(name.encode())

@@ -184,8 +184,8 @@ static char *jstr(jrd *r)
                     goto bad;
                 r->p += 6;
                 cp = 0x10000 + ((cp - 0xD800) << 10) + (lo - 0xDC00);
-            } else if (cp >= 0xDC00 && cp < 0xE000) {
-                goto bad;
+            } else if ((cp >= 0xDC00 && cp < 0xE000) || cp == 0) {
+                goto bad; /* a lone low surrogate, or U+0000, which a C string cannot hold */
             }
             put_utf8(&o, cp);
             break;
@@ -524,6 +524,32 @@ cfa_status cfa_safetensors_tensor(const cfa_safetensors *st, size_t i, cfa_st_te
 {
     if (!st || !out || i >= st->n) return CFA_ERR_INVAL;
     *out = st->t[i];
+    return CFA_OK;
+}
+
+cfa_status cfa_safetensors_names(const cfa_safetensors *st, char *buf, uint64_t cap,
+                                 uint64_t *bytes)
+{
+    if (!st || !bytes || (cap && !buf)) return CFA_ERR_INVAL;
+    uint64_t need = 0;
+    for (size_t i = 0; i < st->n; ++i) need += strlen(st->t[i].name) + 1;
+    *bytes = need;
+    if (!buf) return CFA_OK;
+    if (cap < need) return CFA_ERR_INVAL;
+    char *o = buf;
+    for (size_t i = 0; i < st->n; ++i) {
+        const size_t k = strlen(st->t[i].name) + 1;
+        memcpy(o, st->t[i].name, k);
+        o += k;
+    }
+    return CFA_OK;
+}
+
+cfa_status cfa_safetensors_tensors(const cfa_safetensors *st, size_t first, size_t count,
+                                   cfa_st_tensor *out)
+{
+    if (!st || (count && !out) || first > st->n || count > st->n - first) return CFA_ERR_INVAL;
+    if (count) memcpy(out, st->t + first, count * sizeof *out);
     return CFA_OK;
 }
 

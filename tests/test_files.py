@@ -165,6 +165,7 @@ BAD_HEADERS = [
     b'{"a": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]}',
     b'{"__metadata__": {"x": 1\x002}}',
     b'{"a\x00": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]}}',
+    b'{"a\\u0000b": {"dtype": "F32", "shape": [2], "data_offsets": [0, 8]}}',
 ]
 
 
@@ -183,7 +184,8 @@ ST_ES = {"BOOL": 1, "U8": 1, "I8": 1, "F8_E4M3": 1, "F8_E5M2": 1, "I16": 2, "U16
 def json_reading(raw, file_bytes):
     """The tensor list a strict reading of the header by Python's json module gives, or None
     where the format rejects the header.  The rules: UTF-8 JSON text, no NaN or Infinity; every
-    string a sequence of Unicode scalar values (a lone surrogate escape is rejected); a top-level
+    string a sequence of Unicode scalar values other than U+0000 (a lone surrogate escape or a
+    \\u0000 is rejected); a top-level
     object whose values other than __metadata__ are objects with a known dtype, a shape of at most
     8 integers in [0, 2^63) whose non-zero product fits in 64 bits, and data_offsets [b, e] with
     b <= e <= the data section's size and e - b the shape's byte size.  Repeated names are kept,
@@ -197,7 +199,7 @@ def json_reading(raw, file_bytes):
                 x.encode("utf-8")
             except UnicodeEncodeError:
                 return False
-            return True
+            return "\x00" not in x  # a C string cannot hold U+0000
         if isinstance(x, (list, tuple)):
             return all(scalar_values_only(y) for y in x)
         return True
@@ -241,7 +243,8 @@ def json_reading(raw, file_bytes):
 
 
 _FUZZ_TOKENS = [b"{", b"}", b"[", b"]", b",", b":", b'"', b"\\", b"\\u", b"\\u00", b"\\ud800",
-                b"\\udc00", b"\\ud800\\udc00", b"1e999", b"-1", b"-0", b"01", b"1.5", b"2.0", b"1E2",
+                b"\\udc00", b"\\ud800\\udc00", b"\\u0000", b"1e999", b"-1", b"-0", b"01", b"1.5",
+                b"2.0", b"1E2",
                 b"18446744073709551615", b"18446744073709551616", b"9223372036854775808",
                 b"99999999999999999999999", b"null", b"true", b"NaN", b"\x00", b"\t", b"\n",
                 b"\xff", b"\xc3\xa9", b"\xe2\x82", b"\xed\xa0\x80", b"\xf4\x90\x80\x80", b"\xc0\xaf",
