@@ -107,6 +107,19 @@ int main(void)
     CHECK(53, cfa_safetensors_tensor(st, 0, &t) == CFA_OK);
     CHECK(54, !strcmp(t.name, "w") && t.dtype == CFA_DTYPE_BF16 && t.ndim == 2 &&
                   t.shape[0] == 2 && t.shape[1] == 3 && t.blob_offset == 0 && t.nbytes == 12);
+    cfa_st_tensor all[2];
+    CHECK(57, cfa_safetensors_tensors(st, 0, 1, all) == CFA_OK &&
+                  !memcmp(&all[0], &t, sizeof t));
+    CHECK(58, cfa_safetensors_tensors(st, 0, 2, all) == CFA_ERR_INVAL &&
+                  cfa_safetensors_tensors(st, 2, 0, all) == CFA_ERR_INVAL &&
+                  cfa_safetensors_tensors(st, 1, 0, NULL) == CFA_OK);
+    uint64_t name_bytes = 0;
+    char names[4] = {'x', 'x', 'x', 'x'};
+    CHECK(59, cfa_safetensors_names(st, NULL, 0, &name_bytes) == CFA_OK && name_bytes == 2);
+    CHECK(60, cfa_safetensors_names(st, names, 1, &name_bytes) == CFA_ERR_INVAL &&
+                  names[0] == 'x');
+    CHECK(61, cfa_safetensors_names(st, names, 4, &name_bytes) == CFA_OK &&
+                  !memcmp(names, "w\0xx", 4));
     CHECK(55, cfa_safetensors_close(st) == CFA_OK);
     CHECK(56, cfa_safetensors_parse(hdr, n_hdr, 8 + n_hdr + 11, &st) == CFA_ERR_INVAL);
     printf("ok\n");
