@@ -17,6 +17,8 @@ from workloads import dense_config, moe_config
 from workloads.harness import entries_for
 from workloads.stfile import ST_DTYPE, file_tensors, header_bytes, targets_for, write_safetensors
 
+from test_host_pool import sanitizer_could_not_start
+
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 ST_NAME = {v: k for k, v in ST_DTYPE.items()}
@@ -517,4 +519,6 @@ def test_concurrent_fills_under_sanitizers(tmp_path, sanitizer):
         r = subprocess.run([str(exe), str(path), str(data_offset)], capture_output=True,
                            text=True, timeout=600,
                            env={**os.environ, "TSAN_OPTIONS": "halt_on_error=1 exitcode=66"})
+        if r.returncode != 0 and sanitizer_could_not_start(r.stderr):
+            pytest.skip(f"the {sanitizer} sanitizer runtime cannot start here: " + r.stderr[:200])
         assert r.returncode == 0, (data_offset, r.stdout + r.stderr[-3000:])
