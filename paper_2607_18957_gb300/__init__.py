@@ -149,7 +149,7 @@ def _dtype_codes(dtypes):
     """dtype names or CFA_DTYPE_* codes -> int32 array of codes."""
     if isinstance(dtypes, np.ndarray) and dtypes.dtype.kind in "iu":
         return dtypes.astype(np.int32)
-    if all(type(x) is str for x in dtypes):  # names: one lookup per distinct name
+    if all(isinstance(x, str) for x in dtypes):  # names: one lookup per distinct name
         names, inverse = np.unique(np.asarray(dtypes, dtype=str), return_inverse=True)
         return np.array([DTYPE[k] for k in names.tolist()], dtype=np.int32)[inverse.ravel()]
     memo = {}
