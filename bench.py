@@ -165,6 +165,13 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------------------------
+def attribution_sizes(source_bytes, threads):
+    """Bytes of the pageable source copied to the device (1 GiB) and bytes per thread of the
+    host memcpy (4 GiB split evenly), both capped by the source for a smaller checkpoint."""
+    gib = 1 << 30
+    return min(gib, source_bytes), min(4 * gib, source_bytes) // max(1, threads)
+
+
 def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
     """Where end-to-end time goes: (CFA_OPT_TIMING) per-layer readiness of one pinned load, the
     pinned blob read in place by the kernels (no copy engine), the host link for pinned and
@@ -222,15 +229,12 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
     raw = np.empty(m.source_bytes() + 256, dtype=np.uint8)
     pageable = raw[(-raw.ctypes.data) % 256:][:m.source_bytes()]  # 256-byte aligned view
     pageable[:] = host.numpy()                                   # the same bytes, pageable
-    # 1 GiB of it to the device, and 4 GiB of it through host memcpy (less for a smaller
-    # checkpoint: its whole source, split evenly among the threads)
-    n_h2d = min(gib, pageable.size)
+    n_h2d, part = attribution_sizes(pageable.size, threads)
     dtmp = torch.empty(n_h2d, dtype=torch.uint8, device="cuda")
     src_t = torch.from_numpy(pageable[:n_h2d])
     best = min(_timed(lambda: dtmp.copy_(src_t), stream) for _ in range(5))
     out["h2d_pageable_gbs"] = round(n_h2d / best / 1e6, 2)
     del dtmp
-    part = min(4 * gib, pageable.size) // threads
     dst = np.empty(part * threads, dtype=np.uint8)
 
     def cp(k):

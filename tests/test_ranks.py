@@ -107,3 +107,16 @@ def test_bench_labels_and_traffic_record(monkeypatch):
     monkeypatch.setattr(bench, "kernel_source_hash", lambda: "0" * 64)
     assert bench.recorded_traffic("llama3_8b_bf16") is None
     assert bench.recorded_traffic("no_such_workload") is None
+
+
+def test_attribution_sizes_fit_any_checkpoint():
+    """The pageable H2D and host memcpy measurements never slice past a checkpoint smaller than
+    their 1 and 4 GiB buffers, and split the memcpy evenly among the threads."""
+    import bench
+    gib = 1 << 30
+    for size, threads in [(16_060_000_000, 16), (16_060_000_000, 12), (1_396_744_192, 16),
+                          (125 << 20, 72), (100, 16), (7, 16), (0, 4)]:
+        n_h2d, part = bench.attribution_sizes(size, threads)
+        assert n_h2d == min(gib, size)
+        assert part * threads <= min(4 * gib, size)
+        assert min(4 * gib, size) - part * threads < threads
