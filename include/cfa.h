@@ -64,6 +64,11 @@ typedef int cfa_status;
 #define CFA_ERR_ALIGN    (-11) /* an offset, pointer or size breaks an alignment rule */
 #define CFA_ERR_DEVICE   (-12) /* the unpack kernel's own descriptor check failed */
 #define CFA_ERR_SHAPE    (-13) /* an entry's last dimension differs from its destination's row */
+#define CFA_ERR_SUSPECT  (-14) /* a TMA kernel's wait ran out and so did the wait for its own
+                                  loads in flight: a bulk load may have outlived its CTA, so the
+                                  CUDA context (and the destinations) must be treated as suspect;
+                                  destroy the plan and reset the context before further work */
+#define CFA_ERR_GATHER   (-15) /* the gather callback of a segmented load reported an error */
 
 /* Element types.  Only the element size matters for plain copies; 1-byte types cover int8,
  * uint8 and the fp8 formats. */
@@ -163,6 +168,25 @@ typedef struct cfa_dst {
                                          the column-slice kernel reads them in place from the
                                          pinned memory over the host link, beside the copy ring */
 
+/*
+ * Gather step of a segmented (multi-path) load: section 4.2, "Optimization of Distributed
+ * Loading".  With W ranks cooperating, every chunk is cut into W equal segments of
+ * segment_bytes = chunk_bytes / W; this rank has copied its own segment into
+ * chunk_dev + rank * segment_bytes, and the callback must enqueue on `stream` the collective
+ * that fills the whole device slot chunk_dev[0, W * segment_bytes) with every rank's segment
+ * (an AllGather with send buffer chunk_dev + rank * segment_bytes and receive buffer chunk_dev,
+ * in place).  Once that work completes on `stream` the chunk is Gathered and its unpack runs.
+ * Bytes of segments past the end of the blob are never read, whatever they hold.
+ *
+ * It is called on the thread that calls cfa_load_async, once per chunk, for chunks 0, 1, 2 ...
+ * in order and for every chunk of the blob (so every rank issues the same sequence of
+ * collectives); it must only enqueue work and return (not wait for the GPU), and it returns 0,
+ * or non-zero on failure (the load then stops enqueueing and reports CFA_ERR_GATHER).  Every
+ * rank's plan must have the same blob_bytes, chunk_bytes and seg_world.
+ */
+typedef int (*cfa_gather_fn)(void *user, void *chunk_dev, uint64_t segment_bytes, int32_t world,
+                             int32_t rank, uint32_t chunk, cfa_stream stream);
+
 typedef struct cfa_plan_opts {
     uint64_t chunk_bytes;     /* chunk length S, a multiple of 256; default 512 MiB */
     int32_t host_slots;       /* pinned host staging slots of S bytes, allocated by the first HOST
@@ -180,6 +204,19 @@ typedef struct cfa_plan_opts {
     uint32_t reserved;        /* must be 0 */
     void *workspace;          /* optional device memory for the staging slots (NULL = plan allocates) */
     uint64_t workspace_bytes; /* must be >= dev_slots * chunk_bytes when workspace is given */
+    /* Segmented (multi-path) loading, section 4.2 "Optimization of Distributed Loading":
+     * seg_world > 1 ranks load every chunk together, each copying only its segment (one
+     * seg_world-th of the chunk) from its own source into its own device slot, and `gather`
+     * (above) assembles the chunk in every rank's slot before the unpack.  chunk_bytes must be
+     * a multiple of 256 * seg_world; the device slots are then chunk_bytes long even for a blob
+     * shorter than one chunk.  Loads of such a plan take HOST, PINNED and CALLBACK sources,
+     * never skip a chunk, and stage the rank's whole segments (cfa_stats.staged_bytes), not
+     * only the byte ranges its own pieces read: the other ranks may need any of them.
+     * Default seg_world = 1 (off), seg_rank = 0, gather = NULL. */
+    int32_t seg_world;
+    int32_t seg_rank;         /* this rank, 0 <= seg_rank < seg_world */
+    cfa_gather_fn gather;     /* required when seg_world > 1 */
+    void *gather_user;        /* passed to gather */
 } cfa_plan_opts;
 
 /* Fills *opts with the defaults listed above. */
@@ -300,9 +337,16 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
  * cfa_wait_layer.  Loads on one plan run in the order they were enqueued; the checksums and
  * layer events always refer to the most recently enqueued load.
  *
+ * With seg_world > 1 (segmented plans) each chunk's H2D copy moves only this rank's segment,
+ * then opts.gather assembles the chunk in the device slot on a stream of the plan (the chunk's
+ * Gathered state), and the unpack waits for that instead of the copy.
+ *
  * Errors: CFA_ERR_INVAL (bad source, host-only plan, or a staging kind the plan has no slots
- * for), CFA_ERR_ALIGN, CFA_ERR_CUDA.  Failures that happen later (the callback, a CUDA error)
- * are latched and returned by cfa_wait_layer / cfa_get_checksums for that load.
+ * for; DEVICE and HOST_DIRECT sources on a segmented plan), CFA_ERR_ALIGN, CFA_ERR_CUDA,
+ * CFA_ERR_GATHER (the gather callback failed: the chunks before it were enqueued, the rest of
+ * the load was not; the load's events are still recorded, so waits end, and they report
+ * CFA_ERR_GATHER).  Failures that happen later (the fill callback, a CUDA error) are latched
+ * and returned by cfa_wait_layer / cfa_get_checksums for that load.
  */
 cfa_status cfa_load_async(cfa_plan *plan, const cfa_source *src, cfa_stream stream);
 
@@ -313,7 +357,8 @@ cfa_status cfa_load_async(cfa_plan *plan, const cfa_source *src, cfa_stream stre
  *   consumer == NULL: blocks the host, polling without spinning on the GPU, until the group is
  *                     ready or timeout_ns (< 0: no limit) has passed; then CFA_ERR_TIMEOUT.
  * Errors: CFA_ERR_INVAL (unknown layer, no load yet), CFA_ERR_TIMEOUT, CFA_ERR_SOURCE,
- * CFA_ERR_CUDA, CFA_ERR_DEVICE.
+ * CFA_ERR_GATHER, CFA_ERR_CUDA, CFA_ERR_DEVICE (status word 1 or 2: a descriptor rejected by
+ * the kernel, or a TMA wait that ran out and ended cleanly), CFA_ERR_SUSPECT (status word 3).
  */
 cfa_status cfa_wait_layer(cfa_plan *plan, int32_t layer, cfa_stream consumer, int64_t timeout_ns);
 
@@ -384,15 +429,26 @@ cfa_status cfa_unpack_chunks_async(cfa_plan *plan, uint32_t chunk_begin, uint32_
  *   - all calls on a device share that array: calls serialise on the host, but calls whose GPU
  *     work may overlap (different streams, no ordering between them) race on it;
  *   - the first call on a device does a one-time set-up (it looks up the array's device address
- *     and the kernels' occupancy); make it before any stream capture.
+ *     and the kernels' occupancy); make it before any stream capture.  That address belongs to
+ *     the device's context: do not call this again in a process after cudaDeviceReset;
+ *   - the call blocks the host: the descriptors go up as a copy from pageable host memory,
+ *     which CUDA completes before returning, and which first waits for the work already
+ *     queued on `stream`.  The unpack kernels are enqueued behind it and run after the call
+ *     returns.
  *
  *   entries, n_entries, dsts, n_dsts   as for cfa_plan_create (host arrays, read during the call)
  *   blob_dev, blob_bytes   the blob in device memory (256-byte aligned); must stay valid and
  *                          unchanged until the unpack has run on `stream`
  *   cksum_dev              device array of n_entries uint64 receiving the checksums
  *                          (cleared by the call), or NULL for none
- *   stream                 all GPU work is enqueued here; the call returns without waiting, after
- *                          the descriptors have been handed to the driver
+ *   status_dev             optional device int (4-byte aligned) receiving the kernels' own
+ *                          status word: the call sets it to 0 on `stream`, and a kernel that
+ *                          rejects a work item (its source outside the blob, a misaligned
+ *                          address, a wrong work class) sets it to 1 and leaves that item's
+ *                          bytes unwritten.  The host validation above makes this unreachable
+ *                          for any accepted manifest; read it once `stream` has run the unpack
+ *                          to confirm.  NULL: the status goes to the scratch array's own word
+ *   stream                 all GPU work is enqueued here
  *   err, err_len           optional buffer for a message on failure (NULL for none)
  * Errors: CFA_ERR_INVAL (NULL argument, bad entry, too many work items), CFA_ERR_DTYPE,
  * CFA_ERR_SHAPE, CFA_ERR_OOB, CFA_ERR_ALIGN, CFA_ERR_CUDA.
@@ -400,8 +456,8 @@ cfa_status cfa_unpack_chunks_async(cfa_plan *plan, uint32_t chunk_begin, uint32_
 #define CFA_NOALLOC_MAX_ITEMS 16384
 cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t n_entries,
                               const cfa_dst *dsts, size_t n_dsts, const void *blob_dev,
-                              uint64_t blob_bytes, uint64_t *cksum_dev, cfa_stream stream,
-                              char *err, size_t err_len);
+                              uint64_t blob_bytes, uint64_t *cksum_dev, int *status_dev,
+                              cfa_stream stream, char *err, size_t err_len);
 
 /* ---- checkpoint files (the InDisk end of section 4.2's chunk automaton) ------------------- */
 
@@ -492,6 +548,18 @@ cfa_status cfa_safetensors_close(cfa_safetensors *st);
 cfa_status cfa_file_source_open(const char *path, uint64_t data_offset, uint32_t flags,
                                 cfa_source *out);
 cfa_status cfa_file_source_close(cfa_source *src);
+
+/*
+ * Where rank `rank` of `world` finds its segment of chunk `chunk` in a segmented load (see
+ * cfa_plan_opts.seg_world): *blob_offset receives chunk * chunk_bytes + rank * segment_bytes
+ * and *bytes the part of [*blob_offset, *blob_offset + segment_bytes) inside the blob (0 for a
+ * segment wholly past its end), with segment_bytes = chunk_bytes / world.  Host-only, no CUDA
+ * call.  Errors: CFA_ERR_INVAL (NULL output, world < 1, rank outside [0, world), chunk_bytes not
+ * a positive multiple of 256 * world, chunk past the end of the blob).
+ */
+cfa_status cfa_segment_range(uint64_t blob_bytes, uint64_t chunk_bytes, int32_t world,
+                             int32_t rank, uint32_t chunk, uint64_t *blob_offset,
+                             uint64_t *bytes);
 
 /* Zeroes the plan's checksum buffer on `stream`. */
 cfa_status cfa_reset_checksums(cfa_plan *plan, cfa_stream stream);

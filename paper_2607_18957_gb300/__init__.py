@@ -24,7 +24,7 @@ from . import _lib
 from ._lib import ALL, DTYPE, ENTRY_DTYPE, DST_DTYPE, PIECE_DTYPE  # noqa: F401
 
 __all__ = ["Plan", "Source", "FileSource", "Safetensors", "StTensor", "CfaError", "make_entries",
-           "make_dsts", "ALL", "library_path"]
+           "make_dsts", "ALL", "library_path", "segment_range", "AllGather"]
 
 
 class CfaError(RuntimeError):
@@ -382,6 +382,54 @@ class Safetensors:
                             src_row_stride=stride)
 
 
+def segment_range(blob_bytes, chunk_bytes, world, rank, chunk):
+    """(blob offset, bytes) of rank `rank`'s segment of chunk `chunk` in a segmented load of
+    `world` ranks (cfa_segment_range)."""
+    off, n = ctypes.c_uint64(), ctypes.c_uint64()
+    _check(_lib.load().cfa_segment_range(int(blob_bytes), int(chunk_bytes), int(world),
+                                         int(rank), int(chunk), ctypes.byref(off),
+                                         ctypes.byref(n)))
+    return off.value, n.value
+
+
+class _RawBytes:
+    """`n` bytes at device address `ptr`, seen by torch through __cuda_array_interface__."""
+
+    def __init__(self, ptr, n):
+        self.__cuda_array_interface__ = {"shape": (n,), "typestr": "|u1", "data": (ptr, False),
+                                         "version": 3, "strides": None}
+
+
+class AllGather:
+    """The gather step of a segmented load (section 4.2, "Optimization of Distributed
+    Loading"; section 5: AllGather over a torch.distributed group, NCCL on GPUs): a callable for
+    Plan(gather=...) that gathers every rank's segment into the chunk's slot in place, enqueued
+    on the loader's gather stream.  `device` "cuda" (slot in device memory, the library's case)
+    or "cpu" (host memory: the same exchange over gloo, for tests without a GPU)."""
+
+    def __init__(self, group=None, device="cuda"):
+        self.group = group
+        self.device = device
+
+    def slot(self, ptr, n):
+        import torch
+        if self.device == "cpu":
+            buf = (ctypes.c_uint8 * n).from_address(ptr)
+            return torch.frombuffer(buf, dtype=torch.uint8, count=n)
+        return torch.as_tensor(_RawBytes(ptr, n), device="cuda")
+
+    def __call__(self, chunk_ptr, segment_bytes, world, rank, chunk, stream):
+        import torch
+        import torch.distributed as dist
+        out = self.slot(chunk_ptr, segment_bytes * world)
+        mine = out[rank * segment_bytes:(rank + 1) * segment_bytes]
+        if self.device == "cpu":
+            dist.all_gather_into_tensor(out, mine, group=self.group)
+            return
+        with torch.cuda.stream(torch.cuda.ExternalStream(stream)):
+            dist.all_gather_into_tensor(out, mine, group=self.group)
+
+
 class Plan:
     """A loading plan (cfa_plan): validated manifest, chunk <-> tensor mapping, descriptor table,
     staging slots, streams and events."""
@@ -390,7 +438,11 @@ class Plan:
                  dev_slots=2, fill_threads=8, slab_bytes=262144, tiny_bytes=8192, strict=True,
                  host_only=False, timing=False, bulk=True, no_merge=False, stage_slices=False,
                  device=-1,
-                 workspace=0, workspace_bytes=0):
+                 workspace=0, workspace_bytes=0, world=1, rank=0, gather=None):
+        """world > 1 makes a segmented plan (cfa_plan_opts.seg_world): this process loads
+        rank `rank`'s segment of every chunk and `gather(chunk_ptr, segment_bytes, world, rank,
+        chunk, stream_handle)` assembles each chunk in the device slot (e.g. AllGather(group)).
+        An exception raised by `gather` fails the load with CFA_ERR_GATHER."""
         lib = _lib.load()
         self._lib = lib
         self._handle = None
@@ -417,6 +469,20 @@ class Plan:
                    (_lib.OPT_STAGE_SLICES if stage_slices else 0))
         o.workspace = workspace or None
         o.workspace_bytes = workspace_bytes
+        o.seg_world = world
+        o.seg_rank = rank
+        self._gather = None
+        if gather is not None:
+            def trampoline(_user, chunk_ptr, seg_bytes, w, r, chunk, stream):
+                try:
+                    gather(chunk_ptr, seg_bytes, w, r, chunk, stream or 0)
+                    return 0
+                except Exception as e:  # reported as CFA_ERR_GATHER by the library
+                    self.gather_error = e
+                    return 1
+            self._gather = _lib.GATHER_FN(trampoline)  # kept alive with the plan
+            o.gather = ctypes.cast(self._gather, ctypes.c_void_p).value
+        self.gather_error = None
         h = ctypes.c_void_p()
         ea = entries.arr
         st = lib.cfa_plan_create(ea.ctypes.data if len(ea) else None, len(ea),

@@ -12,7 +12,8 @@ CFA_OK = 0
 STATUS = {0: "CFA_OK", -1: "CFA_ERR_INVAL", -2: "CFA_ERR_OVERLAP", -3: "CFA_ERR_OOB",
           -4: "CFA_ERR_COVERAGE", -5: "CFA_ERR_CUDA", -6: "CFA_ERR_SOURCE", -7: "CFA_ERR_TIMEOUT",
           -8: "CFA_ERR_BUSY", -9: "CFA_ERR_NOMEM", -10: "CFA_ERR_DTYPE", -11: "CFA_ERR_ALIGN",
-          -12: "CFA_ERR_DEVICE", -13: "CFA_ERR_SHAPE"}
+          -12: "CFA_ERR_DEVICE", -13: "CFA_ERR_SHAPE",
+          -14: "CFA_ERR_SUSPECT", -15: "CFA_ERR_GATHER"}
 DTYPE = {"u8": 1, "bf16": 2, "f16": 3, "f32": 4, "i32": 5, "i64": 6, "f64": 7, "i16": 8}
 DTYPE_SIZE = {"u8": 1, "bf16": 2, "f16": 2, "f32": 4, "i32": 4, "i64": 8, "f64": 8, "i16": 2}
 ENTRY_CAST_BF16, ENTRY_CKSUM, ENTRY_CONVERT = 0x1, 0x2, 0x4
@@ -32,6 +33,9 @@ DST_DTYPE = np.dtype([("dev_ptr", "<u8"), ("dtype", "<i4"), ("ndim", "<i4"),
 
 FILL_FN = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_uint64, ctypes.c_void_p,
                            ctypes.c_uint64)
+# cfa_gather_fn(user, chunk_dev, segment_bytes, world, rank, chunk, stream)
+GATHER_FN = ctypes.CFUNCTYPE(ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_uint64,
+                             ctypes.c_int32, ctypes.c_int32, ctypes.c_uint32, ctypes.c_void_p)
 
 
 class PlanOpts(ctypes.Structure):
@@ -40,7 +44,9 @@ class PlanOpts(ctypes.Structure):
                 ("device", ctypes.c_int32), ("slab_bytes", ctypes.c_uint32),
                 ("tiny_bytes", ctypes.c_uint32), ("flags", ctypes.c_uint32),
                 ("reserved", ctypes.c_uint32), ("workspace", ctypes.c_void_p),
-                ("workspace_bytes", ctypes.c_uint64)]
+                ("workspace_bytes", ctypes.c_uint64), ("seg_world", ctypes.c_int32),
+                ("seg_rank", ctypes.c_int32), ("gather", ctypes.c_void_p),
+                ("gather_user", ctypes.c_void_p)]
 
 
 class Source(ctypes.Structure):
@@ -97,12 +103,13 @@ SIGNATURES = {
     "cfa_plan_get_pieces": (ctypes.c_int, [_P, _P, _SZ, _P]),
     "cfa_unpack_chunks_async": (ctypes.c_int, [_P, ctypes.c_uint32, ctypes.c_uint32, _P, _P]),
     "cfa_reset_checksums": (ctypes.c_int, [_P, _P]),
+    "cfa_segment_range": (ctypes.c_int, [_U64, _U64, _I32, _I32, ctypes.c_uint32, _P, _P]),
     "cfa_plan_destroy": (ctypes.c_int, [_P]),
     "cfa_last_error": (ctypes.c_char_p, [_P]),
     "cfa_status_name": (ctypes.c_char_p, [ctypes.c_int]),
     "cfa_abi_sizeof": (_SZ, [ctypes.c_char_p]),
-    "cfa_unpack_noalloc": (ctypes.c_int, [_P, _SZ, _P, _SZ, _P, _U64, _P, _P, ctypes.c_char_p,
-                                          _SZ]),
+    "cfa_unpack_noalloc": (ctypes.c_int, [_P, _SZ, _P, _SZ, _P, _U64, _P, _P, _P,
+                                          ctypes.c_char_p, _SZ]),
     "cfa_safetensors_open": (ctypes.c_int, [ctypes.c_char_p, _P]),
     "cfa_safetensors_parse": (ctypes.c_int, [_P, _U64, _U64, _P]),
     "cfa_safetensors_info": (ctypes.c_int, [_P, _P, _P, _P]),

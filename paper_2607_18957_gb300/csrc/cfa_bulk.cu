@@ -16,9 +16,10 @@
  * No block-wide barrier runs inside the loop.  Plain cp.async.bulk only: no tensor maps, no
  * multicast, one CTA's own shared memory.
  *
- * Every wait is bounded: a wait that runs out sets the status word and ends both loops; the CTA
- * then waits (again bounded) for the loads it issued but did not consume, and for its stores,
- * and returns.
+ * Every wait is bounded: a wait that runs out ends both loops; the CTA then waits (again
+ * bounded) for the loads it issued but did not consume, and for its stores, and returns with
+ * status word 2, or 3 if that drain ran out as well (a load may then still be in flight into
+ * shared memory the CTA no longer owns).
  */
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -279,10 +280,15 @@ __global__ void __launch_bounds__(kThreads) cfa_bulk_kernel(const BulkArgs a)
     }
     __syncthreads();
     if (aborted && threadIdx.x == 0) {
-        atomicCAS(a.status, 0, 2);
-        /* loads issued but not consumed: wait for them (bounded) before shared memory goes */
-        for (uint32_t k = n_consumed; k < n_issued; ++k)
-            mbar_wait(&full[k % kStages], (k / kStages) & 1u, limit);
+        /* loads issued but not consumed: wait for them (bounded) before shared memory goes.  If
+         * one of these waits runs out too, the CTA leaves with a bulk load that may still write
+         * into shared memory it no longer owns: status 3 (over 1 and 2) tells the host that the
+         * context is suspect, not merely that a wait timed out */
+        bool drained = true;
+        for (uint32_t k = n_consumed; k < n_issued && drained; ++k)
+            drained = mbar_wait(&full[k % kStages], (k / kStages) & 1u, limit);
+        if (drained) atomicCAS(a.status, 0, 2);
+        else atomicMax(a.status, 3);
     }
 }
 

@@ -57,6 +57,25 @@ void cfa_plan_opts_default(cfa_plan_opts *o)
     o->slab_bytes = 262144;
     o->tiny_bytes = 8192;
     o->flags = CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK;
+    o->seg_world = 1;
+}
+
+/* Rank `rank`'s segment of chunk `chunk` (section 4.2, distributed loading): the chunk is cut
+ * into `world` equal segments of S / world bytes; the part inside the blob. */
+cfa_status cfa_segment_range(uint64_t blob_bytes, uint64_t chunk_bytes, int32_t world,
+                             int32_t rank, uint32_t chunk, uint64_t *blob_offset,
+                             uint64_t *bytes)
+{
+    if (!blob_offset || !bytes || world < 1 || rank < 0 || rank >= world || chunk_bytes == 0 ||
+        chunk_bytes % (256ull * (uint64_t)world) != 0)
+        return CFA_ERR_INVAL;
+    const uint64_t n_chunks = blob_bytes / chunk_bytes + (blob_bytes % chunk_bytes != 0);
+    if ((uint64_t)chunk >= n_chunks) return CFA_ERR_INVAL;
+    const uint64_t seg = chunk_bytes / (uint64_t)world;
+    const uint64_t lo = (uint64_t)chunk * chunk_bytes + (uint64_t)rank * seg;
+    *blob_offset = lo;
+    *bytes = lo >= blob_bytes ? 0 : (blob_bytes - lo < seg ? blob_bytes - lo : seg);
+    return CFA_OK;
 }
 
 static void fail(char *err, size_t n, const char *fmt, ...)
@@ -360,6 +379,17 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         o.workspace_bytes / (uint64_t)o.dev_slots < o.chunk_bytes) {
         fail(err, errlen, "workspace too small for %d slots of %llu bytes", o.dev_slots,
              (unsigned long long)o.chunk_bytes);
+        return CFA_ERR_INVAL;
+    }
+    if (o.seg_world == 0) o.seg_world = 1;
+    if (o.seg_world < 0 || o.seg_world > 4096 || o.seg_rank < 0 || o.seg_rank >= o.seg_world) {
+        fail(err, errlen, "seg_rank %d outside [0, seg_world = %d)", o.seg_rank, o.seg_world);
+        return CFA_ERR_INVAL;
+    }
+    if (o.seg_world > 1 &&
+        (!o.gather || o.chunk_bytes % (256ull * (uint64_t)o.seg_world) != 0)) {
+        fail(err, errlen, "a segmented plan (seg_world %d) needs a gather function and "
+             "chunk_bytes a multiple of 256 * seg_world", o.seg_world);
         return CFA_ERR_INVAL;
     }
     if (o.workspace && ((uintptr_t)o.workspace & 255u)) {
@@ -756,10 +786,26 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
 
     /* 4b. what each chunk's pieces read: contiguous ranges merged across gaps of at most
      * kCopyGap bytes, and column slices that would move more than twice their bytes as
-     * strided 2-D copies */
+     * strided 2-D copies.  A segmented plan instead copies this rank's whole segment of every
+     * chunk (the other ranks may read any of its bytes). */
     out->copy_first = (uint32_t *)calloc((size_t)n_chunks + 1, sizeof(uint32_t));
     if (!out->copy_first) { st = CFA_ERR_NOMEM; goto done; }
-    {
+    if (o.seg_world > 1) {
+        out->copies = (cfa_copy *)calloc(n_chunks ? n_chunks : 1, sizeof(cfa_copy));
+        if (!out->copies) { st = CFA_ERR_NOMEM; goto done; }
+        for (uint32_t c = 0; c < n_chunks; ++c) {
+            uint64_t lo = 0, len = 0;
+            cfa_segment_range(blob_bytes, S, o.seg_world, o.seg_rank, c, &lo, &len);
+            out->copy_first[c] = (uint32_t)out->n_copies;
+            if (!len) continue;
+            cfa_copy *cp = &out->copies[out->n_copies++];
+            cp->src = lo;
+            cp->width = cp->pitch = len;
+            cp->rows = 1;
+            out->staged_bytes += len;
+        }
+        out->copy_first[n_chunks] = (uint32_t)out->n_copies;
+    } else {
         const uint64_t kCopyGap = 1ull << 20;
         vec cv = {0};
         cv.elem = sizeof(cfa_copy);

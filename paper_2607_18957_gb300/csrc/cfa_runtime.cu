@@ -127,6 +127,11 @@ struct cfa_plan {
     /* pinned sources: column slices read in place over the host link, beside the copy ring */
     cudaStream_t direct_stream = nullptr;
     cudaEvent_t ev_direct = nullptr;
+    /* segmented plans: the gather callback's stream, and per device slot the event after which
+     * the slot holds the whole chunk (the chunk's Gathered state) */
+    bool segmented = false;
+    cudaStream_t gather_stream = nullptr;
+    std::vector<cudaEvent_t> ev_gathered;
     std::vector<cudaEvent_t> ev_dev_free, ev_h2d, ev_host_free, ev_filled, ev_layer;
     cudaEvent_t ev_begin = nullptr, ev_all = nullptr;
     std::vector<cudaEvent_t> t_h2d0, t_h2d1, t_k0, t_k1;
@@ -348,8 +353,10 @@ void release(cfa_plan *p)
                 if (e) cudaEventDestroy(e);
             v.clear();
         };
+        if (p->gather_stream) cudaStreamSynchronize(p->gather_stream);
         kill(p->ev_dev_free);
         kill(p->ev_h2d);
+        kill(p->ev_gathered);
         kill(p->ev_host_free);
         kill(p->ev_filled);
         kill(p->ev_layer);
@@ -370,6 +377,7 @@ void release(cfa_plan *p)
         }
         if (p->fill_stream) cudaStreamDestroy(p->fill_stream);
         if (p->copy_stream) cudaStreamDestroy(p->copy_stream);
+        if (p->gather_stream) cudaStreamDestroy(p->gather_stream);
         if (p->aux_stream) cudaStreamDestroy(p->aux_stream);
         if (p->d_slabs) cudaFree(p->d_slabs);
         if (p->d_tiny) cudaFree(p->d_tiny);
@@ -464,7 +472,11 @@ cfa_status setup_device(cfa_plan *p)
 
     p->n_dev_slots = o.dev_slots;
     p->n_host_slots = o.host_slots;
-    p->slot_bytes = std::min<uint64_t>(hp.chunk_bytes, (hp.blob_bytes + 255) / 256 * 256);
+    /* a segmented plan's gather fills all seg_world segments of the slot, chunk_bytes in all,
+     * even for a blob shorter than one chunk */
+    p->slot_bytes = p->segmented ? hp.chunk_bytes
+                                 : std::min<uint64_t>(hp.chunk_bytes,
+                                                      (hp.blob_bytes + 255) / 256 * 256);
     if (p->n_dev_slots > 0 && p->slot_bytes > 0) {
         if (o.workspace) {
             p->d_slots = static_cast<uint8_t *>(o.workspace);
@@ -500,6 +512,10 @@ cfa_status setup_device(cfa_plan *p)
     };
     if ((st = events(p->ev_dev_free, p->n_dev_slots, false))) return st;
     if ((st = events(p->ev_h2d, p->n_dev_slots, false))) return st;
+    if (p->segmented) {
+        CK(nullptr, cudaStreamCreateWithFlags(&p->gather_stream, cudaStreamNonBlocking));
+        if ((st = events(p->ev_gathered, p->n_dev_slots, false))) return st;
+    }
     if ((st = events(p->ev_host_free, p->n_host_slots, false))) return st;
     if ((st = events(p->ev_filled, p->n_host_slots, false))) return st;
     if ((st = events(p->ev_layer, hp.n_layers, timing))) return st;
@@ -525,6 +541,11 @@ cfa_status check_status_word(cfa_plan *p)
     CK(p, cudaStreamWaitEvent(p->aux_stream, p->ev_all, 0));
     CK(p, cudaMemcpyAsync(&h, p->d_status, sizeof(int), cudaMemcpyDeviceToHost, p->aux_stream));
     CK(p, cudaStreamSynchronize(p->aux_stream));
+    if (h == 3) {
+        set_err(p, "a TMA bulk-copy wait ran out and so did the wait for the CTA's own loads in "
+                   "flight (status word 3): treat the CUDA context as suspect");
+        return CFA_ERR_SUSPECT;
+    }
     if (h) {
         set_err(p, h == 2 ? "a TMA bulk-copy wait ran out (status word 2)"
                           : "the unpack kernel rejected a work item outside its chunk or of the "
@@ -600,7 +621,9 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
         if (hp.layer_last_chunk[l] < 0) p->layers_empty.push_back(l);
         else p->layers_ending[(size_t)hp.layer_last_chunk[l]].push_back(l);
     }
-    p->chunk_busy.assign(hp.n_chunks, 0);
+    p->segmented = hp.opts.seg_world > 1;
+    /* a segmented load takes every chunk: each rank must issue the same gathers */
+    p->chunk_busy.assign(hp.n_chunks, p->segmented ? 1 : 0);
     for (size_t i = 0; i < hp.n_pieces; ++i) p->chunk_busy[hp.pieces[i].chunk] = 1;
     if (!p->host_only) {
         st = setup_device(p);
@@ -671,6 +694,10 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
     }
     const bool staged = kind == CFA_SRC_HOST || kind == CFA_SRC_CALLBACK;
     const bool in_place = kind == CFA_SRC_DEVICE || kind == CFA_SRC_HOST_DIRECT;
+    if (p->segmented && in_place) {
+        set_err(p, "a segmented plan loads from HOST, PINNED or CALLBACK sources only");
+        return CFA_ERR_INVAL;
+    }
     if (kind == CFA_SRC_HOST_DIRECT && hp.blob_bytes) {
         /* page-locked memory is mapped for the device; pageable memory is readable in place
          * only where the device shares the host's page tables */
@@ -763,8 +790,10 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
          * through the slots as strided 2-D copies (slower than plain copies on the copy engine):
          * the column-slice kernels read them over the host link on the direct stream, in chunk
          * order and ahead of the copy ring, and each chunk's readiness also waits for them. */
-        const bool slices_in_place = kind == CFA_SRC_PINNED && hp.n_strided &&
+        const bool slices_in_place = kind == CFA_SRC_PINNED && hp.n_strided && !p->segmented &&
                                      !(hp.opts.flags & CFA_OPT_STAGE_SLICES);
+        const uint64_t seg_bytes = p->segmented ? S / (uint64_t)hp.opts.seg_world : 0;
+        cfa_status gather_failed = CFA_OK;
         const size_t row = (size_t)hp.n_chunks + 1;
         auto has_slices = [&](uint32_t c) {
             for (int k = 0; k < CFA_N_CLASSES; ++k)
@@ -775,7 +804,7 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
         if (slices_in_place) CK(p, cudaStreamWaitEvent(p->direct_stream, p->ev_begin, 0));
         uint32_t k = 0; /* busy chunks so far: they take the slots in turn */
         for (uint32_t c = 0; c < hp.n_chunks; ++c) {
-            if (!p->chunk_busy[c]) {
+            if (!p->chunk_busy[c] || gather_failed) {
                 cfa_status st = record_layers(p, c, c + 1, cs);
                 if (st) return st;
                 continue;
@@ -817,6 +846,28 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             ++k;
             if (staged) CK(p, cudaEventRecord(p->ev_host_free[hs], p->copy_stream));
             CK(p, cudaEventRecord(p->ev_h2d[ds], p->copy_stream));
+            cudaEvent_t ready = p->ev_h2d[ds];
+            if (p->segmented) {
+                /* InGPU for this rank's segment -> Gathered: the caller's collective fills the
+                 * other segments of the slot on the gather stream */
+                CK(p, cudaStreamWaitEvent(p->gather_stream, p->ev_h2d[ds], 0));
+                const int r = hp.opts.gather(hp.opts.gather_user, dslot, seg_bytes,
+                                             hp.opts.seg_world, hp.opts.seg_rank, c,
+                                             reinterpret_cast<cfa_stream>(p->gather_stream));
+                if (r != 0) {
+                    /* the chunks before this one stay enqueued; the rest of the load is not,
+                     * but its events are still recorded so that waits end */
+                    set_err(p, "the gather callback failed on chunk %u (returned %d)", c, r);
+                    gather_failed = CFA_ERR_GATHER;
+                    cx->error.store(CFA_ERR_GATHER);
+                    p->last_h2d = 0; /* no per-chunk copy times for a cut-short load */
+                    cfa_status st = record_layers(p, c, c + 1, cs);
+                    if (st) return st;
+                    continue;
+                }
+                CK(p, cudaEventRecord(p->ev_gathered[ds], p->gather_stream));
+                ready = p->ev_gathered[ds];
+            }
             const bool direct_c = slices_in_place && has_slices(c);
             if (direct_c) {
                 cfa_status st = launch(p, c, c + 1, (uint64_t)(uintptr_t)src->base,
@@ -824,7 +875,7 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
                 if (st) return st;
                 CK(p, cudaEventRecord(p->ev_direct, p->direct_stream));
             }
-            CK(p, cudaStreamWaitEvent(cs, p->ev_h2d[ds], 0));
+            CK(p, cudaStreamWaitEvent(cs, ready, 0));
             cfa_status st = launch(p, c, c + 1, (uint64_t)(uintptr_t)dslot - off, 0, cs, true,
                                    slices_in_place ? LAUNCH_CONTIG : LAUNCH_ALL);
             if (st) return st;
@@ -836,7 +887,7 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
     CK(p, cudaEventRecord(p->ev_all, cs));
     logf("load %llu enqueued: source kind %d, %llu kernel launches, %u staged chunks",
          (unsigned long long)p->n_loads, kind, (unsigned long long)p->last_launches, p->last_h2d);
-    return CFA_OK;
+    return cx->error.load() == CFA_ERR_GATHER ? CFA_ERR_GATHER : CFA_OK;
 }
 
 cfa_status cfa_wait_layer(cfa_plan *p, int32_t layer, cfa_stream consumer, int64_t timeout_ns)
@@ -863,7 +914,7 @@ cfa_status cfa_wait_layer(cfa_plan *p, int32_t layer, cfa_stream consumer, int64
     if (st) return st;
     const int e = p->last->error.load();
     if (e) {
-        set_err(p, "the source callback failed");
+        if (e != CFA_ERR_GATHER) set_err(p, "the source callback failed");
         return e;
     }
     if (layer == CFA_ALL) return check_status_word(p);
@@ -1056,6 +1107,8 @@ const char *cfa_status_name(cfa_status st)
     case CFA_ERR_ALIGN: return "CFA_ERR_ALIGN";
     case CFA_ERR_DEVICE: return "CFA_ERR_DEVICE";
     case CFA_ERR_SHAPE: return "CFA_ERR_SHAPE";
+    case CFA_ERR_SUSPECT: return "CFA_ERR_SUSPECT";
+    case CFA_ERR_GATHER: return "CFA_ERR_GATHER";
     default: return "CFA_ERR_UNKNOWN";
     }
 }
