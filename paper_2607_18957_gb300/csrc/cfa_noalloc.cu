@@ -13,7 +13,13 @@
  * Set-up: the first call on a device looks up the device address of the scratch array with
  * cudaGetSymbolAddress (in host code the array's name is only a stand-in, not a device
  * address) and caches it for that device; make the first call on each device before any stream
- * capture.
+ * capture.  The cached address belongs to the device's current context: after a
+ * cudaDeviceReset the library must not be used again in the process.
+ *
+ * Blocking: the descriptors go up with a copy from pageable host memory, which returns only
+ * once the bytes have been copied, so the call blocks the host until the work already queued
+ * on the stream has run and the copy is done; the unpack kernels themselves run after it
+ * returns.
  *
  * Sharing: every call on a device uses the same scratch array, which keeps the last call's
  * contents.  Calls are serialised on the host by a mutex, but two calls whose GPU work overlaps
@@ -199,8 +205,8 @@ cfa_status setup(int dev, NoallocScratch **scratch)
 extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t n_entries,
                                          const cfa_dst *dsts, size_t n_dsts,
                                          const void *blob_dev, uint64_t blob_bytes,
-                                         uint64_t *cksum_dev, cfa_stream stream_, char *err,
-                                         size_t err_len)
+                                         uint64_t *cksum_dev, int *status_dev,
+                                         cfa_stream stream_, char *err, size_t err_len)
 {
     g_err = err;
     g_err_len = err ? err_len : 0;
@@ -208,6 +214,10 @@ extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t
     if ((n_entries && !entries) || (n_dsts && !dsts) || (blob_bytes && !blob_dev)) {
         say("cfa_unpack_noalloc: NULL argument");
         return CFA_ERR_INVAL;
+    }
+    if ((uintptr_t)status_dev & 3u) {
+        say("cfa_unpack_noalloc: status_dev must be 4-byte aligned");
+        return CFA_ERR_ALIGN;
     }
     if ((uintptr_t)blob_dev & 255u) {
         say("cfa_unpack_noalloc: the blob must be 256-byte aligned");
@@ -287,9 +297,11 @@ extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t
     cfa_status st = setup(dev, &scratch);
     if (st) return st;
 
-    /* the status word and the checksums start at zero; the descriptors are uploaded from the
-     * host array (the call returns once the driver has taken the bytes) */
-    e = cudaMemsetAsync(&scratch->status, 0, sizeof(int), stream);
+    /* the kernels' status word (the caller's, or the scratch's own) and the checksums start at
+     * zero; the descriptors are uploaded from the host array (a pageable copy: the call returns
+     * once the bytes are on the device, after the work queued before it on the stream) */
+    int *status = status_dev ? status_dev : &scratch->status;
+    e = cudaMemsetAsync(status, 0, sizeof(int), stream);
     if (e == cudaSuccess && cksum_dev && n_entries)
         e = cudaMemsetAsync(cksum_dev, 0, n_entries * sizeof(uint64_t), stream);
     if (e == cudaSuccess && total)
@@ -300,7 +312,7 @@ extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t
         e = cfa_launch_unpack(k, scratch->items + base[k][0], count[k][0],
                               scratch->items + base[k][1], count[k][1],
                               (uint64_t)(uintptr_t)blob_dev, 0, 0, blob_bytes,
-                              reinterpret_cast<unsigned long long *>(cksum_dev), &scratch->status,
+                              reinterpret_cast<unsigned long long *>(cksum_dev), status,
                               g_grid_cap[dev][k], stream);
     }
     if (e != cudaSuccess) {

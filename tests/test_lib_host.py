@@ -334,7 +334,7 @@ def _noalloc_status(m, ents=None, blob_ptr=FAKE_BASE, blob_bytes=None):
     err = ctypes.create_string_buffer(512)
     st = lib.cfa_unpack_noalloc(e.arr.ctypes.data, len(e.arr), d.ctypes.data, len(d), blob_ptr,
                                 m.blob_bytes if blob_bytes is None else blob_bytes, None, None,
-                                err, len(err))
+                                None, err, len(err))
     return _lib.STATUS.get(st, str(st)), err.value.decode()
 
 
