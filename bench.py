@@ -1,10 +1,12 @@
 #!/usr/bin/env python3
 """Benchmark of the GB300 checkpoint loader.
 
-One step = one complete load of a synthetic Llama-3-8B-shaped bf16 checkpoint (32 layers, q/k/v
-and gate/up fused; 16.06 GB) into its final per-parameter layout, i.e. every stage of the path:
-chunked staging, host->device transfer (e2e only), the unpack kernel with fused layouts and
-per-tensor checksums, readiness events, and the checksum read-back (e2e only).
+One step = one complete load of a synthetic checkpoint into its final per-parameter layout, i.e.
+every stage of the path: chunked staging, host->device transfer (e2e only), the unpack kernels
+with fused layouts and per-tensor checksums, readiness events, and the checksum read-back (e2e
+only).  The headline workload is the largest one that fits one GPU: a Llama-3-70B-shaped bf16
+checkpoint (80 layers, q/k/v and gate/up fused; 141.1 GB) streamed in 1 GiB chunks from an
+8 GiB pool (the blob is defined periodic with that period).
 
 Printed on one JSON line (rank 0):
   value      unpacked GB/s into the final layout, kernel only: the blob already sits in HBM
@@ -12,10 +14,14 @@ Printed on one JSON line (rank 0):
              destination byte written once, over the device time of K steps
   e2e        the same metric end to end through the C ABI with a pinned HOST blob: every step
              copies the whole checkpoint host->device (cudaMemcpyAsync on the loader's copy
-             stream) and reads the checksums back; also seconds per model and the fraction of
-             the measured host->device bandwidth
-  roofline   the unpack kernel against the measured HBM copy bandwidth
+             stream) and reads the checksums back; also seconds per model, the fraction of the
+             measured host->device bandwidth, and the per-layer ready times of one load
+  roofline   the unpack kernels against the measured HBM copy bandwidth
   cpu_baseline  the oracle (plain CPU loader) on a bounded sample, on this host's cores
+  configs    the same kernel-only and end-to-end figures for the other workloads: 1,000 tiny
+             tensors and the Mixtral workload's 200k extras alone (L2 flushed between steps),
+             Llama-3-8B bf16 (with the end-to-end attribution), Llama-3-8B fp32 -> bf16 (the
+             oracle over the whole model on all host cores), Mixtral-8x7B bf16
 
 --impl reference times the oracle as the reference arm.  --gpus N runs N independent replicas
 (one process per GPU under torchrun); nothing in the path is sharded or exchanged.
@@ -37,6 +43,13 @@ METRIC = "unpacked GB/s into final layout (% of HBM peak); end-to-end H2D load s
 UNIT = "GB/s"
 HBM_FALLBACK_GBS = 6800.0
 L2_BYTES = 129e6
+HEADLINE = "llama3_70b_bf16"
+CONFIGS = ("tiny_1000", "mixtral_extras_200k", "llama3_8b_bf16", "llama3_8b_f32_rne",
+           "mixtral_8x7b_bf16")
+# workloads whose inputs fit in L2: the kernel-only steps flush it (a 1 GiB write) in between
+L2_FLUSHED = ("tiny_1000", "mixtral_extras_200k")
+# the oracle over every tensor (on all host cores) for these; a bounded sample for the others
+CPU_FULL = ("tiny_1000", "llama3_8b_f32_rne")
 
 
 def parse_args():
@@ -45,7 +58,9 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="llama3_8b_bf16")
+    ap.add_argument("--workload", default=HEADLINE)
+    ap.add_argument("--configs", default=",".join(CONFIGS),
+                    help="comma-separated workloads measured after the headline one, or 'none'")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
@@ -66,11 +81,30 @@ def parse_args():
 
 
 # ------------------------------------------------------------------------------------------
+# Small cases of the workloads' kernel classes for ncu captures (a few GB on the device, inputs
+# larger than L2): 2 layers and a 32k vocabulary of the 8B and 70B shapes.
+_SMALL = {
+    "llama3_8b_bf16_2layer_v32k": dict(seed=2, layers=2, hidden=4096, n_q=32, n_kv=8,
+                                       head_dim=128, inter=14336, vocab=32000),
+    # fp32 -> bf16 class, 256-byte aligned tensors (~2.8 GB blob)
+    "llama3_8b_f32_rne_2layer_v32k": dict(seed=3, layers=2, hidden=4096, n_q=32, n_kv=8,
+                                          head_dim=128, inter=14336, vocab=32000,
+                                          src_dtype="f32"),
+    # the same packed at 4-byte offsets with gaps: sources off the 16-byte grid
+    "llama3_8b_f32_rne_2layer_v32k_odd": dict(seed=8, layers=2, hidden=4096, n_q=32, n_kv=8,
+                                              head_dim=128, inter=14336, vocab=32000,
+                                              src_dtype="f32", align=4, jitter=3),
+    # tensor-parallel rank 3 of 8 of the 70B shape: column slices of o and down
+    "llama3_70b_bf16_2layer_v32k_tp8r3": dict(seed=5, layers=2, hidden=8192, n_q=64, n_kv=8,
+                                              head_dim=128, inter=28672, vocab=32000, tp=8,
+                                              rank=3, chunk_bytes=1 << 30),
+}
+
+
 def make_workload(name):
     import workloads
-    if name == "llama3_8b_bf16_2layer_v32k":  # small case for ncu captures (~1.4 GB blob)
-        return workloads.dense_config(name, 2, layers=2, hidden=4096, n_q=32, n_kv=8,
-                                      head_dim=128, inter=14336, vocab=32000)
+    if name in _SMALL:
+        return workloads.dense_config(name, **_SMALL[name])
     try:
         return workloads.named_config(name)
     except KeyError:
@@ -172,7 +206,7 @@ def attribution_sizes(source_bytes, threads):
     return min(gib, source_bytes), min(4 * gib, source_bytes) // max(1, threads)
 
 
-def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
+def attribution(m, host, dsts, entries, stream, args, h2d_gbs, sweep=False):
     """Where end-to-end time goes: (CFA_OPT_TIMING) per-layer readiness of one pinned load, the
     pinned blob read in place by the kernels (no copy engine), the host link for pinned and
     pageable memory, host memcpy with the loader's fill threads, a load from a pageable copy of
@@ -207,6 +241,7 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
                              "median_group": round(float(np.median(t)), 2),
                              "last_group": round(float(t[-1]), 2),
                              "groups": int(t.size), "load_ms": round(st["load_ms"], 2),
+                             "all": [round(float(x), 2) for x in t],
                              "h2d_ms": round(st["h2d_ms"], 2),
                              "unpack_ms": round(st["unpack_ms"], 2)}
     # the same pinned blob read in place by the unpack kernels over NVLink-C2C (no copy
@@ -256,6 +291,9 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
     plan.close()
     out["e2e_pageable_s_per_model"] = round(ms / 1e3, 4)
     out["e2e_pageable_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
+    if sweep:
+        out["fill_threads_sweep"] = fill_thread_sweep(m, pageable, dsts, entries, stream, args,
+                                                      part * threads)
     # the same pageable bytes read in place by the unpack kernel over NVLink-C2C (no staging)
     plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
                     dev_slots=0, host_slots=0, bulk=args.bulk)
@@ -275,6 +313,41 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs):
     out.update(file_attribution(m, pageable, dsts, stream, args, threads))
     del pageable, raw
     return out
+
+
+def fill_thread_sweep(m, pageable, dsts, entries, stream, args, memcpy_bytes):
+    """Host memcpy rate and the pageable load through the pinned ring, per fill thread count:
+    where the host side of the staged path saturates on this machine."""
+    from concurrent.futures import ThreadPoolExecutor
+
+    import numpy as np
+
+    import paper_2607_18957_gb300 as cfa
+    rows = []
+    dst = np.empty(memcpy_bytes, dtype=np.uint8)
+    for t in (4, 8, 16, 32, 48, 64):
+        part = memcpy_bytes // t
+
+        def cp(k):
+            np.copyto(dst[k * part:(k + 1) * part], pageable[k * part:(k + 1) * part])
+        with ThreadPoolExecutor(t) as ex:
+            list(ex.map(cp, range(t)))
+            t0 = time.perf_counter()
+            list(ex.map(cp, range(t)))
+            memcpy_gbs = part * t / (time.perf_counter() - t0) / 1e9
+        plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                        dev_slots=2, host_slots=2, fill_threads=t, bulk=args.bulk)
+        src = cfa.Source.host(pageable.ctypes.data, period=m.period or 0)
+        plan.load_async(src, stream)
+        plan.checksums()
+        ms = min(_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
+                 for _ in range(2))
+        plan.close()
+        rows.append({"threads": t, "host_memcpy_gbs": round(memcpy_gbs, 2),
+                     "e2e_pageable_s_per_model": round(ms / 1e3, 4),
+                     "e2e_pageable_gbs": round(m.blob_bytes / ms / 1e6, 2)})
+    del dst
+    return rows
 
 
 def file_attribution(m, pageable, dsts, stream, args, threads):
@@ -390,43 +463,93 @@ def _timed(fn, stream):
     return a.elapsed_time(b)
 
 
+def host_cores():
+    """Cores this process may run on (the box's own count, not this container's)."""
+    return len(os.sched_getaffinity(0))
+
+
+def _dst_order(m):
+    """Destinations in blob order (by the first blob byte any of their entries reads)."""
+    return sorted(range(m.n_dsts),
+                  key=lambda j: min(int(m.e_offset[i]) for i in m.entries_of_dst(j)))
+
+
+def _oracle_one(m, j):
+    """Destination j through the oracle: (unpack seconds, algorithmic bytes).  Generating the
+    source window is outside the timed call."""
+    import oracle
+    es = m.entries_of_dst(j)
+    lo = min(int(m.e_offset[i]) for i in es)
+    hi = max(int(m.e_offset[i]) + m.e_extent(i) for i in es)
+    window = m.blob_range(lo, hi - lo)
+    t0 = time.perf_counter()
+    r = oracle.unpack(m, window, blob_begin=lo, dsts=[j])
+    dt = time.perf_counter() - t0
+    assert r.status == 0
+    return dt, sum(m.e_nbytes(i) for i in es) + m.d_nbytes(j)
+
+
 def cpu_baseline(m, seconds, steps=None):
     """The oracle, as it stands, on destinations in blob order until `seconds` of CPU time (or
-    one destination per step for the reference arm).  Generation of the sample's blob bytes is
-    outside the timed region.  Returns (GB/s, bytes, secs, description, per-step times)."""
-    import numpy as np
-
-    import oracle
-    from workloads import DTYPE_SIZE
-    order = sorted(range(m.n_dsts),
-                   key=lambda j: min(int(m.e_offset[i]) for i in m.entries_of_dst(j)))
+    one destination per step for the reference arm; seconds=None: every destination).
+    Generation of the sample's blob bytes is outside the timed region.  Returns (GB/s, bytes,
+    secs, description, per-step times)."""
+    order = _dst_order(m)
     done_bytes, busy, used, step_times = 0, 0.0, [], []
     k = 0
     while True:
         j = order[k % len(order)]
         k += 1
-        es = m.entries_of_dst(j)
-        lo = min(int(m.e_offset[i]) for i in es)
-        hi = max(int(m.e_offset[i]) + m.e_extent(i) for i in es)
-        window = m.blob_range(lo, hi - lo)
-        t0 = time.perf_counter()
-        r = oracle.unpack(m, window, blob_begin=lo, dsts=[j])
-        dt = time.perf_counter() - t0
-        assert r.status == 0
-        nb = sum(m.e_nbytes(i) for i in es) + m.d_nbytes(j)
+        dt, nb = _oracle_one(m, j)
         done_bytes += nb
         busy += dt
         used.append(m.d_name[j])
         step_times.append((dt, nb))
-        del window, r
         if steps is not None:
             if len(step_times) >= steps:
                 break
-        elif busy >= seconds or k >= len(order):
+        elif (seconds is not None and busy >= seconds) or k >= len(order):
             break
-    desc = (f"{len(used)} destination tensor(s) of {m.name} in blob order ({used[0]} ...), "
-            f"{done_bytes / 1e9:.2f} GB of algorithmic bytes, single thread")
+    whole = seconds is None and steps is None
+    desc = (f"{'all ' if whole else ''}{len(used)} destination tensor(s) of {m.name} in blob "
+            f"order ({used[0]} ...), {done_bytes / 1e9:.2f} GB of algorithmic bytes, single "
+            "thread")
     return done_bytes / busy / 1e9, done_bytes, busy, desc, step_times
+
+
+_POOL_MANIFESTS = {}
+
+
+def _pool_task(args):
+    key, j = args
+    if key not in _POOL_MANIFESTS:  # a plain exception (not SystemExit) reaches the parent
+        import workloads
+        _POOL_MANIFESTS[key] = workloads.named_config(key)
+    return _oracle_one(_POOL_MANIFESTS[key], j)
+
+
+def cpu_baseline_all_cores(m, key, workers):
+    """The oracle over every destination of `m`, one destination per task, on `workers` spawned
+    processes (each runs the single-threaded oracle as it stands).  Returns the whole-model rate
+    over the wall time of the pool (blob windows generated inside it, in each worker) and the
+    single-thread rate over the oracle calls alone."""
+    import multiprocessing as mp
+    order = _dst_order(m)
+    # largest first, so that the pool does not end on one big tensor
+    order.sort(key=lambda j: -m.d_nbytes(j))
+    ctx = mp.get_context("spawn")
+    with ctx.Pool(workers) as pool:
+        t0 = time.perf_counter()
+        res = pool.map(_pool_task, [(key, j) for j in order], chunksize=1)
+        wall = time.perf_counter() - t0
+    nb = sum(b for _, b in res)
+    busy = sum(t for t, _ in res)
+    return {"value": round(nb / wall / 1e9, 4), "unit": UNIT, "cores": workers,
+            "host_cores": host_cores(), "kind": "oracle",
+            "single_thread_gbs": round(nb / busy / 1e9, 4),
+            "sample": f"all {len(order)} destinations of {m.name} ({nb / 1e9:.2f} GB of "
+                      f"algorithmic bytes) on {workers} processes, one destination per task; "
+                      f"wall {wall:.1f} s including each task's blob-window generation"}
 
 
 def run_reference(args):
@@ -447,8 +570,8 @@ def run_reference(args):
         "data": f"synthetic (seeded counter-based generator; {_BLOB_KIND[m.blob_kind]})",
         "config": {"workload": m.name, "step": "one destination tensor per step, in blob order",
                    "parallelism": "replicas"},
-        "cpu_baseline": {"value": round(gbs, 4), "unit": UNIT, "cores": cores, "kind": "oracle",
-                         "sample": desc},
+        "cpu_baseline": {"value": round(gbs, 4), "unit": UNIT, "cores": cores,
+                         "host_cores": host_cores(), "kind": "oracle", "sample": desc},
         "e2e": {"value": round(gbs, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -500,39 +623,195 @@ def whole_job_gbs(ranks, bytes_this_rank, ms_this_rank):
     return ranks.sum(bytes_this_rank) / (ranks.max(ms_this_rank) / 1e3) / 1e9
 
 
-def run_ours(args):
+def free_memory():
+    """Returns device memory and cached page-locked host memory between workloads."""
+    import gc
+
+    import torch
+    gc.collect()
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    if hasattr(torch._C, "_host_emptyCache"):
+        torch._C._host_emptyCache()
+
+
+def measure_kernel(m, plan, src, stream, ranks, steps, warmup, l2_flush):
+    """Kernel-only steps: `warmup` untimed loads, then `steps` timed ones between a barrier and a
+    synchronize on both sides; with l2_flush a 1 GiB write runs between loads, outside the
+    per-load events.  Returns (total ms, per-load ms list, checksums of the last load)."""
+    import torch
+    flush = torch.empty(1 << 30, dtype=torch.uint8, device="cuda") if l2_flush else None
+    for k in range(warmup):
+        if flush is not None:
+            flush.fill_(k & 255)
+        plan.load_async(src, stream)
+    torch.cuda.synchronize()
+    ranks.barrier()
+    torch.cuda.synchronize()
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for k in range(steps):
+        if flush is not None:
+            flush.fill_((k + 1) & 255)
+        ev[k][0].record(stream)
+        plan.load_async(src, stream)
+        ev[k][1].record(stream)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    ranks.barrier()
+    per_load = [a.elapsed_time(b) for a, b in ev]
+    total = sum(per_load) if l2_flush else t0.elapsed_time(t1)
+    return total, per_load, plan.checksums()
+
+
+def measure_h2d(host, stream):
+    """Host->device copy bandwidth of this machine: 1 GiB from page-locked memory, best of 12."""
+    import torch
+    gib = 1 << 30
+    hsrc = host[:gib] if host.numel() >= gib else torch.empty(gib, dtype=torch.uint8,
+                                                             pin_memory=True)
+    dtmp = torch.empty(gib, dtype=torch.uint8, device="cuda")
+    best = min(_timed(lambda: dtmp.copy_(hsrc, non_blocking=True), stream) for _ in range(12))
+    return gib / (best / 1e3) / 1e9
+
+
+def measure_e2e(m, entries, dsts, host, stream, ranks, steps, warmup, args, ck_want):
+    """End-to-end steps through the C ABI from the pinned host blob: every step copies the
+    staged bytes host->device through two device slots, unpacks, and reads the checksums
+    back.  Returns (ms per step over the slowest rank, per-step ms, staged bytes)."""
     import numpy as np
+    import torch
+
+    import paper_2607_18957_gb300 as cfa
+    plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                    dev_slots=2, host_slots=0, bulk=args.bulk, stage_slices=args.stage_slices)
+    src = cfa.Source.pinned(host.data_ptr(), period=m.period or 0)
+    for _ in range(warmup):
+        plan.load_async(src, stream)
+        plan.checksums()
+    ranks.barrier()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    marks = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    a.record(stream)
+    for k in range(steps):
+        plan.load_async(src, stream)   # H2D of the whole checkpoint + unpack
+        ck = plan.checksums()           # D2H of the step's result
+        marks[k].record(stream)
+    b.record(stream)
+    torch.cuda.synchronize()
+    ranks.barrier()
+    ms = ranks.max(a.elapsed_time(b)) / steps
+    step_ms = [a.elapsed_time(marks[0])] + [marks[k - 1].elapsed_time(marks[k])
+                                            for k in range(1, steps)]
+    assert np.array_equal(ck, ck_want), f"{m.name}: end-to-end checksums differ from the " \
+                                        "kernel-only run"
+    staged = plan.stats()["staged_bytes"]
+    plan.close()
+    return ms, step_ms, staged
+
+
+def measure_workload(name, args, ranks, stream, peak, e2e_steps, attribution_on=False,
+                     h2d_gbs=None):
+    """Kernel-only and end-to-end figures of one workload; frees its memory before returning.
+    Returns a record (dict) plus the manifest."""
     import torch
 
     import paper_2607_18957_gb300 as cfa
     from workloads.harness import DeviceDsts, entries_for, pinned_blob
 
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    ranks = Ranks("nccl", "cuda")
-    world, rank = ranks.world, ranks.rank
-    barrier, max_over_ranks, sum_over_ranks = ranks.barrier, ranks.max, ranks.sum
-
-    m = make_workload(args.workload)
+    m = make_workload(name)
     t_setup = time.time()
-    host = pinned_blob(m)                      # the checkpoint in page-locked host memory
+    host = pinned_blob(m)                      # the checkpoint (or its period) page-locked
     dev_blob = torch.empty(m.source_bytes(), dtype=torch.uint8, device="cuda")
     dev_blob.copy_(host)
     dsts = DeviceDsts(m)
     entries = entries_for(m)
-    stream = torch.cuda.current_stream()
     setup_s = time.time() - t_setup
+    l2_flush = name in L2_FLUSHED
 
     # ---------------- kernel only: the blob already resident in HBM -------------------------
     plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
                     dev_slots=0, host_slots=0, bulk=args.bulk)
     st = plan.stats()
-    algo_bytes = st["bytes_read"] + st["bytes_written"]
+    algo = st["bytes_read"] + st["bytes_written"]
     src = cfa.Source.device(dev_blob.data_ptr(), period=m.period or 0)
-    for _ in range(args.warmup):
-        plan.load_async(src, stream)
-    torch.cuda.synchronize()
-    launches_per_load = plan.stats()["kernel_launches"]
+    total_ms, per_load, ck_dev = measure_kernel(m, plan, src, stream, ranks, args.steps,
+                                                args.warmup, l2_flush)
+    launches = plan.stats()["kernel_launches"]
+    plan.close()
+    del dev_blob
+    torch.cuda.empty_cache()
+    mean_ms = statistics.mean(per_load)
+    achieved = algo / (mean_ms / 1e3) / 1e9
+    rec = {"workload": m.name, "blob_bytes": m.blob_bytes, "tensors": m.n_entries,
+           "destinations": m.n_dsts, "algorithmic_bytes": algo, "chunk_bytes": m.chunk_bytes,
+           "total_ms": total_ms, "steps": args.steps,
+           "value_gbs": whole_job_gbs(ranks, algo * args.steps, total_ms),
+           "kernel_ms": round(mean_ms, 4), "kernel_ms_median": round(statistics.median(per_load), 4),
+           "kernel_ms_min": round(min(per_load), 4), "kernel_gbs": round(achieved, 1),
+           "frac": round(achieved / peak, 4), "launches_per_load": launches,
+           "work_items": {"tma": st["n_bulk"], "slabs": st["n_slabs"], "tiny": st["n_tiny"],
+                          "column_blocks": st["n_strided"]},
+           "pieces": st["n_pieces"],
+           "pieces_per_s": round(st["n_pieces"] / (mean_ms / 1e3), 1),
+           "l2": ("flushed between steps (1 GiB write outside the timed loads)" if l2_flush
+                  else f"no flush: inputs {m.blob_bytes / 1e9:.2f} GB > L2 "
+                       f"{L2_BYTES / 1e6:.0f} MB"),
+           "setup_s": round(setup_s, 2), "_n_bulk": st["n_bulk"]}
+
+    # ---------------- end to end: pinned host blob -> final layout through the C ABI ---------
+    if e2e_steps:
+        if h2d_gbs is None:
+            h2d_gbs = measure_h2d(host, stream)
+        ms, step_ms, staged = measure_e2e(m, entries, dsts, host, stream, ranks, e2e_steps,
+                                          min(args.warmup, 3), args, ck_dev)
+        print(f"{m.name} e2e step ms:", [round(x, 1) for x in step_ms], file=sys.stderr)
+        rec["e2e"] = {
+            "value": round(ranks.sum(algo) / (ms / 1e3) / 1e9, 3), "unit": UNIT,
+            "h2d_bytes_per_step": staged, "d2h_bytes_per_step": 8 * m.n_entries,
+            "seconds_per_model": round(ms / 1e3, 5), "h2d_gbs_measured": round(h2d_gbs, 2),
+            "frac_of_h2d": round((staged / (ms / 1e3) / 1e9) / h2d_gbs, 4),
+            "steps": e2e_steps, "step_ms_median": round(statistics.median(step_ms), 2),
+            "step_ms_max": round(max(step_ms), 2),
+            "source": f"pinned host {'pool of ' + str(m.period >> 30) + ' GiB (periodic blob)' if m.period else 'blob'}, "
+                      f"2 device staging slots of {m.chunk_bytes >> 20} MiB"}
+        if attribution_on and not args.no_attribution:
+            rec["e2e"]["attribution"] = attribution(m, host, dsts, entries, stream, args,
+                                                    h2d_gbs, sweep=(name == "llama3_8b_bf16"))
+    rec["_h2d_gbs"] = h2d_gbs
+    del host, dsts, entries
+    free_memory()
+    return rec, m
+
+
+def _config_record(rec):
+    """The per-workload entry of the `configs` object: kernel-only and end-to-end figures."""
+    out = {k: v for k, v in rec.items() if not k.startswith("_") and
+           k not in ("total_ms", "value_gbs", "steps")}
+    e2e = rec.get("e2e")
+    if e2e:
+        out["e2e"] = {k: e2e[k] for k in ("seconds_per_model", "frac_of_h2d", "h2d_gbs_measured",
+                                          "h2d_bytes_per_step", "step_ms_median", "step_ms_max",
+                                          "steps", "source")}
+        if "attribution" in e2e:
+            out["e2e"]["attribution"] = e2e["attribution"]
+    return out
+
+
+def run_ours(args):
+    import torch
+
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    ranks = Ranks("nccl", "cuda")
+    world, rank = ranks.world, ranks.rank
+    stream = torch.cuda.current_stream()
+    peaks, peak_kind = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", HBM_FALLBACK_GBS))
 
     props = torch.cuda.get_device_properties(local)
     uuid = str(getattr(props, "uuid", "") or "")
@@ -541,26 +820,6 @@ def run_ours(args):
     sampler = ClockSampler(uuid)
     sampler.start()
     time.sleep(0.3)
-    barrier()
-    torch.cuda.synchronize()
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-          for _ in range(args.steps)]
-    t0 = torch.cuda.Event(enable_timing=True)
-    t1 = torch.cuda.Event(enable_timing=True)
-    t0.record(stream)
-    for k in range(args.steps):
-        ev[k][0].record(stream)
-        plan.load_async(src, stream)
-        ev[k][1].record(stream)
-    t1.record(stream)
-    torch.cuda.synchronize()
-    barrier()
-    kernel_ms = t0.elapsed_time(t1)
-    per_load = [a.elapsed_time(b) for a, b in ev]
-    ck_dev = plan.checksums()
-    plan.close()
-    total_ms = max_over_ranks(kernel_ms)
-    value = whole_job_gbs(ranks, algo_bytes * args.steps, kernel_ms)
     # context for the roofline: this GPU's own device copy, taken the way the measured peak was
     # (torch copy_ of 1 Gi bf16 elements, read + write bytes, best of 10)
     ca = torch.empty(1 << 30, dtype=torch.bfloat16, device="cuda")
@@ -569,114 +828,78 @@ def run_ours(args):
     copy_ms = min(_timed(lambda: cb.copy_(ca), stream) for _ in range(10))
     same_box_copy_gbs = 2 * ca.numel() * 2 / (copy_ms / 1e3) / 1e9
     del ca, cb
+    torch.cuda.empty_cache()
 
-    # ---------------- end to end: pinned host blob -> final layout through the C ABI ---------
-    e2e = None
-    h2d_gbs = None
-    if not args.no_e2e:
-        # host->device copy bandwidth of this machine, 1 GiB pinned, best of 10
-        gib = 1 << 30
-        hsrc = host[:gib] if host.numel() >= gib else torch.empty(gib, dtype=torch.uint8,
-                                                                 pin_memory=True)
-        dtmp = torch.empty(gib, dtype=torch.uint8, device="cuda")
-        best = None
-        for _ in range(12):
-            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            a.record(stream)
-            dtmp.copy_(hsrc, non_blocking=True)
-            b.record(stream)
-            b.synchronize()
-            t = a.elapsed_time(b)
-            best = t if best is None else min(best, t)
-        h2d_gbs = gib / (best / 1e3) / 1e9
-        del dtmp
-        e2e_steps = args.e2e_steps or min(args.steps, 20)
-        plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                        dev_slots=2, host_slots=0, bulk=args.bulk,
-                        stage_slices=args.stage_slices)
-        hsrc_all = cfa.Source.pinned(host.data_ptr(), period=m.period or 0)
-        for _ in range(min(args.warmup, 3)):
-            plan.load_async(hsrc_all, stream)
-            plan.checksums()
-        barrier()
-        torch.cuda.synchronize()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        marks = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps)]
-        a.record(stream)
-        for k in range(e2e_steps):
-            plan.load_async(hsrc_all, stream)   # H2D of the whole checkpoint + unpack
-            ck = plan.checksums()                # D2H of the step's result
-            marks[k].record(stream)
-        b.record(stream)
-        torch.cuda.synchronize()
-        barrier()
-        e2e_ms = max_over_ranks(a.elapsed_time(b)) / e2e_steps
-        step_ms = [a.elapsed_time(marks[0])] + [marks[k - 1].elapsed_time(marks[k])
-                                                for k in range(1, e2e_steps)]
-        print("e2e step ms:", [round(x, 1) for x in step_ms], file=sys.stderr)
-        assert np.array_equal(ck, ck_dev), "end-to-end checksums differ from the kernel-only run"
-        plan.close()
-        e2e_gbs = sum_over_ranks(algo_bytes) / (e2e_ms / 1e3) / 1e9
-        staged = st["staged_bytes"]  # what the copies move: the bytes the pieces read
-        e2e = {"value": round(e2e_gbs, 3), "unit": UNIT,
-               "h2d_bytes_per_step": staged, "d2h_bytes_per_step": 8 * m.n_entries,
-               "seconds_per_model": round(e2e_ms / 1e3, 5),
-               "h2d_gbs_measured": round(h2d_gbs, 2),
-               "frac_of_h2d": round((staged / (e2e_ms / 1e3) / 1e9) / h2d_gbs, 4),
-               "steps": e2e_steps, "step_ms_median": round(statistics.median(step_ms), 2),
-               "step_ms_max": round(max(step_ms), 2),
-               "source": f"pinned host blob, 2 device staging slots of {m.chunk_bytes >> 20} MiB"}
-        if not args.no_attribution:
-            e2e["attribution"] = attribution(m, host, dsts, entries, stream, args, h2d_gbs)
+    e2e_steps = 0 if args.no_e2e else (args.e2e_steps or min(args.steps, 20))
+    head, m = measure_workload(args.workload, args, ranks, stream, peak, e2e_steps,
+                               attribution_on=True)
+    h2d_gbs = head["_h2d_gbs"]
+    names = [] if args.configs in ("", "none") else \
+        [n for n in args.configs.split(",") if n and n != args.workload]
+    configs, manifests = {}, {}
+    for name in names:
+        rec, mc = measure_workload(name, args, ranks, stream, peak,
+                                   0 if args.no_e2e else min(e2e_steps, 8),
+                                   attribution_on=(name == "llama3_8b_bf16"), h2d_gbs=h2d_gbs)
+        configs[name] = _config_record(rec)
+        manifests[name] = mc
     clocks = sampler.stop()
 
     # ---------------- the oracle on this host -------------------------------------------------
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         gbs, nb, busy, desc, _ = cpu_baseline(m, args.cpu_seconds)
-        cpu = {"value": round(gbs, 4), "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": desc}
+        cpu = {"value": round(gbs, 4), "unit": UNIT, "cores": 1, "host_cores": host_cores(),
+               "kind": "oracle", "sample": desc}
+        for name, mc in manifests.items():
+            if name == "llama3_8b_f32_rne":
+                configs[name]["cpu_baseline"] = cpu_baseline_all_cores(mc, name, host_cores())
+                continue
+            whole = name in CPU_FULL
+            gbs, nb, busy, desc, _ = cpu_baseline(mc, None if whole else 2.0)
+            configs[name]["cpu_baseline"] = {"value": round(gbs, 4), "unit": UNIT, "cores": 1,
+                                             "host_cores": host_cores(), "kind": "oracle",
+                                             "sample": desc}
 
     if rank != 0:
         ranks.close()
         return
     dtype, cls, cls_desc = path_types(m)
-    if st["n_bulk"]:
+    if head["_n_bulk"]:
         kernel_name = "cfa_bulk_kernel (TMA bulk copies) + cfa_unpack_kernel (heads, tails, tiny)"
     else:
         kernel_name = f"cfa_unpack_kernel<{cls}> ({cls_desc}; 16-byte vectors)"
-    peaks, peak_kind = measured_peaks()
-    peak = float(peaks.get("hbm_gbs", HBM_FALLBACK_GBS))
-    avg_launch_ms = statistics.mean(per_load)
-    achieved = algo_bytes / (avg_launch_ms / 1e3) / 1e9
     line = {
-        "metric": METRIC, "value": round(value, 3), "unit": UNIT, "n_gpus": world,
+        "metric": METRIC, "value": round(head["value_gbs"], 3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": round(total_ms / args.steps, 4), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": dtype,
+        "ms_per_step": round(ranks.max(head["total_ms"]) / args.steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": dtype,
         "data": f"synthetic (seeded counter-based generator; {_BLOB_KIND[m.blob_kind]})",
         "config": {"workload": m.name, "blob_bytes": m.blob_bytes, "tensors": m.n_entries,
-                   "destinations": m.n_dsts, "algorithmic_bytes_per_step": algo_bytes,
-                   "chunk_bytes": m.chunk_bytes, "kernel_source": "device-resident blob",
-                   "l2": f"no flush: inputs {m.blob_bytes / 1e9:.2f} GB > L2 "
-                         f"{L2_BYTES / 1e6:.0f} MB",
+                   "destinations": m.n_dsts, "algorithmic_bytes_per_step":
+                       head["algorithmic_bytes"],
+                   "chunk_bytes": m.chunk_bytes,
+                   "kernel_source": "device-resident blob" + (
+                       f" (periodic: an {m.period >> 30} GiB pool)" if m.period else ""),
+                   "l2": head["l2"],
                    "parallelism": "replicas" if world > 1 else "single GPU"},
-        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak,
-                     "unit": "GB/s", "frac": round(achieved / peak, 4),
-                     "traffic": recorded_traffic(m.name) if st["n_bulk"] else None,
-                     "peak_source": peak_kind,
-                     "kernel": kernel_name,
-                     "launch_ms": round(avg_launch_ms, 4),
+        "roofline": {"bound": "hbm", "achieved": head["kernel_gbs"], "peak": peak,
+                     "unit": "GB/s", "frac": head["frac"],
+                     "traffic": recorded_traffic(m.name) if head["_n_bulk"] else None,
+                     "peak_source": peak_kind, "kernel": kernel_name,
+                     "launch_ms": head["kernel_ms"],
                      "same_box_copy_gbs": round(same_box_copy_gbs, 1),
-                     "frac_of_same_box_copy": round(achieved / same_box_copy_gbs, 4)},
-        "e2e": e2e,
+                     "frac_of_same_box_copy": round(head["kernel_gbs"] / same_box_copy_gbs, 4)},
+        "e2e": head.get("e2e"),
         "cpu_baseline": cpu,
-        "gpu_launches": int(launches_per_load * args.steps),
+        "configs": configs,
+        "gpu_launches": int(head["launches_per_load"] * args.steps),
         "clocks": clocks,
-        "setup_s": round(setup_s, 2),
+        "setup_s": head["setup_s"],
     }
     print(json.dumps(line), flush=True)
     ranks.close()
+
 
 
 def main():
