@@ -94,6 +94,10 @@ _SMALL = {
     "llama3_8b_f32_rne_2layer_v32k_odd": dict(seed=8, layers=2, hidden=4096, n_q=32, n_kv=8,
                                               head_dim=128, inter=14336, vocab=32000,
                                               src_dtype="f32", align=4, jitter=3),
+    # the 70B layer shapes, 1 GiB chunks (~4.5 GB blob): the headline's TMA kernel
+    "llama3_70b_bf16_2layer_v32k": dict(seed=5, layers=2, hidden=8192, n_q=64, n_kv=8,
+                                        head_dim=128, inter=28672, vocab=32000,
+                                        chunk_bytes=1 << 30),
     # tensor-parallel rank 3 of 8 of the 70B shape: column slices of o and down
     "llama3_70b_bf16_2layer_v32k_tp8r3": dict(seed=5, layers=2, hidden=8192, n_q=64, n_kv=8,
                                               head_dim=128, inter=28672, vocab=32000, tp=8,
@@ -120,16 +124,21 @@ def measured_peaks():
         return {"hbm_gbs": HBM_FALLBACK_GBS}, "fallback"
 
 
-def kernel_source_hash():
+KERNEL_SOURCES = ("cfa_unpack.cu", "cfa_bulk.cu", "cfa_device.cuh")
+
+
+def kernel_source_hash(files=KERNEL_SOURCES):
+    """sha256 over the named kernel source files (csrc/), in order."""
     h = hashlib.sha256()
-    for f in ("cfa_unpack.cu", "cfa_bulk.cu", "cfa_device.cuh"):
+    for f in files:
         with open(os.path.join(ROOT, "paper_2607_18957_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()
 
 
 def recorded_traffic(workload):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel is unchanged."""
+    """DRAM bytes per launch from the committed ncu summary, if the sources of the captured
+    kernel (the record's `sources`, else all kernel sources) are unchanged since."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     try:
         with open(path) as f:
@@ -137,9 +146,25 @@ def recorded_traffic(workload):
     except OSError:
         return None
     r = rec.get(workload)
-    if not r or r.get("kernel_sha256") != kernel_source_hash():
+    if not r or r.get("kernel_sha256") != kernel_source_hash(tuple(r.get("sources",
+                                                                          KERNEL_SOURCES))):
         return None
     return r.get("dram_bytes_per_launch")
+
+
+def kernel_names(st):
+    """The unpack kernels one load of a plan with these stats launches."""
+    out = []
+    if st["n_bulk"]:
+        out.append("cfa_bulk_kernel (TMA bulk copies)")
+    if st["n_slabs"]:
+        out.append("cfa_unpack_kernel (16-byte vector slabs" + (", tiny pieces interleaved)"
+                                                               if st["n_tiny"] else ")"))
+    elif st["n_tiny"]:
+        out.append("cfa_tiny_kernel (tiny pieces)")
+    if st["n_strided"]:
+        out.append("cfa_strided_kernel (column slices)")
+    return " + ".join(out)
 
 
 class ClockSampler:
@@ -761,6 +786,7 @@ def measure_workload(name, args, ranks, stream, peak, e2e_steps, attribution_on=
            "l2": ("flushed between steps (1 GiB write outside the timed loads)" if l2_flush
                   else f"no flush: inputs {m.blob_bytes / 1e9:.2f} GB > L2 "
                        f"{L2_BYTES / 1e6:.0f} MB"),
+           "kernels": kernel_names(st),
            "setup_s": round(setup_s, 2), "_n_bulk": st["n_bulk"]}
 
     # ---------------- end to end: pinned host blob -> final layout through the C ABI ---------
@@ -865,10 +891,7 @@ def run_ours(args):
         ranks.close()
         return
     dtype, cls, cls_desc = path_types(m)
-    if head["_n_bulk"]:
-        kernel_name = "cfa_bulk_kernel (TMA bulk copies) + cfa_unpack_kernel (heads, tails, tiny)"
-    else:
-        kernel_name = f"cfa_unpack_kernel<{cls}> ({cls_desc}; 16-byte vectors)"
+    kernel_name = f"{head['kernels']}; dominant work class: {cls_desc}"
     line = {
         "metric": METRIC, "value": round(head["value_gbs"], 3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup,
@@ -885,7 +908,7 @@ def run_ours(args):
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "roofline": {"bound": "hbm", "achieved": head["kernel_gbs"], "peak": peak,
                      "unit": "GB/s", "frac": head["frac"],
-                     "traffic": recorded_traffic(m.name) if head["_n_bulk"] else None,
+                     "traffic": recorded_traffic(m.name),
                      "peak_source": peak_kind, "kernel": kernel_name,
                      "launch_ms": head["kernel_ms"],
                      "same_box_copy_gbs": round(same_box_copy_gbs, 1),

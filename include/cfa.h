@@ -193,7 +193,8 @@ typedef struct cfa_plan_opts {
                                  or CALLBACK load (0 = none); default 2 */
     int32_t dev_slots;        /* device staging slots of S bytes, allocated by cfa_plan_create
                                  (0 = none: DEVICE sources only); default 2 */
-    int32_t fill_threads;     /* host threads copying pageable sources into pinned slots; default 8 */
+    int32_t fill_threads;     /* host threads copying pageable sources into pinned slots; default:
+                                 the CPUs the process may run on, at most 32 */
     int32_t device;           /* CUDA device ordinal; -1 = the current device */
     uint32_t slab_bytes;      /* destination bytes per block-level work item, a multiple of 4096;
                                  default 262144 */

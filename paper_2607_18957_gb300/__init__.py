@@ -435,7 +435,7 @@ class Plan:
     staging slots, streams and events."""
 
     def __init__(self, entries, dsts, blob_bytes, chunk_bytes=512 << 20, host_slots=2,
-                 dev_slots=2, fill_threads=8, slab_bytes=262144, tiny_bytes=8192, strict=True,
+                 dev_slots=2, fill_threads=None, slab_bytes=262144, tiny_bytes=8192, strict=True,
                  host_only=False, timing=False, bulk=True, no_merge=False, stage_slices=False,
                  device=-1,
                  workspace=0, workspace_bytes=0, world=1, rank=0, gather=None):
@@ -457,7 +457,8 @@ class Plan:
         o.chunk_bytes = chunk_bytes
         o.host_slots = host_slots
         o.dev_slots = dev_slots
-        o.fill_threads = fill_threads
+        if fill_threads is not None:  # None: the library's default (one per usable CPU)
+            o.fill_threads = fill_threads
         o.device = device
         o.slab_bytes = slab_bytes
         o.tiny_bytes = tiny_bytes

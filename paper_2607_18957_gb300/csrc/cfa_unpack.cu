@@ -43,6 +43,7 @@ constexpr int kCopyMinBlocks = 3; /* 2-8-byte copy classes: 80 registers, room f
  * three CTAs per SM the copy kernels hold them without spilling; two for the 1-byte class at
  * four CTAs), two for column-slice rows. */
 constexpr int kRealignRounds = 4;
+
 constexpr int kRealignRoundsRows = 2;
 
 struct UnpackArgs {
@@ -378,7 +379,10 @@ __device__ __forceinline__ bool item_ok(const cfa_work &w, const UnpackArgs &a)
            (w.dst & ((1ull << dl) - 1)) == 0;
 }
 
-template <int CLS, int U, int W = 32>
+/* One work item: U 16-byte vectors per thread in flight on the aligned path, UR rounds of W
+ * vectors per lane group on the realigning path (default: four for slabs of the 2-8-byte copy
+ * classes, two for the 1-byte class). */
+template <int CLS, int U, int W = 32, int UR = (U > 1 ? (CLS >= 1 ? kRealignRounds : 2) : 1)>
 __device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs &a, uint32_t tid,
                                              uint32_t nthr)
 {
@@ -389,9 +393,7 @@ __device__ __forceinline__ uint64_t run_item(const cfa_work &w, const UnpackArgs
     if constexpr (C::conv != CFA_CONV_NONE)
         return convert_run<C::ses, C::des, C::conv, (U > 2 ? 2 : U)>(src, dst, w.n, tid, nthr);
     else
-        return copy_run<(1 << CLS), U, (U > 1 ? (CLS >= 1 ? kRealignRounds : 2) : 1), W>(src, dst,
-                                                                       (uint64_t)w.n << CLS, tid,
-                                                                       nthr);
+        return copy_run<(1 << CLS), U, UR, W>(src, dst, (uint64_t)w.n << CLS, tid, nthr);
 }
 
 /* Adds the CTA's accumulated checksum to slot ck; every thread of the CTA must call it. */
@@ -428,7 +430,7 @@ constexpr int kSegs = 32 / kSegLanes;
 constexpr uint32_t kSegMaxBytes = CFA_TINY_SEG_BYTES;
 constexpr uint32_t kTinyPerGroup = kWarps * kSegs;
 
-template <int CLS>
+template <int CLS, int U = 1, int UR = 1>
 __device__ __forceinline__ void run_tiny(const UnpackArgs &a, uint32_t group, uint32_t warp,
                                          uint32_t lane)
 {
@@ -446,7 +448,7 @@ __device__ __forceinline__ void run_tiny(const UnpackArgs &a, uint32_t group, ui
     if (!__any_sync(0xFFFFFFFFu, bytes > kSegMaxBytes)) {
         if (ok) {
             const uint32_t mask = 0xFFu << (seg * kSegLanes);
-            uint64_t v = run_item<CLS, 1, kSegLanes>(w, a, sub, kSegLanes);
+            uint64_t v = run_item<CLS, U, kSegLanes, UR>(w, a, sub, kSegLanes);
 #pragma unroll
             for (int o = kSegLanes / 2; o > 0; o >>= 1) v += __shfl_down_sync(mask, v, o, kSegLanes);
             if (sub == 0 && w.ck != CFA_NO_CK) atomicAdd(a.ck + w.ck, v);
@@ -463,7 +465,7 @@ __device__ __forceinline__ void run_tiny(const UnpackArgs &a, uint32_t group, ui
         wk.ck = __shfl_sync(0xFFFFFFFFu, w.ck, src_lane);
         wk.mode = __shfl_sync(0xFFFFFFFFu, w.mode, src_lane);
         wk.pad = __shfl_sync(0xFFFFFFFFu, w.pad, src_lane);
-        const uint64_t v = warp_sum(run_item<CLS, 1>(wk, a, lane, 32u));
+        const uint64_t v = warp_sum(run_item<CLS, U, 32, UR>(wk, a, lane, 32u));
         if (lane == 0 && wk.ck != CFA_NO_CK) atomicAdd(a.ck + wk.ck, v);
     }
 }
@@ -513,6 +515,134 @@ __global__ void __launch_bounds__(kThreads, (CLS >= 1 && CLS < 4 ? kCopyMinBlock
         }
     }
     if (acc_ck != CFA_NO_CK) block_flush(acc, acc_ck, a.ck, red);
+}
+
+/* A launch of tiny pieces only (no block-level items).  A tiny piece is bound by latency, not
+ * bandwidth: the combined kernel's one vector per lane kept about 2 MB in flight on the whole
+ * GPU, a third of what HBM needs at its latency.  Here every piece is copied by one 8-lane
+ * segment with kUnroll vectors per lane in flight: a piece whose source and destination share
+ * their 16-byte phase (checkpoints packed at 16-byte or wider alignment) in one round trip of up
+ * to 512 bytes, head and tail included (copy_same_phase); other copies and conversions through
+ * run_item with one realigning round.  Each segment fetches the descriptor of its next piece
+ * before copying the current one, so the descriptor load is off the critical path.  Its own
+ * kernel keeps these registers out of the combined kernel's budget. */
+constexpr int kTinyRounds = 1;
+
+/* Bytes [lo, hi) of a 16-byte vector kept, the others zeroed. */
+__device__ __forceinline__ uint4 keep_bytes(uint4 v, uint32_t lo, uint32_t hi)
+{
+    uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int h = min(max((int)hi - 4 * q, 0), 4), l = min(max((int)lo - 4 * q, 0), 4);
+        const uint32_t below_hi = h >= 4 ? 0xFFFFFFFFu : (1u << (8 * h)) - 1u;
+        const uint32_t below_lo = l >= 4 ? 0xFFFFFFFFu : (1u << (8 * l)) - 1u;
+        w[q] &= below_hi & ~below_lo;
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+/* Stores the ES-byte elements of v at byte offsets [lo, hi) of the 16-byte block at dst16. */
+template <int ES>
+__device__ __forceinline__ void store_part(uint8_t *dst16, uint4 v, uint32_t lo, uint32_t hi)
+{
+    typedef typename Elem<ES>::T T;
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int q = 0; q < 16 / ES; ++q) {
+        const uint32_t b = (uint32_t)(q * ES);
+        if (b >= lo && b < hi) {
+            T e;
+            if constexpr (ES == 8)
+                e = ((unsigned long long)w[b / 4 + 1] << 32) | w[b / 4];
+            else
+                e = (T)(w[b / 4] >> (8 * (b % 4)));
+            reinterpret_cast<T *>(dst16)[q] = e;
+        }
+    }
+}
+
+/* A tiny piece whose source and destination share their offset within 16 bytes: rounds of
+ * W x U aligned 16-byte vectors, the piece's partial first and last vectors loaded whole in the
+ * same round (an aligned 16-byte block holding bytes of the piece lies in the same page and
+ * allocation) and stored element by element, so a piece of up to W * U * 16 bytes is one round
+ * trip, not the vector round plus the head and tail rounds of copy_run.  Lane `lane` of W. */
+template <int ES, int U, int W>
+__device__ __forceinline__ uint64_t copy_same_phase(const uint8_t *src, uint8_t *dst,
+                                                    uint32_t nbytes, uint32_t lane)
+{
+    const uint32_t p = (uint32_t)((uintptr_t)src & 15u);
+    const uint4 *s = reinterpret_cast<const uint4 *>(src - p);
+    uint8_t *d = dst - p;
+    const uint32_t end = p + nbytes; /* in bytes from s */
+    const uint32_t nv = (end + 15u) >> 4;
+    uint64_t acc = 0;
+    for (uint32_t base = 0; base < nv; base += W * U) {
+        uint4 v[U];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const uint32_t i = base + u * W + lane;
+            if (i < nv) v[u] = ld_stream(s + i);
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const uint32_t i = base + u * W + lane;
+            if (i >= nv) continue;
+            const uint32_t lo = i == 0 ? p : 0u;
+            const uint32_t hi = end - 16u * i < 16u ? end - 16u * i : 16u;
+            if (lo == 0 && hi == 16u) {
+                st_stream(d + 16u * i, v[u]);
+                acc += vsum<ES>(v[u]);
+            } else {
+                store_part<ES>(d + 16u * i, v[u], lo, hi);
+                acc += vsum<ES>(keep_bytes(v[u], lo, hi));
+            }
+        }
+    }
+    return acc;
+}
+
+template <int CLS>
+__global__ void __launch_bounds__(kThreads, (CLS < 4 ? kCopyMinBlocks : kMinBlocks))
+    cfa_tiny_kernel(const UnpackArgs a)
+{
+    const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
+    const uint32_t seg = lane / kSegLanes, sub = lane % kSegLanes;
+    const uint32_t mask = 0xFFu << (seg * kSegLanes);
+    const uint32_t n_groups = (a.n_tiny + kTinyPerGroup - 1) / kTinyPerGroup;
+    const uint32_t slot = warp * kSegs + seg; /* this segment's piece within a group */
+    uint32_t group = blockIdx.x;
+    cfa_work w{};
+    if (group < n_groups && group * kTinyPerGroup + slot < a.n_tiny)
+        w = a.tiny[group * kTinyPerGroup + slot];
+    while (group < n_groups) {
+        const uint32_t t = group * kTinyPerGroup + slot;
+        const uint32_t next = group + gridDim.x;
+        cfa_work wn{};
+        if (next < n_groups && next * kTinyPerGroup + slot < a.n_tiny)
+            wn = a.tiny[next * kTinyPerGroup + slot];
+        if (t < a.n_tiny) {
+            if (item_ok<CLS>(w, a)) {
+                uint64_t v;
+                const uint64_t off = a.src_period ? w.src % a.src_period : w.src;
+                const uint8_t *src = reinterpret_cast<const uint8_t *>(a.src_base + off);
+                uint8_t *dst = reinterpret_cast<uint8_t *>(w.dst);
+                if (CLS < 4 && (((uintptr_t)src ^ (uintptr_t)dst) & 15u) == 0)
+                    v = copy_same_phase<(CLS < 4 ? (1 << CLS) : 1), kUnroll, kSegLanes>(
+                        src, dst, w.n << (CLS < 4 ? CLS : 0), sub);
+                else
+                    v = run_item<CLS, kUnroll, kSegLanes, kTinyRounds>(w, a, sub, kSegLanes);
+#pragma unroll
+                for (int o = kSegLanes / 2; o > 0; o >>= 1)
+                    v += __shfl_down_sync(mask, v, o, kSegLanes);
+                if (sub == 0 && w.ck != CFA_NO_CK) atomicAdd(a.ck + w.ck, v);
+            } else if (sub == 0) {
+                atomicCAS(a.status, 0, 1);
+            }
+        }
+        w = wn;
+        group = next;
+    }
 }
 
 /* ---- column slices: blocks of strided rows -------------------------------------------- */
@@ -591,6 +721,10 @@ const kernel_fn kKernels[CFA_N_CLASSES] = {
     cfa_unpack_kernel<0>, cfa_unpack_kernel<1>, cfa_unpack_kernel<2>,
     cfa_unpack_kernel<3>, cfa_unpack_kernel<4>, cfa_unpack_kernel<5>,
     cfa_unpack_kernel<6>, cfa_unpack_kernel<7>, cfa_unpack_kernel<8>};
+const kernel_fn kTiny[CFA_N_CLASSES] = {
+    cfa_tiny_kernel<0>, cfa_tiny_kernel<1>, cfa_tiny_kernel<2>,
+    cfa_tiny_kernel<3>, cfa_tiny_kernel<4>, cfa_tiny_kernel<5>,
+    cfa_tiny_kernel<6>, cfa_tiny_kernel<7>, cfa_tiny_kernel<8>};
 
 } // namespace
 
@@ -630,7 +764,10 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
     a.ck = ck;
     a.status = status;
     const uint64_t grid = items < (uint64_t)grid_cap ? items : (uint64_t)grid_cap;
-    kKernels[cls]<<<(unsigned)grid, kThreads, 0, stream>>>(a);
+    /* tiny pieces alone take the tiny kernel (same occupancy class as the combined one, so the
+     * same grid cap holds) */
+    if (n_slabs == 0) kTiny[cls]<<<(unsigned)grid, kThreads, 0, stream>>>(a);
+    else kKernels[cls]<<<(unsigned)grid, kThreads, 0, stream>>>(a);
     return cudaGetLastError();
 }
 

@@ -261,6 +261,38 @@ def test_element_sizes_1_4_8():
         load_and_compare(m, "pinned", chunk=chunk)
 
 
+def _tiny_phase_manifest(n=3000, dst_phase=8, seed=17):
+    """Only tiny pieces (below the 8 KiB line), of every element size: half at source offsets
+    with the destinations' phase within 16 bytes (the tiny kernel's one-round path, partial first
+    and last vectors included), half at other element-aligned offsets (its fallback)."""
+    from workloads import Manifest
+    rng = np.random.default_rng(seed)
+    kinds = [("u8", 1), ("bf16", 2), ("f32", 4), ("i64", 8)]
+    ents, dsts, off = [], [], 0
+    for k in range(n):
+        dt, es = kinds[k % 4]
+        nel = max(1, int(rng.integers(1, 8000)) // es)
+        off = (off + es - 1) // es * es
+        if k % 2 == 0:
+            off += (dst_phase - off) % 16          # the destination's phase
+        else:
+            off += es * int(rng.integers(0, 16 // es))
+        dsts.append({"name": f"d{k}", "dtype": dt, "shape": (nel,)})
+        ents.append({"name": f"e{k}", "dtype": dt, "shape": (nel,), "offset": off, "dst": k})
+        off += nel * es
+    return Manifest("tiny_phases", ents, dsts, off + 32, "bits", seed)
+
+
+@pytest.mark.parametrize("kind", ["device", "pinned", "direct_pinned"])
+def test_tiny_only_launches_at_every_phase(kind):
+    m = _tiny_phase_manifest()
+    # whole-blob chunks (one tiny-only launch), and 64 KiB chunks that cut pieces at chunk
+    # starts (source phase 0) and ends
+    for chunk in (1 << 30, 64 << 10):
+        st = load_and_compare(m, kind, chunk=chunk, misalign=8, host_slots=0)
+        assert st["n_slabs"] == 0 and st["n_bulk"] == 0 and st["n_tiny"] >= m.n_entries
+
+
 def test_back_to_back_loads_and_reuse():
     """Loads on one plan run in order; the plan can be reused; the last load wins."""
     m = cfg_dense()

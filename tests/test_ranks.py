@@ -102,11 +102,17 @@ def test_bench_labels_and_traffic_record(monkeypatch):
     assert dt == "u16+u32+u8" and cls == 0
     with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
         rec = json.load(f)["llama3_8b_bf16"]
-    monkeypatch.setattr(bench, "kernel_source_hash", lambda: rec["kernel_sha256"])
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda files=None: rec["kernel_sha256"])
     assert bench.recorded_traffic("llama3_8b_bf16") == rec["dram_bytes_per_launch"]
-    monkeypatch.setattr(bench, "kernel_source_hash", lambda: "0" * 64)
+    monkeypatch.setattr(bench, "kernel_source_hash", lambda files=None: "0" * 64)
     assert bench.recorded_traffic("llama3_8b_bf16") is None
     assert bench.recorded_traffic("no_such_workload") is None
+    # a record names the sources of the kernel it captured; the hash covers those only
+    monkeypatch.undo()
+    files = tuple(rec.get("sources", bench.KERNEL_SOURCES))
+    assert len(bench.kernel_source_hash(files)) == 64
+    st = {"n_bulk": 3, "n_slabs": 0, "n_tiny": 5, "n_strided": 0}
+    assert bench.kernel_names(st) == "cfa_bulk_kernel (TMA bulk copies) + cfa_tiny_kernel (tiny pieces)"
 
 
 def test_attribution_sizes_fit_any_checkpoint():

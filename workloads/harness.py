@@ -97,12 +97,64 @@ class CallbackSource:
         return s
 
 
+class _HugePinned:
+    """n bytes of page-locked host memory: an anonymous mapping aligned to 512 MiB with
+    MADV_HUGEPAGE (transparent huge pages where the kernel allows them), page-locked with
+    cudaHostRegister after it has been written.  Unregistered and unmapped when the last tensor
+    over it is freed.  torch's pinned allocator instead rounds a request up to a power of two
+    (93.6 GB -> 128 GiB) and uses the base pages."""
+
+    ALIGN = 512 << 20
+
+    def __init__(self, n):
+        self.libc = ctypes.CDLL(None, use_errno=True)
+        self.libc.mmap.restype = ctypes.c_void_p
+        self.libc.mmap.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_int,
+                                   ctypes.c_int, ctypes.c_long]
+        self.libc.munmap.argtypes = [ctypes.c_void_p, ctypes.c_size_t]
+        self.libc.madvise.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int]
+        self.n = n
+        self.size = n + self.ALIGN
+        self.p = self.libc.mmap(None, self.size, 0x3, 0x22, -1, 0)  # RW, PRIVATE|ANONYMOUS
+        if self.p is None or self.p == ctypes.c_void_p(-1).value:
+            raise OSError(ctypes.get_errno(), "mmap of the pinned blob failed")
+        self.base = (self.p + self.ALIGN - 1) // self.ALIGN * self.ALIGN
+        self.libc.madvise(self.base, n, 14)  # MADV_HUGEPAGE; a refusal only costs speed
+        self.registered = False
+
+    def register(self):
+        import torch
+        rc = torch.cuda.cudart().cudaHostRegister(self.base, self.n, 0)
+        if int(getattr(rc, "value", rc)) != 0:
+            raise RuntimeError(f"cudaHostRegister failed ({rc})")
+        self.registered = True
+
+    def __del__(self):
+        try:
+            if self.registered:
+                import torch
+                torch.cuda.cudart().cudaHostUnregister(self.base)
+            self.libc.munmap(self.p, self.size)
+        except Exception:
+            pass
+
+
 def pinned_blob(m, threads=None):
-    """A page-locked torch uint8 tensor holding the source bytes of the manifest's blob."""
+    """A page-locked torch uint8 tensor holding the source bytes of the manifest's blob (huge
+    pages, exact size; torch's pinned allocator if that cannot be had)."""
     import torch
-    t = torch.empty(m.source_bytes(), dtype=torch.uint8, pin_memory=True)
-    m.fill_source_ptr(t.data_ptr(), threads)
-    return t
+    n = m.source_bytes()
+    try:
+        h = _HugePinned(max(n, 1))
+        m.fill_source_ptr(h.base, threads)  # written first, so that the pages are huge
+        h.register()
+    except (OSError, RuntimeError, AttributeError):
+        t = torch.empty(n, dtype=torch.uint8, pin_memory=True)
+        m.fill_source_ptr(t.data_ptr(), threads)
+        return t
+    arr = (ctypes.c_uint8 * max(n, 1)).from_address(h.base)
+    arr._owner = h  # the tensor keeps the array, the array keeps the mapping
+    return torch.frombuffer(arr, dtype=torch.uint8)[:n]
 
 
 def device_blob(m, host=None):
