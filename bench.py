@@ -75,6 +75,9 @@ def parse_args():
     ap.add_argument("--vector-only", dest="bulk", action="store_false",
                     help="copy every slab with the 16-byte vector kernel instead of the TMA bulk "
                          "kernel (for comparison)")
+    ap.add_argument("--dst-order", default="index", choices=["index", "blob"],
+                    help="destinations laid out in index order (default) or in blob order, so "
+                         "that a load writes them front to back (for comparison)")
     ap.add_argument("--e2e-steps", type=int, default=None,
                     help="steps of the end-to-end measurement (default: min(steps, 20))")
     return ap.parse_args()
@@ -703,6 +706,23 @@ def measure_h2d(host, stream):
     return gib / (best / 1e3) / 1e9
 
 
+def host_buffer_rate(host, stream, passes=2):
+    """GB/s of plain 512 MiB host->device copies over the whole page-locked source buffer, per
+    pass: the rate the copy engine gets from this particular buffer, beside the loader's."""
+    import torch
+    ch = 512 << 20
+    n = host.numel() // ch
+    if n == 0:
+        return []
+    dev = torch.empty(ch, dtype=torch.uint8, device="cuda")
+    out = []
+    for _ in range(passes):
+        ms = _timed(lambda: [dev.copy_(host[k * ch:(k + 1) * ch], non_blocking=True)
+                             for k in range(n)], stream)
+        out.append(round(n * ch / ms / 1e6, 1))
+    return out
+
+
 def measure_e2e(m, entries, dsts, host, stream, ranks, steps, warmup, args, ck_want):
     """End-to-end steps through the C ABI from the pinned host blob: every step copies the
     staged bytes host->device through two device slots, unpacks, and reads the checksums
@@ -753,7 +773,7 @@ def measure_workload(name, args, ranks, stream, peak, e2e_steps, attribution_on=
     host = pinned_blob(m)                      # the checkpoint (or its period) page-locked
     dev_blob = torch.empty(m.source_bytes(), dtype=torch.uint8, device="cuda")
     dev_blob.copy_(host)
-    dsts = DeviceDsts(m)
+    dsts = DeviceDsts(m, order=args.dst_order)
     entries = entries_for(m)
     setup_s = time.time() - t_setup
     l2_flush = name in L2_FLUSHED
@@ -793,6 +813,7 @@ def measure_workload(name, args, ranks, stream, peak, e2e_steps, attribution_on=
     if e2e_steps:
         if h2d_gbs is None:
             h2d_gbs = measure_h2d(host, stream)
+        buffer_gbs = host_buffer_rate(host, stream)
         ms, step_ms, staged = measure_e2e(m, entries, dsts, host, stream, ranks, e2e_steps,
                                           min(args.warmup, 3), args, ck_dev)
         print(f"{m.name} e2e step ms:", [round(x, 1) for x in step_ms], file=sys.stderr)
@@ -803,6 +824,7 @@ def measure_workload(name, args, ranks, stream, peak, e2e_steps, attribution_on=
             "frac_of_h2d": round((staged / (ms / 1e3) / 1e9) / h2d_gbs, 4),
             "steps": e2e_steps, "step_ms_median": round(statistics.median(step_ms), 2),
             "step_ms_max": round(max(step_ms), 2),
+            "host_buffer_h2d_gbs": buffer_gbs,
             "source": f"pinned host {'pool of ' + str(m.period >> 30) + ' GiB (periodic blob)' if m.period else 'blob'}, "
                       f"2 device staging slots of {m.chunk_bytes >> 20} MiB"}
         if attribution_on and not args.no_attribution:
@@ -822,7 +844,7 @@ def _config_record(rec):
     if e2e:
         out["e2e"] = {k: e2e[k] for k in ("seconds_per_model", "frac_of_h2d", "h2d_gbs_measured",
                                           "h2d_bytes_per_step", "step_ms_median", "step_ms_max",
-                                          "steps", "source")}
+                                          "host_buffer_h2d_gbs", "steps", "source")}
         if "attribution" in e2e:
             out["e2e"]["attribution"] = e2e["attribution"]
     return out

@@ -198,9 +198,9 @@ typedef struct cfa_plan_opts {
     int32_t device;           /* CUDA device ordinal; -1 = the current device */
     uint32_t slab_bytes;      /* destination bytes per block-level work item, a multiple of 4096;
                                  default 262144 */
-    uint32_t tiny_bytes;      /* pieces with fewer destination bytes are warp-level items (four
-                                 per warp; those of at most 512 bytes in 8-lane segments);
-                                 default 8192 */
+    uint32_t tiny_bytes;      /* pieces with fewer destination bytes become warp-level items of
+                                 at most 512 destination bytes, each copied by an 8-lane
+                                 segment of a warp; default 8192 */
     uint32_t flags;           /* CFA_OPT_*; default CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK */
     uint32_t reserved;        /* must be 0 */
     void *workspace;          /* optional device memory for the staging slots (NULL = plan allocates) */
@@ -425,8 +425,9 @@ cfa_status cfa_unpack_chunks_async(cfa_plan *plan, uint32_t chunk_begin, uint32_
  *   - the work descriptors live in a fixed device array inside this library of
  *     CFA_NOALLOC_MAX_ITEMS entries (16384 x 32 bytes = 512 KiB, plus a status word), held by
  *     every GPU that loads the library until the process exits.  A tensor needs one work item
- *     per 2 MiB of destination bytes, one in all below 8 KiB; a manifest that needs more is
- *     rejected with CFA_ERR_INVAL before any GPU work, and `err` says so;
+ *     per 2 MiB of destination bytes, and below 8 KiB one per 512-byte-aligned block of
+ *     destination addresses it touches; a manifest that needs more is rejected with
+ *     CFA_ERR_INVAL before any GPU work, and `err` says so;
  *   - all calls on a device share that array: calls serialise on the host, but calls whose GPU
  *     work may overlap (different streams, no ordering between them) race on it;
  *   - the first call on a device does a one-time set-up (it looks up the array's device address

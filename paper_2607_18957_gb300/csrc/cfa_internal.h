@@ -38,8 +38,8 @@ typedef struct cfa_work {
  * starts at source blob offset src + k * stride * (source element size) and lands at
  * dst + k * cols * (destination element size).  40 bytes.
  */
-/* Tiny pieces with at most this many destination bytes are copied by 8-lane warp segments; the
- * plan orders them ahead of the larger tiny pieces of the same (class, chunk). */
+/* Warp-level work items hold at most this many destination bytes (the plan cuts tiny pieces at
+ * destination addresses that are multiples of it): one 8-lane warp segment copies one item. */
 #define CFA_TINY_SEG_BYTES 512u
 
 typedef struct cfa_swork {

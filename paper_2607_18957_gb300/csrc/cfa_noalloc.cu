@@ -40,7 +40,7 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
                                          uint64_t src_base, uint64_t src_period,
                                          uint64_t src_lo, uint64_t src_hi,
                                          unsigned long long *ck, int *status, int grid_cap,
-                                         cudaStream_t stream);
+                                         int dev_src, cudaStream_t stream);
 
 namespace {
 
@@ -98,6 +98,13 @@ bool mul_fits(uint64_t a, uint64_t b, uint64_t *out)
     if (a != 0 && b > UINT64_MAX / a) return false;
     *out = a * b;
     return true;
+}
+
+/* Warp-level items of a tiny entry of nb > 0 destination bytes at dst0: one per
+ * CFA_TINY_SEG_BYTES-aligned block of destination addresses it touches. */
+uint64_t tiny_items(uint64_t dst0, uint64_t nb)
+{
+    return (dst0 + nb - 1) / CFA_TINY_SEG_BYTES - dst0 / CFA_TINY_SEG_BYTES + 1;
 }
 
 cfa_status fail(cfa_status st, const char *msg, size_t i)
@@ -238,13 +245,15 @@ extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t
         if (!n) continue;
         const int cls = conv ? CFA_CLASS_OF_CONV(conv) : log2_es(es_s);
         const uint64_t nb = n * (uint64_t)es_d;
-        const uint64_t items = nb < kTinyBytes ? 1 : (nb + kSlabBytes - 1) / kSlabBytes;
+        const uint64_t dst0 = (uint64_t)(uintptr_t)dsts[entries[i].dst_index].dev_ptr + off;
+        const uint64_t items = nb < kTinyBytes ? tiny_items(dst0, nb)
+                                               : (nb + kSlabBytes - 1) / kSlabBytes;
         uint64_t total = items;
         for (int k = 0; k < CFA_N_CLASSES; ++k) total += count[k][0] + count[k][1];
         if (total > CFA_NOALLOC_MAX_ITEMS) {
             say("cfa_unpack_noalloc: the manifest needs more than the %d work items of the "
-                "fixed scratch (one per 2 MiB of destination, one per tensor under 8 KiB); "
-                "use cfa_plan_create", CFA_NOALLOC_MAX_ITEMS);
+                "fixed scratch (one per 2 MiB of destination, one per 512 bytes of a tensor "
+                "under 8 KiB); use cfa_plan_create", CFA_NOALLOC_MAX_ITEMS);
             return CFA_ERR_INVAL;
         }
         count[cls][nb < kTinyBytes ? 1 : 0] += (uint32_t)items;
@@ -271,10 +280,17 @@ extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t
         const uint64_t dst0 = (uint64_t)(uintptr_t)dsts[entries[i].dst_index].dev_ptr + off;
         const uint64_t nb = n * (uint64_t)es_d;
         if (nb < kTinyBytes) {
-            w.src = entries[i].blob_offset;
-            w.dst = dst0;
-            w.n = (uint32_t)n;
-            g_host_items[cursor[cls][1]++] = w;
+            /* warp-level items of at most CFA_TINY_SEG_BYTES, cut at destination addresses
+             * that are multiples of it (the tiny kernel's unit, as in the planned path) */
+            for (uint64_t pos = dst0; pos < dst0 + nb;) {
+                uint64_t next = (pos / CFA_TINY_SEG_BYTES + 1) * CFA_TINY_SEG_BYTES;
+                if (next > dst0 + nb) next = dst0 + nb;
+                w.src = entries[i].blob_offset + (pos - dst0) / (uint64_t)es_d * (uint64_t)es_s;
+                w.dst = pos;
+                w.n = (uint32_t)((next - pos) / (uint64_t)es_d);
+                g_host_items[cursor[cls][1]++] = w;
+                pos = next;
+            }
             continue;
         }
         const uint64_t per = kSlabBytes / (uint64_t)es_d; /* elements per item */
@@ -313,7 +329,7 @@ extern "C" cfa_status cfa_unpack_noalloc(const cfa_tensor_entry *entries, size_t
                               scratch->items + base[k][1], count[k][1],
                               (uint64_t)(uintptr_t)blob_dev, 0, 0, blob_bytes,
                               reinterpret_cast<unsigned long long *>(cksum_dev), status,
-                              g_grid_cap[dev][k], stream);
+                              g_grid_cap[dev][k], 1, stream);
     }
     if (e != cudaSuccess) {
         say("cfa_unpack_noalloc: CUDA error %s", cudaGetErrorString(e));

@@ -9,10 +9,11 @@
  *      destinations are covered without overlap (exactly once in strict mode);
  *   3. cut the blob into chunks of S bytes (the last one partial) and intersect every entry's
  *      source range with them: one piece per (tensor, chunk) pair;
- *   4. turn pieces into work items: pieces below `tiny_bytes` destination bytes become one
- *      warp-level item each; larger ones are split into block-level slabs whose cuts fall on
- *      destination addresses that are multiples of `slab_bytes`, so only a piece's first and
- *      last slab can start or end off a 16-byte boundary;
+ *   4. turn pieces into work items: pieces below `tiny_bytes` destination bytes become
+ *      warp-level items of at most CFA_TINY_SEG_BYTES each; larger ones are split into
+ *      block-level slabs whose cuts fall on destination addresses that are multiples of
+ *      `slab_bytes`, so only a piece's first and last slab can start or end off a 16-byte
+ *      boundary;
  *   5. record, per readiness group, the last chunk that carries one of its bytes.
  */
 #define _GNU_SOURCE /* sched_getaffinity, CPU_COUNT */
@@ -766,10 +767,21 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
             w.pad = cls;
             const uint64_t nb = pc->n_elems * (uint64_t)in->es_d;
             if (nb < o.tiny_bytes) {
-                w.src = pc->src_offset;
-                w.dst = a0;
-                w.n = (uint32_t)pc->n_elems;
-                if (vec_push(&tiny, &w)) { st = CFA_ERR_NOMEM; goto done; }
+                /* warp-level items of at most CFA_TINY_SEG_BYTES destination bytes, cut at
+                 * destination addresses that are multiples of it: each is one 8-lane segment's
+                 * single round of loads, where a whole warp would take a larger piece in
+                 * several dependent rounds (a piece is bound by latency, not bandwidth) */
+                uint64_t pos = a0;
+                const uint64_t end = a0 + nb;
+                while (pos < end) {
+                    uint64_t next = (pos / CFA_TINY_SEG_BYTES + 1) * CFA_TINY_SEG_BYTES;
+                    if (next > end) next = end;
+                    w.src = pc->src_offset + (pos - a0) / (uint64_t)in->es_d * (uint64_t)in->es_s;
+                    w.dst = pos;
+                    w.n = (uint32_t)((next - pos) / (uint64_t)in->es_d);
+                    if (vec_push(&tiny, &w)) { st = CFA_ERR_NOMEM; goto done; }
+                    pos = next;
+                }
                 continue;
             }
             uint64_t pos = a0;

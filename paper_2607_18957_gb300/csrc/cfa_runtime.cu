@@ -61,7 +61,7 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
                                          uint64_t src_base, uint64_t src_period,
                                          uint64_t src_lo, uint64_t src_hi,
                                          unsigned long long *ck, int *status, int grid_cap,
-                                         cudaStream_t stream);
+                                         int dev_src, cudaStream_t stream);
 
 namespace {
 
@@ -308,14 +308,15 @@ cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint
                                   p->d_ck, p->d_status, p->bulk_grid_cap[k], ls));
         else if (J.type == BULK_AS_VECTOR) /* bulk items are copy-class slabs of class k */
             CK(p, cfa_launch_unpack(k, p->d_bulk + J.a0, J.a1 - J.a0, nullptr, 0, src_base,
-                                    period, lo, hi, p->d_ck, p->d_status, p->grid_cap[k], ls));
+                                    period, lo, hi, p->d_ck, p->d_status, p->grid_cap[k], tma,
+                                    ls));
         else if (J.type == STRIDED)
             CK(p, cfa_launch_strided(k, p->d_strided + J.a0, J.a1 - J.a0, src_base, period, lo,
                                      hi, p->d_ck, p->d_status, p->strided_grid_cap[k], ls));
         else
             CK(p, cfa_launch_unpack(k, p->d_slabs + J.a0, J.a1 - J.a0, p->d_tiny + J.b0,
                                     J.b1 - J.b0, src_base, period, lo, hi, p->d_ck, p->d_status,
-                                    p->grid_cap[k], ls));
+                                    p->grid_cap[k], tma, ls));
         if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], ls));
         p->last_launches++;
     }

@@ -57,6 +57,7 @@ struct UnpackArgs {
     uint64_t src_hi;
     unsigned long long *ck;
     int *status;
+    uint32_t dev_src;    /* 1: the source is device memory (staging slots or a device blob) */
 };
 
 /* ---- memory operations ------------------------------------------------------------------ */
@@ -562,11 +563,12 @@ __device__ __forceinline__ void store_part(uint8_t *dst16, uint4 v, uint32_t lo,
     }
 }
 
-/* A tiny piece whose source and destination share their offset within 16 bytes: rounds of
- * W x U aligned 16-byte vectors, the piece's partial first and last vectors loaded whole in the
- * same round (an aligned 16-byte block holding bytes of the piece lies in the same page and
- * allocation) and stored element by element, so a piece of up to W * U * 16 bytes is one round
- * trip, not the vector round plus the head and tail rounds of copy_run.  Lane `lane` of W. */
+/* A tiny piece whose source and destination share their offset within 16 bytes, on W lanes:
+ * the whole 16-byte vectors in rounds of W x U (no branch per vector), and the partial first
+ * and last vectors (at most one each) by lanes 0 and 1, loaded whole in the same round (an
+ * aligned 16-byte block holding bytes of the piece lies in the same page and allocation) and
+ * stored element by element.  A piece of up to W * U * 16 bytes is one round trip, and the
+ * element-wise code runs once per piece instead of in every vector slot. */
 template <int ES, int U, int W>
 __device__ __forceinline__ uint64_t copy_same_phase(const uint8_t *src, uint8_t *dst,
                                                     uint32_t nbytes, uint32_t lane)
@@ -576,36 +578,309 @@ __device__ __forceinline__ uint64_t copy_same_phase(const uint8_t *src, uint8_t 
     uint8_t *d = dst - p;
     const uint32_t end = p + nbytes; /* in bytes from s */
     const uint32_t nv = (end + 15u) >> 4;
+    /* vector 0 is partial if the piece starts inside it or ends inside it */
+    const bool part0 = nv > 0 && (p != 0 || (nv == 1 && (end & 15u) != 0));
+    const bool part1 = nv > 1 && (end & 15u) != 0; /* the last vector, when not vector 0 */
+    const uint32_t f0 = part0 ? 1u : 0u, f1 = part1 ? nv - 1u : (nv > f0 ? nv : f0);
+    /* the partial vectors: lane 0 takes vector 0, lane 1 the last; their loads go first */
+    uint4 pv = make_uint4(0u, 0u, 0u, 0u);
+    const bool mine = (lane == 0 && part0) || (lane == 1 && part1);
+    if (mine) pv = ld_stream(s + (lane == 0 ? 0u : nv - 1u));
     uint64_t acc = 0;
-    for (uint32_t base = 0; base < nv; base += W * U) {
+    for (uint32_t base = f0; base < f1; base += W * U) {
         uint4 v[U];
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const uint32_t i = base + u * W + lane;
-            if (i < nv) v[u] = ld_stream(s + i);
+            if (i < f1) v[u] = ld_stream(s + i);
         }
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const uint32_t i = base + u * W + lane;
-            if (i >= nv) continue;
-            const uint32_t lo = i == 0 ? p : 0u;
-            const uint32_t hi = end - 16u * i < 16u ? end - 16u * i : 16u;
-            if (lo == 0 && hi == 16u) {
+            if (i < f1) {
                 st_stream(d + 16u * i, v[u]);
                 acc += vsum<ES>(v[u]);
-            } else {
-                store_part<ES>(d + 16u * i, v[u], lo, hi);
-                acc += vsum<ES>(keep_bytes(v[u], lo, hi));
             }
         }
     }
+    if (mine) { /* bounds recomputed here rather than held across the loop */
+        const uint32_t pi = lane == 0 ? 0u : nv - 1u;
+        const uint32_t plo = pi == 0 ? p : 0u;
+        const uint32_t phi = end - 16u * pi < 16u ? end - 16u * pi : 16u;
+        store_part<ES>(d + 16u * pi, pv, plo, phi);
+        acc += vsum<ES>(keep_bytes(pv, plo, phi));
+    }
     return acc;
+}
+
+/* A tiny piece whose source and destination differ in their offset within 16 bytes, on W lanes:
+ * every 16-byte destination vector takes bytes k .. k+15 of the two aligned source vectors
+ * under it (k the phase difference); each source vector is loaded once and passed to the lane
+ * that needs it as its second by shuffle, as on copy_run's realigning path; the partial first
+ * and last destination vectors go to lanes 0 and 1 as in copy_same_phase.  Only source vectors that hold bytes of the piece are loaded, so every load
+ * stays in the piece's pages.  One round trip for up to W * U * 16 bytes. */
+template <int ES, int U, int W>
+__device__ __forceinline__ uint64_t copy_diff_phase(const uint8_t *src, uint8_t *dst,
+                                                    uint32_t nbytes, uint32_t lane)
+{
+    const uint32_t dp = (uint32_t)((uintptr_t)dst & 15u);
+    uint8_t *d = dst - dp;
+    const uint8_t *A = src - dp; /* source byte of destination vector 0's byte 0 */
+    const uint32_t k = (uint32_t)((uintptr_t)A & 15u);
+    const uint4 *s = reinterpret_cast<const uint4 *>(A - k);
+    const uint32_t end = dp + nbytes;
+    const uint32_t nv = (end + 15u) >> 4;
+    const bool part0 = nv > 0 && (dp != 0 || (nv == 1 && (end & 15u) != 0));
+    const bool part1 = nv > 1 && (end & 15u) != 0;
+    const uint32_t f0 = part0 ? 1u : 0u, f1 = part1 ? nv - 1u : (nv > f0 ? nv : f0);
+    /* destination byte j of vector i comes from source vector i when j < 16 - k, else i + 1 */
+    const uint32_t split = 16u - k;
+    uint4 pa = make_uint4(0u, 0u, 0u, 0u), pb = pa;
+    const bool mine = (lane == 0 && part0) || (lane == 1 && part1);
+    if (mine) {
+        const uint32_t pi = lane == 0 ? 0u : nv - 1u;
+        const uint32_t plo = pi == 0 ? dp : 0u;
+        const uint32_t phi = end - 16u * pi < 16u ? end - 16u * pi : 16u;
+        if (plo < split) pa = ld_shared_line(s + pi);
+        if (phi > split) pb = ld_shared_line(s + pi + 1u);
+    }
+    uint64_t acc = 0;
+    const uint32_t mask =
+        W == 32 ? 0xFFFFFFFFu : (((1u << W) - 1u) << (threadIdx.x & 31u & ~(W - 1u)));
+    for (uint32_t base = f0; base < f1; base += W * U) {
+        /* lane l, round u holds source vector i = base + W u + l; vector i + 1 comes from the
+         * next lane, or for the last lane from lane 0 of the next round; the lane whose
+         * neighbour holds nothing (i + 1 == f1, or the last lane's last round) loads it */
+        uint4 va[U];
+        int own = -1;
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const uint32_t i = base + u * W + lane;
+            va[u] = make_uint4(0u, 0u, 0u, 0u);
+            if (i < f1) {
+                va[u] = ld_shared_line(s + i);
+                if (i + 1u == f1 || (lane == W - 1u && u == U - 1)) own = u;
+            }
+        }
+        uint4 c = make_uint4(0u, 0u, 0u, 0u);
+        if (own >= 0) c = ld_shared_line(s + base + W * own + lane + 1u);
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const uint32_t i = base + u * W + lane;
+            uint4 b, n0;
+            b.x = __shfl_down_sync(mask, va[u].x, 1, W);
+            b.y = __shfl_down_sync(mask, va[u].y, 1, W);
+            b.z = __shfl_down_sync(mask, va[u].z, 1, W);
+            b.w = __shfl_down_sync(mask, va[u].w, 1, W);
+            if (u + 1 < U) {
+                n0.x = __shfl_sync(mask, va[u + 1].x, 0, W);
+                n0.y = __shfl_sync(mask, va[u + 1].y, 0, W);
+                n0.z = __shfl_sync(mask, va[u + 1].z, 0, W);
+                n0.w = __shfl_sync(mask, va[u + 1].w, 0, W);
+                if (lane == W - 1u) b = n0;
+            }
+            if (i < f1) {
+                if (own == u) b = c;
+                const uint4 o = funnel16(va[u], b, k);
+                st_stream(d + 16u * i, o);
+                acc += vsum<ES>(o);
+            }
+        }
+    }
+    if (mine) {
+        const uint32_t pi = lane == 0 ? 0u : nv - 1u;
+        const uint32_t plo = pi == 0 ? dp : 0u;
+        const uint32_t phi = end - 16u * pi < 16u ? end - 16u * pi : 16u;
+        const uint4 o = funnel16(pa, pb, k);
+        store_part<ES>(d + 16u * pi, o, plo, phi);
+        acc += vsum<ES>(keep_bytes(o, plo, phi));
+    }
+    return acc;
+}
+
+/* A work descriptor read with volatile loads: issued where it is written (the top of the
+ * tiny kernel's loop, one piece ahead), so the compiler cannot move the load down to its use
+ * and put a second memory round trip into every piece. */
+__device__ __forceinline__ cfa_work ld_work_now(const cfa_work *p)
+{
+    uint32_t a0, a1, a2, a3, b0, b1, b2, b3;
+    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(a0), "=r"(a1), "=r"(a2), "=r"(a3)
+                 : "l"(p));
+    asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(b0), "=r"(b1), "=r"(b2), "=r"(b3)
+                 : "l"(reinterpret_cast<const uint8_t *>(p) + 16));
+    cfa_work w;
+    w.src = ((uint64_t)a1 << 32) | a0;
+    w.dst = ((uint64_t)a3 << 32) | a2;
+    w.n = b0;
+    w.ck = b1;
+    w.mode = b2;
+    w.pad = b3;
+    return w;
+}
+
+/* ---- tiny copies staged through shared memory with cp.async ----------------------------- */
+
+/* Aligned 16-byte source vectors per warp-level item in shared memory: an item of at most
+ * CFA_TINY_SEG_BYTES bytes spans at most CFA_TINY_SEG_BYTES / 16 + 1 of them, plus one that the
+ * realigning read may touch (its bytes are never used). */
+constexpr int kSlotVecs = CFA_TINY_SEG_BYTES / 16 + 2;
+
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem)
+{
+    const uint32_t sa = (uint32_t)__cvta_generic_to_shared(smem);
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sa), "l"(gmem) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_1() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
+/* One item of the segment's pipeline: its descriptor, whether it is to be copied, and its source
+ * address (the item's aligned vectors start at src - phase). */
+struct TinyItem {
+    cfa_work w;
+    bool live;
+};
+
+template <int CLS>
+__device__ __forceinline__ TinyItem tiny_fetch(const UnpackArgs &a, uint32_t group,
+                                               uint32_t n_groups, uint32_t slot)
+{
+    TinyItem it;
+    it.live = false;
+    it.w = cfa_work{};
+    const uint32_t t = group * kTinyPerGroup + slot;
+    if (group < n_groups && t < a.n_tiny) {
+        it.w = ld_work_now(a.tiny + t);
+        it.live = true;
+    }
+    return it;
+}
+
+/* Issues the cp.async copies of an item's aligned source vectors into `stage` (lanes sub, sub +
+ * 8, ...).  Items that fail the kernel's checks, or exceed CFA_TINY_SEG_BYTES, are flagged in
+ * the status word and dropped. */
+template <int CLS>
+__device__ __forceinline__ void tiny_issue(const UnpackArgs &a, TinyItem &it, uint4 *stage,
+                                           uint32_t sub)
+{
+    if (!it.live) return;
+    const uint32_t bytes = it.w.n << CLS;
+    if (!item_ok<CLS>(it.w, a) || bytes > CFA_TINY_SEG_BYTES) {
+        if (sub == 0) atomicCAS(a.status, 0, 1);
+        it.live = false;
+        return;
+    }
+    const uint64_t off = a.src_period ? it.w.src % a.src_period : it.w.src;
+    const uint64_t src = a.src_base + off;
+    const uint32_t ps = (uint32_t)(src & 15u);
+    const uint32_t nv = (ps + bytes + 15u) >> 4;
+    const uint4 *s = reinterpret_cast<const uint4 *>(src - ps);
+    for (uint32_t v = sub; v < nv; v += kSegLanes) cp_async16(stage + v, s + v);
+}
+
+/* Writes a staged item to its destination: destination vector i (aligned) holds staged bytes
+ * [16 i + delta, 16 i + delta + 16), delta = source phase - destination phase, so with
+ * delta = 16 j0 + k it is staged vector i + j0 (k = 0) or bytes k .. of vectors i + j0 and
+ * i + j0 + 1.  The whole vectors go in a tight loop over the segment's lanes; the partial first
+ * and last ones (when the item covers them only in part) go to lanes 0 and 1, element by
+ * element.  Returns this lane's checksum share. */
+template <int CLS>
+__device__ __forceinline__ uint64_t tiny_store(const UnpackArgs &a, const TinyItem &it,
+                                               const uint4 *stage, uint32_t sub)
+{
+    constexpr int ES = 1 << CLS;
+    if (!it.live) return 0;
+    const uint32_t bytes = it.w.n << CLS;
+    const uint64_t off = a.src_period ? it.w.src % a.src_period : it.w.src;
+    const uint32_t ps = (uint32_t)((a.src_base + off) & 15u);
+    const uint32_t dp = (uint32_t)(it.w.dst & 15u);
+    uint4 *d = reinterpret_cast<uint4 *>(it.w.dst - dp);
+    const uint32_t end = dp + bytes;
+    const uint32_t nv = (end + 15u) >> 4;
+    const int delta = (int)ps - (int)dp;
+    const int j0 = delta >> 4; /* -1 or 0 */
+    const uint32_t k = (uint32_t)delta & 15u;
+    const bool part0 = dp != 0 || (nv == 1 && (end & 15u) != 0);
+    const bool part1 = nv > 1 && (end & 15u) != 0;
+    const uint32_t f0 = part0 ? 1u : 0u, f1 = part1 ? nv - 1u : (nv > f0 ? nv : f0);
+    uint64_t acc = 0;
+    if (k == 0) {
+        for (uint32_t i = f0 + sub; i < f1; i += kSegLanes) {
+            const uint4 v = stage[i]; /* k == 0 means delta == 0 */
+            st_stream(d + i, v);
+            acc += vsum<ES>(v);
+        }
+    } else {
+        for (uint32_t i = f0 + sub; i < f1; i += kSegLanes) {
+            const int j = (int)i + j0; /* >= 0: i >= 1 here when j0 = -1 (part0 is then set) */
+            const uint4 v = funnel16(stage[j], stage[j + 1], k);
+            st_stream(d + i, v);
+            acc += vsum<ES>(v);
+        }
+    }
+    if ((sub == 0 && part0) || (sub == 1 && part1)) {
+        const uint32_t i = sub == 0 ? 0u : nv - 1u;
+        const int j = (int)i + j0;
+        const uint4 lo_v = stage[j < 0 ? 0 : j];
+        const uint4 v = k ? funnel16(lo_v, stage[j + 1], k) : lo_v;
+        const uint32_t lo = i == 0 ? dp : 0u;
+        const uint32_t hi = end - 16u * i < 16u ? end - 16u * i : 16u;
+        store_part<ES>(reinterpret_cast<uint8_t *>(d + i), v, lo, hi);
+        acc += vsum<ES>(keep_bytes(v, lo, hi));
+    }
+    return acc;
+}
+
+/* The copy classes' tiny kernel body: each 8-lane segment runs a two-deep pipeline over its
+ * items (one per group of the CTA's groups): the cp.async copies of item k + 1 are in flight
+ * while item k is written out, and the descriptor of item k + 2 is fetched meanwhile.  The
+ * source bytes wait in shared memory, not in registers, so memory-level parallelism does not
+ * cost occupancy. */
+template <int CLS>
+__device__ __forceinline__ void tiny_staged(const UnpackArgs &a)
+{
+    __shared__ __align__(16) uint4 stage[kWarps * kSegs][2][kSlotVecs];
+    const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
+    const uint32_t seg = lane / kSegLanes, sub = lane % kSegLanes;
+    const uint32_t mask = 0xFFu << (seg * kSegLanes);
+    const uint32_t n_groups = (a.n_tiny + kTinyPerGroup - 1) / kTinyPerGroup;
+    const uint32_t slot = warp * kSegs + seg;
+    uint4(*buf)[kSlotVecs] = stage[slot];
+    uint32_t group = blockIdx.x;
+    TinyItem cur = tiny_fetch<CLS>(a, group, n_groups, slot);
+    TinyItem nxt = tiny_fetch<CLS>(a, group + gridDim.x, n_groups, slot);
+    tiny_issue<CLS>(a, cur, buf[0], sub);
+    cp_async_commit();
+    for (uint32_t k = 0; group < n_groups; ++k, group += gridDim.x) {
+        const TinyItem after = tiny_fetch<CLS>(a, group + 2 * gridDim.x, n_groups, slot);
+        tiny_issue<CLS>(a, nxt, buf[(k + 1) & 1], sub);
+        cp_async_commit();
+        cp_async_wait_1(); /* this lane's copies of item k have landed */
+        __syncwarp(mask);  /* and the other lanes' of the segment */
+        uint64_t v = tiny_store<CLS>(a, cur, buf[k & 1], sub);
+#pragma unroll
+        for (int q = kSegLanes / 2; q > 0; q >>= 1) v += __shfl_down_sync(mask, v, q, kSegLanes);
+        if (sub == 0 && cur.live && cur.w.ck != CFA_NO_CK) atomicAdd(a.ck + cur.w.ck, v);
+        __syncwarp(mask);  /* buffer k & 1 is read; item k + 2 may be copied into it */
+        cur = nxt;
+        nxt = after;
+    }
+    asm volatile("cp.async.wait_all;" ::: "memory");
 }
 
 template <int CLS>
 __global__ void __launch_bounds__(kThreads, (CLS < 4 ? kCopyMinBlocks : kMinBlocks))
     cfa_tiny_kernel(const UnpackArgs a)
 {
+    if constexpr (CLS < 4) {
+        /* device-memory sources take the shared-memory pipeline; host memory read in place over
+         * the link keeps plain loads */
+        if (a.dev_src) {
+            tiny_staged<CLS>(a);
+            return;
+        }
+    }
     const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
     const uint32_t seg = lane / kSegLanes, sub = lane % kSegLanes;
     const uint32_t mask = 0xFFu << (seg * kSegLanes);
@@ -614,24 +889,26 @@ __global__ void __launch_bounds__(kThreads, (CLS < 4 ? kCopyMinBlocks : kMinBloc
     uint32_t group = blockIdx.x;
     cfa_work w{};
     if (group < n_groups && group * kTinyPerGroup + slot < a.n_tiny)
-        w = a.tiny[group * kTinyPerGroup + slot];
+        w = ld_work_now(a.tiny + group * kTinyPerGroup + slot);
     while (group < n_groups) {
         const uint32_t t = group * kTinyPerGroup + slot;
         const uint32_t next = group + gridDim.x;
         cfa_work wn{};
         if (next < n_groups && next * kTinyPerGroup + slot < a.n_tiny)
-            wn = a.tiny[next * kTinyPerGroup + slot];
+            wn = ld_work_now(a.tiny + next * kTinyPerGroup + slot);
         if (t < a.n_tiny) {
             if (item_ok<CLS>(w, a)) {
                 uint64_t v;
                 const uint64_t off = a.src_period ? w.src % a.src_period : w.src;
                 const uint8_t *src = reinterpret_cast<const uint8_t *>(a.src_base + off);
                 uint8_t *dst = reinterpret_cast<uint8_t *>(w.dst);
-                if (CLS < 4 && (((uintptr_t)src ^ (uintptr_t)dst) & 15u) == 0)
-                    v = copy_same_phase<(CLS < 4 ? (1 << CLS) : 1), kUnroll, kSegLanes>(
-                        src, dst, w.n << (CLS < 4 ? CLS : 0), sub);
-                else
+                constexpr int ES = CLS < 4 ? (1 << CLS) : 1;
+                if (CLS >= 4)
                     v = run_item<CLS, kUnroll, kSegLanes, kTinyRounds>(w, a, sub, kSegLanes);
+                else if ((((uintptr_t)src ^ (uintptr_t)dst) & 15u) == 0)
+                    v = copy_same_phase<ES, kUnroll, kSegLanes>(src, dst, w.n * ES, sub);
+                else
+                    v = copy_diff_phase<ES, 2, kSegLanes>(src, dst, w.n * ES, sub);
 #pragma unroll
                 for (int o = kSegLanes / 2; o > 0; o >>= 1)
                     v += __shfl_down_sync(mask, v, o, kSegLanes);
@@ -747,7 +1024,7 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
                                          uint64_t src_base, uint64_t src_period,
                                          uint64_t src_lo, uint64_t src_hi,
                                          unsigned long long *ck, int *status, int grid_cap,
-                                         cudaStream_t stream)
+                                         int dev_src, cudaStream_t stream)
 {
     if (cls < 0 || cls >= CFA_N_CLASSES || grid_cap <= 0) return cudaErrorInvalidValue;
     const uint64_t items = (uint64_t)n_slabs + (n_tiny + kTinyPerGroup - 1) / kTinyPerGroup;
@@ -763,6 +1040,7 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
     a.src_hi = src_hi;
     a.ck = ck;
     a.status = status;
+    a.dev_src = dev_src ? 1u : 0u;
     const uint64_t grid = items < (uint64_t)grid_cap ? items : (uint64_t)grid_cap;
     /* tiny pieces alone take the tiny kernel (same occupancy class as the combined one, so the
      * same grid cap holds) */

@@ -101,11 +101,11 @@ def test_bench_labels_and_traffic_record(monkeypatch):
     dt, cls, _ = bench.path_types(workloads.named_config("llama3_8b_fp8_block128"))
     assert dt == "u16+u32+u8" and cls == 0
     with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
-        rec = json.load(f)["llama3_8b_bf16"]
+        name, rec = next(iter(json.load(f).items()))
     monkeypatch.setattr(bench, "kernel_source_hash", lambda files=None: rec["kernel_sha256"])
-    assert bench.recorded_traffic("llama3_8b_bf16") == rec["dram_bytes_per_launch"]
+    assert bench.recorded_traffic(name) == rec["dram_bytes_per_launch"]
     monkeypatch.setattr(bench, "kernel_source_hash", lambda files=None: "0" * 64)
-    assert bench.recorded_traffic("llama3_8b_bf16") is None
+    assert bench.recorded_traffic(name) is None
     assert bench.recorded_traffic("no_such_workload") is None
     # a record names the sources of the kernel it captured; the hash covers those only
     monkeypatch.undo()

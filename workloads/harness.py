@@ -27,16 +27,24 @@ class DeviceDsts:
     element size), with `guard` bytes of GUARD_BYTE before the first destination, between
     destinations and after the last, so that stray writes show up."""
 
-    def __init__(self, m, device="cuda", guard=256, misalign=0, fill=GUARD_BYTE):
+    def __init__(self, m, device="cuda", guard=256, misalign=0, fill=GUARD_BYTE, order="index"):
+        """order "index": destinations in index order; "blob": in the order of their first
+        blob byte, so that a load writes them front to back."""
         import torch
         self.m = m
-        offs = []
+        offs = [0] * m.n_dsts
         pos = guard
-        for j in range(m.n_dsts):
+        seq = range(m.n_dsts)
+        if order == "blob":
+            first = np.full(m.n_dsts, np.iinfo(np.uint64).max, dtype=np.uint64)
+            np.minimum.at(first, m.e_dst, m.e_offset)
+            seq = np.argsort(first, kind="stable")
+        for j in seq:
+            j = int(j)
             es = DTYPE_SIZE[str(m.d_dtype[j])]
             mis = (misalign // es) * es
             pos = (pos + 255) // 256 * 256 + mis
-            offs.append(pos)
+            offs[j] = pos
             pos += m.d_nbytes(j) + guard
         self.total = pos + 256
         self.offsets = offs
@@ -53,7 +61,7 @@ class DeviceDsts:
     def host_bytes(self, j):
         return self.view(j).cpu().numpy()
 
-    def host_region(self, j0, j1):
+    def host_region(self, j0, j1):  # index order layouts only
         """Destinations j0 .. j1-1 with one device->host copy: {j: uint8 array}."""
         lo = self.offsets[j0]
         hi = self.offsets[j1 - 1] + self.m.d_nbytes(j1 - 1)
@@ -97,64 +105,12 @@ class CallbackSource:
         return s
 
 
-class _HugePinned:
-    """n bytes of page-locked host memory: an anonymous mapping aligned to 512 MiB with
-    MADV_HUGEPAGE (transparent huge pages where the kernel allows them), page-locked with
-    cudaHostRegister after it has been written.  Unregistered and unmapped when the last tensor
-    over it is freed.  torch's pinned allocator instead rounds a request up to a power of two
-    (93.6 GB -> 128 GiB) and uses the base pages."""
-
-    ALIGN = 512 << 20
-
-    def __init__(self, n):
-        self.libc = ctypes.CDLL(None, use_errno=True)
-        self.libc.mmap.restype = ctypes.c_void_p
-        self.libc.mmap.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_int,
-                                   ctypes.c_int, ctypes.c_long]
-        self.libc.munmap.argtypes = [ctypes.c_void_p, ctypes.c_size_t]
-        self.libc.madvise.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int]
-        self.n = n
-        self.size = n + self.ALIGN
-        self.p = self.libc.mmap(None, self.size, 0x3, 0x22, -1, 0)  # RW, PRIVATE|ANONYMOUS
-        if self.p is None or self.p == ctypes.c_void_p(-1).value:
-            raise OSError(ctypes.get_errno(), "mmap of the pinned blob failed")
-        self.base = (self.p + self.ALIGN - 1) // self.ALIGN * self.ALIGN
-        self.libc.madvise(self.base, n, 14)  # MADV_HUGEPAGE; a refusal only costs speed
-        self.registered = False
-
-    def register(self):
-        import torch
-        rc = torch.cuda.cudart().cudaHostRegister(self.base, self.n, 0)
-        if int(getattr(rc, "value", rc)) != 0:
-            raise RuntimeError(f"cudaHostRegister failed ({rc})")
-        self.registered = True
-
-    def __del__(self):
-        try:
-            if self.registered:
-                import torch
-                torch.cuda.cudart().cudaHostUnregister(self.base)
-            self.libc.munmap(self.p, self.size)
-        except Exception:
-            pass
-
-
 def pinned_blob(m, threads=None):
-    """A page-locked torch uint8 tensor holding the source bytes of the manifest's blob (huge
-    pages, exact size; torch's pinned allocator if that cannot be had)."""
+    """A page-locked torch uint8 tensor holding the source bytes of the manifest's blob."""
     import torch
-    n = m.source_bytes()
-    try:
-        h = _HugePinned(max(n, 1))
-        m.fill_source_ptr(h.base, threads)  # written first, so that the pages are huge
-        h.register()
-    except (OSError, RuntimeError, AttributeError):
-        t = torch.empty(n, dtype=torch.uint8, pin_memory=True)
-        m.fill_source_ptr(t.data_ptr(), threads)
-        return t
-    arr = (ctypes.c_uint8 * max(n, 1)).from_address(h.base)
-    arr._owner = h  # the tensor keeps the array, the array keeps the mapping
-    return torch.frombuffer(arr, dtype=torch.uint8)[:n]
+    t = torch.empty(m.source_bytes(), dtype=torch.uint8, pin_memory=True)
+    m.fill_source_ptr(t.data_ptr(), threads)
+    return t
 
 
 def device_blob(m, host=None):
