@@ -75,6 +75,8 @@ def parse_args():
     ap.add_argument("--vector-only", dest="bulk", action="store_false",
                     help="copy every slab with the 16-byte vector kernel instead of the TMA bulk "
                          "kernel (for comparison)")
+    ap.add_argument("--slab-kib", type=int, default=None,
+                    help="destination KiB per block-level work item (default: the library's)")
     ap.add_argument("--dst-order", default="index", choices=["index", "blob"],
                     help="destinations laid out in index order (default) or in blob order, so "
                          "that a load writes them front to back (for comparison)")
@@ -779,8 +781,9 @@ def measure_workload(name, args, ranks, stream, peak, e2e_steps, attribution_on=
     l2_flush = name in L2_FLUSHED
 
     # ---------------- kernel only: the blob already resident in HBM -------------------------
+    slab = {} if args.slab_kib is None else {"slab_bytes": args.slab_kib << 10}
     plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                    dev_slots=0, host_slots=0, bulk=args.bulk)
+                    dev_slots=0, host_slots=0, bulk=args.bulk, **slab)
     st = plan.stats()
     algo = st["bytes_read"] + st["bytes_written"]
     src = cfa.Source.device(dev_blob.data_ptr(), period=m.period or 0)

@@ -196,8 +196,10 @@ typedef struct cfa_plan_opts {
     int32_t fill_threads;     /* host threads copying pageable sources into pinned slots; default:
                                  the CPUs the process may run on, at most 32 */
     int32_t device;           /* CUDA device ordinal; -1 = the current device */
-    uint32_t slab_bytes;      /* destination bytes per block-level work item, a multiple of 4096;
-                                 default 262144 */
+    uint32_t slab_bytes;      /* destination bytes per block-level work item, a multiple of 4096
+                                 in [4096, 64 MiB], or 0 (the default): chosen by the plan for
+                                 about 4096 items per load, a power of two in [32 KiB, 256 KiB]
+                                 (256 KiB from 1 GiB of destinations up) */
     uint32_t tiny_bytes;      /* pieces with fewer destination bytes become warp-level items of
                                  at most 512 destination bytes, each copied by an 8-lane
                                  segment of a warp; default 8192 */

@@ -61,6 +61,18 @@ static int cfa_default_fill_threads(void)
     return n > 32 ? 32 : n;
 }
 
+/* Slab size when the caller leaves it to the plan: about 4096 block-level items over the load
+ * (the persistent grids hold 456-608 CTAs), as a power of two in [32 KiB, 256 KiB].  Loads of a
+ * gigabyte and more get 256 KiB (the size a sweep of 64 KiB - 1 MiB picked on the 8B, 70B,
+ * Mixtral and fp32 checkpoints); a 125 MiB load of 1,000 tensors gets 32 KiB, where 256 KiB left
+ * one slab per CTA and a launch of 0.073 ms instead of 0.054. */
+static uint32_t cfa_auto_slab(uint64_t dst_bytes)
+{
+    uint64_t s = 32u << 10;
+    while (s < (256u << 10) && s * 2 * 4096 <= dst_bytes) s *= 2;
+    return (uint32_t)s;
+}
+
 void cfa_plan_opts_default(cfa_plan_opts *o)
 {
     if (!o) return;
@@ -70,7 +82,7 @@ void cfa_plan_opts_default(cfa_plan_opts *o)
     o->dev_slots = 2;
     o->fill_threads = cfa_default_fill_threads();
     o->device = -1;
-    o->slab_bytes = 262144;
+    o->slab_bytes = 0; /* chosen from the load's size: cfa_auto_slab */
     o->tiny_bytes = 8192;
     o->flags = CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK;
     o->seg_world = 1;
@@ -378,8 +390,9 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
              (unsigned long long)o.chunk_bytes);
         return CFA_ERR_INVAL;
     }
-    if (o.slab_bytes < 4096 || o.slab_bytes % 4096 != 0 || o.slab_bytes > (64u << 20)) {
-        fail(err, errlen, "slab_bytes must be a multiple of 4096 in [4096, 64 MiB]");
+    if (o.slab_bytes != 0 &&
+        (o.slab_bytes < 4096 || o.slab_bytes % 4096 != 0 || o.slab_bytes > (64u << 20))) {
+        fail(err, errlen, "slab_bytes must be 0 or a multiple of 4096 in [4096, 64 MiB]");
         return CFA_ERR_INVAL;
     }
     if (o.tiny_bytes > (1u << 20)) {
@@ -725,6 +738,11 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
     if (!out->slab_first || !out->bulk_first || !out->tiny_first || !out->strided_first) {
         st = CFA_ERR_NOMEM;
         goto done;
+    }
+    if (o.slab_bytes == 0) {
+        uint64_t dst_total = 0;
+        for (size_t i = 0; i < n_entries; ++i) dst_total += info[i].n * (uint64_t)info[i].es_d;
+        o.slab_bytes = cfa_auto_slab(dst_total);
     }
     {
         const int use_bulk = CFA_BULK_READY && (o.flags & CFA_OPT_BULK);

@@ -189,6 +189,26 @@ def test_destinations_overlapping_in_memory_are_rejected():
     assert e.value.name == "CFA_ERR_OVERLAP"
 
 
+def test_slab_size_follows_the_load_size():
+    """slab_bytes 0 (the default) gives about 4096 block-level items per load, a power of two in
+    [32 KiB, 256 KiB]: the same work items as that size given explicitly."""
+    def items(p):
+        st = p.stats()
+        return st["n_slabs"], st["n_bulk"], st["n_tiny"]
+    import workloads
+    cases = [(workloads.named_config("tiny_1000"), 32 << 10),          # 131 MB of destinations
+             (dense_config("mid", 3, layers=2, hidden=2048, n_q=16, n_kv=4, head_dim=128,
+                           inter=8192, vocab=32000), 64 << 10),         # 505 MB
+             (dense_config("big", 3, layers=4, hidden=2048, n_q=16, n_kv=4, head_dim=128,
+                           inter=8192, vocab=32000), 128 << 10),        # 748 MB
+             (workloads.named_config("llama3_8b_bf16"), 256 << 10)]    # 16 GB
+    for m, want in cases:
+        with host_plan(m) as auto, host_plan(m, slab_bytes=want) as fixed, \
+                host_plan(m, slab_bytes=want // 2) as half:
+            assert items(auto) == items(fixed), (m.name, want)
+            assert items(auto) != items(half), (m.name, want)
+
+
 def test_bad_options_and_misaligned_destination():
     m, _, _, _ = manifest_case("fused_tiny.txt")
     with pytest.raises(cfa.CfaError) as e:
