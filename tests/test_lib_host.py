@@ -47,6 +47,15 @@ def test_struct_layouts_match():
     assert lib.cfa_abi_sizeof(b"cfa_tensor_entry") == 112
     assert lib.cfa_abi_sizeof(b"nonsense") == 0
     assert lib.cfa_status_name(-2) == b"CFA_ERR_OVERLAP"
+    # every status code of cfa.h has its name in the library and in the binding
+    import re
+    with open(os.path.join(ROOT, "include", "cfa.h")) as f:
+        codes = dict((int(v), k) for k, v in
+                     re.findall(r"#define (CFA_OK|CFA_ERR_\w+)\s+\(?(-?\d+)\)?", f.read()))
+    assert codes[-14] == "CFA_ERR_SUSPECT" and codes[-15] == "CFA_ERR_GATHER"
+    for v, name in codes.items():
+        assert lib.cfa_status_name(v) == name.encode(), name
+        assert _lib.STATUS[v] == name
 
 
 FAKE_BASE = 0x7F00_0000_0000
