@@ -32,6 +32,20 @@ static cfa_tensor_entry entry(const char *name, int64_t rows, uint64_t off, int6
     return e;
 }
 
+/* A host-only plan never loads, so its gather step is never called. */
+static int gather_never_called(void *user, void *chunk_dev, uint64_t segment_bytes, int32_t world,
+                               int32_t rank, uint32_t chunk, cfa_stream stream)
+{
+    (void)user;
+    (void)chunk_dev;
+    (void)segment_bytes;
+    (void)world;
+    (void)rank;
+    (void)chunk;
+    (void)stream;
+    return 1;
+}
+
 int main(void)
 {
     CHECK(1, cfa_abi_sizeof("cfa_tensor_entry") == sizeof(cfa_tensor_entry));
@@ -92,6 +106,31 @@ int main(void)
     CHECK(40, cfa_plan_create(e, 3, &d, 1, 392, &o, &plan) == CFA_ERR_OVERLAP && !plan);
     CHECK(41, strstr(cfa_last_error(NULL), "overlap") != NULL);
     CHECK(42, strcmp(cfa_status_name(CFA_ERR_OVERLAP), "CFA_ERR_OVERLAP") == 0);
+
+    /* segmented loading: 2 ranks, one 512-byte chunk holding the 392-byte blob; rank 0's
+     * segment is bytes 0 .. 255, rank 1's 256 .. 391 (136 bytes), and a segmented host-only plan
+     * stages exactly its segment; chunks must be multiples of 256 x ranks, and a segmented plan
+     * without a gather step is refused */
+    uint64_t so = 0, sn = 0;
+    CHECK(50, cfa_segment_range(392, 512, 2, 1, 0, &so, &sn) == CFA_OK && so == 256 && sn == 136);
+    CHECK(51, cfa_segment_range(392, 512, 2, 0, 0, &so, &sn) == CFA_OK && so == 0 && sn == 256);
+    CHECK(52, cfa_segment_range(392, 256, 2, 0, 0, &so, &sn) == CFA_ERR_INVAL);
+    CHECK(57, cfa_segment_range(392, 512, 2, 0, 1, &so, &sn) == CFA_ERR_INVAL);
+    e[1] = entry("k", 2, 328, 8);
+    o.chunk_bytes = 512;
+    o.seg_world = 2;
+    o.seg_rank = 1;
+    plan = NULL;
+    CHECK(53, cfa_plan_create(e, 3, &d, 1, 392, &o, &plan) == CFA_ERR_INVAL && !plan);
+    o.gather = gather_never_called;
+    CHECK(54, cfa_plan_create(e, 3, &d, 1, 392, &o, &plan) == CFA_OK && plan);
+    cfa_stats sst;
+    CHECK(55, cfa_get_stats(plan, &sst) == CFA_OK && sst.staged_bytes == 136);
+    CHECK(56, cfa_plan_destroy(plan) == CFA_OK);
+    o.seg_world = 1;
+    o.seg_rank = 0;
+    o.gather = NULL;
+    o.chunk_bytes = 256;
 
     /* a safetensors header in memory */
     static const char hdr[] = "{\"__metadata__\":{\"format\":\"pt\"},"

@@ -237,6 +237,22 @@ def test_gpu_segmented_load_matches_the_oracle(source_kind, world, rank):
 
 
 @pytest.mark.gpu
+@pytest.mark.parametrize("source_kind", ["pinned", "host"])
+def test_gpu_segmented_load_of_a_tensor_parallel_rank_with_conversions(source_kind):
+    """A rank's plan with column slices (read by the column-slice kernel from the gathered slot)
+    and fp32 -> bf16 conversions, over segments of 3 ranks."""
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    torch.cuda.set_device(0)
+    m = workloads.dense_config("seg_tp", 83, layers=2, hidden=256, n_q=4, n_kv=2, head_dim=64,
+                               inter=640, vocab=700, src_dtype="f32", align=4, jitter=3, tp=2,
+                               rank=1)
+    m.chunk_bytes = 256 * 3 * 128  # 96 KiB chunks: rows and tensors cross chunk boundaries
+    _gpu_case(m, source_kind, 3, 2, host_slots=2, dev_slots=2)
+
+
+@pytest.mark.gpu
 def test_gpu_segmented_load_of_a_blob_shorter_than_one_chunk():
     import torch
     if not torch.cuda.is_available():
