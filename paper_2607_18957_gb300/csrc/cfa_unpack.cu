@@ -24,6 +24,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "cfa_device.cuh"
 #include "cfa_internal.h"
 
@@ -744,12 +746,13 @@ struct TinyItem {
 
 template <int CLS>
 __device__ __forceinline__ TinyItem tiny_fetch(const UnpackArgs &a, uint32_t group,
-                                               uint32_t n_groups, uint32_t slot)
+                                               uint32_t n_groups, uint32_t slot,
+                                               uint32_t per_group)
 {
     TinyItem it;
     it.live = false;
     it.w = cfa_work{};
-    const uint32_t t = group * kTinyPerGroup + slot;
+    const uint32_t t = group * per_group + slot;
     if (group < n_groups && t < a.n_tiny) {
         it.w = ld_work_now(a.tiny + t);
         it.live = true;
@@ -760,7 +763,7 @@ __device__ __forceinline__ TinyItem tiny_fetch(const UnpackArgs &a, uint32_t gro
 /* Issues the cp.async copies of an item's aligned source vectors into `stage` (lanes sub, sub +
  * 8, ...).  Items that fail the kernel's checks, or exceed CFA_TINY_SEG_BYTES, are flagged in
  * the status word and dropped. */
-template <int CLS>
+template <int CLS, int L>
 __device__ __forceinline__ void tiny_issue(const UnpackArgs &a, TinyItem &it, uint4 *stage,
                                            uint32_t sub)
 {
@@ -776,7 +779,7 @@ __device__ __forceinline__ void tiny_issue(const UnpackArgs &a, TinyItem &it, ui
     const uint32_t ps = (uint32_t)(src & 15u);
     const uint32_t nv = (ps + bytes + 15u) >> 4;
     const uint4 *s = reinterpret_cast<const uint4 *>(src - ps);
-    for (uint32_t v = sub; v < nv; v += kSegLanes) cp_async16(stage + v, s + v);
+    for (uint32_t v = sub; v < nv; v += L) cp_async16(stage + v, s + v);
 }
 
 /* Writes a staged item to its destination: destination vector i (aligned) holds staged bytes
@@ -785,7 +788,7 @@ __device__ __forceinline__ void tiny_issue(const UnpackArgs &a, TinyItem &it, ui
  * i + j0 + 1.  The whole vectors go in a tight loop over the segment's lanes; the partial first
  * and last ones (when the item covers them only in part) go to lanes 0 and 1, element by
  * element.  Returns this lane's checksum share. */
-template <int CLS>
+template <int CLS, int L>
 __device__ __forceinline__ uint64_t tiny_store(const UnpackArgs &a, const TinyItem &it,
                                                const uint4 *stage, uint32_t sub)
 {
@@ -806,13 +809,13 @@ __device__ __forceinline__ uint64_t tiny_store(const UnpackArgs &a, const TinyIt
     const uint32_t f0 = part0 ? 1u : 0u, f1 = part1 ? nv - 1u : (nv > f0 ? nv : f0);
     uint64_t acc = 0;
     if (k == 0) {
-        for (uint32_t i = f0 + sub; i < f1; i += kSegLanes) {
+        for (uint32_t i = f0 + sub; i < f1; i += L) {
             const uint4 v = stage[i]; /* k == 0 means delta == 0 */
             st_stream(d + i, v);
             acc += vsum<ES>(v);
         }
     } else {
-        for (uint32_t i = f0 + sub; i < f1; i += kSegLanes) {
+        for (uint32_t i = f0 + sub; i < f1; i += L) {
             const int j = (int)i + j0; /* >= 0: i >= 1 here when j0 = -1 (part0 is then set) */
             const uint4 v = funnel16(stage[j], stage[j + 1], k);
             st_stream(d + i, v);
@@ -832,37 +835,46 @@ __device__ __forceinline__ uint64_t tiny_store(const UnpackArgs &a, const TinyIt
     return acc;
 }
 
-/* The copy classes' tiny kernel body: each 8-lane segment runs a two-deep pipeline over its
- * items (one per group of the CTA's groups): the cp.async copies of item k + 1 are in flight
- * while item k is written out, and the descriptor of item k + 2 is fetched meanwhile.  The
- * source bytes wait in shared memory, not in registers, so memory-level parallelism does not
- * cost occupancy. */
+/* The copy classes' tiny kernel body: each group of kStagedLanes lanes runs a two-deep pipeline
+ * over its items (one per group of the CTA's groups of items): the cp.async copies of item k + 1
+ * are in flight while item k is written out, and the descriptor of item k + 2 is fetched
+ * meanwhile.  The source bytes wait in shared memory (dynamic: two slots per lane group), not
+ * in registers, so memory-level parallelism does not cost occupancy; with four lanes per item a
+ * warp carries eight items at once, so the per-item work (descriptor, checks, checksum
+ * reduction) takes half the warp instructions it would with eight lanes. */
+constexpr int kStagedLanes = 4;
+constexpr int kStagedPerWarp = 32 / kStagedLanes;
+constexpr uint32_t kStagedPerGroup = kWarps * kStagedPerWarp;
+constexpr uint32_t kStagedSmem = kStagedPerGroup * 2 * kSlotVecs * sizeof(uint4);
+
 template <int CLS>
 __device__ __forceinline__ void tiny_staged(const UnpackArgs &a)
 {
-    __shared__ __align__(16) uint4 stage[kWarps * kSegs][2][kSlotVecs];
+    constexpr int L = kStagedLanes;
+    extern __shared__ __align__(16) uint4 tiny_stage[];
     const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
-    const uint32_t seg = lane / kSegLanes, sub = lane % kSegLanes;
-    const uint32_t mask = 0xFFu << (seg * kSegLanes);
-    const uint32_t n_groups = (a.n_tiny + kTinyPerGroup - 1) / kTinyPerGroup;
-    const uint32_t slot = warp * kSegs + seg;
-    uint4(*buf)[kSlotVecs] = stage[slot];
+    const uint32_t seg = lane / L, sub = lane % L;
+    const uint32_t mask = ((1u << L) - 1u) << (seg * L);
+    const uint32_t n_groups = (a.n_tiny + kStagedPerGroup - 1) / kStagedPerGroup;
+    const uint32_t slot = warp * kStagedPerWarp + seg;
+    uint4 *buf0 = tiny_stage + (size_t)slot * 2 * kSlotVecs, *buf1 = buf0 + kSlotVecs;
     uint32_t group = blockIdx.x;
-    TinyItem cur = tiny_fetch<CLS>(a, group, n_groups, slot);
-    TinyItem nxt = tiny_fetch<CLS>(a, group + gridDim.x, n_groups, slot);
-    tiny_issue<CLS>(a, cur, buf[0], sub);
+    TinyItem cur = tiny_fetch<CLS>(a, group, n_groups, slot, kStagedPerGroup);
+    TinyItem nxt = tiny_fetch<CLS>(a, group + gridDim.x, n_groups, slot, kStagedPerGroup);
+    tiny_issue<CLS, L>(a, cur, buf0, sub);
     cp_async_commit();
     for (uint32_t k = 0; group < n_groups; ++k, group += gridDim.x) {
-        const TinyItem after = tiny_fetch<CLS>(a, group + 2 * gridDim.x, n_groups, slot);
-        tiny_issue<CLS>(a, nxt, buf[(k + 1) & 1], sub);
+        const TinyItem after =
+            tiny_fetch<CLS>(a, group + 2 * gridDim.x, n_groups, slot, kStagedPerGroup);
+        tiny_issue<CLS, L>(a, nxt, (k & 1) ? buf0 : buf1, sub);
         cp_async_commit();
         cp_async_wait_1(); /* this lane's copies of item k have landed */
-        __syncwarp(mask);  /* and the other lanes' of the segment */
-        uint64_t v = tiny_store<CLS>(a, cur, buf[k & 1], sub);
+        __syncwarp(mask);  /* and the other lanes' of the group */
+        uint64_t v = tiny_store<CLS, L>(a, cur, (k & 1) ? buf1 : buf0, sub);
 #pragma unroll
-        for (int q = kSegLanes / 2; q > 0; q >>= 1) v += __shfl_down_sync(mask, v, q, kSegLanes);
+        for (int q = L / 2; q > 0; q >>= 1) v += __shfl_down_sync(mask, v, q, L);
         if (sub == 0 && cur.live && cur.w.ck != CFA_NO_CK) atomicAdd(a.ck + cur.w.ck, v);
-        __syncwarp(mask);  /* buffer k & 1 is read; item k + 2 may be copied into it */
+        __syncwarp(mask);  /* the slot of item k is read; item k + 2 may be copied into it */
         cur = nxt;
         nxt = after;
     }
@@ -1003,6 +1015,22 @@ const kernel_fn kTiny[CFA_N_CLASSES] = {
     cfa_tiny_kernel<3>, cfa_tiny_kernel<4>, cfa_tiny_kernel<5>,
     cfa_tiny_kernel<6>, cfa_tiny_kernel<7>, cfa_tiny_kernel<8>};
 
+/* Lets the tiny kernel of copy class cls use kStagedSmem bytes of dynamic shared memory on the
+ * current device (over the 48 KiB default), once per device and class. */
+cudaError_t tiny_smem_ready(int cls)
+{
+    static std::atomic<unsigned char> done[64][4];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64 || cls < 0 || cls >= 4) return cudaErrorInvalidValue;
+    if (done[dev][cls].load(std::memory_order_acquire)) return cudaSuccess;
+    e = cudaFuncSetAttribute(kTiny[cls], cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)kStagedSmem);
+    if (e == cudaSuccess) done[dev][cls].store(1, std::memory_order_release);
+    return e;
+}
+
 } // namespace
 
 /* Resident CTAs per SM of the class-cls kernel (0 if it cannot run). */
@@ -1043,9 +1071,18 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
     a.dev_src = dev_src ? 1u : 0u;
     const uint64_t grid = items < (uint64_t)grid_cap ? items : (uint64_t)grid_cap;
     /* tiny pieces alone take the tiny kernel (same occupancy class as the combined one, so the
-     * same grid cap holds) */
-    if (n_slabs == 0) kTiny[cls]<<<(unsigned)grid, kThreads, 0, stream>>>(a);
-    else kKernels[cls]<<<(unsigned)grid, kThreads, 0, stream>>>(a);
+     * same grid cap holds); its copy classes stage device-memory sources in dynamic shared
+     * memory */
+    if (n_slabs == 0) {
+        const bool staged = cls < 4 && dev_src;
+        if (staged) {
+            cudaError_t e = tiny_smem_ready(cls);
+            if (e != cudaSuccess) return e;
+        }
+        kTiny[cls]<<<(unsigned)grid, kThreads, staged ? kStagedSmem : 0, stream>>>(a);
+    } else {
+        kKernels[cls]<<<(unsigned)grid, kThreads, 0, stream>>>(a);
+    }
     return cudaGetLastError();
 }
 
