@@ -889,9 +889,18 @@ def run_ours(args):
         [n for n in args.configs.split(",") if n and n != args.workload]
     configs, manifests = {}, {}
     for name in names:
-        rec, mc = measure_workload(name, args, ranks, stream, peak,
-                                   0 if args.no_e2e else min(e2e_steps, 8),
-                                   attribution_on=(name == "llama3_8b_bf16"), h2d_gbs=h2d_gbs)
+        try:
+            rec, mc = measure_workload(name, args, ranks, stream, peak,
+                                       0 if args.no_e2e else min(e2e_steps, 8),
+                                       attribution_on=(name == "llama3_8b_bf16"),
+                                       h2d_gbs=h2d_gbs)
+        except Exception as e:  # noqa: BLE001 -- one workload must not cost the whole line
+            if world > 1:
+                raise  # the ranks' collectives would no longer match
+            print(f"{name}: {type(e).__name__}: {e}", file=sys.stderr, flush=True)
+            configs[name] = {"error": f"{type(e).__name__}: {e}"[:300]}
+            free_memory()
+            continue
         configs[name] = _config_record(rec)
         manifests[name] = mc
     clocks = sampler.stop()
@@ -903,14 +912,18 @@ def run_ours(args):
         cpu = {"value": round(gbs, 4), "unit": UNIT, "cores": 1, "host_cores": host_cores(),
                "kind": "oracle", "sample": desc}
         for name, mc in manifests.items():
-            if name == "llama3_8b_f32_rne":
-                configs[name]["cpu_baseline"] = cpu_baseline_all_cores(mc, name, host_cores())
-                continue
-            whole = name in CPU_FULL
-            gbs, nb, busy, desc, _ = cpu_baseline(mc, None if whole else 2.0)
-            configs[name]["cpu_baseline"] = {"value": round(gbs, 4), "unit": UNIT, "cores": 1,
-                                             "host_cores": host_cores(), "kind": "oracle",
-                                             "sample": desc}
+            try:
+                if name == "llama3_8b_f32_rne":
+                    configs[name]["cpu_baseline"] = cpu_baseline_all_cores(mc, name,
+                                                                           host_cores())
+                    continue
+                whole = name in CPU_FULL
+                gbs, nb, busy, desc, _ = cpu_baseline(mc, None if whole else 2.0)
+                configs[name]["cpu_baseline"] = {"value": round(gbs, 4), "unit": UNIT,
+                                                 "cores": 1, "host_cores": host_cores(),
+                                                 "kind": "oracle", "sample": desc}
+            except Exception as e:  # noqa: BLE001 -- reported in the line, not fatal
+                configs[name]["cpu_baseline"] = {"error": f"{type(e).__name__}: {e}"[:300]}
 
     if rank != 0:
         ranks.close()
