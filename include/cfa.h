@@ -201,8 +201,8 @@ typedef struct cfa_plan_opts {
                                  about 4096 items per load, a power of two in [32 KiB, 256 KiB]
                                  (256 KiB from 1 GiB of destinations up) */
     uint32_t tiny_bytes;      /* pieces with fewer destination bytes become warp-level items of
-                                 at most 512 destination bytes, each copied by an 8-lane
-                                 segment of a warp; default 8192 */
+                                 at most 512 destination bytes, each copied by four or eight
+                                 lanes of a warp; default 8192 */
     uint32_t flags;           /* CFA_OPT_*; default CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK */
     uint32_t reserved;        /* must be 0 */
     void *workspace;          /* optional device memory for the staging slots (NULL = plan allocates) */
@@ -215,7 +215,7 @@ typedef struct cfa_plan_opts {
      * shorter than one chunk.  Loads of such a plan take HOST, PINNED and CALLBACK sources,
      * never skip a chunk, and stage the rank's whole segments (cfa_stats.staged_bytes), not
      * only the byte ranges its own pieces read: the other ranks may need any of them.
-     * Default seg_world = 1 (off), seg_rank = 0, gather = NULL. */
+     * Default seg_world = 1 (0 and 1 are off), seg_rank = 0, gather = NULL. */
     int32_t seg_world;
     int32_t seg_rank;         /* this rank, 0 <= seg_rank < seg_world */
     cfa_gather_fn gather;     /* required when seg_world > 1 */
