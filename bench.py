@@ -267,6 +267,19 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs, sweep=False):
                        "chunks": [[round(float(x), 4) for x in row] for row in tl],
                        "layer_ready_ms": [round(float(x), 4) for x in t]}, f)
     plan.close()
+    # the same staged load with all of each chunk on the copy engine, and all of it pulled by
+    # the SMs (the default splits each chunk's ranges half and half)
+    for pct, key in ((0, "e2e_copy_engine_only"), (100, "e2e_sm_pull_only")):
+        plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                        dev_slots=2, host_slots=0, bulk=args.bulk,
+                        stage_slices=args.stage_slices, pull_percent=pct)
+        src = cfa.Source.pinned(host.data_ptr(), period=m.period or 0)
+        plan.load_async(src, stream)
+        plan.checksums()
+        steps = [_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
+                 for _ in range(3)]
+        plan.close()
+        out[key + "_step_ms"] = [round(x, 1) for x in steps]
     out["layer_ready_ms"] = {"first_group": round(float(t[0]), 2),
                              "median_group": round(float(np.median(t)), 2),
                              "last_group": round(float(t[-1]), 2),

@@ -204,7 +204,14 @@ typedef struct cfa_plan_opts {
                                  at most 512 destination bytes, each copied by four or eight
                                  lanes of a warp; default 8192 */
     uint32_t flags;           /* CFA_OPT_*; default CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK */
-    uint32_t reserved;        /* must be 0 */
+    uint32_t pull_percent;    /* staged loads: the share, in percent (0-100), of each chunk's
+                                 contiguous byte ranges that the plan's pull kernel copies into
+                                 the device slot with SM loads over the host link, beside the
+                                 copy engine's copies of the rest (0 = copy engine only).  On
+                                 GB300 the SMs read page-locked memory at the link rate even
+                                 from buffers the copy engine reads at half of it; the price is
+                                 one CTA per SM for the length of the transfer.  Default 50;
+                                 no effect on segmented plans and strided 2-D copies */
     void *workspace;          /* optional device memory for the staging slots (NULL = plan allocates) */
     uint64_t workspace_bytes; /* must be >= dev_slots * chunk_bytes when workspace is given */
     /* Segmented (multi-path) loading, section 4.2 "Optimization of Distributed Loading":

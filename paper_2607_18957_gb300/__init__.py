@@ -438,7 +438,8 @@ class Plan:
                  dev_slots=2, fill_threads=None, slab_bytes=0, tiny_bytes=8192, strict=True,
                  host_only=False, timing=False, bulk=True, no_merge=False, stage_slices=False,
                  device=-1,
-                 workspace=0, workspace_bytes=0, world=1, rank=0, gather=None):
+                 workspace=0, workspace_bytes=0, world=1, rank=0, gather=None,
+                 pull_percent=None):
         """world > 1 makes a segmented plan (cfa_plan_opts.seg_world): this process loads
         rank `rank`'s segment of every chunk and `gather(chunk_ptr, segment_bytes, world, rank,
         chunk, stream_handle)` assembles each chunk in the device slot (e.g. AllGather(group)).
@@ -470,6 +471,8 @@ class Plan:
                    (_lib.OPT_STAGE_SLICES if stage_slices else 0))
         o.workspace = workspace or None
         o.workspace_bytes = workspace_bytes
+        if pull_percent is not None:  # None: the library's default
+            o.pull_percent = pull_percent
         o.seg_world = world
         o.seg_rank = rank
         self._gather = None

@@ -43,7 +43,7 @@ class PlanOpts(ctypes.Structure):
                 ("dev_slots", ctypes.c_int32), ("fill_threads", ctypes.c_int32),
                 ("device", ctypes.c_int32), ("slab_bytes", ctypes.c_uint32),
                 ("tiny_bytes", ctypes.c_uint32), ("flags", ctypes.c_uint32),
-                ("reserved", ctypes.c_uint32), ("workspace", ctypes.c_void_p),
+                ("pull_percent", ctypes.c_uint32), ("workspace", ctypes.c_void_p),
                 ("workspace_bytes", ctypes.c_uint64), ("seg_world", ctypes.c_int32),
                 ("seg_rank", ctypes.c_int32), ("gather", ctypes.c_void_p),
                 ("gather_user", ctypes.c_void_p)]

@@ -86,6 +86,7 @@ void cfa_plan_opts_default(cfa_plan_opts *o)
     o->tiny_bytes = 8192;
     o->flags = CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK;
     o->seg_world = 1;
+    o->pull_percent = 50;
 }
 
 /* Rank `rank`'s segment of chunk `chunk` (section 4.2, distributed loading): the chunk is cut
@@ -400,7 +401,7 @@ cfa_status cfa_host_plan_build(const cfa_tensor_entry *entries, size_t n_entries
         return CFA_ERR_INVAL;
     }
     if (o.host_slots < 0 || o.dev_slots < 0 || o.fill_threads < 0 || o.fill_threads > 256 ||
-        o.reserved != 0 || o.device < -1) {
+        o.pull_percent > 100 || o.device < -1) {
         fail(err, errlen, "bad slot, thread or device option");
         return CFA_ERR_INVAL;
     }

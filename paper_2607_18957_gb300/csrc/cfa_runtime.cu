@@ -56,6 +56,8 @@ extern "C" cudaError_t cfa_launch_bulk(int log2es, const cfa_work *items, uint32
                                        unsigned long long *ck, int *status, int grid_cap,
                                        cudaStream_t stream);
 extern "C" cudaError_t cfa_bulk_selftest_timeout(int *status_host);
+extern "C" cudaError_t cfa_launch_pull(const void *src, void *dst, uint64_t bytes, int grid,
+                                       cudaStream_t stream);
 extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_t n_slabs,
                                          const cfa_work *tiny, uint32_t n_tiny,
                                          uint64_t src_base, uint64_t src_period,
@@ -132,6 +134,11 @@ struct cfa_plan {
     bool segmented = false;
     cudaStream_t gather_stream = nullptr;
     std::vector<cudaEvent_t> ev_gathered;
+    /* staged loads with pull_percent > 0: the SM pull kernel's stream, and per device slot the
+     * event after which the pulled part of the chunk is in the slot */
+    cudaStream_t pull_stream = nullptr;
+    std::vector<cudaEvent_t> ev_pulled;
+    int n_sms = 0;
     std::vector<cudaEvent_t> ev_dev_free, ev_h2d, ev_host_free, ev_filled, ev_layer;
     cudaEvent_t ev_begin = nullptr, ev_all = nullptr;
     std::vector<cudaEvent_t> t_h2d0, t_h2d1, t_k0, t_k1;
@@ -355,6 +362,8 @@ void release(cfa_plan *p)
             v.clear();
         };
         if (p->gather_stream) cudaStreamSynchronize(p->gather_stream);
+        if (p->pull_stream) cudaStreamSynchronize(p->pull_stream);
+        kill(p->ev_pulled);
         kill(p->ev_dev_free);
         kill(p->ev_h2d);
         kill(p->ev_gathered);
@@ -379,6 +388,7 @@ void release(cfa_plan *p)
         if (p->fill_stream) cudaStreamDestroy(p->fill_stream);
         if (p->copy_stream) cudaStreamDestroy(p->copy_stream);
         if (p->gather_stream) cudaStreamDestroy(p->gather_stream);
+        if (p->pull_stream) cudaStreamDestroy(p->pull_stream);
         if (p->aux_stream) cudaStreamDestroy(p->aux_stream);
         if (p->d_slabs) cudaFree(p->d_slabs);
         if (p->d_tiny) cudaFree(p->d_tiny);
@@ -407,6 +417,7 @@ cfa_status setup_device(cfa_plan *p)
     }
     int sms = 0;
     CK(nullptr, cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, p->device));
+    p->n_sms = sms;
     CK(nullptr, cudaDeviceGetAttribute(&p->pageable_access, cudaDevAttrPageableMemoryAccess,
                                        p->device));
     for (int k = 0; k < CFA_N_CLASSES; ++k) {
@@ -516,6 +527,10 @@ cfa_status setup_device(cfa_plan *p)
     if (p->segmented) {
         CK(nullptr, cudaStreamCreateWithFlags(&p->gather_stream, cudaStreamNonBlocking));
         if ((st = events(p->ev_gathered, p->n_dev_slots, false))) return st;
+    }
+    if (o.pull_percent > 0 && !p->segmented && p->n_dev_slots > 0) {
+        CK(nullptr, cudaStreamCreateWithFlags(&p->pull_stream, cudaStreamNonBlocking));
+        if ((st = events(p->ev_pulled, p->n_dev_slots, false))) return st;
     }
     if ((st = events(p->ev_host_free, p->n_host_slots, false))) return st;
     if ((st = events(p->ev_filled, p->n_host_slots, false))) return st;
@@ -803,6 +818,21 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             return false;
         };
         if (slices_in_place) CK(p, cudaStreamWaitEvent(p->direct_stream, p->ev_begin, 0));
+        /* the SM pull path: a share of each contiguous range goes to the pull kernel on the
+         * pull stream, the rest to the copy engine; the device must be able to read the host
+         * memory the chunk comes from (page-locked memory, or any memory with pageable access) */
+        bool pull_on = p->pull_stream != nullptr && hp.opts.pull_percent > 0;
+        if (pull_on && kind == CFA_SRC_PINNED && !p->pageable_access) {
+            cudaPointerAttributes at;
+            std::memset(&at, 0, sizeof at);
+            if (cudaPointerGetAttributes(&at, src->base) != cudaSuccess) {
+                cudaGetLastError();
+                at.type = cudaMemoryTypeUnregistered;
+            }
+            pull_on = at.type == cudaMemoryTypeHost;
+        }
+        if (pull_on) CK(p, cudaStreamWaitEvent(p->pull_stream, p->ev_begin, 0));
+        constexpr uint64_t kMinPull = 64u << 10; /* smaller shares stay with the copy engine */
         uint32_t k = 0; /* busy chunks so far: they take the slots in turn */
         for (uint32_t c = 0; c < hp.n_chunks; ++c) {
             if (!p->chunk_busy[c] || gather_failed) {
@@ -828,15 +858,37 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             uint8_t *dslot = p->d_slots + (uint64_t)ds * p->slot_bytes;
             CK(p, cudaStreamWaitEvent(p->copy_stream, p->ev_dev_free[ds], 0));
             if (timing) CK(p, cudaEventRecord(p->t_h2d0[c], p->copy_stream));
+            bool pulled = false;
             /* InMem -> InGPU: only the ranges the chunk's pieces read */
             for (uint32_t k = hp.copy_first[c]; k < hp.copy_first[c + 1]; ++k) {
                 const cfa_copy &cp = hp.copies[k];
                 const uint64_t at = cp.src - off;
                 if (slices_in_place && cp.rows > 1) continue; /* read in place instead */
-                if (cp.rows == 1)
-                    CK(p, cudaMemcpyAsync(dslot + at, static_cast<const uint8_t *>(hsrc) + at,
-                                          cp.width, cudaMemcpyHostToDevice, p->copy_stream));
-                else
+                if (cp.rows == 1) {
+                    /* bytes [at, at + ce) by the copy engine, the rest by the pull kernel; the
+                     * cut sits on a 16-byte boundary of the slot */
+                    uint64_t ce = cp.width;
+                    if (pull_on) {
+                        const uint64_t want = cp.width - cp.width * hp.opts.pull_percent / 100;
+                        const uint64_t cut = (at + want + 15) / 16 * 16 - at;
+                        if (cut < cp.width && cp.width - cut >= kMinPull) ce = cut;
+                    }
+                    if (ce)
+                        CK(p, cudaMemcpyAsync(dslot + at,
+                                              static_cast<const uint8_t *>(hsrc) + at, ce,
+                                              cudaMemcpyHostToDevice, p->copy_stream));
+                    if (ce < cp.width) {
+                        if (!pulled) {
+                            CK(p, cudaStreamWaitEvent(p->pull_stream, p->ev_dev_free[ds], 0));
+                            if (staged)
+                                CK(p, cudaStreamWaitEvent(p->pull_stream, p->ev_filled[hs], 0));
+                            pulled = true;
+                        }
+                        CK(p, cfa_launch_pull(static_cast<const uint8_t *>(hsrc) + at + ce,
+                                              dslot + at + ce, cp.width - ce, p->n_sms,
+                                              p->pull_stream));
+                    }
+                } else
                     CK(p, cudaMemcpy2DAsync(dslot + at, cp.pitch,
                                             static_cast<const uint8_t *>(hsrc) + at, cp.pitch,
                                             cp.width, cp.rows, cudaMemcpyHostToDevice,
@@ -845,8 +897,17 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             if (timing) CK(p, cudaEventRecord(p->t_h2d1[c], p->copy_stream));
             p->last_h2d++;
             ++k;
-            if (staged) CK(p, cudaEventRecord(p->ev_host_free[hs], p->copy_stream));
             CK(p, cudaEventRecord(p->ev_h2d[ds], p->copy_stream));
+            if (pulled) {
+                /* both transfers must be done before the unpack, and before the pinned host
+                 * slot is refilled: the caller's stream waits for both and marks the slot free */
+                CK(p, cudaEventRecord(p->ev_pulled[ds], p->pull_stream));
+                CK(p, cudaStreamWaitEvent(cs, p->ev_pulled[ds], 0));
+                CK(p, cudaStreamWaitEvent(cs, p->ev_h2d[ds], 0));
+                if (staged) CK(p, cudaEventRecord(p->ev_host_free[hs], cs));
+            } else if (staged) {
+                CK(p, cudaEventRecord(p->ev_host_free[hs], p->copy_stream));
+            }
             cudaEvent_t ready = p->ev_h2d[ds];
             if (p->segmented) {
                 /* InGPU for this rank's segment -> Gathered: the caller's collective fills the

@@ -934,6 +934,36 @@ __global__ void __launch_bounds__(kThreads, (CLS < 4 ? kCopyMinBlocks : kMinBloc
     }
 }
 
+/* ---- host -> device pull over the host link --------------------------------------------- */
+
+/* Copies bytes [0, n) from src (host memory the device reads over NVLink-C2C: page-locked, or any
+ * memory on devices that read pageable memory) to dst (device memory), which share their offset
+ * within 16 bytes: head and tail bytes one by one, the body in 16-byte vectors, four in flight
+ * per thread.  The staged pipeline's second transfer path beside the copy engine. */
+__global__ void __launch_bounds__(kThreads) cfa_pull_kernel(const uint8_t *__restrict__ src,
+                                                            uint8_t *__restrict__ dst, uint64_t n)
+{
+    const uint64_t tid = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const uint64_t nthr = (uint64_t)gridDim.x * blockDim.x;
+    uint64_t head = (16u - ((uintptr_t)dst & 15u)) & 15u;
+    if (head > n) head = n;
+    for (uint64_t e = tid; e < head; e += nthr) dst[e] = src[e];
+    const uint4 *s = reinterpret_cast<const uint4 *>(src + head);
+    uint4 *d = reinterpret_cast<uint4 *>(dst + head);
+    const uint64_t nv = (n - head) >> 4;
+    uint64_t i = tid;
+    for (; i + 3 * nthr < nv; i += 4 * nthr) {
+        const uint4 a = ld_stream(s + i), b = ld_stream(s + i + nthr);
+        const uint4 c = ld_stream(s + i + 2 * nthr), e = ld_stream(s + i + 3 * nthr);
+        st_stream(d + i, a);
+        st_stream(d + i + nthr, b);
+        st_stream(d + i + 2 * nthr, c);
+        st_stream(d + i + 3 * nthr, e);
+    }
+    for (; i < nv; i += nthr) st_stream(d + i, ld_stream(s + i));
+    for (uint64_t e = head + (nv << 4) + tid; e < n; e += nthr) dst[e] = src[e];
+}
+
 /* ---- column slices: blocks of strided rows -------------------------------------------- */
 
 struct StridedArgs {
@@ -1083,6 +1113,19 @@ extern "C" cudaError_t cfa_launch_unpack(int cls, const cfa_work *slabs, uint32_
     } else {
         kKernels[cls]<<<(unsigned)grid, kThreads, 0, stream>>>(a);
     }
+    return cudaGetLastError();
+}
+
+/* Pulls `bytes` from host memory at src into device memory at dst (same offset within 16
+ * bytes) on `stream` with a grid of `grid` CTAs. */
+extern "C" cudaError_t cfa_launch_pull(const void *src, void *dst, uint64_t bytes, int grid,
+                                       cudaStream_t stream)
+{
+    if (!bytes) return cudaSuccess;
+    if (!src || !dst || grid <= 0 || (((uintptr_t)src ^ (uintptr_t)dst) & 15u))
+        return cudaErrorInvalidValue;
+    cfa_pull_kernel<<<grid, kThreads, 0, stream>>>(static_cast<const uint8_t *>(src),
+                                                   static_cast<uint8_t *>(dst), bytes);
     return cudaGetLastError();
 }
 

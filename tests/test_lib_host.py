@@ -226,6 +226,11 @@ def test_bad_options_and_misaligned_destination():
     with pytest.raises(cfa.CfaError) as e:
         host_plan(m, slab_bytes=1000)
     assert e.value.name == "CFA_ERR_INVAL"
+    with pytest.raises(cfa.CfaError) as e:
+        host_plan(m, pull_percent=101)
+    assert e.value.name == "CFA_ERR_INVAL"
+    for pct in (0, 50, 100):
+        host_plan(m, pull_percent=pct).close()
     d = fake_dsts(m)
     d[0] = (d[0][0] + 1, d[0][1], d[0][2])
     with pytest.raises(cfa.CfaError) as e:
