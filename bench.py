@@ -324,16 +324,21 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs, sweep=False):
         out["host_memcpy_gbs"] = round(dst.size / (time.perf_counter() - t0) / 1e9, 2)
     out["host_threads"] = threads
     del dst
-    plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                    dev_slots=2, host_slots=2, fill_threads=threads, bulk=args.bulk)
-    src = cfa.Source.host(pageable.ctypes.data, period=m.period or 0)
-    plan.load_async(src, stream)
-    plan.checksums()
-    ms = min(_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
-             for _ in range(2))
-    plan.close()
-    out["e2e_pageable_s_per_model"] = round(ms / 1e3, 4)
-    out["e2e_pageable_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
+    # a pageable copy of the checkpoint as a HOST source: by default the SM pull kernel reads it
+    # straight into the device slots; with pull_percent 0 the fill threads copy it into the
+    # pinned ring and the copy engine takes it from there
+    for pct, key in ((None, "e2e_pageable"), (0, "e2e_pageable_ring")):
+        kw = {} if pct is None else {"pull_percent": pct}
+        plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
+                        dev_slots=2, host_slots=2, fill_threads=threads, bulk=args.bulk, **kw)
+        src = cfa.Source.host(pageable.ctypes.data, period=m.period or 0)
+        plan.load_async(src, stream)
+        plan.checksums()
+        ms = min(_timed(lambda: (plan.load_async(src, stream), plan.checksums()), stream)
+                 for _ in range(2))
+        plan.close()
+        out[key + "_s_per_model"] = round(ms / 1e3, 4)
+        out[key + "_gbs"] = round(m.blob_bytes / ms / 1e6, 2)
     if sweep:
         out["fill_threads_sweep"] = fill_thread_sweep(m, pageable, dsts, entries, stream, args,
                                                       part * threads)
@@ -379,7 +384,8 @@ def fill_thread_sweep(m, pageable, dsts, entries, stream, args, memcpy_bytes):
             list(ex.map(cp, range(t)))
             memcpy_gbs = part * t / (time.perf_counter() - t0) / 1e9
         plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                        dev_slots=2, host_slots=2, fill_threads=t, bulk=args.bulk)
+                        dev_slots=2, host_slots=2, fill_threads=t, bulk=args.bulk,
+                        pull_percent=0)  # the fill threads' ring, not the SM pull
         src = cfa.Source.host(pageable.ctypes.data, period=m.period or 0)
         plan.load_async(src, stream)
         plan.checksums()

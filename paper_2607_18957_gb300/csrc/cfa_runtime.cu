@@ -708,7 +708,13 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
         set_err(p, "pinned and device sources must be 256-byte aligned");
         return CFA_ERR_ALIGN;
     }
-    const bool staged = kind == CFA_SRC_HOST || kind == CFA_SRC_CALLBACK;
+    /* a pageable source on a device that reads pageable memory, with the pull path on: the pull
+     * kernel reads it straight into the device slots (no fill threads, no pinned host slots,
+     * no host memcpy); the copy engine cannot read pageable memory without blocking the call,
+     * so it takes no share, and column slices are read in place by their kernel */
+    const bool host_pull = kind == CFA_SRC_HOST && p->pull_stream && hp.opts.pull_percent > 0 &&
+                           p->pageable_access && ((uintptr_t)src->base & 15u) == 0;
+    const bool staged = (kind == CFA_SRC_HOST && !host_pull) || kind == CFA_SRC_CALLBACK;
     const bool in_place = kind == CFA_SRC_DEVICE || kind == CFA_SRC_HOST_DIRECT;
     if (p->segmented && in_place) {
         set_err(p, "a segmented plan loads from HOST, PINNED or CALLBACK sources only");
@@ -806,8 +812,9 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
          * through the slots as strided 2-D copies (slower than plain copies on the copy engine):
          * the column-slice kernels read them over the host link on the direct stream, in chunk
          * order and ahead of the copy ring, and each chunk's readiness also waits for them. */
-        const bool slices_in_place = kind == CFA_SRC_PINNED && hp.n_strided && !p->segmented &&
-                                     !(hp.opts.flags & CFA_OPT_STAGE_SLICES);
+        const bool slices_in_place =
+            ((kind == CFA_SRC_PINNED && !(hp.opts.flags & CFA_OPT_STAGE_SLICES)) || host_pull) &&
+            hp.n_strided && !p->segmented;
         const uint64_t seg_bytes = p->segmented ? S / (uint64_t)hp.opts.seg_world : 0;
         cfa_status gather_failed = CFA_OK;
         const size_t row = (size_t)hp.n_chunks + 1;
@@ -868,7 +875,9 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
                     /* bytes [at, at + ce) by the copy engine, the rest by the pull kernel; the
                      * cut sits on a 16-byte boundary of the slot */
                     uint64_t ce = cp.width;
-                    if (pull_on) {
+                    if (host_pull) {
+                        ce = 0;
+                    } else if (pull_on) {
                         const uint64_t want = cp.width - cp.width * hp.opts.pull_percent / 100;
                         const uint64_t cut = (at + want + 15) / 16 * 16 - at;
                         if (cut < cp.width && cp.width - cut >= kMinPull) ce = cut;
