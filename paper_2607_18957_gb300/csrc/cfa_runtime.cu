@@ -99,6 +99,13 @@ struct DeviceGuard {
     }
 };
 
+/* Bytes of one half of the checksum buffer: a word per entry (at least one) and the status
+ * word after them, so that one clear resets both. */
+inline size_t ck_clear_bytes(size_t n_entries)
+{
+    return ((n_entries ? n_entries : 1) + 1) * sizeof(unsigned long long);
+}
+
 } // namespace
 
 /* Kernels of one launch group beyond the first run on up to this many side streams. */
@@ -114,8 +121,17 @@ struct cfa_plan {
     int strided_grid_cap[CFA_N_CLASSES] = {0};
     cfa_work *d_slabs = nullptr, *d_tiny = nullptr, *d_bulk = nullptr;
     cfa_swork *d_strided = nullptr;
+    /* Two halves of checksums + status word: a load accumulates into the half cleared before
+     * it began and clears the other half, its predecessor's, on ck_stream beside its own work,
+     * so no clear sits between a load's start and its first kernel.  d_ck / d_status point into
+     * the half of the last load (or of cfa_unpack_chunks_async and cfa_reset_checksums). */
+    unsigned long long *d_ck_mem = nullptr;
+    size_t ck_half_words = 0;
+    int ck_half = 0;
     unsigned long long *d_ck = nullptr;
     int *d_status = nullptr;
+    cudaStream_t ck_stream = nullptr;
+    cudaEvent_t ev_ck_clear = nullptr;
     uint8_t *d_slots = nullptr;
     bool own_slots = false;
     uint64_t slot_bytes = 0;
@@ -347,6 +363,14 @@ cfa_status make_event(cfa_plan *p, cudaEvent_t *ev, bool timing)
     return CFA_OK;
 }
 
+/* Points d_ck / d_status at half h of the checksum buffer. */
+void use_ck_half(cfa_plan *p, int h)
+{
+    p->ck_half = h;
+    p->d_ck = p->d_ck_mem + (size_t)h * p->ck_half_words;
+    p->d_status = reinterpret_cast<int *>(p->d_ck + (p->ck_half_words - 1));
+}
+
 void release(cfa_plan *p)
 {
     if (!p) return;
@@ -356,6 +380,7 @@ void release(cfa_plan *p)
         if (p->copy_stream) cudaStreamSynchronize(p->copy_stream);
         if (p->ev_all) cudaEventSynchronize(p->ev_all);
         if (p->aux_stream) cudaStreamSynchronize(p->aux_stream);
+        if (p->ck_stream) cudaStreamSynchronize(p->ck_stream);
         auto kill = [](std::vector<cudaEvent_t> &v) {
             for (cudaEvent_t e : v)
                 if (e) cudaEventDestroy(e);
@@ -377,6 +402,8 @@ void release(cfa_plan *p)
         if (p->ev_begin) cudaEventDestroy(p->ev_begin);
         if (p->ev_all) cudaEventDestroy(p->ev_all);
         if (p->ev_fork) cudaEventDestroy(p->ev_fork);
+        if (p->ev_ck_clear) cudaEventDestroy(p->ev_ck_clear);
+        if (p->ck_stream) cudaStreamDestroy(p->ck_stream);
         if (p->direct_stream) cudaStreamSynchronize(p->direct_stream);
         if (p->ev_direct) cudaEventDestroy(p->ev_direct);
         if (p->direct_stream) cudaStreamDestroy(p->direct_stream);
@@ -394,8 +421,7 @@ void release(cfa_plan *p)
         if (p->d_tiny) cudaFree(p->d_tiny);
         if (p->d_bulk) cudaFree(p->d_bulk);
         if (p->d_strided) cudaFree(p->d_strided);
-        if (p->d_ck) cudaFree(p->d_ck);
-        if (p->d_status) cudaFree(p->d_status);
+        if (p->d_ck_mem) cudaFree(p->d_ck_mem);
         if (p->own_slots && p->d_slots) cudaFree(p->d_slots);
         if (p->h_slots) cudaFreeHost(p->h_slots);
     }
@@ -473,14 +499,15 @@ cfa_status setup_device(cfa_plan *p)
             CK(nullptr, cudaMemcpy(p->d_strided, hp.strided, hp.n_strided * sizeof(cfa_swork),
                                    cudaMemcpyHostToDevice));
     }
-    const size_t ck_bytes = (hp.n_entries ? hp.n_entries : 1) * sizeof(unsigned long long);
-    if (cudaMalloc(&p->d_ck, ck_bytes) != cudaSuccess ||
-        cudaMalloc(&p->d_status, sizeof(int)) != cudaSuccess) {
+    /* two halves of checksums with the status word after them: one clear resets both */
+    const size_t ck_bytes = ck_clear_bytes(hp.n_entries);
+    p->ck_half_words = ck_bytes / sizeof(unsigned long long);
+    if (cudaMalloc(&p->d_ck_mem, 2 * ck_bytes) != cudaSuccess) {
         set_err(nullptr, "cudaMalloc of the checksum buffer failed");
         return CFA_ERR_NOMEM;
     }
-    CK(nullptr, cudaMemset(p->d_ck, 0, ck_bytes));
-    CK(nullptr, cudaMemset(p->d_status, 0, sizeof(int)));
+    CK(nullptr, cudaMemset(p->d_ck_mem, 0, 2 * ck_bytes));
+    use_ck_half(p, 0);
 
     p->n_dev_slots = o.dev_slots;
     p->n_host_slots = o.host_slots;
@@ -506,6 +533,8 @@ cfa_status setup_device(cfa_plan *p)
     CK(nullptr, cudaStreamCreateWithFlags(&p->fill_stream, cudaStreamNonBlocking));
     CK(nullptr, cudaStreamCreateWithFlags(&p->copy_stream, cudaStreamNonBlocking));
     CK(nullptr, cudaStreamCreateWithFlags(&p->aux_stream, cudaStreamNonBlocking));
+    CK(nullptr, cudaStreamCreateWithFlags(&p->ck_stream, cudaStreamNonBlocking));
+    if ((st = make_event(nullptr, &p->ev_ck_clear, false))) return st;
     for (int j = 0; j < kSideStreams; ++j) {
         CK(nullptr, cudaStreamCreateWithFlags(&p->side_stream[j], cudaStreamNonBlocking));
         if ((st = make_event(nullptr, &p->ev_join[j], false))) return st;
@@ -781,14 +810,23 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
     p->last_h2d = 0;
     const bool timing = (hp.opts.flags & CFA_OPT_TIMING) != 0;
 
-    /* the load starts after the previous load of this plan and after prior work on cs */
+    /* the load starts after the previous load of this plan, after prior work on cs and after
+     * the clear of the checksum half it takes; it clears the other half for the next load */
     CK(p, cudaStreamWaitEvent(cs, p->ev_all, 0));
+    CK(p, cudaStreamWaitEvent(cs, p->ev_ck_clear, 0));
     CK(p, cudaEventRecord(p->ev_begin, cs));
     CK(p, cudaStreamWaitEvent(p->fill_stream, p->ev_begin, 0));
     CK(p, cudaStreamWaitEvent(p->copy_stream, p->ev_begin, 0));
-    if (hp.any_cksum)
-        CK(p, cudaMemsetAsync(p->d_ck, 0, hp.n_entries * sizeof(unsigned long long), cs));
-    CK(p, cudaMemsetAsync(p->d_status, 0, sizeof(int), cs));
+    use_ck_half(p, p->ck_half ^ 1);
+    {
+        unsigned long long *other = p->d_ck_mem + (size_t)(p->ck_half ^ 1) * p->ck_half_words;
+        CK(p, cudaStreamWaitEvent(p->ck_stream, p->ev_begin, 0));
+        if (hp.any_cksum)
+            CK(p, cudaMemsetAsync(other, 0, ck_clear_bytes(hp.n_entries), p->ck_stream));
+        else
+            CK(p, cudaMemsetAsync(other + (p->ck_half_words - 1), 0, sizeof(int), p->ck_stream));
+        CK(p, cudaEventRecord(p->ev_ck_clear, p->ck_stream));
+    }
     for (uint32_t l : p->layers_empty) CK(p, cudaEventRecord(p->ev_layer[l], cs));
 
     if (in_place) {
@@ -1142,9 +1180,8 @@ cfa_status cfa_reset_checksums(cfa_plan *p, cfa_stream stream)
 {
     if (!p || p->host_only) return CFA_ERR_INVAL;
     DeviceGuard g(p->device);
-    CK(p, cudaMemsetAsync(p->d_ck, 0, (p->hp.n_entries ? p->hp.n_entries : 1) * 8,
+    CK(p, cudaMemsetAsync(p->d_ck, 0, ck_clear_bytes(p->hp.n_entries),
                           reinterpret_cast<cudaStream_t>(stream)));
-    CK(p, cudaMemsetAsync(p->d_status, 0, sizeof(int), reinterpret_cast<cudaStream_t>(stream)));
     return CFA_OK;
 }
 

@@ -312,6 +312,39 @@ def test_back_to_back_loads_and_reuse():
     assert np.array_equal(ck, ref.cksum)
 
 
+def test_checksums_of_each_load_are_its_own():
+    """A load accumulates into the checksum half cleared before it and clears the other one for
+    the next load: read after each of several alternating loads, the checksums are that load's
+    alone; cfa_reset_checksums then clears the current half for cfa_unpack_chunks_async."""
+    m = cfg_dense()
+    blob, ref = reference(m)
+    other = np.random.default_rng(2).integers(0, 256, size=blob.size, dtype=np.uint8)
+    ref_other = oracle.unpack(m, other)
+    d = DeviceDsts(m)
+    a = torch.from_numpy(other).to("cuda")
+    b = torch.from_numpy(blob).pin_memory()
+    S = 256 << 10
+    with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=S) as plan:
+        for k in range(5):
+            if k % 2 == 0:
+                plan.load_async(cfa.Source.device(a.data_ptr()))
+                want = ref_other.cksum
+            else:
+                plan.load_async(cfa.Source.pinned(b.data_ptr()))
+                want = ref.cksum
+            assert np.array_equal(plan.checksums(), want), k
+        plan.reset_checksums()
+        stage = torch.empty(S, dtype=torch.uint8, device="cuda")
+        for c in range(plan.info()["n_chunks"]):
+            part = other[c * S:(c + 1) * S]
+            stage[:part.size].copy_(torch.from_numpy(part))
+            plan.unpack_chunks_async(c, c + 1, stage.data_ptr())
+        torch.cuda.synchronize()
+        assert np.array_equal(plan.checksums(), ref_other.cksum)
+    for j in range(m.n_dsts):
+        assert np.array_equal(d.host_bytes(j), ref_other.dst[j])
+
+
 def test_layer_readiness_consumer_stream_and_host():
     m = dense_config("dense_layers", 65, layers=4, hidden=512, n_q=8, n_kv=2, head_dim=64,
                      inter=1536, vocab=1000)
