@@ -251,7 +251,7 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs, sweep=False):
     out = {"h2d_pinned_gbs": round(h2d_gbs, 2)}
     # first, next to the end-to-end steps: per-layer readiness of one timed pinned load
     plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                    dev_slots=2, host_slots=0, timing=True, bulk=args.bulk,
+                    dev_slots=3, host_slots=0, timing=True, bulk=args.bulk,
                     stage_slices=args.stage_slices)
     plan.load_async(cfa.Source.pinned(host.data_ptr(), period=m.period or 0), stream)
     plan.wait_layer()
@@ -261,17 +261,18 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs, sweep=False):
         tl = plan.timeline()
         with open(args.timeline, "w") as f:
             json.dump({"workload": m.name, "chunk_bytes": m.chunk_bytes,
-                       "source": "pinned host blob, 2 device staging slots",
+                       "source": "pinned host blob, 3 device staging slots",
                        "columns": ["h2d_begin_ms", "h2d_end_ms", "unpack_begin_ms",
                                    "unpack_end_ms"],
                        "chunks": [[round(float(x), 4) for x in row] for row in tl],
                        "layer_ready_ms": [round(float(x), 4) for x in t]}, f)
     plan.close()
-    # the same staged load with all of each chunk on the copy engine, and all of it pulled by
-    # the SMs (the default splits each chunk's ranges half and half)
-    for pct, key in ((0, "e2e_copy_engine_only"), (100, "e2e_sm_pull_only")):
+    # the same staged load with all of each chunk on the copy engine, and with each chunk's
+    # ranges split half and half between the copy engine and the SM pull kernel (the default
+    # pulls all of it)
+    for pct, key in ((0, "e2e_copy_engine_only"), (50, "e2e_half_copy_engine")):
         plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                        dev_slots=2, host_slots=0, bulk=args.bulk,
+                        dev_slots=3, host_slots=0, bulk=args.bulk,
                         stage_slices=args.stage_slices, pull_percent=pct)
         src = cfa.Source.pinned(host.data_ptr(), period=m.period or 0)
         plan.load_async(src, stream)
@@ -330,7 +331,7 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs, sweep=False):
     for pct, key in ((None, "e2e_pageable"), (0, "e2e_pageable_ring")):
         kw = {} if pct is None else {"pull_percent": pct}
         plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                        dev_slots=2, host_slots=2, fill_threads=threads, bulk=args.bulk, **kw)
+                        dev_slots=3, host_slots=2, fill_threads=threads, bulk=args.bulk, **kw)
         src = cfa.Source.host(pageable.ctypes.data, period=m.period or 0)
         plan.load_async(src, stream)
         plan.checksums()
@@ -384,7 +385,7 @@ def fill_thread_sweep(m, pageable, dsts, entries, stream, args, memcpy_bytes):
             list(ex.map(cp, range(t)))
             memcpy_gbs = part * t / (time.perf_counter() - t0) / 1e9
         plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                        dev_slots=2, host_slots=2, fill_threads=t, bulk=args.bulk,
+                        dev_slots=3, host_slots=2, fill_threads=t, bulk=args.bulk,
                         pull_percent=0)  # the fill threads' ring, not the SM pull
         src = cfa.Source.host(pageable.ctypes.data, period=m.period or 0)
         plan.load_async(src, stream)
@@ -430,7 +431,7 @@ def file_attribution(m, pageable, dsts, stream, args, threads):
         write_s = time.perf_counter() - t0
         st = cfa.Safetensors.open(path)
         plan = cfa.Plan(st.entries(targets_for(m)), dsts.cfa_dsts, st.data_bytes,
-                        chunk_bytes=m.chunk_bytes, dev_slots=2, host_slots=2,
+                        chunk_bytes=m.chunk_bytes, dev_slots=3, host_slots=2,
                         fill_threads=threads, bulk=args.bulk)
         with cfa.Source.file(path, st.data_offset) as src:
             plan.load_async(src, stream)
@@ -753,7 +754,7 @@ def measure_e2e(m, entries, dsts, host, stream, ranks, steps, warmup, args, ck_w
 
     import paper_2607_18957_gb300 as cfa
     plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                    dev_slots=2, host_slots=0, bulk=args.bulk, stage_slices=args.stage_slices)
+                    dev_slots=3, host_slots=0, bulk=args.bulk, stage_slices=args.stage_slices)
     src = cfa.Source.pinned(host.data_ptr(), period=m.period or 0)
     for _ in range(warmup):
         plan.load_async(src, stream)
@@ -848,7 +849,7 @@ def measure_workload(name, args, ranks, stream, peak, e2e_steps, attribution_on=
             "step_ms_max": round(max(step_ms), 2),
             "host_buffer_h2d_gbs": buffer_gbs,
             "source": f"pinned host {'pool of ' + str(m.period >> 30) + ' GiB (periodic blob)' if m.period else 'blob'}, "
-                      f"2 device staging slots of {m.chunk_bytes >> 20} MiB"}
+                      f"3 device staging slots of {m.chunk_bytes >> 20} MiB"}
         if attribution_on and not args.no_attribution:
             rec["e2e"]["attribution"] = attribution(m, host, dsts, entries, stream, args,
                                                     h2d_gbs, sweep=(name == "llama3_8b_bf16"))

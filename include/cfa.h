@@ -155,7 +155,9 @@ typedef struct cfa_dst {
 #define CFA_OPT_STRICT_COVERAGE 0x1u  /* every destination byte must be written exactly once */
 #define CFA_OPT_HOST_ONLY       0x2u  /* build and validate on the host only: no CUDA call is made,
                                          cfa_plan_get_pieces works, loads return CFA_ERR_INVAL */
-#define CFA_OPT_TIMING          0x4u  /* record per-chunk timing events (cfa_get_stats, timeline) */
+#define CFA_OPT_TIMING          0x4u  /* record per-chunk timing events (cfa_get_stats, timeline);
+                                         a staged chunk's transfer then begins after the previous
+                                         chunk's has ended on both transfer paths */
 #define CFA_OPT_BULK            0x8u  /* copy cast-free slabs whose source, destination and
                                          length are multiples of 16 bytes with the TMA bulk-copy
                                          kernel; without it every slab takes the 16-byte vector
@@ -192,7 +194,8 @@ typedef struct cfa_plan_opts {
     int32_t host_slots;       /* pinned host staging slots of S bytes, allocated by the first HOST
                                  or CALLBACK load (0 = none); default 2 */
     int32_t dev_slots;        /* device staging slots of S bytes, allocated by cfa_plan_create
-                                 (0 = none: DEVICE sources only); default 2 */
+                                 (0 = none: DEVICE sources only); default 3, so that a chunk's
+                                 unpack has two transfers' time before its slot is needed */
     int32_t fill_threads;     /* host threads copying pageable sources into pinned slots; default:
                                  the CPUs the process may run on, at most 32 */
     int32_t device;           /* CUDA device ordinal; -1 = the current device */
@@ -210,8 +213,9 @@ typedef struct cfa_plan_opts {
                                  copy engine's copies of the rest (0 = copy engine only).  On
                                  GB300 the SMs read page-locked memory at the link rate even
                                  from buffers the copy engine reads at half of it; the price is
-                                 one CTA per SM for the length of the transfer.  Default 50;
-                                 no effect on segmented plans and strided 2-D copies */
+                                 one CTA per SM for the length of the transfer.  Default 100
+                                 (all of it pulled); no effect on segmented plans and strided
+                                 2-D copies */
     void *workspace;          /* optional device memory for the staging slots (NULL = plan allocates) */
     uint64_t workspace_bytes; /* must be >= dev_slots * chunk_bytes when workspace is given */
     /* Segmented (multi-path) loading, section 4.2 "Optimization of Distributed Loading":

@@ -435,7 +435,7 @@ class Plan:
     staging slots, streams and events."""
 
     def __init__(self, entries, dsts, blob_bytes, chunk_bytes=512 << 20, host_slots=2,
-                 dev_slots=2, fill_threads=None, slab_bytes=0, tiny_bytes=8192, strict=True,
+                 dev_slots=3, fill_threads=None, slab_bytes=0, tiny_bytes=8192, strict=True,
                  host_only=False, timing=False, bulk=True, no_merge=False, stage_slices=False,
                  device=-1,
                  workspace=0, workspace_bytes=0, world=1, rank=0, gather=None,

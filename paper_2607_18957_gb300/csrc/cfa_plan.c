@@ -79,14 +79,14 @@ void cfa_plan_opts_default(cfa_plan_opts *o)
     memset(o, 0, sizeof *o);
     o->chunk_bytes = 512ull << 20;
     o->host_slots = 2;
-    o->dev_slots = 2;
+    o->dev_slots = 3;
     o->fill_threads = cfa_default_fill_threads();
     o->device = -1;
     o->slab_bytes = 0; /* chosen from the load's size: cfa_auto_slab */
     o->tiny_bytes = 8192;
     o->flags = CFA_OPT_STRICT_COVERAGE | CFA_OPT_BULK;
     o->seg_world = 1;
-    o->pull_percent = 50;
+    o->pull_percent = 100;
 }
 
 /* Rank `rank`'s segment of chunk `chunk` (section 4.2, distributed loading): the chunk is cut

@@ -280,12 +280,13 @@ void CUDART_CB fill_host_fn(void *arg)
  * one kernel's last CTAs overlap the next kernel's first instead of the GPU draining between
  * them.  With tma = false (a source in host memory, read over the host link) the aligned slabs
  * planned for the TMA kernel are copied by the vector kernel instead: bulk copies are for
- * device memory. */
+ * device memory.  grid_div > 1 divides every kernel's grid cap by it. */
 enum { LAUNCH_CONTIG = 1, LAUNCH_STRIDED = 2, LAUNCH_ALL = 3 };
 
 cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint64_t period,
-                  cudaStream_t s, bool tma = true, int what = LAUNCH_ALL)
+                  cudaStream_t s, bool tma = true, int what = LAUNCH_ALL, int grid_div = 1)
 {
+    auto cap = [grid_div](int c) { return std::max(1, c / grid_div); };
     const cfa_host_plan &hp = p->hp;
     const uint64_t lo = (uint64_t)c0 * hp.chunk_bytes;
     const uint64_t hi = std::min<uint64_t>(hp.blob_bytes, (uint64_t)c1 * hp.chunk_bytes);
@@ -328,18 +329,18 @@ cfa_status launch(cfa_plan *p, uint32_t c0, uint32_t c1, uint64_t src_base, uint
         }
         if (J.type == BULK)
             CK(p, cfa_launch_bulk(k, p->d_bulk + J.a0, J.a1 - J.a0, src_base, period, lo, hi,
-                                  p->d_ck, p->d_status, p->bulk_grid_cap[k], ls));
+                                  p->d_ck, p->d_status, cap(p->bulk_grid_cap[k]), ls));
         else if (J.type == BULK_AS_VECTOR) /* bulk items are copy-class slabs of class k */
             CK(p, cfa_launch_unpack(k, p->d_bulk + J.a0, J.a1 - J.a0, nullptr, 0, src_base,
-                                    period, lo, hi, p->d_ck, p->d_status, p->grid_cap[k], tma,
-                                    ls));
+                                    period, lo, hi, p->d_ck, p->d_status, cap(p->grid_cap[k]),
+                                    tma, ls));
         else if (J.type == STRIDED)
             CK(p, cfa_launch_strided(k, p->d_strided + J.a0, J.a1 - J.a0, src_base, period, lo,
-                                     hi, p->d_ck, p->d_status, p->strided_grid_cap[k], ls));
+                                     hi, p->d_ck, p->d_status, cap(p->strided_grid_cap[k]), ls));
         else
             CK(p, cfa_launch_unpack(k, p->d_slabs + J.a0, J.a1 - J.a0, p->d_tiny + J.b0,
                                     J.b1 - J.b0, src_base, period, lo, hi, p->d_ck, p->d_status,
-                                    p->grid_cap[k], tma, ls));
+                                    cap(p->grid_cap[k]), tma, ls));
         if (timing) CK(p, cudaEventRecord(p->t_k1[p->last_launches], ls));
         p->last_launches++;
     }
@@ -878,7 +879,17 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
         }
         if (pull_on) CK(p, cudaStreamWaitEvent(p->pull_stream, p->ev_begin, 0));
         constexpr uint64_t kMinPull = 64u << 10; /* smaller shares stay with the copy engine */
+        /* A staged chunk's unpack runs beside the next chunk's transfer: at a quarter of the
+         * grid it still outruns the host link many times over, and it leaves most SMs to the
+         * pull kernel, whose CTAs would otherwise wait for a full-grid unpack to end before
+         * they start (the link idle meanwhile).  The last chunk, which nothing follows, takes
+         * the whole grid. */
+        constexpr int kStagedGridDiv = 4;
+        uint32_t last_busy = 0;
+        for (uint32_t c = 0; c < hp.n_chunks; ++c)
+            if (p->chunk_busy[c]) last_busy = c;
         uint32_t k = 0; /* busy chunks so far: they take the slots in turn */
+        cudaEvent_t prev_h2d_end = nullptr; /* CFA_OPT_TIMING: the last transfer's end event */
         for (uint32_t c = 0; c < hp.n_chunks; ++c) {
             if (!p->chunk_busy[c] || gather_failed) {
                 cfa_status st = record_layers(p, c, c + 1, cs);
@@ -902,7 +913,12 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             }
             uint8_t *dslot = p->d_slots + (uint64_t)ds * p->slot_bytes;
             CK(p, cudaStreamWaitEvent(p->copy_stream, p->ev_dev_free[ds], 0));
-            if (timing) CK(p, cudaEventRecord(p->t_h2d0[c], p->copy_stream));
+            if (timing) {
+                /* with CFA_OPT_TIMING a chunk's transfer (copy engine and pull) begins after the
+                 * previous chunk's has ended, so that each interval is that chunk's alone */
+                if (prev_h2d_end) CK(p, cudaStreamWaitEvent(p->copy_stream, prev_h2d_end, 0));
+                CK(p, cudaEventRecord(p->t_h2d0[c], p->copy_stream));
+            }
             bool pulled = false;
             /* InMem -> InGPU: only the ranges the chunk's pieces read */
             for (uint32_t k = hp.copy_first[c]; k < hp.copy_first[c + 1]; ++k) {
@@ -929,6 +945,8 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
                             CK(p, cudaStreamWaitEvent(p->pull_stream, p->ev_dev_free[ds], 0));
                             if (staged)
                                 CK(p, cudaStreamWaitEvent(p->pull_stream, p->ev_filled[hs], 0));
+                            if (timing)
+                                CK(p, cudaStreamWaitEvent(p->pull_stream, p->t_h2d0[c], 0));
                             pulled = true;
                         }
                         CK(p, cfa_launch_pull(static_cast<const uint8_t *>(hsrc) + at + ce,
@@ -941,7 +959,10 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
                                             cp.width, cp.rows, cudaMemcpyHostToDevice,
                                             p->copy_stream));
             }
-            if (timing) CK(p, cudaEventRecord(p->t_h2d1[c], p->copy_stream));
+            if (timing && !pulled) {
+                CK(p, cudaEventRecord(p->t_h2d1[c], p->copy_stream));
+                prev_h2d_end = p->t_h2d1[c];
+            }
             p->last_h2d++;
             ++k;
             CK(p, cudaEventRecord(p->ev_h2d[ds], p->copy_stream));
@@ -949,8 +970,17 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
                 /* both transfers must be done before the unpack, and before the pinned host
                  * slot is refilled: the caller's stream waits for both and marks the slot free */
                 CK(p, cudaEventRecord(p->ev_pulled[ds], p->pull_stream));
-                CK(p, cudaStreamWaitEvent(cs, p->ev_pulled[ds], 0));
-                CK(p, cudaStreamWaitEvent(cs, p->ev_h2d[ds], 0));
+                if (timing) {
+                    /* the transfer ends when both paths have: its end event follows both,
+                     * and the unpack waits for that event */
+                    CK(p, cudaStreamWaitEvent(p->pull_stream, p->ev_h2d[ds], 0));
+                    CK(p, cudaEventRecord(p->t_h2d1[c], p->pull_stream));
+                    CK(p, cudaStreamWaitEvent(cs, p->t_h2d1[c], 0));
+                    prev_h2d_end = p->t_h2d1[c];
+                } else {
+                    CK(p, cudaStreamWaitEvent(cs, p->ev_pulled[ds], 0));
+                    CK(p, cudaStreamWaitEvent(cs, p->ev_h2d[ds], 0));
+                }
                 if (staged) CK(p, cudaEventRecord(p->ev_host_free[hs], cs));
             } else if (staged) {
                 CK(p, cudaEventRecord(p->ev_host_free[hs], p->copy_stream));
@@ -986,7 +1016,8 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
             }
             CK(p, cudaStreamWaitEvent(cs, ready, 0));
             cfa_status st = launch(p, c, c + 1, (uint64_t)(uintptr_t)dslot - off, 0, cs, true,
-                                   slices_in_place ? LAUNCH_CONTIG : LAUNCH_ALL);
+                                   slices_in_place ? LAUNCH_CONTIG : LAUNCH_ALL,
+                                   c == last_busy ? 1 : kStagedGridDiv);
             if (st) return st;
             CK(p, cudaEventRecord(p->ev_dev_free[ds], cs));
             if (direct_c) CK(p, cudaStreamWaitEvent(cs, p->ev_direct, 0));

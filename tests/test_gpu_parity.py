@@ -518,13 +518,16 @@ def test_two_plans_load_at_once_from_two_threads():
         plan.close()
 
 
-def test_timeline_orders_copies_before_unpacks():
+@pytest.mark.parametrize("slots,pull", [(3, None), (2, None), (2, 0), (3, 50)])
+def test_timeline_orders_copies_before_unpacks(slots, pull):
+    """Per-chunk timeline of a staged load (the transfer's interval covers the copy engine's
+    copies and the pull kernel's, whichever ran)."""
     m = CONFIGS["dense"]()
     blob, ref = reference(m)
     keep = []
     d = DeviceDsts(m)
     with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=1 << 20,
-                  timing=True) as plan:
+                  timing=True, dev_slots=slots, pull_percent=pull) as plan:
         plan.load_async(make_source("pinned", m, blob, keep))
         plan.wait_layer()
         t = plan.timeline()
@@ -535,8 +538,8 @@ def test_timeline_orders_copies_before_unpacks():
         assert ran.sum() >= n - 1
         # a chunk is unpacked only after its copy into the device slot has finished
         assert (t[ran, 2] >= t[ran, 1] - 1e-3).all() and (t[ran, 3] >= t[ran, 2]).all()
-        # with two device slots, chunk c + 2's copy waits for chunk c's unpack
-        assert (t[2:, 0] >= t[:-2, 3] - 1e-3)[ran[:-2]].all()
+        # with k device slots, chunk c + k's transfer waits for chunk c's unpack
+        assert (t[slots:, 0] >= t[:-slots, 3] - 1e-3)[ran[:-slots]].all()
         # a device-resident source: no copies, one merged launch over every chunk
         plan.load_async(make_source("device", m, blob, keep))
         plan.wait_layer()
@@ -557,7 +560,7 @@ def test_staged_load_skips_chunks_no_piece_reads(kind):
     keep = []
     d = DeviceDsts(m)
     with cfa.Plan(entries_for(m), d.cfa_dsts, m.blob_bytes, chunk_bytes=64 << 10,
-                  timing=True, fill_threads=4) as plan:
+                  timing=True, fill_threads=4, dev_slots=2) as plan:
         n = plan.info()["n_chunks"]
         busy = np.zeros(n, dtype=bool)
         busy[plan.pieces()["chunk"]] = True
@@ -575,7 +578,7 @@ def test_staged_load_skips_chunks_no_piece_reads(kind):
             tb = t[busy]
             assert (tb[:, 0] >= 0).all() and (tb[:, 1] >= tb[:, 0]).all()
             assert (tb[:, 2] >= tb[:, 1] - 1e-3).all() and (tb[:, 3] >= tb[:, 2]).all()
-            assert (tb[1:, 0] >= tb[:-1, 1] - 1e-3).all()  # one copy stream, chunk order
+            assert (tb[1:, 0] >= tb[:-1, 1] - 1e-3).all()  # transfers in chunk order
             # the slot of busy chunk k + 2 is the slot of busy chunk k
             assert (tb[2:, 0] >= tb[:-2, 3] - 1e-3).all()
             lt = plan.layer_times()
