@@ -337,11 +337,14 @@ cfa_status cfa_plan_create(const cfa_tensor_entry *entries, size_t n_entries,
 
 /*
  * Enqueues one complete load of the blob into the destinations and returns without waiting.
- * Every chunk goes through: host staging (HOST: copied by the plan's fill threads; CALLBACK:
- * written by src->fill; PINNED, DEVICE and HOST_DIRECT: none), a host->device copy on the
- * plan's copy stream (none for DEVICE and HOST_DIRECT), and the unpack kernels on `stream`
- * that write all pieces of the chunk (DEVICE sources merge all chunks into one launch per work
- * class).  Staging and copies move only the byte ranges the chunk's pieces read (strided 2-D
+ * Every chunk goes through: host staging (HOST without pageable access, or with pull_percent
+ * 0: copied by the plan's fill threads; CALLBACK: written by src->fill; PINNED, DEVICE and
+ * HOST_DIRECT: none), a host->device transfer into a device slot (none for DEVICE and
+ * HOST_DIRECT): the plan's pull kernel on a stream of the plan for pull_percent of each
+ * contiguous range, the copy engine on the plan's copy stream for the rest and for strided 2-D
+ * copies; and the unpack kernels on `stream` that write all pieces of the chunk (DEVICE sources
+ * merge all chunks into one launch per work class; a staged chunk's unpack, beside the next
+ * transfer, runs on a quarter of the grid, the last chunk's on all of it).  Staging and copies move only the byte ranges the chunk's pieces read (strided 2-D
  * copies for column slices), so a tensor-parallel rank moves about its share of the
  * checkpoint; cfa_stats.staged_bytes gives the total.  A chunk no piece reads (an
  * expert-parallel rank's view of other ranks' experts) is skipped altogether: no fill, no copy,
