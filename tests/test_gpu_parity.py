@@ -180,6 +180,18 @@ def test_parity_sources(cfg, kind):
 
 
 @pytest.mark.parametrize("cfg", list(CONFIGS))
+@pytest.mark.parametrize("kind", ["pinned", "callback", "host"])
+@pytest.mark.parametrize("pull,slots", [(0, 2), (50, 3), (100, 1)])
+def test_parity_transfer_paths(cfg, kind, pull, slots):
+    """Staged loads through the copy engine alone, split half and half with the pull kernel,
+    and pulled alone through a single device slot (every transfer then waits for the previous
+    chunk's unpack), at chunk sizes whose ranges go to both paths."""
+    m = CONFIGS[cfg]()
+    stats = load_and_compare(m, kind, chunk=(1 << 20) + 4096, pull_percent=pull, dev_slots=slots)
+    assert stats["staged_bytes"] > 0
+
+
+@pytest.mark.parametrize("cfg", list(CONFIGS))
 @pytest.mark.parametrize("chunk", [256, 4096 + 256, 3 << 20, 1 << 30])
 def test_parity_chunk_sizes(cfg, chunk):
     """Theorem 2: the chunking (any chunk length) must not change the loaded state."""
