@@ -755,7 +755,7 @@ def host_buffer_rate(host, stream, passes=2):
 
 def measure_e2e(m, entries, dsts, host, stream, ranks, steps, warmup, args, ck_want):
     """End-to-end steps through the C ABI from the pinned host blob: every step copies the
-    staged bytes host->device through two device slots, unpacks, and reads the checksums
+    staged bytes host->device through three device slots, unpacks, and reads the checksums
     back.  Returns (ms per step over the slowest rank, per-step ms, staged bytes)."""
     import numpy as np
     import torch

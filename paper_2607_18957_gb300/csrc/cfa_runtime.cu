@@ -818,15 +818,18 @@ cfa_status cfa_load_async(cfa_plan *p, const cfa_source *src, cfa_stream stream_
     CK(p, cudaEventRecord(p->ev_begin, cs));
     CK(p, cudaStreamWaitEvent(p->fill_stream, p->ev_begin, 0));
     CK(p, cudaStreamWaitEvent(p->copy_stream, p->ev_begin, 0));
-    use_ck_half(p, p->ck_half ^ 1);
     {
-        unsigned long long *other = p->d_ck_mem + (size_t)(p->ck_half ^ 1) * p->ck_half_words;
+        /* the half the previous load used is cleared for the next load; this load switches to
+         * the other one only once that clear is enqueued, so a load that fails here leaves the
+         * clean half for the next */
+        unsigned long long *prev = p->d_ck;
         CK(p, cudaStreamWaitEvent(p->ck_stream, p->ev_begin, 0));
         if (hp.any_cksum)
-            CK(p, cudaMemsetAsync(other, 0, ck_clear_bytes(hp.n_entries), p->ck_stream));
+            CK(p, cudaMemsetAsync(prev, 0, ck_clear_bytes(hp.n_entries), p->ck_stream));
         else
-            CK(p, cudaMemsetAsync(other + (p->ck_half_words - 1), 0, sizeof(int), p->ck_stream));
+            CK(p, cudaMemsetAsync(prev + (p->ck_half_words - 1), 0, sizeof(int), p->ck_stream));
         CK(p, cudaEventRecord(p->ev_ck_clear, p->ck_stream));
+        use_ck_half(p, p->ck_half ^ 1);
     }
     for (uint32_t l : p->layers_empty) CK(p, cudaEventRecord(p->ev_layer[l], cs));
 
