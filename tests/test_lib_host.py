@@ -333,6 +333,26 @@ def test_default_options_take_the_bulk_path():
         assert st["n_bulk"] == 0 and st["n_slabs"] > 0
 
 
+def test_default_staging_options_match_the_header():
+    """The documented staging defaults: 512 MiB chunks, 2 pinned and 3 device slots, the whole
+    of each range pulled by the SMs, automatic slab size, 8 KiB tiny threshold; the binding's
+    Plan() takes the same device slot count and leaves pull_percent to the library."""
+    import ctypes
+    import inspect
+    import re
+    lib = _lib.load()
+    o = _lib.PlanOpts()
+    lib.cfa_plan_opts_default(ctypes.byref(o))
+    assert (o.chunk_bytes, o.host_slots, o.dev_slots) == (512 << 20, 2, 3)
+    assert (o.pull_percent, o.slab_bytes, o.tiny_bytes, o.seg_world) == (100, 0, 8192, 1)
+    params = inspect.signature(cfa.Plan).parameters
+    assert params["dev_slots"].default == o.dev_slots
+    assert params["pull_percent"].default is None
+    hdr = open(os.path.join(os.path.dirname(__file__), "..", "include", "cfa.h")).read()
+    assert re.search(r"dev_slots;.*?default 3", hdr, re.S)
+    assert re.search(r"pull_percent;.*?Default 100", hdr, re.S)
+
+
 def test_log_lines_on_request():
     """CFA_LOG=1 prints one line per plan and per error on stderr (a child process, so the
     variable is read fresh)."""
