@@ -333,6 +333,27 @@ __device__ uint64_t convert_run(const uint8_t *__restrict__ src, uint8_t *__rest
                 x[u][0] = a.x & 0xFFFFu; x[u][1] = a.x >> 16; x[u][2] = a.y & 0xFFFFu;
                 x[u][3] = a.y >> 16; x[u][4] = a.z & 0xFFFFu; x[u][5] = a.z >> 16;
                 x[u][6] = a.w & 0xFFFFu; x[u][7] = a.w >> 16;
+            } else if (SES == 4 && ((uintptr_t)src & 7u) == 0) {
+                /* 8-byte aligned: four 8-byte loads instead of eight 4-byte ones */
+                const uint2 *s2 = reinterpret_cast<const uint2 *>(src + 32ull * g);
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const uint2 v = __ldg(s2 + q);
+                    x[u][2 * q] = v.x;
+                    x[u][2 * q + 1] = v.y;
+                }
+            } else if (SES == 4) {
+                /* 4 mod 8: the first and last elements alone, the six between as 8-byte pairs */
+                const uint32_t *s1 = reinterpret_cast<const uint32_t *>(src + 32ull * g);
+                const uint2 *s2 = reinterpret_cast<const uint2 *>(s1 + 1);
+                x[u][0] = __ldg(s1);
+#pragma unroll
+                for (int q = 0; q < 3; ++q) {
+                    const uint2 v = __ldg(s2 + q);
+                    x[u][1 + 2 * q] = v.x;
+                    x[u][2 + 2 * q] = v.y;
+                }
+                x[u][7] = __ldg(s1 + 7);
             } else {
 #pragma unroll
                 for (int q = 0; q < 8; ++q)
