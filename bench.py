@@ -267,10 +267,10 @@ def attribution(m, host, dsts, entries, stream, args, h2d_gbs, sweep=False):
                        "chunks": [[round(float(x), 4) for x in row] for row in tl],
                        "layer_ready_ms": [round(float(x), 4) for x in t]}, f)
     plan.close()
-    # the same staged load with all of each chunk on the copy engine, and with each chunk's
-    # ranges split half and half between the copy engine and the SM pull kernel (the default
-    # pulls all of it)
-    for pct, key in ((0, "e2e_copy_engine_only"), (50, "e2e_half_copy_engine")):
+    # the same staged load with each chunk's ranges split half and half between the copy engine
+    # and the SM pull kernel (the default pulls all of it; the copy engine alone is in every
+    # workload's e2e record)
+    for pct, key in ((50, "e2e_half_copy_engine"),):
         plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
                         dev_slots=3, host_slots=0, bulk=args.bulk,
                         stage_slices=args.stage_slices, pull_percent=pct)
@@ -753,7 +753,8 @@ def host_buffer_rate(host, stream, passes=2):
     return out
 
 
-def measure_e2e(m, entries, dsts, host, stream, ranks, steps, warmup, args, ck_want):
+def measure_e2e(m, entries, dsts, host, stream, ranks, steps, warmup, args, ck_want,
+                pull_percent=None):
     """End-to-end steps through the C ABI from the pinned host blob: every step copies the
     staged bytes host->device through three device slots, unpacks, and reads the checksums
     back.  Returns (ms per step over the slowest rank, per-step ms, staged bytes)."""
@@ -762,7 +763,8 @@ def measure_e2e(m, entries, dsts, host, stream, ranks, steps, warmup, args, ck_w
 
     import paper_2607_18957_gb300 as cfa
     plan = cfa.Plan(entries, dsts.cfa_dsts, m.blob_bytes, chunk_bytes=m.chunk_bytes,
-                    dev_slots=3, host_slots=0, bulk=args.bulk, stage_slices=args.stage_slices)
+                    dev_slots=3, host_slots=0, bulk=args.bulk, stage_slices=args.stage_slices,
+                    pull_percent=pull_percent)
     src = cfa.Source.pinned(host.data_ptr(), period=m.period or 0)
     for _ in range(warmup):
         plan.load_async(src, stream)
@@ -869,6 +871,14 @@ def measure_workload(name, args, ranks, stream, peak, e2e_steps, attribution_on=
             "host_buffer_h2d_gbs": buffer_gbs,
             "source": f"pinned host {'pool of ' + str(m.period >> 30) + ' GiB (periodic blob)' if m.period else 'blob'}, "
                       f"3 device staging slots of {m.chunk_bytes >> 20} MiB"}
+        # the same staged load with every transfer on the copy engine (`cudaMemcpyAsync` on the
+        # plan's copy stream, pull_percent 0) instead of the default pull kernel
+        ce_ms, ce_steps, _ = measure_e2e(m, entries, dsts, host, stream, ranks, 3, 1, args,
+                                         ck_dev, pull_percent=0)
+        rec["e2e"]["copy_engine_only"] = {
+            "seconds_per_model": round(ce_ms / 1e3, 5),
+            "frac_of_h2d": round((staged / (ce_ms / 1e3) / 1e9) / h2d_gbs, 4),
+            "step_ms": [round(x, 1) for x in ce_steps]}
         if attribution_on and not args.no_attribution:
             rec["e2e"]["attribution"] = attribution(m, host, dsts, entries, stream, args,
                                                     h2d_gbs, sweep=(name == "llama3_8b_bf16"))
@@ -886,7 +896,8 @@ def _config_record(rec):
     if e2e:
         out["e2e"] = {k: e2e[k] for k in ("seconds_per_model", "frac_of_h2d", "h2d_gbs_measured",
                                           "h2d_bytes_per_step", "step_ms_median", "step_ms_max",
-                                          "host_buffer_h2d_gbs", "steps", "source")}
+                                          "host_buffer_h2d_gbs", "steps", "source",
+                                          "copy_engine_only")}
         if "attribution" in e2e:
             out["e2e"]["attribution"] = e2e["attribution"]
     return out
