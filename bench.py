@@ -932,8 +932,10 @@ def run_ours(args):
     torch.cuda.empty_cache()
 
     e2e_steps = 0 if args.no_e2e else (args.e2e_steps or min(args.steps, 20))
+    # the attribution (pageable copies, a safetensors file of the 8B, fill-thread sweeps) is a
+    # single-GPU diagnostic: replicas would multiply its host memory and disk use by N
     head, m = measure_workload(args.workload, args, ranks, stream, peak, e2e_steps,
-                               attribution_on=True)
+                               attribution_on=(world == 1))
     h2d_gbs = head["_h2d_gbs"]
     names = [] if args.configs in ("", "none") else \
         [n for n in args.configs.split(",") if n and n != args.workload]
@@ -942,7 +944,8 @@ def run_ours(args):
         try:
             rec, mc = measure_workload(name, args, ranks, stream, peak,
                                        0 if args.no_e2e else min(e2e_steps, 8),
-                                       attribution_on=(name == "llama3_8b_bf16"),
+                                       attribution_on=(name == "llama3_8b_bf16" and
+                                                       world == 1),
                                        h2d_gbs=h2d_gbs)
         except Exception as e:  # noqa: BLE001 -- one workload must not cost the whole line
             if world > 1:
