@@ -619,7 +619,7 @@ def run_reference(args):
         "vs_baseline": None, "dtype": path_types(m)[0],
         "data": f"synthetic (seeded counter-based generator; {_BLOB_KIND[m.blob_kind]})",
         "config": {"workload": m.name, "step": "one destination tensor per step, in blob order",
-                   "parallelism": "replicas"},
+                   "parallelism": "rank 0 of replicas" if args.gpus > 1 else "single host"},
         "cpu_baseline": {"value": round(gbs, 4), "unit": UNIT, "cores": cores,
                          "host_cores": host_cores(), "kind": "oracle", "sample": desc},
         "e2e": {"value": round(gbs, 4), "unit": UNIT, "h2d_bytes_per_step": 0,
